@@ -1,0 +1,104 @@
+/*
+ * domino_oracle.h -- plain fp64 CPU oracle of the Domino draft-side block step.
+ *
+ * TEST INFRASTRUCTURE ONLY.  This library exists to check the CUDA path; it is
+ * called from the tests, from the package smoke check and from the CPU-baseline
+ * leg of the benchmark, never from the product path.  It shares no code, header,
+ * table or helper with the CUDA library (include/domino.h) and includes nothing
+ * from it.
+ *
+ * Conventions
+ *   - bf16 tensors are passed as raw uint16_t bit patterns and widened exactly to
+ *     double; every intermediate is double; nothing is rounded in between.
+ *   - Row-major everywhere; a weight [rows, cols] has element (r, c) at r*cols + c.
+ *   - A NULL bias means a zero bias.
+ *   - Return codes: 0 ok, ORACLE_ERR_ARG (-1) for bad sizes or pointers,
+ *     ORACLE_ERR_TOKEN (-2) for a prefix id outside [0, V).
+ *
+ * Notation follows the paper (Domino, arXiv 2605.29707): B sequences, K draft
+ * positions, hidden size H, vocabulary V, GRU state size Ds (d_s), correction
+ * rank R (r), top-k width k, N tree nodes per sequence.
+ */
+#ifndef DOMINO_ORACLE_H
+#define DOMINO_ORACLE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ORACLE_ERR_ARG (-1)
+#define ORACLE_ERR_TOKEN (-2)
+
+/* Exact bf16 -> double widening. */
+double oracle_bf16_to_double(uint16_t b);
+
+/* O1, section 4.1.2 "Causal Encoder": E_j is the token embedding of prefix id j.
+ * emb: bf16 [V, H]; ids: [n]; E: double [n, H]. */
+int oracle_embed(const uint16_t* emb, int V, int H, const int32_t* ids, int n, double* E);
+
+/* O2, section 4.1.2 causal-encoder equation S_{i-1} = GRU(E_{<=i-1}).
+ * GRU with torch.nn.GRU gate conventions (gate blocks r | z | n):
+ *   r = sigmoid(W_ir x + b_ir + W_hr h + b_hr)
+ *   z = sigmoid(W_iz x + b_iz + W_hz h + b_hz)
+ *   n = tanh(W_in x + b_in + r * (W_hn h + b_hn))
+ *   h' = (1 - z) * n + z * h,  starting from h = 0.
+ * E: double [K, Hin]; w_ih bf16 [3Ds, Hin]; w_hh bf16 [3Ds, Ds]; b_ih, b_hh bf16 [3Ds] or NULL.
+ * S: double [K, Ds], S[j] = state after absorbing E_0..E_j. */
+int oracle_gru(const double* E, int K, int Hin, int Ds, const uint16_t* w_ih, const uint16_t* w_hh,
+               const uint16_t* b_ih, const uint16_t* b_hh, double* S);
+
+/* O3, section 4.1.2 low-rank correction equation: u_j = SiLU(W1 [hidden_j ; S_j] + b1).
+ * hidden: double [K, H]; S: double [K, Ds]; w1 bf16 [R, H + Ds] (columns 0..H-1 multiply
+ * hidden, H..H+Ds-1 multiply S); b1 bf16 [R] or NULL.  u: double [K, R]. */
+int oracle_lowrank(const double* hidden, const double* S, int K, int H, int Ds, int R,
+                   const uint16_t* w1, const uint16_t* b1, double* u);
+
+/* O4, section 4.1.1 base-logit equation plus section 4.1.2 residual:
+ *   z_j[v] = W_lm[v] . hidden_j + W2[v] . u_j + b2[v].
+ * hidden: double [K, H]; u: double [K, R] (ignored when R == 0); w_lm bf16 [V, H];
+ * w2 bf16 [V, R] or NULL (no correction); b2 bf16 [V] or NULL.  z: double [K, V].
+ * nthreads > 1 splits the (row, vocab) grid across OpenMP threads. */
+int oracle_logits(const double* hidden, const double* u, int K, int H, int V, int R,
+                  const uint16_t* w_lm, const uint16_t* w2, const uint16_t* b2, double* z,
+                  int nthreads);
+
+/* O5: log-softmax of each row: lse = m + log(sum_v exp(z - m)), logp = z - lse. */
+int oracle_log_softmax(const double* z, int n, int V, double* logp, double* lse);
+
+/* O6: the k best entries of each row ordered by (value descending, id ascending). */
+int oracle_topk(const double* logp, int n, int V, int k, int32_t* ids, double* vals);
+
+/* O7, draft tree: best-first selection of N nodes.  The frontier starts with the k
+ * depth-1 candidates of position 0; each pop takes the candidate with the greatest
+ * (score, then lower token id, then lower parent index); a popped node of depth d < K
+ * pushes its k children from position d's top-k list with score = parent score + logp.
+ * topk_ids / topk_logp: [K, k].  Outputs [N]: parent (-1 for the root/anchor), token,
+ * depth (1..K), score (cumulative log-probability). */
+int oracle_tree(const int32_t* topk_ids, const double* topk_logp, int K, int k, int N,
+                int32_t* parent, int32_t* token, int32_t* depth, double* score);
+
+/* The whole step for the sequences listed in seqs (nseq of them; seqs == NULL means
+ * all B in order).  Output arrays are indexed by the position in that list.
+ *   hidden bf16 [B, K, H], prefix_ids [B, K], w_lm bf16 [V, H], emb bf16 [V, H],
+ *   w_ih [3Ds, H], w_hh [3Ds, Ds], b_ih/b_hh [3Ds] or NULL, w1 [R, H+Ds], b1 [R] or NULL,
+ *   w2 [V, R] or NULL, b2 [V] or NULL.
+ * Outputs: logp_full [nseq, K, V] or NULL, lse [nseq, K] or NULL,
+ *   topk_ids/topk_logp [nseq, K, k], tree_* [nseq, N]. */
+int oracle_draft_step(const uint16_t* hidden, const int32_t* prefix_ids, const uint16_t* w_lm,
+                      const uint16_t* emb, const uint16_t* w_ih, const uint16_t* w_hh,
+                      const uint16_t* b_ih, const uint16_t* b_hh, const uint16_t* w1,
+                      const uint16_t* b1, const uint16_t* w2, const uint16_t* b2, int B, int K,
+                      int H, int V, int Ds, int R, int k, int N, const int32_t* seqs, int nseq,
+                      double* logp_full, double* lse, int32_t* topk_ids, double* topk_logp,
+                      int32_t* tree_parent, int32_t* tree_token, int32_t* tree_depth,
+                      double* tree_score, int nthreads);
+
+/* Number of OpenMP threads the oracle would use for nthreads <= 0 (all available). */
+int oracle_max_threads(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

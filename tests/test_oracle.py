@@ -1,0 +1,371 @@
+"""Pins for the fp64 CPU oracle (CPU only).
+
+Each test ties one oracle step to something other than the oracle itself: a
+hand-worked example from tests/golden/, a library routine that computes a special
+case (torch.nn.GRU, scipy's log-softmax, a stable library sort), brute-force
+enumeration, an invariant the method guarantees, or the parameter count the paper
+states.
+"""
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def bf16(x):
+    """float values that are exact in bf16 -> uint16 bit patterns (truncation is exact here)."""
+    a = np.asarray(x, dtype=np.float32)
+    bits = a.view(np.uint32)
+    assert np.all((bits & 0xFFFF) == 0), "value not exactly representable in bf16"
+    return (bits >> 16).astype(np.uint16)
+
+
+def rand_bf16(rng, shape, std):
+    x = torch.from_numpy(rng.standard_normal(shape).astype(np.float32) * std)
+    return x.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+
+
+def to_f64(b):
+    return (np.asarray(b, np.uint16).astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def _ev(expr):
+    return eval(expr, {"__builtins__": {}}, {"log": math.log, "exp": math.exp})
+
+
+def load(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return json.load(f)
+
+
+# ----------------------------------------------------------------------------- hand cases
+
+def test_bf16_widening_exact():
+    assert oracle.bf16_to_double(0x3F80) == 1.0
+    assert oracle.bf16_to_double(0xC000) == -2.0
+    assert oracle.bf16_to_double(0x3F00) == 0.5
+    assert oracle.bf16_to_double(0x3C23) == float(np.float32(np.uint32(0x3C230000).view(np.float32)))
+
+
+@pytest.mark.parametrize("name", ["hand_case_a.json", "hand_case_b.json"])
+def test_hand_cases_head_off(name):
+    g = load(name)
+    V, H, K, k, N = g["V"], g["H"], g["K"], g["k"], g["N"]
+    w = {"w_lm": bf16(g["w_lm"])}
+    hidden = bf16(g["hidden"]).reshape(1, K, H)
+    ids = np.asarray(g["prefix_ids"], np.int32).reshape(1, K)
+    out = oracle.draft_step(w, hidden, ids, k, N, want_logp_full=True)
+    assert out["topk_ids"][0].tolist() == g["expect_topk_ids"]
+    assert out["tree_parent"][0].tolist() == g["expect_tree_parent"]
+    assert out["tree_token"][0].tolist() == g["expect_tree_token"]
+    assert out["tree_depth"][0].tolist() == g["expect_tree_depth"]
+    for i, e in enumerate(g["expect_tree_score"]):
+        assert out["tree_score"][0, i] == pytest.approx(_ev(e), abs=1e-12)
+    if "expect_lse" in g:
+        for j, e in enumerate(g["expect_lse"]):
+            assert out["lse"][0, j] == pytest.approx(_ev(e), abs=1e-12)
+    if "expect_logp" in g:
+        for j in range(K):
+            for v in range(V):
+                assert out["logp_full"][0, j, v] == pytest.approx(_ev(g["expect_logp"][j][v]), abs=1e-12)
+
+
+def test_hand_case_c_head_on():
+    g = load("hand_case_c.json")
+    K, k, N, tol = g["K"], g["k"], g["N"], g["tolerance"]
+    w = {n: bf16(g[n]) for n in ("w_lm", "emb", "w_ih", "w_hh", "b_ih", "b_hh", "w1", "b1", "w2", "b2")}
+    hidden = bf16(g["hidden"]).reshape(1, K, g["H"])
+    ids = np.asarray(g["prefix_ids"], np.int32).reshape(1, K)
+    # step by step
+    E = oracle.embed(w["emb"], ids[0])
+    assert E.tolist() == [[1.0, 0.0], [0.0, 1.0]]
+    S = oracle.gru(E, w["w_ih"], w["w_hh"], w["b_ih"], w["b_hh"])
+    assert S[:, 0] == pytest.approx(g["expect_S"], abs=tol)
+    u = oracle.lowrank(to_f64(hidden[0]), S, w["w1"], w["b1"])
+    assert u[:, 0] == pytest.approx(g["expect_u"], abs=tol)
+    # whole step
+    out = oracle.draft_step(w, hidden, ids, k, N, want_logp_full=True)
+    assert out["logp_full"][0] == pytest.approx(np.asarray(g["expect_logp"]), abs=tol)
+    assert out["topk_ids"][0].tolist() == g["expect_topk_ids"]
+    assert out["tree_parent"][0].tolist() == g["expect_tree_parent"]
+    assert out["tree_token"][0].tolist() == g["expect_tree_token"]
+    assert out["tree_depth"][0].tolist() == g["expect_tree_depth"]
+    assert out["tree_score"][0] == pytest.approx(g["expect_tree_score"], abs=tol)
+
+
+# ----------------------------------------------------------------------------- GRU
+
+@pytest.mark.parametrize("Hin,Ds,K", [(12, 8, 5), (40, 24, 7), (8, 1, 3)])
+def test_gru_matches_torch_nn_gru_fp64(Hin, Ds, K):
+    """torch.nn.GRU (a library GRU) in float64 is the reference for the recurrence."""
+    rng = np.random.default_rng(Hin * 100 + Ds)
+    w_ih = rand_bf16(rng, (3 * Ds, Hin), 0.3)
+    w_hh = rand_bf16(rng, (3 * Ds, Ds), 0.3)
+    b_ih = rand_bf16(rng, (3 * Ds,), 0.3)
+    b_hh = rand_bf16(rng, (3 * Ds,), 0.3)
+    E = rng.standard_normal((K, Hin))
+    S = oracle.gru(E, w_ih, w_hh, b_ih, b_hh)
+    gru = torch.nn.GRU(Hin, Ds, bias=True).double()
+    with torch.no_grad():
+        gru.weight_ih_l0.copy_(torch.from_numpy(to_f64(w_ih)))
+        gru.weight_hh_l0.copy_(torch.from_numpy(to_f64(w_hh)))
+        gru.bias_ih_l0.copy_(torch.from_numpy(to_f64(b_ih)))
+        gru.bias_hh_l0.copy_(torch.from_numpy(to_f64(b_hh)))
+        ref, _ = gru(torch.from_numpy(E).unsqueeze(1))
+    np.testing.assert_allclose(S, ref[:, 0].numpy(), atol=1e-12, rtol=0)
+    # and without biases (NULL means zero)
+    S0 = oracle.gru(E, w_ih, w_hh)
+    with torch.no_grad():
+        gru.bias_ih_l0.zero_(); gru.bias_hh_l0.zero_()
+        ref0, _ = gru(torch.from_numpy(E).unsqueeze(1))
+    np.testing.assert_allclose(S0, ref0[:, 0].numpy(), atol=1e-12, rtol=0)
+
+
+# ----------------------------------------------------------------------------- softmax / top-k
+
+def test_log_softmax_matches_scipy_and_normalises():
+    from scipy.special import log_softmax as sp_lsm
+    rng = np.random.default_rng(1)
+    z = rng.standard_normal((6, 1000)) * 5
+    lp, lse = oracle.log_softmax(z)
+    np.testing.assert_allclose(lp, sp_lsm(z, axis=1), atol=1e-12, rtol=0)
+    np.testing.assert_allclose(np.exp(lp).sum(1), 1.0, atol=1e-12)
+    assert np.all(lp <= 0)
+    # shift invariance and the uniform special case
+    lp2, _ = oracle.log_softmax(z + 123.25)
+    np.testing.assert_allclose(lp2, lp, atol=1e-10)
+    lpu, lseu = oracle.log_softmax(np.zeros((2, 77)))
+    np.testing.assert_allclose(lpu, -math.log(77), atol=1e-14)
+    np.testing.assert_allclose(lseu, math.log(77), atol=1e-14)
+
+
+def test_topk_matches_stable_library_sort_with_ties():
+    rng = np.random.default_rng(2)
+    lp = np.round(rng.standard_normal((10, 300)) * 2) / 4  # coarse grid -> many exact ties
+    for k in (1, 5, 17, 300):
+        ids, vals = oracle.topk(lp, k)
+        for i in range(lp.shape[0]):
+            order = np.lexsort((np.arange(300), -lp[i]))  # value desc, then id asc
+            assert ids[i].tolist() == order[:k].tolist()
+            assert vals[i].tolist() == lp[i, order[:k]].tolist()
+
+
+# ----------------------------------------------------------------------------- tree
+
+def _random_lists(rng, K, k, V=50, ties=False):
+    ids = np.stack([rng.choice(V, size=k, replace=False) for _ in range(K)]).astype(np.int32)
+    lp = -np.sort(rng.exponential(1.0, size=(K, k)), axis=1)
+    if ties:
+        lp = np.round(lp * 4) / 4
+        # keep each list ordered by (value desc, id asc)
+        for j in range(K):
+            o = np.lexsort((ids[j], -lp[j]))
+            ids[j], lp[j] = ids[j][o], lp[j][o]
+    return ids, lp
+
+
+def _paths(K, k):
+    for d in range(1, K + 1):
+        yield from itertools.product(range(k), repeat=d)
+
+
+def _node_path(par, tok, dep, i, ids):
+    path = []
+    while i >= 0:
+        d = dep[i]
+        path.append(int(np.where(ids[d - 1] == tok[i])[0][0]))
+        i = par[i]
+    return tuple(reversed(path))
+
+
+@pytest.mark.parametrize("K,k", [(3, 3), (2, 4), (4, 2), (1, 5)])
+def test_tree_matches_brute_force_enumeration(K, k):
+    rng = np.random.default_rng(K * 10 + k)
+    ids, lp = _random_lists(rng, K, k)
+    allp = list(_paths(K, k))
+    scores = {p: sum(lp[d, c] for d, c in enumerate(p)) for p in allp}
+    ranked = sorted(allp, key=lambda p: -scores[p])
+    for N in range(1, len(allp) + 1):
+        par, tok, dep, sc = oracle.tree(ids, lp, N)
+        got = {_node_path(par, tok, dep, i, ids) for i in range(N)}
+        assert got == set(ranked[:N])
+        np.testing.assert_allclose(sc, sorted((scores[p] for p in ranked[:N]), reverse=True),
+                                   atol=1e-12)
+
+
+@pytest.mark.parametrize("ties", [False, True])
+def test_tree_invariants(ties):
+    rng = np.random.default_rng(7 + ties)
+    K, k, N = 5, 4, 40
+    ids, lp = _random_lists(rng, K, k, ties=ties)
+    par, tok, dep, sc = oracle.tree(ids, lp, N)
+    for i in range(N):
+        assert par[i] < i
+        d = dep[i]
+        assert 1 <= d <= K
+        q = int(np.where(ids[d - 1] == tok[i])[0][0])
+        base = 0.0 if par[i] < 0 else sc[par[i]]
+        assert (d == 1) == (par[i] < 0)
+        if par[i] >= 0:
+            assert dep[par[i]] == d - 1
+        assert sc[i] == base + lp[d - 1, q]  # cumulative score = parent's + own log-prob
+        if i:
+            assert sc[i] <= sc[i - 1]
+    # no node appears twice
+    assert len({(par[i], tok[i]) for i in range(N)}) == N
+
+
+def test_tree_special_cases():
+    rng = np.random.default_rng(11)
+    K, k = 6, 4
+    ids, lp = _random_lists(rng, K, k)
+    # k = 1, N = K: the chain of per-position argmaxes
+    par, tok, dep, sc = oracle.tree(ids[:, :1], lp[:, :1], K)
+    assert tok.tolist() == ids[:, 0].tolist()
+    assert par.tolist() == [-1] + list(range(K - 1))
+    np.testing.assert_allclose(sc, np.cumsum(lp[:, 0]), atol=1e-12)
+    # K = 1: the top-N of position 0
+    par, tok, dep, sc = oracle.tree(ids[:1], lp[:1], 3)
+    assert tok.tolist() == ids[0, :3].tolist() and par.tolist() == [-1, -1, -1]
+    # N = 1: the argmax of position 0
+    par, tok, dep, sc = oracle.tree(ids, lp, 1)
+    assert tok.tolist() == [ids[0, 0]] and sc.tolist() == [lp[0, 0]]
+    # N above the size of the tree is rejected
+    with pytest.raises(oracle.OracleError):
+        oracle.tree(ids[:2, :2], lp[:2, :2], 7)
+
+
+# ----------------------------------------------------------------------------- whole step
+
+def _small_workload(rng, B=2, K=5, H=24, V=64, Ds=16, R=8, biases=True):
+    w = {
+        "w_lm": rand_bf16(rng, (V, H), 0.3), "emb": rand_bf16(rng, (V, H), 0.5),
+        "w_ih": rand_bf16(rng, (3 * Ds, H), 0.3), "w_hh": rand_bf16(rng, (3 * Ds, Ds), 0.3),
+        "w1": rand_bf16(rng, (R, H + Ds), 0.3), "w2": rand_bf16(rng, (V, R), 0.5),
+        "b_ih": None, "b_hh": None, "b1": None, "b2": None,
+    }
+    if biases:
+        w["b_ih"] = rand_bf16(rng, (3 * Ds,), 0.2)
+        w["b_hh"] = rand_bf16(rng, (3 * Ds,), 0.2)
+        w["b1"] = rand_bf16(rng, (R,), 0.2)
+        w["b2"] = rand_bf16(rng, (V,), 0.2)
+    hidden = rand_bf16(rng, (B, K, H), 1.0)
+    ids = rng.integers(0, V, size=(B, K)).astype(np.int32)
+    return w, hidden, ids
+
+
+def test_causality_position_j_sees_ids_0_to_j_only():
+    """Section 4.1.2: S_{i-1} summarises the tokens before position i (anchor first)."""
+    rng = np.random.default_rng(3)
+    w, hidden, ids = _small_workload(rng, B=1)
+    K = ids.shape[1]
+    base = oracle.draft_step(w, hidden, ids, 4, 6, want_logp_full=True)["logp_full"][0]
+    for jp in range(K):
+        ids2 = ids.copy()
+        ids2[0, jp] = (ids2[0, jp] + 17) % w["w_lm"].shape[0]
+        lp = oracle.draft_step(w, hidden, ids2, 4, 6, want_logp_full=True)["logp_full"][0]
+        assert np.array_equal(lp[:jp], base[:jp])           # earlier positions untouched
+        assert np.abs(lp[jp] - base[jp]).max() > 1e-6        # position jp sees id jp
+        if jp + 1 < K:
+            assert np.abs(lp[jp + 1:] - base[jp + 1:]).max() > 1e-6
+
+
+def test_correction_off_gives_base_distribution():
+    """Table 4 'w/o Domino head': with W2 = 0 the refined distribution is the base one."""
+    rng = np.random.default_rng(4)
+    w, hidden, ids = _small_workload(rng)
+    w_off = dict(w, w2=np.zeros_like(w["w2"]))
+    on0 = oracle.draft_step(w_off, hidden, ids, 4, 6, want_logp_full=True)
+    off = oracle.draft_step(dict(w, w2=None), hidden, ids, 4, 6, want_logp_full=True)
+    np.testing.assert_array_equal(on0["logp_full"], off["logp_full"])
+    # base logits: hidden . W_lm^T + b2 (library matmul as the special-case reference)
+    from scipy.special import log_softmax as sp_lsm
+    z = to_f64(hidden).reshape(-1, hidden.shape[-1]) @ to_f64(w["w_lm"]).T + to_f64(w["b2"])
+    np.testing.assert_allclose(off["logp_full"].reshape(z.shape), sp_lsm(z, axis=1), atol=1e-12)
+
+
+def test_uniform_bias_shift_leaves_distribution_unchanged():
+    rng = np.random.default_rng(5)
+    w, hidden, ids = _small_workload(rng, biases=False)
+    a = oracle.draft_step(w, hidden, ids, 4, 6, want_logp_full=True)
+    b2 = np.full(w["w_lm"].shape[0], bf16([2.5])[0], np.uint16)
+    b = oracle.draft_step(dict(w, b2=b2), hidden, ids, 4, 6, want_logp_full=True)
+    np.testing.assert_allclose(a["logp_full"], b["logp_full"], atol=1e-12)
+    assert a["topk_ids"].tolist() == b["topk_ids"].tolist()
+
+
+def test_step_equals_composition_and_sequence_selection():
+    rng = np.random.default_rng(6)
+    w, hidden, ids = _small_workload(rng, B=3)
+    k, N = 4, 9
+    full = oracle.draft_step(w, hidden, ids, k, N, want_logp_full=True)
+    sel = oracle.draft_step(w, hidden, ids, k, N, seqs=[2, 0], want_logp_full=True)
+    for si, b in enumerate([2, 0]):
+        for key in ("logp_full", "topk_ids", "topk_logp", "tree_parent", "tree_token", "tree_score"):
+            np.testing.assert_array_equal(sel[key][si], full[key][b])
+    b = 1
+    E = oracle.embed(w["emb"], ids[b])
+    S = oracle.gru(E, w["w_ih"], w["w_hh"], w["b_ih"], w["b_hh"])
+    u = oracle.lowrank(to_f64(hidden[b]), S, w["w1"], w["b1"])
+    z = oracle.logits(to_f64(hidden[b]), u, w["w_lm"], w["w2"], w["b2"])
+    lp, lse = oracle.log_softmax(z)
+    np.testing.assert_array_equal(lp, full["logp_full"][b])
+    tid, tlp = oracle.topk(lp, k)
+    np.testing.assert_array_equal(tid, full["topk_ids"][b])
+    par, tok, dep, sc = oracle.tree(tid, tlp, N)
+    np.testing.assert_array_equal(tok, full["tree_token"][b])
+
+
+def test_lowrank_concat_order_hidden_then_state():
+    """W1 acts on [H_i; S_{i-1}]: the first H columns see hidden, the rest the state."""
+    H, Ds = 3, 2
+    hidden = np.array([[1.0, 2.0, 3.0]])
+    S = np.array([[10.0, 20.0]])
+    w1 = bf16([[1, 0, 0, 0, 0], [0, 0, 0, 1, 0], [0, 0, 0, 0, 0.5]])
+    u = oracle.lowrank(hidden, S, w1)
+    silu = lambda x: x / (1 + math.exp(-x))
+    assert u[0].tolist() == pytest.approx([silu(1.0), silu(10.0), silu(10.0)], abs=1e-14)
+
+
+def test_bad_token_and_bad_args():
+    rng = np.random.default_rng(8)
+    w, hidden, ids = _small_workload(rng, B=1)
+    bad = ids.copy(); bad[0, 2] = w["w_lm"].shape[0]
+    with pytest.raises(oracle.OracleError) as e:
+        oracle.draft_step(w, hidden, bad, 4, 6)
+    assert e.value.rc == oracle.ERR_TOKEN
+    bad[0, 2] = -1
+    with pytest.raises(oracle.OracleError):
+        oracle.draft_step(w, hidden, bad, 4, 6)
+    with pytest.raises(oracle.OracleError):
+        oracle.draft_step(w, hidden, ids, 0, 6)
+
+
+def test_parameter_count_matches_paper_56M():
+    """The head adds 'only 56M parameters' for Qwen3-8B (d_s = 1024, r = 256, H = 4096,
+    V = 151936).  The shapes the oracle takes must add up to that figure."""
+    H, V, Ds, R = 4096, 151936, 1024, 256
+    gru = 3 * Ds * H + 3 * Ds * Ds + 2 * 3 * Ds   # w_ih, w_hh, b_ih, b_hh
+    w1 = R * (H + Ds)                              # W1 over [H_i; S_{i-1}]
+    w2 = V * R                                     # W2 to the full vocabulary
+    total = gru + w1 + w2
+    assert total == 55_941_120
+    assert round(total / 1e6) == 56
+    # the oracle accepts exactly these shapes (tiny V to keep it fast)
+    rng = np.random.default_rng(9)
+    Vs = 8
+    w = {"w_lm": rand_bf16(rng, (Vs, H), 0.02), "emb": rand_bf16(rng, (Vs, H), 0.02),
+         "w_ih": rand_bf16(rng, (3 * Ds, H), 0.02), "w_hh": rand_bf16(rng, (3 * Ds, Ds), 0.02),
+         "b_ih": None, "b_hh": None, "w1": rand_bf16(rng, (R, H + Ds), 0.02), "b1": None,
+         "w2": rand_bf16(rng, (Vs, R), 0.02), "b2": None}
+    hidden = rand_bf16(rng, (1, 2, H), 1.0)
+    out = oracle.draft_step(w, hidden, np.array([[1, 2]], np.int32), 2, 3)
+    assert out["topk_ids"].shape == (1, 2, 2)
