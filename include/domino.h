@@ -1,0 +1,150 @@
+/*
+ * domino.h -- C ABI of the GB300 (sm_103a) Domino draft-side block step.
+ *
+ * Method: Domino (arXiv 2605.29707).  Given the parallel draft backbone's hidden states for
+ * a K-position draft block and the block's prefix tokens, one call computes, for every
+ * sequence b and draft position j:
+ *   base logits          L_base = W_lm . hidden[b, j]                 (section 4.1.1, LM-head eq.)
+ *   causal state         S_j = GRU(E_0 .. E_j), E_i = emb[prefix_ids[b, i]], h starts at 0
+ *                                                                      (section 4.1.2, encoder eq.)
+ *   low-rank correction  dL = W2 . SiLU(W1 [hidden[b, j]; S_j] + b1) + b2
+ *                                                                      (section 4.1.2, correction eq.)
+ *   final logits         L = L_base + dL                               (section 4.1.2, residual)
+ *   log-softmax of L, its k best tokens (value descending, then token id ascending), and
+ *   the draft tree: the N nodes of highest cumulative log-probability below the anchor,
+ *   chosen best-first with ties to the lower token id and then the lower parent index; a
+ *   node at depth d takes its token from position d-1's top-k list ("Tree" cost, Fig. 1).
+ * prefix_ids[b, 0] is the anchor (last verified token); prefix_ids[b, j >= 1] is the token
+ * drafted for position j-1.  Full logits never reach memory.
+ *
+ * Conventions for every entry point
+ *   - All tensors are row-major and contiguous.  bf16 tensors are raw IEEE bfloat16.
+ *   - Device pointers are owned by the caller; the library never allocates, frees or keeps
+ *     them.  Work is enqueued on `stream` (a cudaStream_t passed as void*; NULL = legacy
+ *     default stream).  domino_draft_step does not synchronise.
+ *   - Synchronous argument checks return a negative DOMINO_ERR_* code before anything is
+ *     enqueued.  Errors found on the device (a prefix id outside [0, V), a device-side wait
+ *     that ran out) are written to a status word inside the workspace and read back by
+ *     domino_check_status; the device never traps or asserts.
+ *   - The library runs on sm_103 devices only (GB300); elsewhere it returns
+ *     DOMINO_ERR_UNSUPPORTED.
+ */
+#ifndef DOMINO_H
+#define DOMINO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define DOMINO_ABI_VERSION 1
+
+#if defined(__GNUC__)
+#define DOMINO_API __attribute__((visibility("default")))
+#else
+#define DOMINO_API
+#endif
+
+enum domino_status {
+  DOMINO_OK = 0,
+  DOMINO_ERR_INVALID_ARG = -1, /* NULL required pointer, size <= 0, k > V, N > sum_{d=1..K} k^d,
+                                  workspace too small */
+  DOMINO_ERR_UNSUPPORTED = -2, /* outside the supported envelope: H, Ds or R not a multiple of 8,
+                                  a tensor pointer not 16-byte aligned, k > 32, N > 256, K > 64,
+                                  Ds > 2048, V >= 2^22, or not an sm_103 device */
+  DOMINO_ERR_CUDA = -3,        /* a CUDA runtime call or kernel launch failed */
+  DOMINO_ERR_TIMEOUT = -4,     /* device: a bounded wait (pipeline barrier, grid barrier) ran out */
+  DOMINO_ERR_BAD_TOKEN = -5    /* device: a prefix id outside [0, V) */
+};
+
+/* The Domino head's weights (section 4.1.2), all device pointers to bf16.
+ * GRU: torch.nn.GRU layout, gate blocks r | z | n:
+ *   w_ih [3*Ds, H], w_hh [3*Ds, Ds], b_ih [3*Ds] or NULL, b_hh [3*Ds] or NULL.
+ *   r = sigmoid(W_ir x + b_ir + W_hr h + b_hr); z = sigmoid(W_iz x + b_iz + W_hz h + b_hz);
+ *   n = tanh(W_in x + b_in + r * (W_hn h + b_hn)); h' = (1 - z) * n + z * h.
+ * emb [V, H]: the target's token embedding table feeding the GRU (may alias w_lm when the
+ *   target ties them); only the rows named by prefix_ids are read.
+ * w1 [R, H + Ds]: columns 0..H-1 multiply hidden, columns H..H+Ds-1 multiply S; b1 [R] or NULL.
+ * w2 [V, R]; b2 [V] or NULL.
+ * Ds = d_s (1024 in the paper), R = r (256 in the paper).  R == 0 or w2 == NULL turns the
+ * correction branch off: the step then returns log softmax(W_lm . hidden + b2), the base
+ * distribution of the paper's Table 4 "w/o Domino head" (b2 still applies when given), and
+ * emb / w_ih / w_hh / w1 / b1 are not read. */
+typedef struct domino_head_weights {
+  const void* emb;
+  const void* w_ih;
+  const void* w_hh;
+  const void* b_ih;
+  const void* b_hh;
+  const void* w1;
+  const void* b1;
+  const void* w2;
+  const void* b2;
+  int Ds;
+  int R;
+} domino_head_weights;
+
+/* Bytes of device workspace domino_draft_step needs for these sizes on the current device
+ * (the split of the work depends on the device's SM count).  Returns 0 when the sizes are
+ * invalid or unsupported.  R = 0 (or a head without w2) sizes the correction-off step. */
+DOMINO_API size_t domino_workspace_bytes(int B, int K, int H, int V, int Ds, int R, int k, int N);
+
+/* One draft-side block step.
+ *   hidden      bf16 [B, K, H]   backbone hidden states of the K draft positions
+ *   prefix_ids  int32 [B, K]     anchor then drafted tokens (see above)
+ *   w_lm        bf16 [V, H]      frozen target LM head (nn.Linear layout)
+ *   head        Domino head weights (host struct holding device pointers); NULL = head off
+ *   k           top-k width, 1 <= k <= min(32, V)
+ *   N           tree nodes per sequence, 1 <= N <= min(256, sum_{d=1..K} k^d)
+ * Outputs (device):
+ *   topk_ids    int32 [B, K, k]  per position, log-prob descending, ties to the lower id
+ *   topk_logp   fp32  [B, K, k]  refined log-probabilities log softmax(L)[id]
+ *   tree_parent int32 [B, N]     parent node index, -1 for a child of the anchor; parent < i
+ *   tree_token  int32 [B, N]
+ *   tree_depth  int32 [B, N]     1..K
+ *   tree_score  fp32  [B, N] or NULL   cumulative log-probability, non-increasing in i
+ * workspace: device buffer of at least domino_workspace_bytes(...) bytes, 256-byte aligned;
+ * one workspace must not be shared by steps that overlap in time.
+ * Returns DOMINO_OK once everything is enqueued, or a negative code (nothing enqueued). */
+DOMINO_API int domino_draft_step(const void* hidden, const int32_t* prefix_ids, const void* w_lm,
+                      const domino_head_weights* head, int B, int K, int H, int V, int k, int N,
+                      int32_t* topk_ids, float* topk_logp, int32_t* tree_parent,
+                      int32_t* tree_token, int32_t* tree_depth, float* tree_score,
+                      void* workspace, size_t workspace_bytes, void* stream);
+
+/* The same step with the per-step inputs and the outputs in HOST memory (pinned memory
+ * recommended) and the weights on the device.  hidden / prefix_ids are copied into the
+ * workspace, the step runs, the outputs are copied back, and the call synchronises the
+ * stream before returning.  The workspace must hold
+ * domino_workspace_bytes_host(...) bytes.  Returns DOMINO_OK or the first error, including
+ * device-side errors (it calls domino_check_status itself). */
+DOMINO_API size_t domino_workspace_bytes_host(int B, int K, int H, int V, int Ds, int R, int k, int N);
+DOMINO_API int domino_draft_step_host(const void* hidden_host, const int32_t* prefix_ids_host,
+                           const void* w_lm, const domino_head_weights* head, int B, int K,
+                           int H, int V, int k, int N, int32_t* topk_ids_host,
+                           float* topk_logp_host, int32_t* tree_parent_host,
+                           int32_t* tree_token_host, int32_t* tree_depth_host,
+                           float* tree_score_host, void* workspace, size_t workspace_bytes,
+                           void* stream);
+
+/* Synchronises `stream` and returns the device status word of the last step that used
+ * `workspace`: DOMINO_OK, DOMINO_ERR_BAD_TOKEN or DOMINO_ERR_TIMEOUT (DOMINO_ERR_CUDA if the
+ * read itself fails).  Each domino_draft_step clears the word when it starts. */
+DOMINO_API int domino_check_status(const void* workspace, void* stream);
+
+/* Static, human-readable name of a status code. */
+DOMINO_API const char* domino_status_string(int status);
+
+/* DOMINO_ABI_VERSION of the loaded library. */
+DOMINO_API int domino_abi_version(void);
+
+/* Number of kernel launches one domino_draft_step makes for these sizes (head on when
+ * R > 0), so a caller can count device work. */
+DOMINO_API int domino_launches_per_step(int B, int K, int H, int V, int Ds, int R, int k, int N);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* DOMINO_H */

@@ -1,0 +1,141 @@
+"""ctypes binding of the C ABI in include/domino.h (argument marshalling only).
+
+Every function here has the name of the C entry point it calls.  Tensor arguments may be
+torch tensors (their data_ptr() is passed) or raw integer addresses; the library itself
+does all the work.  Loading fails loudly when libdomino.so has not been built: there is no
+fallback implementation.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libdomino.so")
+
+DOMINO_OK = 0
+DOMINO_ERR_INVALID_ARG = -1
+DOMINO_ERR_UNSUPPORTED = -2
+DOMINO_ERR_CUDA = -3
+DOMINO_ERR_TIMEOUT = -4
+DOMINO_ERR_BAD_TOKEN = -5
+
+# every entry point declared in include/domino.h
+SYMBOLS = ("domino_workspace_bytes", "domino_draft_step", "domino_workspace_bytes_host",
+           "domino_draft_step_host", "domino_check_status", "domino_status_string",
+           "domino_abi_version", "domino_launches_per_step")
+
+
+class domino_head_weights(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in
+                ("emb", "w_ih", "w_hh", "b_ih", "b_hh", "w1", "b1", "w2", "b2")] + \
+               [("Ds", ctypes.c_int), ("R", ctypes.c_int)]
+
+
+class DominoError(RuntimeError):
+    def __init__(self, code: int, what: str = ""):
+        super().__init__(f"{what}: {domino_status_string(code)} ({code})" if what else domino_status_string(code))
+        self.code = code
+
+
+_lib = None
+
+
+def load():
+    """Load libdomino.so (raises if it is missing)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: build it with __graft_entry__.build() "
+                           "(there is no non-CUDA implementation)")
+    lib = ctypes.CDLL(LIB_PATH)
+    P, I, S = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+    lib.domino_workspace_bytes.argtypes = [I] * 8
+    lib.domino_workspace_bytes.restype = S
+    lib.domino_workspace_bytes_host.argtypes = [I] * 8
+    lib.domino_workspace_bytes_host.restype = S
+    step_args = [P, P, P, ctypes.POINTER(domino_head_weights)] + [I] * 6 + [P] * 6 + [P, S, P]
+    lib.domino_draft_step.argtypes = step_args
+    lib.domino_draft_step.restype = I
+    lib.domino_draft_step_host.argtypes = step_args
+    lib.domino_draft_step_host.restype = I
+    lib.domino_check_status.argtypes = [P, P]
+    lib.domino_check_status.restype = I
+    lib.domino_status_string.argtypes = [I]
+    lib.domino_status_string.restype = ctypes.c_char_p
+    lib.domino_abi_version.argtypes = []
+    lib.domino_abi_version.restype = I
+    lib.domino_launches_per_step.argtypes = [I] * 8
+    lib.domino_launches_per_step.restype = I
+    _lib = lib
+    return lib
+
+
+def _addr(x):
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    if hasattr(x, "data_ptr"):
+        return x.data_ptr()
+    if hasattr(x, "ctypes"):  # numpy array
+        return x.ctypes.data
+    raise TypeError(f"cannot take the address of {type(x)}")
+
+
+def _stream(s):
+    if s is None:
+        return None
+    if isinstance(s, int):
+        return s
+    return s.cuda_stream  # torch.cuda.Stream
+
+
+def make_head(emb=None, w_ih=None, w_hh=None, b_ih=None, b_hh=None, w1=None, b1=None, w2=None, b2=None,
+              Ds=0, R=0) -> domino_head_weights:
+    return domino_head_weights(_addr(emb), _addr(w_ih), _addr(w_hh), _addr(b_ih), _addr(b_hh), _addr(w1),
+                               _addr(b1), _addr(w2), _addr(b2), int(Ds), int(R))
+
+
+def domino_workspace_bytes(B, K, H, V, Ds, R, k, N) -> int:
+    return int(load().domino_workspace_bytes(B, K, H, V, Ds, R, k, N))
+
+
+def domino_workspace_bytes_host(B, K, H, V, Ds, R, k, N) -> int:
+    return int(load().domino_workspace_bytes_host(B, K, H, V, Ds, R, k, N))
+
+
+def domino_draft_step(hidden, prefix_ids, w_lm, head, B, K, H, V, k, N, topk_ids, topk_logp, tree_parent,
+                      tree_token, tree_depth, tree_score, workspace, workspace_bytes, stream=None) -> int:
+    h = ctypes.byref(head) if head is not None else None
+    return int(load().domino_draft_step(_addr(hidden), _addr(prefix_ids), _addr(w_lm), h, B, K, H, V, k, N,
+                                        _addr(topk_ids), _addr(topk_logp), _addr(tree_parent),
+                                        _addr(tree_token), _addr(tree_depth), _addr(tree_score),
+                                        _addr(workspace), int(workspace_bytes), _stream(stream)))
+
+
+def domino_draft_step_host(hidden_host, prefix_ids_host, w_lm, head, B, K, H, V, k, N, topk_ids_host,
+                           topk_logp_host, tree_parent_host, tree_token_host, tree_depth_host, tree_score_host,
+                           workspace, workspace_bytes, stream=None) -> int:
+    h = ctypes.byref(head) if head is not None else None
+    return int(load().domino_draft_step_host(
+        _addr(hidden_host), _addr(prefix_ids_host), _addr(w_lm), h, B, K, H, V, k, N, _addr(topk_ids_host),
+        _addr(topk_logp_host), _addr(tree_parent_host), _addr(tree_token_host), _addr(tree_depth_host),
+        _addr(tree_score_host), _addr(workspace), int(workspace_bytes), _stream(stream)))
+
+
+def domino_check_status(workspace, stream=None) -> int:
+    return int(load().domino_check_status(_addr(workspace), _stream(stream)))
+
+
+def domino_status_string(code: int) -> str:
+    return load().domino_status_string(int(code)).decode()
+
+
+def domino_abi_version() -> int:
+    return int(load().domino_abi_version())
+
+
+def domino_launches_per_step(B, K, H, V, Ds, R, k, N) -> int:
+    return int(load().domino_launches_per_step(B, K, H, V, Ds, R, k, N))

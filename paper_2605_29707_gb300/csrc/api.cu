@@ -1,0 +1,456 @@
+// api.cu -- host side of the C ABI declared in include/domino.h: argument checks, the launch
+// plan for the current device, workspace layout, TMA tensor maps and the launch sequence.
+//
+// Launch sequence of one step (all on the caller's stream):
+//   memset   clear the status word and the GRU grid-barrier counter
+//   gather   E_j = emb[prefix_ids] (section 4.1.2) and the prefix-id range check
+//   tc store Xp = E . W_ih^T            (tcgen05, split-K fp32 partials)
+//   tc store Up = hidden . W1[:, :H]^T  (tcgen05, split-K fp32 partials)
+//   gru      S_j = GRU(E_0..E_j); u = SiLU(Up + S . W1[:, H:]^T + b1)   (cooperative)
+//   tc soft  logits = [hidden | u] . [W_lm | W2]^T + b2, online max / sum-exp / top-k
+//   tree     merge the partials -> lse, top-k log-probs; best-first draft tree
+// With the correction branch off only memset, gather (id check), tc soft and tree run.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <string.h>
+
+#include <mutex>
+
+#include "domino.h"
+#include "kernels.h"
+
+namespace {
+
+using dm::TcParams;
+
+constexpr int kMaxTopk = 32;
+constexpr int kMaxN = 256;
+constexpr int kMaxK = 64;
+constexpr int kMaxDs = 2048;
+constexpr int kMaxV = 1 << 22;
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
+int ceil_div(int a, int b) { return (a + b - 1) / b; }
+int pow2_at_least(int x, int lo) {
+  int v = lo;
+  while (v < x) v <<= 1;
+  return v;
+}
+
+struct StorePlan {
+  bool swap = false;
+  int bn = 0, tok_tiles = 0, w_tiles = 0, nkb = 0, splits = 0, kb_per_split = 0, total_items = 0, grid = 0;
+};
+
+struct Plan {
+  int B, K, H, V, Ds, R, k, N, M;
+  bool head;
+  int num_sms;
+  // fused vocabulary GEMM
+  bool swap;
+  int bn, kmax, rec, tok_tiles, w_tiles, nchunks, w_per_chunk, grid;
+  StorePlan xg, ug;
+  int gru_grid, gru_units;
+  // workspace layout (offsets in bytes)
+  size_t off_ctrl, off_E, off_xpart, off_upart, off_S, off_u, off_part, dev_total;
+  size_t off_hid, off_ids, off_tid, off_tlp, off_tpar, off_ttok, off_tdep, off_tsc, host_total;
+};
+
+// Orientation: up to 128 tokens ride on the MMA's N dimension (weights fill the 128-row
+// operand); more tokens take the 128-row operand with 256 weight rows per tile.
+void choose_orientation(int M, bool* swap, int* bn) {
+  if (M <= 128) {
+    *swap = true;
+    *bn = pow2_at_least(M, 16);
+  } else {
+    *swap = false;
+    *bn = 256;
+  }
+}
+
+StorePlan plan_store(int M, int rows_w, int nkb, int num_sms) {
+  StorePlan s;
+  choose_orientation(M, &s.swap, &s.bn);
+  s.tok_tiles = s.swap ? ceil_div(M, s.bn) : ceil_div(M, 128);
+  s.w_tiles = s.swap ? ceil_div(rows_w, 128) : ceil_div(rows_w, s.bn);
+  s.nkb = nkb;
+  const int items = s.tok_tiles * s.w_tiles;
+  int splits = num_sms / items;
+  if (splits < 1) splits = 1;
+  if (splits > nkb) splits = nkb;
+  s.kb_per_split = ceil_div(nkb, splits);
+  s.splits = ceil_div(nkb, s.kb_per_split);
+  s.total_items = items * s.splits;
+  s.grid = s.total_items < num_sms ? s.total_items : num_sms;
+  return s;
+}
+
+long long tree_capacity(int K, int k) {  // sum_{d=1..K} k^d, saturated
+  long long cap = 0, pw = 1;
+  for (int d = 1; d <= K; ++d) {
+    pw *= k;
+    cap += pw;
+    if (cap > (1LL << 40)) return 1LL << 40;
+    if (pw > (1LL << 40)) pw = 1LL << 40;
+  }
+  return cap;
+}
+
+int device_sms(int* sms, int* major, int* minor) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return DOMINO_ERR_CUDA;
+  if (cudaDeviceGetAttribute(sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return DOMINO_ERR_CUDA;
+  if (cudaDeviceGetAttribute(major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess) return DOMINO_ERR_CUDA;
+  if (cudaDeviceGetAttribute(minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess) return DOMINO_ERR_CUDA;
+  return DOMINO_OK;
+}
+
+// Size checks that do not need pointers.  Returns DOMINO_OK or an error code.
+int check_sizes(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head) {
+  if (B <= 0 || K <= 0 || H <= 0 || V <= 0 || k <= 0 || N <= 0) return DOMINO_ERR_INVALID_ARG;
+  if (k > V) return DOMINO_ERR_INVALID_ARG;
+  if (static_cast<long long>(N) > tree_capacity(K, k)) return DOMINO_ERR_INVALID_ARG;
+  if (head && (Ds <= 0 || R < 0)) return DOMINO_ERR_INVALID_ARG;
+  if (H % 8 != 0 || k > kMaxTopk || N > kMaxN || K > kMaxK || V >= kMaxV) return DOMINO_ERR_UNSUPPORTED;
+  if (head && (Ds % 8 != 0 || R % 8 != 0 || Ds > kMaxDs)) return DOMINO_ERR_UNSUPPORTED;
+  if (static_cast<long long>(B) * K > (1LL << 24)) return DOMINO_ERR_UNSUPPORTED;
+  return DOMINO_OK;
+}
+
+int make_plan(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head, Plan* P) {
+  int rc = check_sizes(B, K, H, V, Ds, R, k, N, head);
+  if (rc != DOMINO_OK) return rc;
+  int sms = 0, major = 0, minor = 0;
+  rc = device_sms(&sms, &major, &minor);
+  if (rc != DOMINO_OK) return rc;
+  if (major != 10 || minor != 3) return DOMINO_ERR_UNSUPPORTED;
+  Plan& p = *P;
+  memset(&p, 0, sizeof p);
+  p.B = B; p.K = K; p.H = H; p.V = V; p.k = k; p.N = N;
+  p.head = head;
+  p.Ds = head ? Ds : 0;
+  p.R = head ? R : 0;
+  p.M = B * K;
+  p.num_sms = sms;
+  const int M = p.M;
+
+  choose_orientation(M, &p.swap, &p.bn);
+  p.kmax = k <= 16 ? 16 : 32;
+  p.rec = dm::kSoftmaxRecWords(p.kmax);
+  p.tok_tiles = p.swap ? ceil_div(M, p.bn) : ceil_div(M, 128);
+  p.w_tiles = p.swap ? ceil_div(V, 128) : ceil_div(V, p.bn);
+  int per_tok = sms / p.tok_tiles;
+  if (per_tok < 1) per_tok = 1;
+  p.w_per_chunk = ceil_div(p.w_tiles, per_tok);
+  p.nchunks = ceil_div(p.w_tiles, p.w_per_chunk);
+  p.grid = p.tok_tiles * p.nchunks;
+
+  if (head) {
+    p.xg = plan_store(M, 3 * Ds, ceil_div(H, 64), sms);
+    p.ug = plan_store(M, R, ceil_div(H, 64), sms);
+    p.gru_grid = dm::gru_grid(Ds, sms, &p.gru_units);
+    if (dm::gru_smem_bytes(Ds, p.gru_units) == 0) return DOMINO_ERR_UNSUPPORTED;
+  }
+
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off = align_up(off + bytes);
+    return o;
+  };
+  p.off_ctrl = take(256);
+  if (head) {
+    p.off_E = take(static_cast<size_t>(M) * H * 2);
+    p.off_xpart = take(static_cast<size_t>(p.xg.splits) * M * 3 * Ds * 4);
+    p.off_upart = take(static_cast<size_t>(p.ug.splits) * M * R * 4);
+    p.off_S = take(static_cast<size_t>(M) * Ds * 4);
+    p.off_u = take(static_cast<size_t>(M) * R * 2);
+  }
+  p.off_part = take(static_cast<size_t>(M) * p.nchunks * p.rec * 4);
+  p.dev_total = off;
+  p.off_hid = take(static_cast<size_t>(M) * H * 2);
+  p.off_ids = take(static_cast<size_t>(M) * 4);
+  p.off_tid = take(static_cast<size_t>(M) * k * 4);
+  p.off_tlp = take(static_cast<size_t>(M) * k * 4);
+  p.off_tpar = take(static_cast<size_t>(B) * N * 4);
+  p.off_ttok = take(static_cast<size_t>(B) * N * 4);
+  p.off_tdep = take(static_cast<size_t>(B) * N * 4);
+  p.off_tsc = take(static_cast<size_t>(B) * N * 4);
+  p.host_total = off;
+  return DOMINO_OK;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  });
+  return fn;
+}
+
+// 2-D bf16 tensor map: `rows` rows of `inner` elements, `stride_elems` apart; boxes of
+// 64 x box_rows with 128-byte swizzling; out-of-range elements read as zero.
+bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t stride_elems,
+              uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {inner, rows};
+  cuuint64_t strides[1] = {stride_elems * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Maps for one GEMM: activations X [M, inner] (row stride xs) and weights W [rows_w, inner]
+// (row stride ws), in A/B order for the orientation.
+bool gemm_maps(CUtensorMap* a, CUtensorMap* b, bool swap, int bn, const void* X, int M, int inner, int xs,
+               const void* W, int rows_w, int ws) {
+  if (swap) return make_map(a, W, inner, rows_w, ws, 128) && make_map(b, X, inner, M, xs, bn);
+  return make_map(a, X, inner, M, xs, 128) && make_map(b, W, inner, rows_w, ws, bn);
+}
+
+int cuda_rc(cudaError_t e) { return e == cudaSuccess ? DOMINO_OK : DOMINO_ERR_CUDA; }
+
+int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* w_lm, const domino_head_weights* hw,
+             int32_t* topk_ids, float* topk_logp, int32_t* tpar, int32_t* ttok, int32_t* tdep, float* tsc,
+             uint8_t* ws, cudaStream_t st) {
+  const int M = P.M, H = P.H, V = P.V, Ds = P.Ds, R = P.R;
+  int* status = reinterpret_cast<int*>(ws + P.off_ctrl);
+  unsigned* barrier = reinterpret_cast<unsigned*>(ws + P.off_ctrl + 64);
+  if (cudaMemsetAsync(ws + P.off_ctrl, 0, 256, st) != cudaSuccess) return DOMINO_ERR_CUDA;
+
+  __nv_bfloat16* E = P.head ? reinterpret_cast<__nv_bfloat16*>(ws + P.off_E) : nullptr;
+  dm::GatherParams gp{ids, P.head ? static_cast<const __nv_bfloat16*>(hw->emb) : nullptr, E, M, H, V, status};
+  int rc = cuda_rc(dm::launch_gather(gp, st));
+  if (rc) return rc;
+
+  __nv_bfloat16* u = nullptr;
+  if (P.head) {
+    float* xpart = reinterpret_cast<float*>(ws + P.off_xpart);
+    float* upart = reinterpret_cast<float*>(ws + P.off_upart);
+    u = reinterpret_cast<__nv_bfloat16*>(ws + P.off_u);
+    // X partials: E [M, H] . W_ih [3Ds, H]^T
+    {
+      const dm::TcParams base{};
+      TcParams tp = base;
+      const StorePlan& g = P.xg;
+      CUtensorMap maps[4];
+      if (!gemm_maps(&maps[0], &maps[1], g.swap, g.bn, E, M, H, H, hw->w_ih, 3 * Ds, H)) return DOMINO_ERR_CUDA;
+      maps[2] = maps[0];
+      maps[3] = maps[1];
+      tp.nkb1 = g.nkb; tp.nkb2 = 0;
+      tp.rows_tok = M; tp.rows_w = 3 * Ds;
+      tp.tok_tiles = g.tok_tiles; tp.w_tiles = g.w_tiles;
+      tp.splits = g.splits; tp.kb_per_split = g.kb_per_split; tp.total_items = g.total_items;
+      tp.w_evict_first = 0;
+      tp.out = xpart; tp.ld_out = 3 * Ds;
+      tp.status = status;
+      rc = cuda_rc(dm::launch_tc_gemm(dm::kModeStore, g.bn, g.swap, 16, maps, tp, g.grid, st));
+      if (rc) return rc;
+    }
+    // U partials: hidden [M, H] . W1[:, :H]^T (W1 rows are H + Ds long)
+    {
+      const dm::TcParams base{};
+      TcParams tp = base;
+      const StorePlan& g = P.ug;
+      CUtensorMap maps[4];
+      if (!gemm_maps(&maps[0], &maps[1], g.swap, g.bn, hidden, M, H, H, hw->w1, R, H + Ds)) return DOMINO_ERR_CUDA;
+      maps[2] = maps[0];
+      maps[3] = maps[1];
+      tp.nkb1 = g.nkb; tp.nkb2 = 0;
+      tp.rows_tok = M; tp.rows_w = R;
+      tp.tok_tiles = g.tok_tiles; tp.w_tiles = g.w_tiles;
+      tp.splits = g.splits; tp.kb_per_split = g.kb_per_split; tp.total_items = g.total_items;
+      tp.w_evict_first = 0;
+      tp.out = upart; tp.ld_out = R;
+      tp.status = status;
+      rc = cuda_rc(dm::launch_tc_gemm(dm::kModeStore, g.bn, g.swap, 16, maps, tp, g.grid, st));
+      if (rc) return rc;
+    }
+    dm::GruParams gr{};
+    gr.xpart = xpart; gr.xsplits = P.xg.splits;
+    gr.upart = upart; gr.usplits = P.ug.splits;
+    gr.w_hh = static_cast<const __nv_bfloat16*>(hw->w_hh);
+    gr.b_ih = static_cast<const __nv_bfloat16*>(hw->b_ih);
+    gr.b_hh = static_cast<const __nv_bfloat16*>(hw->b_hh);
+    gr.w1 = static_cast<const __nv_bfloat16*>(hw->w1);
+    gr.b1 = static_cast<const __nv_bfloat16*>(hw->b1);
+    gr.B = P.B; gr.K = P.K; gr.H = H; gr.Ds = Ds; gr.R = R;
+    gr.units = P.gru_units;
+    gr.S = reinterpret_cast<float*>(ws + P.off_S);
+    gr.u = u;
+    gr.barrier = barrier;
+    gr.status = status;
+    rc = cuda_rc(dm::launch_gru(gr, P.gru_grid, st));
+    if (rc) return rc;
+  }
+
+  // fused vocabulary GEMM with the online softmax / top-k epilogue
+  {
+    const dm::TcParams base{};
+    TcParams tp = base;
+    CUtensorMap maps[4];
+    if (!gemm_maps(&maps[0], &maps[1], P.swap, P.bn, hidden, M, H, H, w_lm, V, H)) return DOMINO_ERR_CUDA;
+    if (P.head) {
+      if (!gemm_maps(&maps[2], &maps[3], P.swap, P.bn, u, M, R, R, hw->w2, V, R)) return DOMINO_ERR_CUDA;
+    } else {
+      maps[2] = maps[0];
+      maps[3] = maps[1];
+    }
+    tp.nkb1 = ceil_div(H, 64);
+    tp.nkb2 = P.head ? ceil_div(R, 64) : 0;
+    tp.rows_tok = M; tp.rows_w = V;
+    tp.tok_tiles = P.tok_tiles; tp.w_tiles = P.w_tiles;
+    tp.nchunks = P.nchunks; tp.w_per_chunk = P.w_per_chunk;
+    tp.w_evict_first = P.tok_tiles == 1 ? 1 : 0;
+    tp.bias = hw ? static_cast<const __nv_bfloat16*>(hw->b2) : nullptr;
+    tp.out = reinterpret_cast<float*>(ws + P.off_part);
+    tp.status = status;
+    rc = cuda_rc(dm::launch_tc_gemm(dm::kModeSoftmax, P.bn, P.swap, P.kmax, maps, tp, P.grid, st));
+    if (rc) return rc;
+  }
+
+  dm::TreeParams tr{};
+  tr.partials = reinterpret_cast<const float*>(ws + P.off_part);
+  tr.nchunks = P.nchunks;
+  tr.kmax = P.kmax;
+  tr.B = P.B; tr.K = P.K; tr.k = P.k; tr.N = P.N;
+  tr.topk_ids = topk_ids; tr.topk_logp = topk_logp;
+  tr.tree_parent = tpar; tr.tree_token = ttok; tr.tree_depth = tdep; tr.tree_score = tsc;
+  return cuda_rc(dm::launch_merge_tree(tr, st));
+}
+
+bool head_active(const domino_head_weights* hw) { return hw != nullptr && hw->w2 != nullptr && hw->R > 0; }
+
+int check_pointers(const void* hidden, const int32_t* ids, const void* w_lm, const domino_head_weights* hw,
+                   bool head) {
+  if (!hidden || !ids || !w_lm) return DOMINO_ERR_INVALID_ARG;
+  if (head && (!hw->emb || !hw->w_ih || !hw->w_hh || !hw->w1 || !hw->w2)) return DOMINO_ERR_INVALID_ARG;
+  if (!aligned16(hidden) || !aligned16(w_lm)) return DOMINO_ERR_UNSUPPORTED;
+  if (head && (!aligned16(hw->emb) || !aligned16(hw->w_ih) || !aligned16(hw->w_hh) || !aligned16(hw->w1) ||
+               !aligned16(hw->w2)))
+    return DOMINO_ERR_UNSUPPORTED;
+  return DOMINO_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t domino_workspace_bytes(int B, int K, int H, int V, int Ds, int R, int k, int N) {
+  Plan P;
+  if (make_plan(B, K, H, V, Ds, R, k, N, R > 0, &P) != DOMINO_OK) return 0;
+  return P.dev_total;
+}
+
+size_t domino_workspace_bytes_host(int B, int K, int H, int V, int Ds, int R, int k, int N) {
+  Plan P;
+  if (make_plan(B, K, H, V, Ds, R, k, N, R > 0, &P) != DOMINO_OK) return 0;
+  return P.host_total;
+}
+
+int domino_draft_step(const void* hidden, const int32_t* prefix_ids, const void* w_lm,
+                      const domino_head_weights* head, int B, int K, int H, int V, int k, int N,
+                      int32_t* topk_ids, float* topk_logp, int32_t* tree_parent, int32_t* tree_token,
+                      int32_t* tree_depth, float* tree_score, void* workspace, size_t workspace_bytes,
+                      void* stream) {
+  const bool hd = head_active(head);
+  if (!topk_ids || !topk_logp || !tree_parent || !tree_token || !tree_depth || !workspace)
+    return DOMINO_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(workspace) & (kAlign - 1)) != 0) return DOMINO_ERR_INVALID_ARG;
+  int rc = check_pointers(hidden, prefix_ids, w_lm, head, hd);
+  if (rc) return rc;
+  Plan P;
+  rc = make_plan(B, K, H, V, hd ? head->Ds : 0, hd ? head->R : 0, k, N, hd, &P);
+  if (rc) return rc;
+  if (workspace_bytes < P.dev_total) return DOMINO_ERR_INVALID_ARG;
+  return run_step(P, hidden, prefix_ids, w_lm, head, topk_ids, topk_logp, tree_parent, tree_token, tree_depth,
+                  tree_score, static_cast<uint8_t*>(workspace), static_cast<cudaStream_t>(stream));
+}
+
+int domino_draft_step_host(const void* hidden_host, const int32_t* prefix_ids_host, const void* w_lm,
+                           const domino_head_weights* head, int B, int K, int H, int V, int k, int N,
+                           int32_t* topk_ids_host, float* topk_logp_host, int32_t* tree_parent_host,
+                           int32_t* tree_token_host, int32_t* tree_depth_host, float* tree_score_host,
+                           void* workspace, size_t workspace_bytes, void* stream) {
+  const bool hd = head_active(head);
+  if (!hidden_host || !prefix_ids_host || !w_lm || !topk_ids_host || !topk_logp_host || !tree_parent_host ||
+      !tree_token_host || !tree_depth_host || !workspace)
+    return DOMINO_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(workspace) & (kAlign - 1)) != 0) return DOMINO_ERR_INVALID_ARG;
+  Plan P;
+  int rc = make_plan(B, K, H, V, hd ? head->Ds : 0, hd ? head->R : 0, k, N, hd, &P);
+  if (rc) return rc;
+  if (workspace_bytes < P.host_total) return DOMINO_ERR_INVALID_ARG;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t M = P.M;
+  void* d_hid = ws + P.off_hid;
+  int32_t* d_ids = reinterpret_cast<int32_t*>(ws + P.off_ids);
+  rc = check_pointers(d_hid, d_ids, w_lm, head, hd);
+  if (rc) return rc;
+  if (cudaMemcpyAsync(d_hid, hidden_host, M * H * 2, cudaMemcpyHostToDevice, st) != cudaSuccess) return DOMINO_ERR_CUDA;
+  if (cudaMemcpyAsync(d_ids, prefix_ids_host, M * 4, cudaMemcpyHostToDevice, st) != cudaSuccess) return DOMINO_ERR_CUDA;
+  int32_t* d_tid = reinterpret_cast<int32_t*>(ws + P.off_tid);
+  float* d_tlp = reinterpret_cast<float*>(ws + P.off_tlp);
+  int32_t* d_par = reinterpret_cast<int32_t*>(ws + P.off_tpar);
+  int32_t* d_tok = reinterpret_cast<int32_t*>(ws + P.off_ttok);
+  int32_t* d_dep = reinterpret_cast<int32_t*>(ws + P.off_tdep);
+  float* d_sc = reinterpret_cast<float*>(ws + P.off_tsc);
+  rc = run_step(P, d_hid, d_ids, w_lm, head, d_tid, d_tlp, d_par, d_tok, d_dep, d_sc, ws, st);
+  if (rc) return rc;
+  const size_t BN = static_cast<size_t>(P.B) * N;
+  cudaError_t e = cudaSuccess;
+  e = e ? e : cudaMemcpyAsync(topk_ids_host, d_tid, M * k * 4, cudaMemcpyDeviceToHost, st);
+  e = e ? e : cudaMemcpyAsync(topk_logp_host, d_tlp, M * k * 4, cudaMemcpyDeviceToHost, st);
+  e = e ? e : cudaMemcpyAsync(tree_parent_host, d_par, BN * 4, cudaMemcpyDeviceToHost, st);
+  e = e ? e : cudaMemcpyAsync(tree_token_host, d_tok, BN * 4, cudaMemcpyDeviceToHost, st);
+  e = e ? e : cudaMemcpyAsync(tree_depth_host, d_dep, BN * 4, cudaMemcpyDeviceToHost, st);
+  if (tree_score_host) e = e ? e : cudaMemcpyAsync(tree_score_host, d_sc, BN * 4, cudaMemcpyDeviceToHost, st);
+  if (e != cudaSuccess) return DOMINO_ERR_CUDA;
+  return domino_check_status(workspace, stream);
+}
+
+int domino_check_status(const void* workspace, void* stream) {
+  if (!workspace) return DOMINO_ERR_INVALID_ARG;
+  int h = 0;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(&h, workspace, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess) return DOMINO_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return DOMINO_ERR_CUDA;
+  return h;
+}
+
+const char* domino_status_string(int status) {
+  switch (status) {
+    case DOMINO_OK: return "DOMINO_OK";
+    case DOMINO_ERR_INVALID_ARG: return "DOMINO_ERR_INVALID_ARG";
+    case DOMINO_ERR_UNSUPPORTED: return "DOMINO_ERR_UNSUPPORTED";
+    case DOMINO_ERR_CUDA: return "DOMINO_ERR_CUDA";
+    case DOMINO_ERR_TIMEOUT: return "DOMINO_ERR_TIMEOUT";
+    case DOMINO_ERR_BAD_TOKEN: return "DOMINO_ERR_BAD_TOKEN";
+    default: return "DOMINO_ERR_UNKNOWN";
+  }
+}
+
+int domino_abi_version(void) { return DOMINO_ABI_VERSION; }
+
+int domino_launches_per_step(int B, int K, int H, int V, int Ds, int R, int k, int N) {
+  (void)B; (void)K; (void)H; (void)V; (void)Ds; (void)k; (void)N;
+  return R > 0 ? 6 : 3;  // gather, [X gemm, U gemm, gru,] vocab gemm, merge+tree
+}
+
+}  // extern "C"

@@ -1,0 +1,462 @@
+// tc_gemm.cuh -- persistent tcgen05 GEMM for sm_103a with two K segments and two epilogues.
+//
+// Warp roles (192 threads):
+//   warp 0      one thread issues TMA tile loads into a STAGES-deep shared-memory ring;
+//   warp 1      allocates TMEM; one thread issues tcgen05.mma (M = 128, N = BN, K = 16 per
+//               instruction) into one of two TMEM accumulators and commits to mbarriers;
+//   warps 2..5  epilogue: tcgen05.ld the finished accumulator and either
+//               - softmax mode: fold every logit into a per-(token, CTA) running max, running
+//                 sum of exp and a top-KMAX list (value desc, id asc), so that the logits never
+//                 leave the chip (the vocabulary projection of section 4.1.1 plus the W2 term
+//                 of section 4.1.2 in one accumulator), or
+//               - store mode: write fp32 partial sums (split-K) of a plain projection.
+// The two accumulators let the epilogue of tile i overlap the main loop of tile i+1.
+#pragma once
+
+#include <math.h>
+
+#include "kernels.h"
+#include "ptx.cuh"
+
+namespace dm {
+
+template <int BN, bool SWAP, int MODE, int KMAX>
+struct TcCfg {
+  static constexpr int kABytes = 128 * 128;  // 128 rows x 64 bf16
+  static constexpr int kBBytes = BN * 128;   // BN rows x 64 bf16
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kTPT = SWAP ? 128 / BN : 1;  // epilogue threads per token (swap)
+  static constexpr int kTrStride = 128 + kTPT;      // conflict-free transpose pitch (floats)
+  static constexpr int kTrBytes = (SWAP && MODE == kModeSoftmax) ? BN * kTrStride * 4 : 0;
+  static constexpr int kBudget = 200 * 1024;
+  static constexpr int kSt0 = (kBudget - kTrBytes) / kStageBytes;
+  static constexpr int kStages = kSt0 > 8 ? 8 : kSt0;
+  static constexpr int kTmemCols =
+      (2 * BN <= 32) ? 32 : (2 * BN <= 64) ? 64 : (2 * BN <= 128) ? 128 : (2 * BN <= 256) ? 256 : 512;
+  static constexpr int kBarBytes = 256;
+  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kTrBytes + kBarBytes;
+  static constexpr int kRec = 2 + 2 * KMAX;
+  static_assert(kStages >= 2, "pipeline needs at least two stages");
+  static_assert(kSmemBytes > 116 * 1024, "one CTA per SM keeps TMEM allocation uncontended");
+  static_assert(BN % 16 == 0 && BN >= 16 && BN <= 256, "UMMA N for M = 128");
+};
+
+struct TcItem {
+  int tok, w, kb0, kb1, split;
+};
+
+template <int MODE>
+__device__ __forceinline__ bool tc_get_item(const TcParams& p, int i, TcItem& it) {
+  const int nkb = p.nkb1 + p.nkb2;
+  if (MODE == kModeSoftmax) {
+    const int tok = blockIdx.x % p.tok_tiles;
+    const int chunk = blockIdx.x / p.tok_tiles;
+    const int w = chunk * p.w_per_chunk + i;
+    if (chunk >= p.nchunks || i >= p.w_per_chunk || w >= p.w_tiles) return false;
+    it.tok = tok; it.w = w; it.kb0 = 0; it.kb1 = nkb; it.split = 0;
+    return true;
+  } else {
+    const int idx = blockIdx.x + i * gridDim.x;
+    if (idx >= p.total_items) return false;
+    const int split = idx % p.splits;
+    const int rest = idx / p.splits;
+    it.w = rest % p.w_tiles;
+    it.tok = rest / p.w_tiles;
+    it.split = split;
+    it.kb0 = split * p.kb_per_split;
+    it.kb1 = min(nkb, it.kb0 + p.kb_per_split);
+    return true;
+  }
+}
+
+// Running log-sum-exp state and top-KMAX list of one token over a stream of logits.
+template <int KM>
+struct OnlineTopK {
+  float mx, se;
+  float tv[KM];
+  int ti[KM];
+
+  __device__ __forceinline__ void init() {
+    mx = -INFINITY;
+    se = 0.f;
+#pragma unroll
+    for (int q = 0; q < KM; ++q) { tv[q] = -INFINITY; ti[q] = -1; }
+  }
+
+  // Stream insert: ids arrive in increasing order, so an equal value never displaces an
+  // earlier (lower) id.
+  __device__ __forceinline__ void push(float x, int id) {
+    if (x > mx) {
+      se = se * __expf(mx - x) + 1.f;
+      mx = x;
+    } else {
+      se += __expf(x - mx);
+    }
+    if (x > tv[KM - 1]) {
+#pragma unroll
+      for (int q = 0; q < KM; ++q) {
+        const bool sw = x > tv[q];
+        const float a = tv[q];
+        const int b = ti[q];
+        tv[q] = sw ? x : a;
+        ti[q] = sw ? id : b;
+        x = sw ? a : x;
+        id = sw ? b : id;
+      }
+    }
+  }
+
+  // Keyed insert (value desc, then id asc) for merging lists from other streams.
+  __device__ __forceinline__ void insert_keyed(float x, int id) {
+    const bool better_than_last =
+        x > tv[KM - 1] || (x == tv[KM - 1] && (unsigned)id < (unsigned)ti[KM - 1]);
+    if (!better_than_last) return;
+#pragma unroll
+    for (int q = 0; q < KM; ++q) {
+      const bool sw = x > tv[q] || (x == tv[q] && (unsigned)id < (unsigned)ti[q]);
+      const float a = tv[q];
+      const int b = ti[q];
+      tv[q] = sw ? x : a;
+      ti[q] = sw ? id : b;
+      x = sw ? a : x;
+      id = sw ? b : id;
+    }
+  }
+
+  __device__ __forceinline__ void merge_lse(float omx, float ose) {
+    const float m = fmaxf(mx, omx);
+    if (m == -INFINITY) return;
+    const float a = (mx == -INFINITY) ? 0.f : se * __expf(mx - m);
+    const float b = (omx == -INFINITY) ? 0.f : ose * __expf(omx - m);
+    mx = m;
+    se = a + b;
+  }
+
+  // Merge with the state held by lane (laneid ^ offset).
+  __device__ __forceinline__ void merge_shfl_xor(int offset) {
+    const float omx = __shfl_xor_sync(0xffffffffu, mx, offset);
+    const float ose = __shfl_xor_sync(0xffffffffu, se, offset);
+    float ov[KM];
+    int oi[KM];
+#pragma unroll
+    for (int q = 0; q < KM; ++q) {
+      ov[q] = __shfl_xor_sync(0xffffffffu, tv[q], offset);
+      oi[q] = __shfl_xor_sync(0xffffffffu, ti[q], offset);
+    }
+    merge_lse(omx, ose);
+#pragma unroll
+    for (int q = 0; q < KM; ++q) insert_keyed(ov[q], oi[q]);
+  }
+
+  __device__ __forceinline__ void store(float* rec) const {
+    rec[0] = mx;
+    rec[1] = se;
+#pragma unroll
+    for (int q = 0; q < KM; ++q) {
+      rec[2 + q] = tv[q];
+      reinterpret_cast<int*>(rec)[2 + KM + q] = ti[q];
+    }
+  }
+};
+
+// Returns the OR of `pred` over the 128 epilogue threads (named barrier 1).
+__device__ __forceinline__ bool epi_any(bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.or.pred q, 1, 128, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)pred)
+      : "memory");
+  return r != 0;
+}
+
+template <int BN, bool SWAP, int MODE, int KMAX>
+__global__ void __launch_bounds__(192, 1)
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
+                   const __grid_constant__ CUtensorMap tmA2, const __grid_constant__ CUtensorMap tmB2,
+                   const TcParams p) {
+  using C = TcCfg<BN, SWAP, MODE, KMAX>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + C::kStages * C::kABytes;
+  float* tr = reinterpret_cast<float*>(sB + C::kStages * C::kBBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(tr) + C::kTrBytes);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + C::kStages;
+  uint64_t* tfull = bars + 2 * C::kStages;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* drain = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 128);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (threadIdx.x == 32) {
+    tma_prefetch_desc(&tmA1);
+    tma_prefetch_desc(&tmB1);
+    if (p.nkb2 > 0) {
+      tma_prefetch_desc(&tmA2);
+      tma_prefetch_desc(&tmB2);
+    }
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, C::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      const uint64_t pol_w = p.w_evict_first ? l2_policy_evict_first() : l2_policy_evict_normal();
+      const uint64_t pol_t = l2_policy_evict_last();
+      const uint64_t polA = SWAP ? pol_w : pol_t;
+      const uint64_t polB = SWAP ? pol_t : pol_w;
+      int stage = 0;
+      uint32_t phase = 0;
+      int issued = 0;
+      bool ok = true;
+      TcItem it;
+      for (int i = 0; ok && tc_get_item<MODE>(p, i, it); ++i) {
+        for (int kb = it.kb0; kb < it.kb1; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, p.status)) { ok = false; break; }
+          mbar_arrive_expect_tx(&full[stage], C::kStageBytes);
+          const bool seg2 = kb >= p.nkb1;
+          const int kx = (seg2 ? kb - p.nkb1 : kb) * 64;
+          const int ay = SWAP ? it.w * 128 : it.tok * 128;
+          const int by = SWAP ? it.tok * BN : it.w * BN;
+          tma_load_2d(sA + stage * C::kABytes, seg2 ? &tmA2 : &tmA1, &full[stage], kx, ay, polA);
+          tma_load_2d(sB + stage * C::kBBytes, seg2 ? &tmB2 : &tmB1, &full[stage], kx, by, polB);
+          ++issued;
+          if (++stage == C::kStages) { stage = 0; phase ^= 1u; }
+        }
+      }
+      // Let every load this thread issued land before the CTA can exit (each is the last
+      // one on its stage; a completed phase of that parity returns at once).
+      const int outstanding = issued < C::kStages ? issued : C::kStages;
+      for (int j = 1; j <= outstanding; ++j) {
+        int s = stage - j;
+        uint32_t ph = phase;
+        if (s < 0) { s += C::kStages; ph ^= 1u; }
+        const long long t0 = clock64();
+        while (!mbar_try_wait(&full[s], ph)) {
+          if (clock64() - t0 > kWaitCycles) { set_status(p.status, kStatusTimeout); break; }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t kIdesc = idesc_bf16_f32(128, BN);
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      TcItem it;
+      for (int i = 0; ok && tc_get_item<MODE>(p, i, it); ++i) {
+        const int ab = i & 1;
+        const uint32_t aph = (i >> 1) & 1;
+        if (!mbar_wait(&tempty[ab], aph ^ 1u, abort_flag, p.status)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(ab * BN);
+        for (int kb = it.kb0; kb < it.kb1; ++kb) {
+          if (!mbar_wait(&full[stage], phase, abort_flag, p.status)) { ok = false; break; }
+          tc_fence_after();
+          const uint64_t da = smem_desc_sw128(smem_u32(sA + stage * C::kABytes));
+          const uint64_t db = smem_desc_sw128(smem_u32(sB + stage * C::kBBytes));
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk) {
+            tc_mma_bf16(d_tmem, da + static_cast<uint64_t>(2 * kk), db + static_cast<uint64_t>(2 * kk),
+                        kIdesc, (kb > it.kb0 || kk > 0) ? 1u : 0u);
+          }
+          tc_commit(&empty[stage]);
+          if (++stage == C::kStages) { stage = 0; phase ^= 1u; }
+        }
+        if (ok) tc_commit(&tfull[ab]);
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue (128 threads)
+    const int q = warp & 3;  // TMEM lanes 32q .. 32q+31 belong to this warp
+    const int ep = threadIdx.x - 64;
+    const uint32_t lane_off = static_cast<uint32_t>(32 * q) << 16;
+    OnlineTopK<KMAX> st;
+    if (MODE == kModeSoftmax) st.init();
+    bool aborted = false;
+    TcItem it;
+    it.tok = 0;
+    for (int i = 0; tc_get_item<MODE>(p, i, it); ++i) {
+      const int ab = i & 1;
+      const uint32_t aph = (i >> 1) & 1;
+      const bool ok = mbar_wait(&tfull[ab], aph, abort_flag, p.status);
+      if (epi_any(!ok)) { aborted = true; break; }
+      tc_fence_after();
+      const uint32_t tcol = tmem_base + lane_off + static_cast<uint32_t>(ab * BN);
+
+      if constexpr (MODE == kModeStore) {
+        if constexpr (SWAP) {
+          const int n = it.w * 128 + 32 * q + lane;
+          float* out = p.out + static_cast<size_t>(it.split) * p.rows_tok * p.ld_out;
+#pragma unroll
+          for (int c0 = 0; c0 < BN; c0 += (BN < 32 ? BN : 32)) {
+            float r[BN < 32 ? 16 : 32];
+            if constexpr (BN < 32) tc_ld_x16(tcol + c0, r); else tc_ld_x32(tcol + c0, r);
+            tc_wait_ld();
+#pragma unroll
+            for (int j = 0; j < (BN < 32 ? 16 : 32); ++j) {
+              const int tok = it.tok * BN + c0 + j;
+              if (tok < p.rows_tok && n < p.rows_w) out[static_cast<size_t>(tok) * p.ld_out + n] = r[j];
+            }
+          }
+        } else {
+          const int tok = it.tok * 128 + 32 * q + lane;
+          float* orow = p.out + (static_cast<size_t>(it.split) * p.rows_tok + tok) * p.ld_out;
+#pragma unroll 1
+          for (int c0 = 0; c0 < BN; c0 += 32) {
+            float r[32];
+            tc_ld_x32(tcol + c0, r);
+            tc_wait_ld();
+            const int n0 = it.w * BN + c0;
+            if (tok < p.rows_tok) {
+              if (n0 + 32 <= p.rows_w) {
+#pragma unroll
+                for (int j = 0; j < 32; j += 4)
+                  *reinterpret_cast<float4*>(orow + n0 + j) = make_float4(r[j], r[j + 1], r[j + 2], r[j + 3]);
+              } else {
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                  if (n0 + j < p.rows_w) orow[n0 + j] = r[j];
+              }
+            }
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(&tempty[ab]);
+      } else if constexpr (SWAP) {
+        // vocabulary rows on TMEM lanes, tokens on columns: stage through shared memory so
+        // that each thread owns one token and a strided slice of the tile's vocabulary
+        const int vrow = 32 * q + lane;
+        const int v = it.w * 128 + vrow;
+        const bool vvalid = v < p.rows_w;
+        const float bv = (p.bias != nullptr && vvalid) ? __bfloat162float(p.bias[v]) : 0.f;
+#pragma unroll
+        for (int c0 = 0; c0 < BN; c0 += (BN < 32 ? BN : 32)) {
+          float r[BN < 32 ? 16 : 32];
+          if constexpr (BN < 32) tc_ld_x16(tcol + c0, r); else tc_ld_x32(tcol + c0, r);
+          tc_wait_ld();
+#pragma unroll
+          for (int j = 0; j < (BN < 32 ? 16 : 32); ++j) tr[(c0 + j) * C::kTrStride + vrow] = r[j] + bv;
+        }
+        tc_fence_before();
+        mbar_arrive(&tempty[ab]);
+        named_bar_sync(1, 128);
+        const int tt = ep / C::kTPT;
+        const int sub = ep % C::kTPT;
+        const int vbase = it.w * 128;
+        const float* trow = tr + tt * C::kTrStride;
+#pragma unroll 4
+        for (int jj = 0; jj < BN; ++jj) {
+          const int vl = sub + C::kTPT * jj;
+          if (vbase + vl < p.rows_w) st.push(trow[vl], vbase + vl);
+        }
+        named_bar_sync(1, 128);
+      } else {
+        // tokens on TMEM lanes: each thread streams its own row across the vocabulary tile
+#pragma unroll 1
+        for (int c0 = 0; c0 < BN; c0 += 32) {
+          float r[32];
+          tc_ld_x32(tcol + c0, r);
+          tc_wait_ld();
+          const int v0 = it.w * BN + c0;
+          if (v0 + 32 <= p.rows_w) {
+            if (p.bias != nullptr) {
+#pragma unroll
+              for (int j = 0; j < 32; ++j) st.push(r[j] + __bfloat162float(p.bias[v0 + j]), v0 + j);
+            } else {
+#pragma unroll
+              for (int j = 0; j < 32; ++j) st.push(r[j], v0 + j);
+            }
+          } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+              const int v = v0 + j;
+              if (v < p.rows_w) st.push(r[j] + (p.bias ? __bfloat162float(p.bias[v]) : 0.f), v);
+            }
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(&tempty[ab]);
+      }
+    }
+
+    if (MODE == kModeSoftmax && !aborted) {
+      const int tok_tile = blockIdx.x % p.tok_tiles;
+      const int chunk = blockIdx.x / p.tok_tiles;
+      if constexpr (SWAP) {
+#pragma unroll
+        for (int off = C::kTPT / 2; off >= 1; off >>= 1) st.merge_shfl_xor(off);
+        const int tt = ep / C::kTPT;
+        const int tok = tok_tile * BN + tt;
+        if (ep % C::kTPT == 0 && tok < p.rows_tok)
+          st.store(p.out + (static_cast<size_t>(tok) * p.nchunks + chunk) * C::kRec);
+      } else {
+        const int tok = tok_tile * 128 + 32 * q + lane;
+        if (tok < p.rows_tok) st.store(p.out + (static_cast<size_t>(tok) * p.nchunks + chunk) * C::kRec);
+      }
+    }
+  }
+
+  // ------------------------------------------------------------ teardown
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    if (lane == 0) {
+      // every MMA this thread issued must be finished before the TMEM is released
+      tc_commit(drain);
+      const long long t0 = clock64();
+      while (!mbar_try_wait(drain, 0)) {
+        if (clock64() - t0 > kWaitCycles) { set_status(p.status, kStatusTimeout); break; }
+      }
+    }
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::kTmemCols);
+  }
+}
+
+template <int BN, bool SWAP, int MODE, int KMAX>
+cudaError_t launch_tc_instance(const CUtensorMap* maps, const TcParams& p, int grid, cudaStream_t stream) {
+  using C = TcCfg<BN, SWAP, MODE, KMAX>;
+  auto kern = tc_gemm_kernel<BN, SWAP, MODE, KMAX>;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  kern<<<grid, 192, C::kSmemBytes, stream>>>(maps[0], maps[1], maps[2], maps[3], p);
+  return cudaGetLastError();
+}
+
+}  // namespace dm

@@ -1,0 +1,67 @@
+"""CPU checks of the C-ABI boundary: the library loads without a GPU, exports every entry
+point include/domino.h declares, and rejects bad arguments before touching the device."""
+import os
+import re
+
+import pytest
+
+from paper_2605_29707_gb300 import binding
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _lib():
+    if not os.path.exists(binding.LIB_PATH):
+        from paper_2605_29707_gb300 import build
+        build.build()
+    return binding.load()
+
+
+def declared_entry_points():
+    with open(os.path.join(ROOT, "include", "domino.h")) as f:
+        text = f.read()
+    return re.findall(r"DOMINO_API\s+[\w\s\*]+?\b(domino_\w+)\s*\(", text)
+
+
+def test_header_and_binding_agree():
+    names = declared_entry_points()
+    assert len(names) >= 8
+    assert sorted(names) == sorted(binding.SYMBOLS)
+
+
+def test_library_loads_and_exports_every_declared_symbol():
+    lib = _lib()
+    for name in declared_entry_points():
+        assert hasattr(lib, name), name
+    assert binding.domino_abi_version() == 1
+
+
+def test_status_strings():
+    _lib()
+    assert binding.domino_status_string(0) == "DOMINO_OK"
+    assert binding.domino_status_string(-5) == "DOMINO_ERR_BAD_TOKEN"
+    assert binding.domino_status_string(-4) == "DOMINO_ERR_TIMEOUT"
+    assert binding.domino_status_string(12345) == "DOMINO_ERR_UNKNOWN"
+
+
+def test_invalid_sizes_rejected_without_device():
+    _lib()
+    good = dict(B=1, K=16, H=4096, V=151936, Ds=1024, R=256, k=8, N=16)
+    for bad in (dict(B=0), dict(K=-1), dict(H=0), dict(V=0), dict(k=0), dict(N=0), dict(k=200, V=100),
+                dict(K=2, k=2, N=7), dict(H=4100), dict(k=33), dict(N=257), dict(K=65), dict(V=1 << 22),
+                dict(Ds=1000), dict(R=100), dict(Ds=4096)):
+        args = dict(good, **bad)
+        assert binding.domino_workspace_bytes(*args.values()) == 0, bad
+
+
+def test_null_pointers_rejected_before_any_cuda_call():
+    _lib()
+    rc = binding.domino_draft_step(None, None, None, None, 1, 4, 64, 100, 2, 3, None, None, None, None, None,
+                                   None, None, 0)
+    assert rc == binding.DOMINO_ERR_INVALID_ARG
+
+
+def test_launch_count_query():
+    _lib()
+    assert binding.domino_launches_per_step(1, 16, 4096, 151936, 1024, 256, 8, 16) == 6
+    assert binding.domino_launches_per_step(1, 16, 4096, 151936, 0, 0, 8, 16) == 3
