@@ -1,0 +1,442 @@
+#!/usr/bin/env python3
+"""Benchmark of the Domino draft-side block step on GB300; prints ONE JSON line.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--config NAME]
+
+Workload: the Qwen3-8B-shaped batch-1 K=16 draft step (H=4096, V=151936, d_s=1024, r=256,
+k=8, N=16), the configuration the metric's target is stated on; synthetic seeded inputs
+(paper_2605_29707_gb300/inputs.py).  A step is one domino_draft_step call: embedding gather,
+GRU input projection, W1 hidden projection, GRU recurrence + low-rank code, fused vocabulary
+GEMM with online softmax/top-k, merge + tree.
+
+value   draft blocks/s over all ranks (B blocks per step per rank), device-timed with CUDA
+        events around exactly K steps, inputs resident in HBM; the weights (1.4 GB) exceed
+        the 129 MB L2, so no flush is needed between steps.
+e2e     the same metric through domino_draft_step_host: per step, hidden + prefix ids are
+        copied from pinned host memory and the top-k lists and tree are copied back.
+roofline  the dominant kernel (vocabulary GEMM + softmax/top-k): algorithmic bytes (or
+        FLOPs) per launch / its mean CUDA-event duration in the timed region.
+Multi-GPU: one process per GPU (torchrun); each rank runs its own independent draft step
+(sequences are independent problems), no collective on the data path: weak scaling.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "µs per draft step & draft blocks/s (1 GB300); LM-head HBM GB/s / roofline %"
+UNIT = "draft blocks/s"
+DEFAULT_CONFIG = "qwen3-8b"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+VOCAB_SOURCES = ["paper_2605_29707_gb300/csrc/tc_gemm.cuh", "paper_2605_29707_gb300/csrc/tc_softmax.cu",
+                 "paper_2605_29707_gb300/csrc/ptx.cuh"]
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "vocab_gemm_traffic.json")
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", str(rank)))
+    return rank, world, local
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        p["source"] = "measured"
+        return p
+    p = dict(FALLBACK_PEAKS)
+    p["source"] = "fallback"
+    return p
+
+
+def source_sha(paths):
+    h = hashlib.sha256()
+    for p in paths:
+        with open(os.path.join(ROOT, p), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 100 ms while running."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    NAMES = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(prefix="clocks_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.FIELDS}", "--format=csv,noheader",
+                 "-lms", "100", "-f", self.path], stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        time.sleep(0.15)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, reasons, n = [], None, set(), 0
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1].split()[0]))
+                    smax = float(parts[2].split()[0])
+                except ValueError:
+                    continue
+                n += 1
+                for name, val in zip(self.NAMES, parts[5:9]):
+                    if val.lower().startswith("active"):
+                        reasons.add(name)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax,
+                "reasons": sorted(reasons), "samples": n}
+
+
+def vocab_plan(cfg, num_sms):
+    """Tile plan of the vocabulary GEMM (mirrors the library's host plan) for byte counting."""
+    M = cfg.M
+    if M <= 128:
+        swap, bn = True, max(16, 1 << (M - 1).bit_length())
+        tok_tiles, w_tiles = -(-M // bn), -(-cfg.V // 128)
+    else:
+        swap, bn = False, 256
+        tok_tiles, w_tiles = -(-M // 128), -(-cfg.V // 256)
+    per_tok = max(1, num_sms // tok_tiles)
+    wpc = -(-w_tiles // per_tok)
+    nchunks = -(-w_tiles // wpc)
+    kmax = 16 if cfg.k <= 16 else 32
+    return dict(swap=swap, bn=bn, nchunks=nchunks, rec_words=2 + 2 * kmax, grid=tok_tiles * nchunks)
+
+
+def vocab_work(cfg, num_sms, has_b2=False):
+    """Algorithmic bytes and FLOPs of one vocabulary-GEMM launch: every W_lm and W2 row once,
+    the activations once, the per-chunk partial records written once (logits never stored)."""
+    M, V, H, R = cfg.M, cfg.V, cfg.H, cfg.R
+    plan = vocab_plan(cfg, num_sms)
+    weights = V * (H + R) * 2 + (V * 2 if has_b2 else 0)
+    acts = M * (H + R) * 2
+    partials = M * plan["nchunks"] * plan["rec_words"] * 4
+    return {"bytes": weights + acts + partials, "flops": 2.0 * M * V * (H + R), "per_unit_bytes": (H + R) * 2,
+            "units": V, "plan": plan}
+
+
+def step_work(cfg):
+    """Whole-step algorithmic bytes (every weight once + activations) and FLOPs."""
+    M, V, H, R, Ds = cfg.M, cfg.V, cfg.H, cfg.R, cfg.Ds
+    weights = (V * H + V * R + 3 * Ds * H + 3 * Ds * Ds + R * (H + Ds)) * 2
+    acts = M * H * 2 * 2 + M * 4  # hidden, gathered embedding rows, ids
+    flops = 2.0 * M * (H * V + R * V + 3 * Ds * H + 3 * Ds * Ds + (H + Ds) * R)
+    return {"bytes": weights + acts, "flops": flops}
+
+
+def roofline_entry(kind_bytes, kind_flops, ms, peaks, sustained):
+    hbm = peaks["hbm_gbs"]
+    tens = peaks["bf16_tflops_sustained" if sustained else "bf16_tflops"]
+    t_mem = kind_bytes / (hbm * 1e9)
+    t_flop = kind_flops / (tens * 1e12)
+    if t_mem >= t_flop:
+        achieved = kind_bytes / (ms * 1e-3) / 1e9
+        return {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
+                "frac": round(achieved / hbm, 4), "peak_source": peaks["source"]}
+    achieved = kind_flops / (ms * 1e-3) / 1e12
+    return {"bound": "tensor", "achieved": round(achieved, 1), "peak": tens, "unit": "TFLOP/s",
+            "frac": round(achieved / tens, 4),
+            "peak_source": peaks["source"] + (" sustained" if sustained else " burst")}
+
+
+def traffic_for(cfg_name):
+    if not os.path.exists(TRAFFIC_FILE):
+        return None, "no ncu record"
+    with open(TRAFFIC_FILE) as f:
+        rec = json.load(f)
+    if rec.get("source_sha") != source_sha(VOCAB_SOURCES):
+        return None, "kernel changed since the ncu capture"
+    ent = rec.get("configs", {}).get(cfg_name)
+    if not ent:
+        return None, "no capture for this workload"
+    return ent["traffic_bytes_per_launch"], ent.get("note", "")
+
+
+def dev_bf16(a, device):
+    import numpy as np
+    import torch
+    return torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).to(device)
+
+
+# ---------------------------------------------------------------------------- CPU oracle legs
+def oracle_full_step_seconds(wl, budget_s, max_steps=1000):
+    """Times whole oracle steps (all positions, all vocabulary rows) for about budget_s."""
+    import oracle
+    c = wl.cfg
+    times = []
+    t_end = time.perf_counter() + budget_s
+    while len(times) < max_steps and (not times or time.perf_counter() < t_end):
+        t0 = time.perf_counter()
+        oracle.draft_step(wl.weights, wl.hidden, wl.prefix_ids, c.k, c.N, seqs=[0])
+        times.append(time.perf_counter() - t0)
+    return statistics.mean(times), len(times)
+
+
+def cpu_baseline(wl, budget_s=12.0):
+    import oracle
+    sec, n = oracle_full_step_seconds(wl, budget_s)
+    c = wl.cfg
+    return {"value": round(1.0 / sec, 4), "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
+            "sample": f"{n} whole oracle steps of one sequence ({c.K} positions x {c.V} vocabulary rows, fp64, "
+                      f"OpenMP), {sec:.3f} s each; blocks/s = 1/seconds per step"}
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    import numpy as np
+    import oracle
+    from paper_2605_29707_gb300 import inputs
+    oracle.build()
+    wl = inputs.make_workload(args.config)
+    c, w = wl.cfg, wl.weights
+    hid = (wl.hidden[0].astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    ids = wl.prefix_ids[0]
+    # the correction branch's state (GRU + low-rank code) once per block, timed
+    t0 = time.perf_counter()
+    E = oracle.embed(w["emb"], ids)
+    S = oracle.gru(E, w["w_ih"], w["w_hh"], w["b_ih"], w["b_hh"])
+    u = oracle.lowrank(hid, S, w["w1"], w["b1"])
+    t_head = time.perf_counter() - t0
+    # calibrate one vocabulary slice, then size the per-step sample to the time budget
+    probe = 2048
+    t0 = time.perf_counter()
+    z = oracle.logits(hid, u, w["w_lm"][:probe], w["w2"][:probe], None if w["b2"] is None else w["b2"][:probe])
+    oracle.topk(oracle.log_softmax(z)[0], c.k)
+    t_probe = time.perf_counter() - t0
+    budget = float(os.environ.get("DOMINO_REF_BUDGET_S", "90"))
+    per_step = budget / max(1, args.steps + args.warmup)
+    Vs = int(min(c.V, max(128, probe * per_step / max(t_probe, 1e-6))))
+    times = []
+    for i in range(args.warmup + args.steps):
+        v0 = (i * Vs) % max(1, c.V - Vs + 1)
+        t0 = time.perf_counter()
+        z = oracle.logits(hid, u, w["w_lm"][v0:v0 + Vs], w["w2"][v0:v0 + Vs],
+                          None if w["b2"] is None else w["b2"][v0:v0 + Vs])
+        lp, _ = oracle.log_softmax(z)
+        oracle.topk(lp, min(c.k, Vs))
+        if i >= args.warmup:
+            times.append(time.perf_counter() - t0)
+    t_tree0 = time.perf_counter()
+    oracle.tree(np.zeros((c.K, c.k), np.int32) + np.arange(c.k, dtype=np.int32), -np.tile(np.arange(c.k, dtype=np.float64), (c.K, 1)) - 1.0, c.N)
+    t_tree = time.perf_counter() - t_tree0
+    sec_step = t_head + statistics.mean(times) * (c.V / Vs) + t_tree
+    value = c.B / sec_step
+    cores = oracle.max_threads()
+    sample = (f"{args.steps} timed samples, each the fp64 oracle's logits, log-softmax and top-k for all {c.K} "
+              f"positions over a {Vs}-row vocabulary slice ({Vs / c.V:.4f} of the step); the GRU + low-rank code "
+              f"({t_head:.3f} s) and the tree are timed once per block; seconds per block = head + mean slice "
+              f"time x V/slice + tree = {sec_step:.3f} s")
+    line = {"impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(sec_step * 1e3, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": config_dict(c, world),
+            "cpu_baseline": {"value": round(value, 4), "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": round(value, 4), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def config_dict(c, world):
+    return {"workload": f"{c.name}: B={c.B} K={c.K} H={c.H} V={c.V} d_s={c.Ds} r={c.R} k={c.k} N={c.N}",
+            "B": c.B, "K": c.K, "H": c.H, "V": c.V, "d_s": c.Ds, "r": c.R, "k": c.k, "N": c.N,
+            "parallelism": f"replicas x{world} (independent sequences per GPU)",
+            "l2": "no flush: weights (W_lm alone 1.2 GB at H=4096) exceed the 129 MB L2"}
+
+
+# ---------------------------------------------------------------------------- our arm
+def run_ours(args):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    rank, world, local = dist_env()
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo", init_method="env://")
+    device = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(device)
+
+    from paper_2605_29707_gb300 import binding, inputs
+    from paper_2605_29707_gb300.step import DraftStep
+
+    wl = inputs.make_workload(args.config)
+    c = wl.cfg
+    st = DraftStep(wl.weights, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=device)
+    hidden = dev_bf16(wl.hidden, device)
+    ids = torch.from_numpy(wl.prefix_ids).to(device)
+    stream = torch.cuda.current_stream(device)
+    launches = st.launches_per_step()
+    num_sms = torch.cuda.get_device_properties(device).multi_processor_count
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    for _ in range(args.warmup):
+        rc = st.enqueue(hidden, ids, stream)
+        if rc != 0:
+            raise binding.DominoError(rc, "warm-up step")
+    rc = binding.domino_check_status(st.workspace, stream)
+    if rc != 0:
+        raise binding.DominoError(rc, "warm-up device status")
+
+    # ---- timed region: exactly K steps, per-kernel events on the launching stream
+    sampler = ClockSampler(local)
+    sampler.start()
+    barrier()
+    torch.cuda.synchronize(device)
+    binding.domino_timing_begin(args.steps * launches)
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    bad = 0
+    for _ in range(args.steps):
+        bad |= st.enqueue(hidden, ids, stream) != 0
+    ev1.record(stream)
+    torch.cuda.synchronize(device)
+    barrier()
+    kern = binding.domino_timing_end()
+    clocks = sampler.stop()
+    if bad:
+        raise RuntimeError("a timed step returned an error")
+    rc = binding.domino_check_status(st.workspace, stream)
+    if rc != 0:
+        raise binding.DominoError(rc, "timed device status")
+    ms = ev0.elapsed_time(ev1)
+    if world > 1:
+        t = torch.tensor([ms], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_step = ms / args.steps
+    value = world * c.B * args.steps / (ms / 1e3)
+
+    # ---- e2e through the host-buffer entry point (pinned inputs and outputs)
+    M = c.M
+    h_hidden = torch.from_numpy(wl.hidden.view(np.int16)).pin_memory()
+    h_ids = torch.from_numpy(wl.prefix_ids).pin_memory()
+    host = {"topk_ids": torch.empty(M * c.k, dtype=torch.int32).pin_memory(),
+            "topk_logp": torch.empty(M * c.k, dtype=torch.float32).pin_memory(),
+            "tree_parent": torch.empty(c.B * c.N, dtype=torch.int32).pin_memory(),
+            "tree_token": torch.empty(c.B * c.N, dtype=torch.int32).pin_memory(),
+            "tree_depth": torch.empty(c.B * c.N, dtype=torch.int32).pin_memory(),
+            "tree_score": torch.empty(c.B * c.N, dtype=torch.float32).pin_memory()}
+    n_e2e = max(3, min(args.steps, 1000))
+    for _ in range(3):
+        st.run_host(h_hidden, h_ids, host, stream)
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(n_e2e):
+        rc = st.run_host(h_hidden, h_ids, host, stream)
+        if rc != 0:
+            raise binding.DominoError(rc, "host-buffer step")
+    t_e2e = time.perf_counter() - t0
+    if world > 1:
+        t = torch.tensor([t_e2e], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        t_e2e = float(t.item())
+    e2e_value = world * c.B * n_e2e / t_e2e
+    h2d = M * c.H * 2 + M * 4
+    d2h = M * c.k * 8 + c.B * c.N * 16 + 4
+
+    # ---- roofline of the dominant kernel, measured in the timed region
+    peaks = load_peaks()
+    dominant = max(kern, key=lambda n: kern[n][0])
+    vw = vocab_work(c, num_sms, has_b2=wl.weights.get("b2") is not None)
+    vk_ms, vk_n = kern["vocab_gemm_softmax_topk"]
+    vk_mean = vk_ms / max(1, vk_n)
+    roof = roofline_entry(vw["bytes"], vw["flops"], vk_mean, peaks, sustained=True)
+    traffic, traffic_note = traffic_for(c.name)
+    roof.update({"kernel": "vocab_gemm_softmax_topk", "traffic": traffic,
+                 "algorithmic_bytes_per_launch": vw["bytes"], "algorithmic_flops_per_launch": vw["flops"],
+                 "mean_launch_us": round(vk_mean * 1e3, 2), "launches": vk_n, "traffic_note": traffic_note,
+                 "share_of_step": round(vk_ms / max(1e-9, sum(v[0] for v in kern.values())), 4)})
+    sw = step_work(c)
+    step_roof = max(sw["bytes"] / (peaks["hbm_gbs"] * 1e9), sw["flops"] / (peaks["bf16_tflops_sustained"] * 1e12))
+    breakdown = {n: {"us_per_launch": round(v[0] / max(1, v[1]) * 1e3, 2), "launches": v[1]} for n, v in kern.items()}
+
+    line = {
+        "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms_step, 5), "us_per_step": round(ms_step * 1e3, 2),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded, Qwen3-shaped, random-init weights)", "config": config_dict(c, world),
+        "roofline": roof,
+        "step_roofline": {"us": round(step_roof * 1e6, 2), "frac": round(step_roof / (ms_step * 1e-3), 4),
+                          "bytes": sw["bytes"], "flops": sw["flops"],
+                          "note": "max(every weight once / HBM peak, FLOPs / sustained bf16 peak)"},
+        "kernel_breakdown": breakdown, "dominant_kernel": dominant,
+        "e2e": {"value": round(e2e_value, 3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "steps": n_e2e, "api": "domino_draft_step_host (synchronous per step)"},
+        "gpu_launches": args.steps * launches, "clocks": clocks,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl, args.cpu_seconds)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=4000)
+    ap.add_argument("--warmup", type=int, default=30)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", default=DEFAULT_CONFIG)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -144,6 +144,25 @@ DOMINO_API int domino_abi_version(void);
  * R > 0), so a caller can count device work. */
 DOMINO_API int domino_launches_per_step(int B, int K, int H, int V, int Ds, int R, int k, int N);
 
+/* Per-kernel device timing, for the per-component latency breakdown the paper reports in
+ * its Fig. 1 (LM head, Domino head, tree).  After domino_timing_begin(max_launches), every
+ * kernel the library enqueues (up to max_launches of them, on any stream) is bracketed by a
+ * pair of CUDA events.  domino_timing_end() waits for those events, stops recording and writes
+ * for each kernel kind (index = DOMINO_KERNEL_*) the summed device time in milliseconds and
+ * the number of launches; kinds beyond nkinds are dropped.  Not thread-safe: one recording at
+ * a time per process.  Returns DOMINO_OK or DOMINO_ERR_CUDA / DOMINO_ERR_INVALID_ARG. */
+enum domino_kernel_kind {
+  DOMINO_KERNEL_GATHER = 0,       /* E_j = emb[prefix id], id range check */
+  DOMINO_KERNEL_GRU_INPUT = 1,    /* E . W_ih^T on tensor cores (split-K partials) */
+  DOMINO_KERNEL_W1_HIDDEN = 2,    /* hidden . W1[:, :H]^T on tensor cores (split-K partials) */
+  DOMINO_KERNEL_GRU = 3,          /* GRU recurrence over K positions, then u = SiLU(...) */
+  DOMINO_KERNEL_VOCAB = 4,        /* [hidden | u] . [W_lm | W2]^T with online softmax / top-k */
+  DOMINO_KERNEL_TREE = 5,         /* merge to log-probs and top-k; best-first tree */
+  DOMINO_KERNEL_KINDS = 6
+};
+DOMINO_API int domino_timing_begin(int max_launches);
+DOMINO_API int domino_timing_end(float* total_ms, int* launches, int nkinds);
+
 #ifdef __cplusplus
 }
 #endif

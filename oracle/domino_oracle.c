@@ -79,6 +79,10 @@ int oracle_gru(const double* E, int K, int Hin, int Ds, const uint16_t* w_ih, co
   }
   for (int j = 0; j < K; ++j) {
     const double* x = E + (long)j * Hin;
+    /* the 3Ds gate rows are independent dot products; threads split the rows only */
+#ifdef _OPENMP
+#pragma omp parallel for schedule(static)
+#endif
     for (int g = 0; g < G; ++g) {
       double a = b_ih ? bf(b_ih, g) : 0.0;
       for (int c = 0; c < Hin; ++c) a += bf(w_ih, (long)g * Hin + c) * x[c];
@@ -105,6 +109,9 @@ int oracle_lowrank(const double* hidden, const double* S, int K, int H, int Ds, 
                    const uint16_t* w1, const uint16_t* b1, double* u) {
   if (!hidden || !S || !w1 || !u || K <= 0 || H <= 0 || Ds <= 0 || R <= 0) return ORACLE_ERR_ARG;
   const long ld = (long)H + Ds;
+#ifdef _OPENMP
+#pragma omp parallel for collapse(2) schedule(static)
+#endif
   for (int j = 0; j < K; ++j) {
     for (int q = 0; q < R; ++q) {
       double a = b1 ? bf(b1, q) : 0.0;

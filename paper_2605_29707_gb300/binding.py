@@ -23,7 +23,9 @@ DOMINO_ERR_BAD_TOKEN = -5
 # every entry point declared in include/domino.h
 SYMBOLS = ("domino_workspace_bytes", "domino_draft_step", "domino_workspace_bytes_host",
            "domino_draft_step_host", "domino_check_status", "domino_status_string",
-           "domino_abi_version", "domino_launches_per_step")
+           "domino_abi_version", "domino_launches_per_step", "domino_timing_begin", "domino_timing_end")
+
+KERNEL_KINDS = ("gather", "gru_input_proj", "w1_hidden_proj", "gru", "vocab_gemm_softmax_topk", "merge_tree")
 
 
 class domino_head_weights(ctypes.Structure):
@@ -68,6 +70,10 @@ def load():
     lib.domino_abi_version.restype = I
     lib.domino_launches_per_step.argtypes = [I] * 8
     lib.domino_launches_per_step.restype = I
+    lib.domino_timing_begin.argtypes = [I]
+    lib.domino_timing_begin.restype = I
+    lib.domino_timing_end.argtypes = [P, P, I]
+    lib.domino_timing_end.restype = I
     _lib = lib
     return lib
 
@@ -139,3 +145,18 @@ def domino_abi_version() -> int:
 
 def domino_launches_per_step(B, K, H, V, Ds, R, k, N) -> int:
     return int(load().domino_launches_per_step(B, K, H, V, Ds, R, k, N))
+
+
+def domino_timing_begin(max_launches: int) -> int:
+    return int(load().domino_timing_begin(int(max_launches)))
+
+
+def domino_timing_end() -> dict:
+    """Stops per-kernel timing; returns {kind name: (total ms, launches)}."""
+    n = len(KERNEL_KINDS)
+    ms = (ctypes.c_float * n)()
+    cnt = (ctypes.c_int * n)()
+    rc = int(load().domino_timing_end(ctypes.cast(ms, ctypes.c_void_p), ctypes.cast(cnt, ctypes.c_void_p), n))
+    if rc != 0:
+        raise DominoError(rc, "domino_timing_end")
+    return {KERNEL_KINDS[i]: (float(ms[i]), int(cnt[i])) for i in range(n)}

@@ -17,6 +17,7 @@
 #include <string.h>
 
 #include <mutex>
+#include <vector>
 
 #include "domino.h"
 #include "kernels.h"
@@ -55,6 +56,7 @@ struct Plan {
   StorePlan xg, ug;
   int gru_grid, gru_units;
   // workspace layout (offsets in bytes)
+  size_t ctrl_bytes;
   size_t off_ctrl, off_E, off_xpart, off_upart, off_S, off_u, off_part, dev_total;
   size_t off_hid, off_ids, off_tid, off_tlp, off_tpar, off_ttok, off_tdep, off_tsc, host_total;
 };
@@ -152,7 +154,7 @@ int make_plan(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head
     p.xg = plan_store(M, 3 * Ds, ceil_div(H, 64), sms);
     p.ug = plan_store(M, R, ceil_div(H, 64), sms);
     p.gru_grid = dm::gru_grid(Ds, sms, &p.gru_units);
-    if (dm::gru_smem_bytes(Ds, p.gru_units) == 0) return DOMINO_ERR_UNSUPPORTED;
+    if (dm::gru_smem_bytes(Ds, p.gru_units, M, B) == 0) return DOMINO_ERR_UNSUPPORTED;
   }
 
   size_t off = 0;
@@ -161,7 +163,8 @@ int make_plan(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head
     off = align_up(off + bytes);
     return o;
   };
-  p.off_ctrl = take(256);
+  p.ctrl_bytes = align_up(256 + static_cast<size_t>(B) * 4);
+  p.off_ctrl = take(p.ctrl_bytes);
   if (head) {
     p.off_E = take(static_cast<size_t>(M) * H * 2);
     p.off_xpart = take(static_cast<size_t>(p.xg.splits) * M * 3 * Ds * 4);
@@ -225,17 +228,43 @@ bool gemm_maps(CUtensorMap* a, CUtensorMap* b, bool swap, int bn, const void* X,
 
 int cuda_rc(cudaError_t e) { return e == cudaSuccess ? DOMINO_OK : DOMINO_ERR_CUDA; }
 
+// ---------------------------------------------------------------- per-kernel timing
+struct Timing {
+  bool on = false;
+  int used = 0;
+  std::vector<cudaEvent_t> start, stop;
+  std::vector<int> kind;
+};
+Timing g_timing;
+
+// Brackets one launch with an event pair when timing is on; returns the slot or -1.
+int timing_open(int kind, cudaStream_t st) {
+  Timing& t = g_timing;
+  if (!t.on || t.used >= static_cast<int>(t.start.size())) return -1;
+  const int i = t.used++;
+  t.kind[i] = kind;
+  cudaEventRecord(t.start[i], st);
+  return i;
+}
+
+void timing_close(int slot, cudaStream_t st) {
+  if (slot >= 0) cudaEventRecord(g_timing.stop[slot], st);
+}
+
 int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* w_lm, const domino_head_weights* hw,
              int32_t* topk_ids, float* topk_logp, int32_t* tpar, int32_t* ttok, int32_t* tdep, float* tsc,
              uint8_t* ws, cudaStream_t st) {
   const int M = P.M, H = P.H, V = P.V, Ds = P.Ds, R = P.R;
   int* status = reinterpret_cast<int*>(ws + P.off_ctrl);
   unsigned* barrier = reinterpret_cast<unsigned*>(ws + P.off_ctrl + 64);
-  if (cudaMemsetAsync(ws + P.off_ctrl, 0, 256, st) != cudaSuccess) return DOMINO_ERR_CUDA;
+  unsigned* seq_done = reinterpret_cast<unsigned*>(ws + P.off_ctrl + 256);
+  if (cudaMemsetAsync(ws + P.off_ctrl, 0, P.ctrl_bytes, st) != cudaSuccess) return DOMINO_ERR_CUDA;
 
   __nv_bfloat16* E = P.head ? reinterpret_cast<__nv_bfloat16*>(ws + P.off_E) : nullptr;
   dm::GatherParams gp{ids, P.head ? static_cast<const __nv_bfloat16*>(hw->emb) : nullptr, E, M, H, V, status};
+  int ts = timing_open(DOMINO_KERNEL_GATHER, st);
   int rc = cuda_rc(dm::launch_gather(gp, st));
+  timing_close(ts, st);
   if (rc) return rc;
 
   __nv_bfloat16* u = nullptr;
@@ -259,7 +288,9 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
       tp.w_evict_first = 0;
       tp.out = xpart; tp.ld_out = 3 * Ds;
       tp.status = status;
+      ts = timing_open(DOMINO_KERNEL_GRU_INPUT, st);
       rc = cuda_rc(dm::launch_tc_gemm(dm::kModeStore, g.bn, g.swap, 16, maps, tp, g.grid, st));
+      timing_close(ts, st);
       if (rc) return rc;
     }
     // U partials: hidden [M, H] . W1[:, :H]^T (W1 rows are H + Ds long)
@@ -278,7 +309,9 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
       tp.w_evict_first = 0;
       tp.out = upart; tp.ld_out = R;
       tp.status = status;
+      ts = timing_open(DOMINO_KERNEL_W1_HIDDEN, st);
       rc = cuda_rc(dm::launch_tc_gemm(dm::kModeStore, g.bn, g.swap, 16, maps, tp, g.grid, st));
+      timing_close(ts, st);
       if (rc) return rc;
     }
     dm::GruParams gr{};
@@ -295,7 +328,9 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
     gr.u = u;
     gr.barrier = barrier;
     gr.status = status;
+    ts = timing_open(DOMINO_KERNEL_GRU, st);
     rc = cuda_rc(dm::launch_gru(gr, P.gru_grid, st));
+    timing_close(ts, st);
     if (rc) return rc;
   }
 
@@ -320,18 +355,24 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
     tp.bias = hw ? static_cast<const __nv_bfloat16*>(hw->b2) : nullptr;
     tp.out = reinterpret_cast<float*>(ws + P.off_part);
     tp.status = status;
+    ts = timing_open(DOMINO_KERNEL_VOCAB, st);
     rc = cuda_rc(dm::launch_tc_gemm(dm::kModeSoftmax, P.bn, P.swap, P.kmax, maps, tp, P.grid, st));
+    timing_close(ts, st);
     if (rc) return rc;
   }
 
   dm::TreeParams tr{};
   tr.partials = reinterpret_cast<const float*>(ws + P.off_part);
+  tr.seq_done = seq_done;
   tr.nchunks = P.nchunks;
   tr.kmax = P.kmax;
   tr.B = P.B; tr.K = P.K; tr.k = P.k; tr.N = P.N;
   tr.topk_ids = topk_ids; tr.topk_logp = topk_logp;
   tr.tree_parent = tpar; tr.tree_token = ttok; tr.tree_depth = tdep; tr.tree_score = tsc;
-  return cuda_rc(dm::launch_merge_tree(tr, st));
+  ts = timing_open(DOMINO_KERNEL_TREE, st);
+  rc = cuda_rc(dm::launch_merge_tree(tr, st));
+  timing_close(ts, st);
+  return rc;
 }
 
 bool head_active(const domino_head_weights* hw) { return hw != nullptr && hw->w2 != nullptr && hw->R > 0; }
@@ -447,6 +488,43 @@ const char* domino_status_string(int status) {
 }
 
 int domino_abi_version(void) { return DOMINO_ABI_VERSION; }
+
+int domino_timing_begin(int max_launches) {
+  if (max_launches <= 0) return DOMINO_ERR_INVALID_ARG;
+  Timing& t = g_timing;
+  while (static_cast<int>(t.start.size()) < max_launches) {
+    cudaEvent_t a, b;
+    if (cudaEventCreate(&a) != cudaSuccess) return DOMINO_ERR_CUDA;
+    if (cudaEventCreate(&b) != cudaSuccess) return DOMINO_ERR_CUDA;
+    t.start.push_back(a);
+    t.stop.push_back(b);
+    t.kind.push_back(0);
+  }
+  t.used = 0;
+  t.on = true;
+  return DOMINO_OK;
+}
+
+int domino_timing_end(float* total_ms, int* launches, int nkinds) {
+  Timing& t = g_timing;
+  t.on = false;
+  if (nkinds < 0 || (nkinds > 0 && (!total_ms || !launches))) return DOMINO_ERR_INVALID_ARG;
+  for (int i = 0; i < nkinds; ++i) {
+    total_ms[i] = 0.f;
+    launches[i] = 0;
+  }
+  for (int i = 0; i < t.used; ++i) {
+    if (cudaEventSynchronize(t.stop[i]) != cudaSuccess) return DOMINO_ERR_CUDA;
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, t.start[i], t.stop[i]) != cudaSuccess) return DOMINO_ERR_CUDA;
+    if (t.kind[i] < nkinds) {
+      total_ms[t.kind[i]] += ms;
+      launches[t.kind[i]] += 1;
+    }
+  }
+  t.used = 0;
+  return DOMINO_OK;
+}
 
 int domino_launches_per_step(int B, int K, int H, int V, int Ds, int R, int k, int N) {
   (void)B; (void)K; (void)H; (void)V; (void)Ds; (void)k; (void)N;

@@ -38,13 +38,17 @@ __device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
   return v;
 }
 
-// Bounded grid barrier on a monotonically increasing counter.  The outcome is uniform over
-// the CTA: false means this CTA gave up (status set to DOMINO_ERR_TIMEOUT).
+__device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Bounded grid barrier on a monotonically increasing counter (release on arrival, acquire
+// while polling).  The outcome is uniform over the CTA: false means this CTA gave up and
+// recorded DOMINO_ERR_TIMEOUT.
 __device__ bool grid_barrier(unsigned* counter, unsigned target, int* status, volatile int* flag) {
   __syncthreads();
   if (threadIdx.x == 0) {
-    __threadfence();
-    atomicAdd(counter, 1u);
+    red_release_add(counter, 1u);
     int ok = 1;
     const long long t0 = clock64();
     while (ld_acquire_u32(counter) < target) {
@@ -54,11 +58,18 @@ __device__ bool grid_barrier(unsigned* counter, unsigned target, int* status, vo
         break;
       }
     }
-    __threadfence();
     *flag = ok;
   }
   __syncthreads();
   return *flag != 0;
+}
+
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gmem_src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem_dst)), "l"(gmem_src) : "memory");
+}
+
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
 }
 
 __device__ __forceinline__ float dot8_bf16(const uint4 w, const float4 h0, const float4 h1) {
@@ -88,28 +99,64 @@ __device__ __forceinline__ float bf_or0(const __nv_bfloat16* p, int i) {
   return p ? __bfloat162float(p[i]) : 0.f;
 }
 
+// Shared-memory layout of one GRU CTA (U hidden units, M = B*K rows, BG staged sequences):
+//   whh [3][U][Ds] bf16 | xs [M][3][U] f32 (input-gate sums + b_ih) | bh [3][U] f32 (b_hh)
+//   | hs [BG][Ds] f32 (h_{t-1}) | gs [BG][3][U] f32 (W_hh . h_{t-1}) | flag
+struct GruSmem {
+  size_t whh, xs, bh, hs, gs, flag, total;
+};
+
+__host__ __device__ inline GruSmem gru_layout(int Ds, int U, int M, int BG) {
+  GruSmem L;
+  size_t o = 0;
+  L.whh = o; o += static_cast<size_t>(3) * U * Ds * 2;
+  L.xs = o;  o += static_cast<size_t>(M) * 3 * U * 4;
+  L.bh = o;  o += static_cast<size_t>(3) * U * 4;
+  o = (o + 15) & ~static_cast<size_t>(15);
+  L.hs = o;  o += static_cast<size_t>(BG) * Ds * 4;
+  L.gs = o;  o += static_cast<size_t>(BG) * 3 * U * 4;
+  L.flag = o; o += 16;
+  L.total = o;
+  return L;
+}
+
 __global__ void __launch_bounds__(kGruThreads) gru_kernel(const GruParams p, const int BG) {
   extern __shared__ __align__(16) uint8_t gsm[];
   const int U = p.units, Ds = p.Ds, K = p.K, B = p.B, R = p.R, H = p.H;
   const int M = B * K;
   const int j0 = blockIdx.x * U;
   const int Uc = min(U, Ds - j0);
-  __nv_bfloat16* whh = reinterpret_cast<__nv_bfloat16*>(gsm);         // [3][U][Ds]
-  float* hs = reinterpret_cast<float*>(gsm + static_cast<size_t>(3) * U * Ds * 2);  // [BG][Ds]
-  float* gs = hs + static_cast<size_t>(BG) * Ds;                       // [BG][3U]
-  volatile int* flag = reinterpret_cast<volatile int*>(gs + static_cast<size_t>(BG) * 3 * U);
+  const GruSmem L = gru_layout(Ds, U, M, BG);
+  __nv_bfloat16* whh = reinterpret_cast<__nv_bfloat16*>(gsm + L.whh);
+  float* xs = reinterpret_cast<float*>(gsm + L.xs);
+  float* bh = reinterpret_cast<float*>(gsm + L.bh);
+  float* hs = reinterpret_cast<float*>(gsm + L.hs);
+  float* gs = reinterpret_cast<float*>(gsm + L.gs);
+  volatile int* flag = reinterpret_cast<volatile int*>(gsm + L.flag);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   constexpr int kWarps = kGruThreads / 32;
 
-  // this CTA's rows of W_hh: gate g, unit j0 + jl
+  // this CTA's rows of W_hh (gate g, unit j0 + jl), copied asynchronously
   const int rowlen8 = Ds / 8;
   for (int e = tid; e < 3 * Uc * rowlen8; e += kGruThreads) {
     const int c8 = e % rowlen8;
     const int r = e / rowlen8;
     const int g = r / Uc, jl = r % Uc;
-    reinterpret_cast<uint4*>(whh + (static_cast<size_t>(g) * U + jl) * Ds)[c8] =
-        __ldg(reinterpret_cast<const uint4*>(p.w_hh + (static_cast<size_t>(g) * Ds + j0 + jl) * Ds) + c8);
+    cp_async16(whh + (static_cast<size_t>(g) * U + jl) * Ds + c8 * 8,
+               p.w_hh + (static_cast<size_t>(g) * Ds + j0 + jl) * Ds + c8 * 8);
   }
+  // input-gate sums for every row and this CTA's units: b_ih + sum over split-K partials
+  for (int e = tid; e < M * 3 * Uc; e += kGruThreads) {
+    const int jl = e % Uc;
+    const int g = (e / Uc) % 3;
+    const int m = e / (3 * Uc);
+    const int col = g * Ds + j0 + jl;
+    float a = bf_or0(p.b_ih, col);
+    for (int s = 0; s < p.xsplits; ++s) a += __ldg(p.xpart + (static_cast<size_t>(s) * M + m) * 3 * Ds + col);
+    xs[(static_cast<size_t>(m) * 3 + g) * U + jl] = a;
+  }
+  for (int e = tid; e < 3 * Uc; e += kGruThreads) bh[(e / Uc) * U + e % Uc] = bf_or0(p.b_hh, (e / Uc) * Ds + j0 + e % Uc);
+  cp_async_wait_all();
   __syncthreads();
 
   for (int t = 0; t < K; ++t) {
@@ -123,7 +170,7 @@ __global__ void __launch_bounds__(kGruThreads) gru_kernel(const GruParams p, con
               reinterpret_cast<const float4*>(p.S + (static_cast<size_t>(b0 + bb) * K + (t - 1)) * Ds) + c4);
         }
         __syncthreads();
-        // g_hh = W_hh[rows of this CTA] . h_{t-1}
+        // W_hh[rows of this CTA] . h_{t-1}
         for (int d = warp; d < 3 * Uc * nb; d += kWarps) {
           const int r = d % (3 * Uc), bb = d / (3 * Uc);
           const int g = r / Uc, jl = r % Uc;
@@ -137,7 +184,7 @@ __global__ void __launch_bounds__(kGruThreads) gru_kernel(const GruParams p, con
             acc += dot8_bf16(wv, h0, h1);
           }
           acc = warp_sum(acc);
-          if (lane == 0) gs[bb * 3 * U + g * U + jl] = acc;
+          if (lane == 0) gs[(bb * 3 + g) * U + jl] = acc;
         }
         __syncthreads();
       }
@@ -146,24 +193,18 @@ __global__ void __launch_bounds__(kGruThreads) gru_kernel(const GruParams p, con
         const int bb = e / Uc, jl = e % Uc;
         const int j = j0 + jl;
         const int m = (b0 + bb) * K + t;
-        float xr = bf_or0(p.b_ih, j), xz = bf_or0(p.b_ih, Ds + j), xn = bf_or0(p.b_ih, 2 * Ds + j);
-        for (int s = 0; s < p.xsplits; ++s) {
-          const float* xp = p.xpart + (static_cast<size_t>(s) * M + m) * 3 * Ds;
-          xr += xp[j];
-          xz += xp[Ds + j];
-          xn += xp[2 * Ds + j];
-        }
-        float hr = bf_or0(p.b_hh, j), hz = bf_or0(p.b_hh, Ds + j), hn = bf_or0(p.b_hh, 2 * Ds + j);
+        const float* x = xs + static_cast<size_t>(m) * 3 * U;
+        float hr = bh[jl], hz = bh[U + jl], hn = bh[2 * U + jl];
         float hprev = 0.f;
         if (t > 0) {
-          hr += gs[bb * 3 * U + jl];
-          hz += gs[bb * 3 * U + U + jl];
-          hn += gs[bb * 3 * U + 2 * U + jl];
+          hr += gs[(bb * 3 + 0) * U + jl];
+          hz += gs[(bb * 3 + 1) * U + jl];
+          hn += gs[(bb * 3 + 2) * U + jl];
           hprev = hs[static_cast<size_t>(bb) * Ds + j];
         }
-        const float r = 1.f / (1.f + expf(-(xr + hr)));
-        const float z = 1.f / (1.f + expf(-(xz + hz)));
-        const float n = tanhf(xn + r * hn);
+        const float r = 1.f / (1.f + expf(-(x[jl] + hr)));
+        const float z = 1.f / (1.f + expf(-(x[U + jl] + hz)));
+        const float n = tanhf(x[2 * U + jl] + r * hn);
         p.S[static_cast<size_t>(m) * Ds + j] = (1.f - z) * n + z * hprev;
       }
       __syncthreads();
@@ -188,10 +229,11 @@ __global__ void __launch_bounds__(kGruThreads) gru_kernel(const GruParams p, con
         const float4 h1 = __ldcg(reinterpret_cast<const float4*>(srow + c + 4));
         acc += dot8_bf16(wv, h0, h1);
       }
+      // the hidden half arrives as split-K partial sums; the lanes add them in parallel
+      for (int s = lane; s < p.usplits; s += 32) acc += __ldg(p.upart + (static_cast<size_t>(s) * M + m) * R + q);
       acc = warp_sum(acc);
       if (lane == 0) {
-        float a = acc + bq;
-        for (int s = 0; s < p.usplits; ++s) a += p.upart[(static_cast<size_t>(s) * M + m) * R + q];
+        const float a = acc + bq;
         p.u[static_cast<size_t>(m) * R + q] = __float2bfloat16_rn(a / (1.f + expf(-a)));
       }
     }
@@ -211,38 +253,35 @@ int gru_grid(int Ds, int num_sms, int* units) {
   return G;
 }
 
-static int gru_bg(int Ds, int U) {
-  const size_t whh = static_cast<size_t>(3) * U * Ds * 2;
-  const size_t budget = 220 * 1024;
-  if (whh + Ds * 4 + 12 * U + 64 > budget) return 0;
-  size_t bg = (budget - whh - 64) / (static_cast<size_t>(Ds) * 4 + 12 * U);
-  return bg > 8 ? 8 : static_cast<int>(bg);
+static constexpr size_t kGruSmemBudget = 220 * 1024;
+
+static int gru_bg(int Ds, int U, int M, int B) {
+  int bg = B < 8 ? B : 8;
+  while (bg > 1 && gru_layout(Ds, U, M, bg).total > kGruSmemBudget) --bg;
+  return gru_layout(Ds, U, M, bg).total > kGruSmemBudget ? 0 : bg;
 }
 
-size_t gru_smem_bytes(int Ds, int units) {
-  const int bg = gru_bg(Ds, units);
-  if (bg == 0) return 0;
-  return static_cast<size_t>(3) * units * Ds * 2 + static_cast<size_t>(bg) * Ds * 4 +
-         static_cast<size_t>(bg) * 12 * units + 64;
+size_t gru_smem_bytes(int Ds, int units, int M, int B) {
+  const int bg = gru_bg(Ds, units, M, B);
+  return bg == 0 ? 0 : gru_layout(Ds, units, M, bg).total;
 }
 
 cudaError_t launch_gru(const GruParams& p, int grid, cudaStream_t stream) {
-  const int bg = gru_bg(p.Ds, p.units);
-  const size_t smem = gru_smem_bytes(p.Ds, p.units);
+  const int M = p.B * p.K;
+  const int bg = gru_bg(p.Ds, p.units, M, p.B);
   if (bg == 0) return cudaErrorInvalidValue;
-  cudaError_t e = cudaFuncSetAttribute(gru_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
-  if (e != cudaSuccess) return e;
-  int per_sm = 0, dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, gru_kernel, kGruThreads, smem);
-  if (e != cudaSuccess) return e;
-  if (per_sm * sms < grid) return cudaErrorCooperativeLaunchTooLarge;
+  const size_t smem = gru_layout(p.Ds, p.units, M, bg).total;
+  static size_t attr_smem = 0;
+  if (smem > attr_smem) {
+    cudaError_t e = cudaFuncSetAttribute(gru_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    attr_smem = smem;
+  }
   GruParams pp = p;
   int bgv = bg;
   void* args[] = {&pp, &bgv};
-  e = cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(gru_kernel), dim3(grid), dim3(kGruThreads), args,
-                                  smem, stream);
+  cudaError_t e = cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(gru_kernel), dim3(grid),
+                                              dim3(kGruThreads), args, smem, stream);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

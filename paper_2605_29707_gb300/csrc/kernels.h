@@ -28,7 +28,7 @@ struct TcParams {
   int splits, kb_per_split, total_items;
   int w_evict_first;
   const __nv_bfloat16* bias;  // softmax: b2 [V] or nullptr
-  float* out;                 // softmax: partial records [M][nchunks][rec]; store: [splits][M][ld_out]
+  float* out;                 // softmax: partial records [M][rec fields][nchunks]; store: [splits][M][ld_out]
   int ld_out;
   int* status;
 };
@@ -67,12 +67,13 @@ struct GruParams {
   int* status;
 };
 int gru_grid(int Ds, int num_sms, int* units);
-size_t gru_smem_bytes(int Ds, int units);
+size_t gru_smem_bytes(int Ds, int units, int M, int B);  // 0 = does not fit
 cudaError_t launch_gru(const GruParams& p, int grid, cudaStream_t stream);
 
 // ---------------------------------------------------------------- merge + tree
 struct TreeParams {
-  const float* partials;  // [M][nchunks][rec]
+  const float* partials;  // [M][rec fields][nchunks]
+  unsigned int* seq_done; // [B] zeroed counters: rows of each sequence merged so far
   int nchunks, kmax;
   int B, K, k, N;
   int32_t* topk_ids;      // [B, K, k]

@@ -148,13 +148,15 @@ struct OnlineTopK {
     for (int q = 0; q < KM; ++q) insert_keyed(ov[q], oi[q]);
   }
 
-  __device__ __forceinline__ void store(float* rec) const {
-    rec[0] = mx;
-    rec[1] = se;
+  // Partial records are stored field-major: field f of chunk c at base[f * stride + c], so a
+  // merge kernel reading one field of consecutive chunks issues coalesced loads.
+  __device__ __forceinline__ void store(float* base, int stride) const {
+    base[0] = mx;
+    base[stride] = se;
 #pragma unroll
     for (int q = 0; q < KM; ++q) {
-      rec[2 + q] = tv[q];
-      reinterpret_cast<int*>(rec)[2 + KM + q] = ti[q];
+      base[(2 + q) * stride] = tv[q];
+      reinterpret_cast<int*>(base)[(2 + KM + q) * stride] = ti[q];
     }
   }
 };
@@ -419,10 +421,10 @@ __global__ void __launch_bounds__(192, 1)
         const int tt = ep / C::kTPT;
         const int tok = tok_tile * BN + tt;
         if (ep % C::kTPT == 0 && tok < p.rows_tok)
-          st.store(p.out + (static_cast<size_t>(tok) * p.nchunks + chunk) * C::kRec);
+          st.store(p.out + static_cast<size_t>(tok) * C::kRec * p.nchunks + chunk, p.nchunks);
       } else {
         const int tok = tok_tile * 128 + 32 * q + lane;
-        if (tok < p.rows_tok) st.store(p.out + (static_cast<size_t>(tok) * p.nchunks + chunk) * C::kRec);
+        if (tok < p.rows_tok) st.store(p.out + static_cast<size_t>(tok) * C::kRec * p.nchunks + chunk, p.nchunks);
       }
     }
   }

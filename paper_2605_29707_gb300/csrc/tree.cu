@@ -1,13 +1,18 @@
 // tree.cu -- merge of the per-CTA softmax partials into log-probabilities and top-k lists,
-// then the best-first draft tree (the "Tree" cost of the paper's Fig. 1), one CTA per sequence.
+// then the best-first draft tree (the "Tree" cost of the paper's Fig. 1).
 //
-// Merge: one warp per draft position combines the (max, sum-exp, top-KMAX) records of every
-// vocabulary chunk into lse = max + log(sum) and the k best (value desc, id asc) tokens, with
-// logp = logit - lse.
-// Tree: warp 0 selects N nodes best-first.  The frontier is every child of an already selected
-// node (or of the anchor) not yet selected; the next node is the frontier entry with the greatest
-// (score, lower token id, lower parent index).  For each expanded node ("slot") the warp caches
-// its best remaining child, so a step is one argmax over the slots plus two child refreshes.
+// Merge: one CTA per draft row (sequence b, position j).  Thread c reads chunk c's record
+// (running max, sum of exp, top-KMAX list; field-major, so the loads are coalesced), the CTA
+// reduces lse = max + log(sum) and extracts the k best (value desc, id asc) tokens; logp =
+// logit - lse.
+// Tree: the CTA that merges the last row of a sequence (atomic counter) selects N nodes
+// best-first with one warp.  The frontier is every child (from its position's top-k list) of
+// the anchor or of an already selected node that is not selected yet; the next node is the
+// frontier entry with the greatest (score, lower token id, lower parent index).  Each expanded
+// node ("slot") caches its best remaining child.  Children of a slot have non-increasing scores
+// (sorted log-probs plus the same parent score), so the best remaining child is the first
+// unselected one, or a lower-token child of exactly the same score; one lane refreshes a slot
+// by that short scan.
 #include <math.h>
 
 #include "kernels.h"
@@ -15,13 +20,20 @@
 
 namespace dm {
 
-constexpr int kTreeThreads = 512;
+constexpr int kMergeThreads = 256;
 constexpr int kMaxK = 64;
 constexpr int kMaxTopk = 32;
 constexpr int kMaxN = 256;
 
+__device__ __forceinline__ void warp_argmax2(uint32_t hi, uint32_t lo, uint32_t& mhi, uint32_t& mlo, int& src) {
+  mhi = __reduce_max_sync(0xffffffffu, hi);
+  mlo = __reduce_max_sync(0xffffffffu, hi == mhi ? lo : 0u);
+  const unsigned ball = __ballot_sync(0xffffffffu, hi == mhi && lo == mlo);
+  src = __ffs(ball) - 1;
+}
+
 template <int KM>
-__device__ __forceinline__ void lane_insert(float (&tv)[KM], int (&ti)[KM], float x, int id) {
+__device__ __forceinline__ void insert_keyed(float (&tv)[KM], int (&ti)[KM], float x, int id) {
 #pragma unroll
   for (int q = 0; q < KM; ++q) {
     const bool sw = x > tv[q] || (x == tv[q] && (unsigned)id < (unsigned)ti[q]);
@@ -34,160 +46,190 @@ __device__ __forceinline__ void lane_insert(float (&tv)[KM], int (&ti)[KM], floa
   }
 }
 
-__device__ __forceinline__ void warp_argmax2(uint32_t hi, uint32_t lo, uint32_t& mhi, uint32_t& mlo,
-                                             int& src) {
-  mhi = __reduce_max_sync(0xffffffffu, hi);
-  mlo = __reduce_max_sync(0xffffffffu, hi == mhi ? lo : 0u);
-  const unsigned ball = __ballot_sync(0xffffffffu, hi == mhi && lo == mlo);
-  src = __ffs(ball) - 1;
+__device__ __forceinline__ void lse_merge(float& mx, float& se, float om, float os) {
+  const float nm = fmaxf(mx, om);
+  if (nm == -INFINITY) return;
+  se = (mx == -INFINITY ? 0.f : se * __expf(mx - nm)) + (om == -INFINITY ? 0.f : os * __expf(om - nm));
+  mx = nm;
+}
+
+struct TreeSlots {
+  float score[kMaxN + 1];
+  int depth[kMaxN + 1];
+  unsigned mask[kMaxN + 1];
+  unsigned hi[kMaxN + 1];
+  unsigned lo[kMaxN + 1];
+  int j[kMaxN + 1];
+};
+
+// Best remaining child of slot s (one thread).
+__device__ __forceinline__ void refresh_slot(TreeSlots& S, int s, const float* lp, const int* ids, int K, int k) {
+  const int d = S.depth[s];
+  if (d >= K) { S.hi[s] = 0u; return; }
+  const unsigned all = (k == 32) ? 0xffffffffu : ((1u << k) - 1u);
+  const unsigned avail = ~S.mask[s] & all;
+  if (avail == 0u) { S.hi[s] = 0u; return; }
+  const int j0 = __ffs(avail) - 1;
+  const float base = S.score[s];
+  const float* row_lp = lp + d * k;
+  const int* row_id = ids + d * k;
+  const float best_sc = base + row_lp[j0];
+  int best_j = j0, best_tok = row_id[j0];
+  for (int j = j0 + 1; j < k; ++j) {
+    const float sc = base + row_lp[j];
+    if (sc < best_sc) break;
+    if (!((S.mask[s] >> j) & 1u) && row_id[j] < best_tok) { best_j = j; best_tok = row_id[j]; }
+  }
+  S.hi[s] = f32_ord(best_sc);
+  S.lo[s] = ((0x3FFFFFu - static_cast<unsigned>(best_tok)) << 10) | (0x3FFu - static_cast<unsigned>(s));
+  S.j[s] = best_j;
 }
 
 template <int KM>
-__global__ void __launch_bounds__(kTreeThreads) merge_tree_kernel(const TreeParams p) {
+__global__ void __launch_bounds__(kMergeThreads) merge_tree_kernel(const TreeParams p) {
+  constexpr int F = 2 + 2 * KM;
+  constexpr int kWarps = kMergeThreads / 32;
+  __shared__ float s_mx[kWarps], s_se[kWarps];
+  __shared__ unsigned s_hi[kWarps], s_lo[kWarps];
+  __shared__ int s_src[kWarps];
+  __shared__ int s_win, s_last;
   __shared__ float s_lp[kMaxK * kMaxTopk];
   __shared__ int s_id[kMaxK * kMaxTopk];
-  __shared__ float sl_score[kMaxN + 1];
-  __shared__ int sl_depth[kMaxN + 1];
-  __shared__ unsigned sl_popped[kMaxN + 1];
-  __shared__ unsigned sl_hi[kMaxN + 1];
-  __shared__ unsigned sl_lo[kMaxN + 1];
-  __shared__ int sl_j[kMaxN + 1];
+  __shared__ TreeSlots S;
 
-  const int b = blockIdx.x;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  constexpr int kWarps = kTreeThreads / 32;
-  constexpr int kRec = 2 + 2 * KM;
-  const int K = p.K, k = p.k, N = p.N;
+  const int m = blockIdx.x;
+  const int K = p.K, k = p.k, N = p.N, nch = p.nchunks;
+  const int b = m / K;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const float* base = p.partials + static_cast<size_t>(m) * F * nch;
+  const int* ibase = reinterpret_cast<const int*>(base);
 
-  // ---------------------------------------------------------------- merge
-  for (int j = warp; j < K; j += kWarps) {
-    const int m = b * K + j;
-    float mx = -INFINITY, se = 0.f;
-    float tv[KM];
-    int ti[KM];
+  // ------------------------------------------------------------ this thread's chunks
+  float mx = -INFINITY, se = 0.f;
+  float tv[KM];
+  int ti[KM];
 #pragma unroll
-    for (int q = 0; q < KM; ++q) { tv[q] = -INFINITY; ti[q] = -1; }
-    for (int c = lane; c < p.nchunks; c += 32) {
-      const float* r = p.partials + (static_cast<size_t>(m) * p.nchunks + c) * kRec;
-      const float cm = r[0], cs = r[1];
-      const float nm = fmaxf(mx, cm);
-      if (nm != -INFINITY) {
-        se = (mx == -INFINITY ? 0.f : se * __expf(mx - nm)) + (cm == -INFINITY ? 0.f : cs * __expf(cm - nm));
-        mx = nm;
-      }
-      for (int q = 0; q < KM; ++q) {  // the chunk's list is sorted: stop at the first loser
-        const float x = r[2 + q];
-        const int id = reinterpret_cast<const int*>(r)[2 + KM + q];
-        if (!(x > tv[KM - 1] || (x == tv[KM - 1] && (unsigned)id < (unsigned)ti[KM - 1]))) break;
-        lane_insert<KM>(tv, ti, x, id);
-      }
-    }
+  for (int q = 0; q < KM; ++q) { tv[q] = -INFINITY; ti[q] = -1; }
+  for (int c = tid; c < nch; c += kMergeThreads) {
+    const float cm = __ldg(base + c), cs = __ldg(base + nch + c);
+    float v[KM];
+    int id[KM];
 #pragma unroll
-    for (int o = 16; o; o >>= 1) {
-      const float om = __shfl_xor_sync(0xffffffffu, mx, o);
-      const float os = __shfl_xor_sync(0xffffffffu, se, o);
-      const float nm = fmaxf(mx, om);
-      if (nm != -INFINITY) {
-        se = (mx == -INFINITY ? 0.f : se * __expf(mx - nm)) + (om == -INFINITY ? 0.f : os * __expf(om - nm));
-        mx = nm;
-      }
+    for (int q = 0; q < KM; ++q) {
+      v[q] = __ldg(base + (2 + q) * nch + c);
+      id[q] = __ldg(ibase + (2 + KM + q) * nch + c);
     }
-    const float lse = mx + logf(se);
-    for (int q = 0; q < k; ++q) {
-      uint32_t mhi, mlo;
-      int src;
-      warp_argmax2(f32_ord(tv[0]), ~static_cast<uint32_t>(ti[0]), mhi, mlo, src);
-      const float val = __shfl_sync(0xffffffffu, tv[0], src);
-      const int id = __shfl_sync(0xffffffffu, ti[0], src);
-      if (lane == src) {
+    lse_merge(mx, se, cm, cs);
+    if (c == tid) {
 #pragma unroll
-        for (int i = 0; i + 1 < KM; ++i) { tv[i] = tv[i + 1]; ti[i] = ti[i + 1]; }
-        tv[KM - 1] = -INFINITY;
-        ti[KM - 1] = -1;
-      }
-      if (lane == 0) {
-        const float lp = val - lse;
-        p.topk_ids[static_cast<size_t>(m) * k + q] = id;
-        p.topk_logp[static_cast<size_t>(m) * k + q] = lp;
-        s_id[j * k + q] = id;
-        s_lp[j * k + q] = lp;
-      }
+      for (int q = 0; q < KM; ++q) { tv[q] = v[q]; ti[q] = id[q]; }
+    } else {
+#pragma unroll
+      for (int q = 0; q < KM; ++q) insert_keyed<KM>(tv, ti, v[q], id[q]);
     }
+  }
+
+  // ------------------------------------------------------------ lse over the CTA
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    const float om = __shfl_xor_sync(0xffffffffu, mx, o);
+    const float os = __shfl_xor_sync(0xffffffffu, se, o);
+    lse_merge(mx, se, om, os);
+  }
+  if (lane == 0) { s_mx[warp] = mx; s_se[warp] = se; }
+  __syncthreads();
+  mx = -INFINITY;
+  se = 0.f;
+#pragma unroll
+  for (int w = 0; w < kWarps; ++w) lse_merge(mx, se, s_mx[w], s_se[w]);
+  const float lse = mx + logf(se);
+
+  // ------------------------------------------------------------ k best heads, one per round
+  for (int q = 0; q < k; ++q) {
+    uint32_t mhi, mlo;
+    int src;
+    warp_argmax2(f32_ord(tv[0]), ~static_cast<uint32_t>(ti[0]), mhi, mlo, src);
+    if (lane == 0) { s_hi[warp] = mhi; s_lo[warp] = mlo; s_src[warp] = warp * 32 + src; }
+    __syncthreads();
+    if (warp == 0) {
+      const uint32_t h = lane < kWarps ? s_hi[lane] : 0u;
+      const uint32_t l = lane < kWarps ? s_lo[lane] : 0u;
+      uint32_t wh, wl;
+      int ws;
+      warp_argmax2(h, l, wh, wl, ws);
+      if (lane == 0) s_win = s_src[ws];
+    }
+    __syncthreads();
+    if (tid == s_win) {
+      p.topk_ids[static_cast<size_t>(m) * k + q] = ti[0];
+      p.topk_logp[static_cast<size_t>(m) * k + q] = tv[0] - lse;
+#pragma unroll
+      for (int i = 0; i + 1 < KM; ++i) { tv[i] = tv[i + 1]; ti[i] = ti[i + 1]; }
+      tv[KM - 1] = -INFINITY;
+      ti[KM - 1] = -1;
+    }
+  }
+
+  // ------------------------------------------------------------ last row of the sequence?
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) s_last = (atomicAdd(p.seq_done + b, 1u) == static_cast<unsigned>(K - 1));
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const size_t rows = static_cast<size_t>(b) * K * k;
+  for (int e = tid; e < K * k; e += kMergeThreads) {
+    s_id[e] = __ldcg(p.topk_ids + rows + e);
+    s_lp[e] = __ldcg(p.topk_logp + rows + e);
   }
   __syncthreads();
   if (warp != 0) return;
 
-  // ---------------------------------------------------------------- tree (warp 0)
-  // slot 0 is the anchor; slot i+1 is node i.  Child key: hi = ordered score, lo = token
-  // (lower wins) then parent (lower wins); hi == 0 marks "no child left".
-  auto refresh = [&](int s) {
-    const int d = sl_depth[s];
-    uint32_t hi = 0, lo = 0;
-    if (lane < k && !((sl_popped[s] >> lane) & 1u)) {
-      const float sc = sl_score[s] + s_lp[d * k + lane];
-      hi = f32_ord(sc);
-      lo = ((0x3FFFFFu - static_cast<uint32_t>(s_id[d * k + lane])) << 10) | (0x3FFu - static_cast<uint32_t>(s));
-    }
-    uint32_t mhi, mlo;
-    int src;
-    warp_argmax2(hi, lo, mhi, mlo, src);
-    if (lane == 0) {
-      sl_hi[s] = mhi;
-      sl_lo[s] = mlo;
-      sl_j[s] = src;
-    }
-    __syncwarp();
-  };
-
+  // ------------------------------------------------------------ tree (warp 0)
+  const size_t ob = static_cast<size_t>(b) * N;
   if (lane == 0) {
-    sl_score[0] = 0.f;
-    sl_depth[0] = 0;
-    sl_popped[0] = 0u;
+    S.score[0] = 0.f;
+    S.depth[0] = 0;
+    S.mask[0] = 0u;
+    refresh_slot(S, 0, s_lp, s_id, K, k);
   }
   __syncwarp();
-  refresh(0);
-  const size_t ob = static_cast<size_t>(b) * N;
   for (int i = 0; i < N; ++i) {
-    uint32_t hi = 0, lo = 0;
+    uint32_t hi = 0u, lo = 0u;
     int sb = -1;
     for (int s = lane; s <= i; s += 32) {
-      const uint32_t h = sl_hi[s], l = sl_lo[s];
-      if (h > hi || (h == hi && h != 0 && l > lo)) { hi = h; lo = l; sb = s; }
+      const uint32_t h = S.hi[s], l = S.lo[s];
+      if (h > hi || (h == hi && h != 0u && l > lo)) { hi = h; lo = l; sb = s; }
     }
     uint32_t mhi, mlo;
     int src;
     warp_argmax2(hi, lo, mhi, mlo, src);
     const int s = __shfl_sync(0xffffffffu, sb, src);
-    const int jj = sl_j[s];
-    const int d = sl_depth[s];
-    const int tok = s_id[d * k + jj];
-    const float sc = sl_score[s] + s_lp[d * k + jj];
-    __syncwarp();
     if (lane == 0) {
+      const int jj = S.j[s];
+      const int d = S.depth[s];
+      const int tok = s_id[d * k + jj];
+      const float sc = S.score[s] + s_lp[d * k + jj];
       p.tree_parent[ob + i] = s - 1;
       p.tree_token[ob + i] = tok;
       p.tree_depth[ob + i] = d + 1;
       if (p.tree_score) p.tree_score[ob + i] = sc;
-      sl_score[i + 1] = sc;
-      sl_depth[i + 1] = d + 1;
-      sl_popped[i + 1] = 0u;
-      sl_popped[s] |= 1u << jj;
+      S.score[i + 1] = sc;
+      S.depth[i + 1] = d + 1;
+      S.mask[i + 1] = 0u;
+      S.mask[s] |= 1u << jj;
+      refresh_slot(S, s, s_lp, s_id, K, k);
+      refresh_slot(S, i + 1, s_lp, s_id, K, k);
     }
     __syncwarp();
-    refresh(s);
-    if (d + 1 < K) {
-      refresh(i + 1);
-    } else {
-      if (lane == 0) sl_hi[i + 1] = 0u;
-      __syncwarp();
-    }
   }
 }
 
 cudaError_t launch_merge_tree(const TreeParams& p, cudaStream_t stream) {
   if (p.K > kMaxK || p.k > kMaxTopk || p.N > kMaxN) return cudaErrorInvalidValue;
-  if (p.kmax == 16) merge_tree_kernel<16><<<p.B, kTreeThreads, 0, stream>>>(p);
-  else if (p.kmax == 32) merge_tree_kernel<32><<<p.B, kTreeThreads, 0, stream>>>(p);
+  const int rows = p.B * p.K;
+  if (p.kmax == 16) merge_tree_kernel<16><<<rows, kMergeThreads, 0, stream>>>(p);
+  else if (p.kmax == 32) merge_tree_kernel<32><<<rows, kMergeThreads, 0, stream>>>(p);
   else return cudaErrorInvalidValue;
   return cudaGetLastError();
 }

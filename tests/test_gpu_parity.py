@@ -127,7 +127,7 @@ def test_unsupported_and_invalid_arguments_on_device():
                 workspace=st.workspace, workspace_bytes=st.ws_bytes)
     assert binding.domino_draft_step(**args) == 0
     assert binding.domino_draft_step(**dict(args, workspace_bytes=st.ws_bytes - 1)) == binding.DOMINO_ERR_INVALID_ARG
-    assert binding.domino_draft_step(**dict(args, N=15)) == binding.DOMINO_ERR_INVALID_ARG  # > 2 + 4 + 8
+    assert binding.domino_draft_step(**dict(args, N=31)) == binding.DOMINO_ERR_INVALID_ARG  # > 2+4+8+16
     assert binding.domino_draft_step(**dict(args, hidden=hidden.data_ptr() + 2)) == binding.DOMINO_ERR_UNSUPPORTED
     assert binding.domino_draft_step(**dict(args, k=33)) in (binding.DOMINO_ERR_UNSUPPORTED,
                                                              binding.DOMINO_ERR_INVALID_ARG)
