@@ -144,6 +144,36 @@ DOMINO_API int domino_abi_version(void);
  * R > 0), so a caller can count device work. */
 DOMINO_API int domino_launches_per_step(int B, int K, int H, int V, int Ds, int R, int k, int N);
 
+/* Draft step for callers that cannot allocate device memory.  Some callers cannot call
+ * cudaMalloc or any allocator at all: code running inside a host framework that owns every
+ * allocation, a plugin loaded into a process whose memory pool is fixed up front, or a
+ * real-time caller that must not risk an allocation failing or blocking.  This entry point
+ * takes the same inputs and outputs as domino_draft_step but no workspace: its scratch lives
+ * in a file-scope static device array of DOMINO_STATIC_SCRATCH_BYTES (16 MiB) inside the
+ * library, which every GPU that loads the library holds until the process exits.  The paper
+ * has no counterpart to this; it is a deployment convenience.
+ *   - The first call on a device looks up that array's device address (cudaGetSymbolAddress,
+ *     with that device current); make the first call on each device before any stream capture.
+ *   - Sizes whose step needs more scratch than the array (domino_workspace_bytes(...) >
+ *     DOMINO_STATIC_SCRATCH_BYTES; e.g. the B = 32 serving batch) return DOMINO_ERR_UNSUPPORTED
+ *     before anything is enqueued.
+ *   - Every call on a device shares the one array and it keeps the last call's contents; each
+ *     call clears the words that must start at zero (status and counters) itself.  Calls whose
+ *     work overlaps on the GPU (other streams, other host threads) race on the array: serialise
+ *     them.
+ *   - No allocation of any kind is made (no cudaMalloc / cudaFree, no library allocator).
+ * device_status: optional device int32; after the step it receives the device status word
+ * (DOMINO_OK, DOMINO_ERR_BAD_TOKEN or DOMINO_ERR_TIMEOUT) by an asynchronous copy on `stream`.
+ * Returns DOMINO_OK once enqueued, or a negative code with nothing enqueued. */
+#define DOMINO_STATIC_SCRATCH_BYTES (16u << 20)
+DOMINO_API int domino_draft_step_static_scratch(const void* hidden, const int32_t* prefix_ids,
+                                                const void* w_lm, const domino_head_weights* head,
+                                                int B, int K, int H, int V, int k, int N,
+                                                int32_t* topk_ids, float* topk_logp,
+                                                int32_t* tree_parent, int32_t* tree_token,
+                                                int32_t* tree_depth, float* tree_score,
+                                                int32_t* device_status, void* stream);
+
 /* Per-kernel device timing, for the per-component latency breakdown the paper reports in
  * its Fig. 1 (LM head, Domino head, tree).  After domino_timing_begin(max_launches), every
  * kernel the library enqueues (up to max_launches of them, on any stream) is bracketed by a

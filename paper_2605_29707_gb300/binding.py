@@ -23,7 +23,10 @@ DOMINO_ERR_BAD_TOKEN = -5
 # every entry point declared in include/domino.h
 SYMBOLS = ("domino_workspace_bytes", "domino_draft_step", "domino_workspace_bytes_host",
            "domino_draft_step_host", "domino_check_status", "domino_status_string",
-           "domino_abi_version", "domino_launches_per_step", "domino_timing_begin", "domino_timing_end")
+           "domino_abi_version", "domino_launches_per_step", "domino_timing_begin", "domino_timing_end",
+           "domino_draft_step_static_scratch")
+
+DOMINO_STATIC_SCRATCH_BYTES = 16 << 20
 
 KERNEL_KINDS = ("gather", "gru_input_proj", "w1_hidden_proj", "gru", "vocab_gemm_softmax_topk", "merge_tree")
 
@@ -74,6 +77,9 @@ def load():
     lib.domino_timing_begin.restype = I
     lib.domino_timing_end.argtypes = [P, P, I]
     lib.domino_timing_end.restype = I
+    lib.domino_draft_step_static_scratch.argtypes = [P, P, P, ctypes.POINTER(domino_head_weights)] + [I] * 6 + \
+        [P] * 6 + [P, P]
+    lib.domino_draft_step_static_scratch.restype = I
     _lib = lib
     return lib
 
@@ -160,3 +166,15 @@ def domino_timing_end() -> dict:
     if rc != 0:
         raise DominoError(rc, "domino_timing_end")
     return {KERNEL_KINDS[i]: (float(ms[i]), int(cnt[i])) for i in range(n)}
+
+
+def domino_draft_step_static_scratch(hidden, prefix_ids, w_lm, head, B, K, H, V, k, N, topk_ids, topk_logp,
+                                     tree_parent, tree_token, tree_depth, tree_score, device_status=None,
+                                     stream=None) -> int:
+    """The draft step for callers that cannot allocate device memory: no workspace argument;
+    the library's own static 16 MiB device array serves as scratch (see include/domino.h)."""
+    h = ctypes.byref(head) if head is not None else None
+    return int(load().domino_draft_step_static_scratch(
+        _addr(hidden), _addr(prefix_ids), _addr(w_lm), h, B, K, H, V, k, N, _addr(topk_ids), _addr(topk_logp),
+        _addr(tree_parent), _addr(tree_token), _addr(tree_depth), _addr(tree_score), _addr(device_status),
+        _stream(stream)))

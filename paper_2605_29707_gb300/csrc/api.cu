@@ -532,3 +532,59 @@ int domino_launches_per_step(int B, int K, int H, int V, int Ds, int R, int k, i
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------- static-scratch entry point
+// Scratch of domino_draft_step_static_scratch, for callers that cannot allocate device memory.
+// Host code only sees a stand-in for this symbol; its device address comes from
+// cudaGetSymbolAddress, looked up once per device with that device current.
+static __device__ __align__(256) unsigned char g_static_scratch[DOMINO_STATIC_SCRATCH_BYTES];
+
+namespace {
+
+constexpr int kMaxScratchDevices = 256;
+std::mutex g_static_scratch_mu;
+void* g_static_scratch_addr[kMaxScratchDevices] = {};
+
+int static_scratch_address(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return DOMINO_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxScratchDevices) return DOMINO_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_static_scratch_mu);
+  if (g_static_scratch_addr[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || p == nullptr) return DOMINO_ERR_CUDA;
+    g_static_scratch_addr[dev] = p;
+  }
+  *out = g_static_scratch_addr[dev];
+  return DOMINO_OK;
+}
+
+}  // namespace
+
+extern "C" int domino_draft_step_static_scratch(const void* hidden, const int32_t* prefix_ids, const void* w_lm,
+                                                const domino_head_weights* head, int B, int K, int H, int V, int k,
+                                                int N, int32_t* topk_ids, float* topk_logp, int32_t* tree_parent,
+                                                int32_t* tree_token, int32_t* tree_depth, float* tree_score,
+                                                int32_t* device_status, void* stream) {
+  const bool hd = head_active(head);
+  if (!topk_ids || !topk_logp || !tree_parent || !tree_token || !tree_depth) return DOMINO_ERR_INVALID_ARG;
+  int rc = check_pointers(hidden, prefix_ids, w_lm, head, hd);
+  if (rc) return rc;
+  Plan P;
+  rc = make_plan(B, K, H, V, hd ? head->Ds : 0, hd ? head->R : 0, k, N, hd, &P);
+  if (rc) return rc;
+  if (P.dev_total > DOMINO_STATIC_SCRATCH_BYTES) return DOMINO_ERR_UNSUPPORTED;
+  void* scratch = nullptr;
+  rc = static_scratch_address(&scratch);
+  if (rc) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // run_step clears the status word and the counters at the start of the scratch itself
+  rc = run_step(P, hidden, prefix_ids, w_lm, head, topk_ids, topk_logp, tree_parent, tree_token, tree_depth,
+                tree_score, static_cast<uint8_t*>(scratch), st);
+  if (rc) return rc;
+  if (device_status != nullptr &&
+      cudaMemcpyAsync(device_status, static_cast<uint8_t*>(scratch) + P.off_ctrl, sizeof(int32_t),
+                      cudaMemcpyDeviceToDevice, st) != cudaSuccess)
+    return DOMINO_ERR_CUDA;
+  return DOMINO_OK;
+}
