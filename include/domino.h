@@ -184,8 +184,11 @@ DOMINO_API int domino_draft_step_static_scratch(const void* hidden, const int32_
 enum domino_kernel_kind {
   DOMINO_KERNEL_GATHER = 0,       /* E_j = emb[prefix id], id range check */
   DOMINO_KERNEL_GRU_INPUT = 1,    /* E . W_ih^T on tensor cores (split-K partials) */
-  DOMINO_KERNEL_W1_HIDDEN = 2,    /* hidden . W1[:, :H]^T on tensor cores (split-K partials) */
-  DOMINO_KERNEL_GRU = 3,          /* GRU recurrence over K positions, then u = SiLU(...) */
+  DOMINO_KERNEL_W1_HIDDEN = 2,    /* W1 projection on tensor cores (split-K partials): the hidden
+                                     half before the GRU for M <= 128; both halves after it, plus
+                                     the SiLU finalize, for larger M */
+  DOMINO_KERNEL_GRU = 3,          /* GRU recurrence over K positions (and u = SiLU(...) for
+                                     M <= 128) */
   DOMINO_KERNEL_VOCAB = 4,        /* [hidden | u] . [W_lm | W2]^T with online softmax / top-k */
   DOMINO_KERNEL_TREE = 5,         /* merge to log-probs and top-k; best-first tree */
   DOMINO_KERNEL_KINDS = 6

@@ -54,10 +54,13 @@ struct Plan {
   bool swap;
   int bn, kmax, rec, tok_tiles, w_tiles, nchunks, w_per_chunk, grid;
   StorePlan xg, ug;
-  int gru_grid, gru_units;
+  dm::GruPlan gru;
+  bool u_in_gru;  // small M: u finished inside the GRU kernel; large M: W1 GEMM + finalize
+  bool overlap;   // vocab GEMM launched as a programmatic dependent of the GRU (deferred W2)
+  int tmem_cols;  // TMEM columns of the vocab GEMM
   // workspace layout (offsets in bytes)
   size_t ctrl_bytes;
-  size_t off_ctrl, off_E, off_xpart, off_upart, off_S, off_u, off_part, dev_total;
+  size_t off_ctrl, off_E, off_xpart, off_upart, off_xs, off_hx, off_S, off_u, off_part, dev_total;
   size_t off_hid, off_ids, off_tid, off_tlp, off_tpar, off_ttok, off_tdep, off_tsc, host_total;
 };
 
@@ -151,11 +154,20 @@ int make_plan(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head
   p.grid = p.tok_tiles * p.nchunks;
 
   if (head) {
+    p.u_in_gru = p.swap;
     p.xg = plan_store(M, 3 * Ds, ceil_div(H, 64), sms);
-    p.ug = plan_store(M, R, ceil_div(H, 64), sms);
-    p.gru_grid = dm::gru_grid(Ds, sms, &p.gru_units);
-    if (dm::gru_smem_bytes(Ds, p.gru_units, M, B) == 0) return DOMINO_ERR_UNSUPPORTED;
+    // small M: hidden half of W1 before the GRU; large M: both halves of W1 after it
+    p.ug = plan_store(M, R, p.u_in_gru ? ceil_div(H, 64) : ceil_div(H, 64) + ceil_div(Ds, 64), sms);
+    p.gru = dm::gru_plan(B, Ds, sms);
+    if (p.gru.smem == 0) return DOMINO_ERR_UNSUPPORTED;
+    // Overlap the GRU with the W_lm stream when a deferred-mode vocab CTA and a GRU CTA fit on
+    // one SM (228 KB of shared memory, 1 KB reserved per CTA) and every tile of a CTA can keep
+    // its own TMEM accumulator until u is ready.
+    const int vsm = dm::tc_softmax_deferred_smem(p.bn);
+    p.overlap = p.u_in_gru && vsm > 0 && p.w_per_chunk * p.bn <= 512 &&
+                static_cast<size_t>(vsm) + p.gru.smem + 2048 <= 228 * 1024;
   }
+  p.tmem_cols = pow2_at_least(p.overlap ? p.w_per_chunk * p.bn : 2 * p.bn, 32);
 
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -169,7 +181,9 @@ int make_plan(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head
     p.off_E = take(static_cast<size_t>(M) * H * 2);
     p.off_xpart = take(static_cast<size_t>(p.xg.splits) * M * 3 * Ds * 4);
     p.off_upart = take(static_cast<size_t>(p.ug.splits) * M * R * 4);
-    p.off_S = take(static_cast<size_t>(M) * Ds * 4);
+    p.off_xs = take(static_cast<size_t>(M) * 3 * Ds * 4);
+    p.off_hx = take(static_cast<size_t>(M) * Ds * 4);
+    p.off_S = take(static_cast<size_t>(M) * Ds * 2);
     p.off_u = take(static_cast<size_t>(M) * R * 2);
   }
   p.off_part = take(static_cast<size_t>(M) * p.nchunks * p.rec * 4);
@@ -261,7 +275,8 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
   if (cudaMemsetAsync(ws + P.off_ctrl, 0, P.ctrl_bytes, st) != cudaSuccess) return DOMINO_ERR_CUDA;
 
   __nv_bfloat16* E = P.head ? reinterpret_cast<__nv_bfloat16*>(ws + P.off_E) : nullptr;
-  dm::GatherParams gp{ids, P.head ? static_cast<const __nv_bfloat16*>(hw->emb) : nullptr, E, M, H, V, status};
+  uint32_t* hx = P.head ? reinterpret_cast<uint32_t*>(ws + P.off_hx) : nullptr;
+  dm::GatherParams gp{ids, P.head ? static_cast<const __nv_bfloat16*>(hw->emb) : nullptr, E, hx, M, H, V, Ds, status};
   int ts = timing_open(DOMINO_KERNEL_GATHER, st);
   int rc = cuda_rc(dm::launch_gather(gp, st));
   timing_close(ts, st);
@@ -286,6 +301,7 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
       tp.tok_tiles = g.tok_tiles; tp.w_tiles = g.w_tiles;
       tp.splits = g.splits; tp.kb_per_split = g.kb_per_split; tp.total_items = g.total_items;
       tp.w_evict_first = 0;
+      tp.tmem_cols = pow2_at_least(2 * g.bn, 32);
       tp.out = xpart; tp.ld_out = 3 * Ds;
       tp.status = status;
       ts = timing_open(DOMINO_KERNEL_GRU_INPUT, st);
@@ -293,25 +309,37 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
       timing_close(ts, st);
       if (rc) return rc;
     }
-    // U partials: hidden [M, H] . W1[:, :H]^T (W1 rows are H + Ds long)
-    {
+    __nv_bfloat16* S = reinterpret_cast<__nv_bfloat16*>(ws + P.off_S);
+    // W1 GEMM: hidden [M, H] . W1[:, :H]^T (+ S [M, Ds] . W1[:, H:]^T on the large-M path)
+    auto w1_gemm = [&](bool both) -> int {
       const dm::TcParams base{};
       TcParams tp = base;
       const StorePlan& g = P.ug;
       CUtensorMap maps[4];
       if (!gemm_maps(&maps[0], &maps[1], g.swap, g.bn, hidden, M, H, H, hw->w1, R, H + Ds)) return DOMINO_ERR_CUDA;
-      maps[2] = maps[0];
-      maps[3] = maps[1];
-      tp.nkb1 = g.nkb; tp.nkb2 = 0;
+      if (both) {
+        const void* w1b = static_cast<const __nv_bfloat16*>(hw->w1) + H;
+        if (!gemm_maps(&maps[2], &maps[3], g.swap, g.bn, S, M, Ds, Ds, w1b, R, H + Ds)) return DOMINO_ERR_CUDA;
+      } else {
+        maps[2] = maps[0];
+        maps[3] = maps[1];
+      }
+      tp.nkb1 = ceil_div(H, 64);
+      tp.nkb2 = both ? ceil_div(Ds, 64) : 0;
       tp.rows_tok = M; tp.rows_w = R;
       tp.tok_tiles = g.tok_tiles; tp.w_tiles = g.w_tiles;
       tp.splits = g.splits; tp.kb_per_split = g.kb_per_split; tp.total_items = g.total_items;
       tp.w_evict_first = 0;
+      tp.tmem_cols = pow2_at_least(2 * g.bn, 32);
       tp.out = upart; tp.ld_out = R;
       tp.status = status;
-      ts = timing_open(DOMINO_KERNEL_W1_HIDDEN, st);
-      rc = cuda_rc(dm::launch_tc_gemm(dm::kModeStore, g.bn, g.swap, 16, maps, tp, g.grid, st));
-      timing_close(ts, st);
+      const int slot = timing_open(DOMINO_KERNEL_W1_HIDDEN, st);
+      const int r = cuda_rc(dm::launch_tc_gemm(dm::kModeStore, g.bn, g.swap, 16, maps, tp, g.grid, st));
+      timing_close(slot, st);
+      return r;
+    };
+    if (P.u_in_gru) {
+      rc = w1_gemm(false);
       if (rc) return rc;
     }
     dm::GruParams gr{};
@@ -323,15 +351,25 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
     gr.w1 = static_cast<const __nv_bfloat16*>(hw->w1);
     gr.b1 = static_cast<const __nv_bfloat16*>(hw->b1);
     gr.B = P.B; gr.K = P.K; gr.H = H; gr.Ds = Ds; gr.R = R;
-    gr.units = P.gru_units;
-    gr.S = reinterpret_cast<float*>(ws + P.off_S);
-    gr.u = u;
-    gr.barrier = barrier;
+    gr.units = P.gru.units; gr.gu = P.gru.gu; gr.gb = P.gru.gb; gr.bc = P.gru.bc;
+    gr.xs = reinterpret_cast<float*>(ws + P.off_xs);
+    gr.hx = hx;
+    gr.s_out = P.u_in_gru ? nullptr : S;
+    gr.u = P.u_in_gru ? u : nullptr;
     gr.status = status;
     ts = timing_open(DOMINO_KERNEL_GRU, st);
-    rc = cuda_rc(dm::launch_gru(gr, P.gru_grid, st));
+    rc = cuda_rc(dm::launch_gru(gr, P.gru, st));
     timing_close(ts, st);
     if (rc) return rc;
+    if (!P.u_in_gru) {
+      rc = w1_gemm(true);
+      if (rc) return rc;
+      dm::UFinalParams uf{upart, P.ug.splits, M, R, static_cast<const __nv_bfloat16*>(hw->b1), u};
+      ts = timing_open(DOMINO_KERNEL_W1_HIDDEN, st);
+      rc = cuda_rc(dm::launch_u_finalize(uf, st));
+      timing_close(ts, st);
+      if (rc) return rc;
+    }
   }
 
   // fused vocabulary GEMM with the online softmax / top-k epilogue
@@ -352,11 +390,16 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
     tp.tok_tiles = P.tok_tiles; tp.w_tiles = P.w_tiles;
     tp.nchunks = P.nchunks; tp.w_per_chunk = P.w_per_chunk;
     tp.w_evict_first = P.tok_tiles == 1 ? 1 : 0;
+    tp.defer = P.overlap ? 1 : 0;
+    tp.tmem_cols = P.tmem_cols;
     tp.bias = hw ? static_cast<const __nv_bfloat16*>(hw->b2) : nullptr;
     tp.out = reinterpret_cast<float*>(ws + P.off_part);
     tp.status = status;
     ts = timing_open(DOMINO_KERNEL_VOCAB, st);
-    rc = cuda_rc(dm::launch_tc_gemm(dm::kModeSoftmax, P.bn, P.swap, P.kmax, maps, tp, P.grid, st));
+    if (P.overlap)
+      rc = cuda_rc(dm::launch_tc_softmax_deferred(P.bn, P.kmax, maps, tp, P.grid, st));
+    else
+      rc = cuda_rc(dm::launch_tc_gemm(dm::kModeSoftmax, P.bn, P.swap, P.kmax, maps, tp, P.grid, st));
     timing_close(ts, st);
     if (rc) return rc;
   }
@@ -527,8 +570,11 @@ int domino_timing_end(float* total_ms, int* launches, int nkinds) {
 }
 
 int domino_launches_per_step(int B, int K, int H, int V, int Ds, int R, int k, int N) {
-  (void)B; (void)K; (void)H; (void)V; (void)Ds; (void)k; (void)N;
-  return R > 0 ? 6 : 3;  // gather, [X gemm, U gemm, gru,] vocab gemm, merge+tree
+  (void)H; (void)V; (void)Ds; (void)k; (void)N;
+  if (R <= 0) return 3;  // gather (id check), vocab GEMM, merge + tree
+  // small M: gather, X GEMM, W1-hidden GEMM, GRU (+u), vocab GEMM, merge + tree;
+  // large M: gather, X GEMM, GRU, W1 GEMM, u finalize, vocab GEMM, merge + tree
+  return static_cast<long long>(B) * K <= 128 ? 6 : 7;
 }
 
 }  // extern "C"

@@ -1,12 +1,13 @@
-// gru.cu -- embedding gather (E_j, section 4.1.2) and the GRU causal encoder
-// S_{i-1} = GRU(E_{<=i-1}) followed by the low-rank code u = SiLU(W1 [H_i; S_{i-1}] + b1).
+// gru.cu -- embedding gather (E_j, section 4.1.2), the GRU causal encoder
+// S_{i-1} = GRU(E_{<=i-1}) and the low-rank code u = SiLU(W1 [H_i; S_{i-1}] + b1).
 //
-// The recurrence is the only sequential part of the step: K dependent steps.  One cooperative
-// launch keeps a slice of W_hh resident in each CTA's shared memory for all K steps (CTA c owns
-// hidden units [c*U, c*U+U) and the three gate rows r|z|n of each), exchanges the new state
-// through global memory (L2) and separates the steps with a bounded grid barrier.  After the
-// last step the same CTAs finish u: the hidden half of W1 was computed earlier by the
-// tensor-core projection (split-K partial sums); the state half is added here.
+// The recurrence is the only sequential part of the step: K dependent steps, each needing the
+// full previous state of a sequence.  One cooperative launch keeps the W_hh rows of a block of
+// hidden units resident in shared memory for all K steps and computes W_hh . h_{t-1} on the
+// tensor cores (mma.sync, bf16 operands, fp32 accumulation).  States cross CTAs through L2 as
+// tagged words (bf16 value in the high half, a non-zero flag in the low half; one row per
+// (sequence, position), cleared by the gather kernel), so a CTA waits for exactly the data it
+// reads: no grid barrier and no release fence.  Every wait is bounded.
 #include <math.h>
 
 #include "kernels.h"
@@ -15,12 +16,19 @@
 namespace dm {
 
 constexpr int kGruThreads = 256;
+constexpr int kGruWarps = kGruThreads / 32;
+constexpr int kChunkSeqs = 32;  // sequences staged per MMA pass (4 n-tiles of 8)
 
+// ---------------------------------------------------------------------------- gather
 __global__ void __launch_bounds__(128) gather_kernel(const GatherParams p) {
   const int m = blockIdx.x;
   const int id = p.ids[m];
   const bool ok = id >= 0 && id < p.V;
   if (!ok && threadIdx.x == 0) set_status(p.status, kStatusBadToken);
+  if (p.hx != nullptr) {
+    uint4* hrow = reinterpret_cast<uint4*>(p.hx + static_cast<size_t>(m) * p.Ds);
+    for (int c = threadIdx.x; c < p.Ds / 4; c += blockDim.x) hrow[c] = make_uint4(0, 0, 0, 0);
+  }
   if (p.E == nullptr) return;
   uint4* dst = reinterpret_cast<uint4*>(p.E + static_cast<size_t>(m) * p.H);
   const uint4* src = reinterpret_cast<const uint4*>(p.emb + static_cast<size_t>(ok ? id : 0) * p.H);
@@ -32,36 +40,37 @@ cudaError_t launch_gather(const GatherParams& p, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
-__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
-  unsigned v;
-  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+// ---------------------------------------------------------------------------- helpers
+__device__ __forceinline__ uint4 ld_relaxed_v4(const uint32_t* p) {
+  uint4 v;
+  asm volatile("ld.relaxed.gpu.global.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p)
+               : "memory");
   return v;
 }
 
-__device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
-  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+// Reads 4 tagged state words, re-reading until all four carry the "written" flag.  Returns
+// false if that takes longer than kWaitCycles (the caller reports DOMINO_ERR_TIMEOUT).
+__device__ __forceinline__ bool poll_v4(const uint32_t* p, uint4& v) {
+  v = ld_relaxed_v4(p);
+  if ((v.x & v.y & v.z & v.w & 1u) != 0u) return true;
+  const long long t0 = clock64();
+  while (true) {
+    v = ld_relaxed_v4(p);
+    if ((v.x & v.y & v.z & v.w & 1u) != 0u) return true;
+    if (clock64() - t0 > kWaitCycles) return false;
+  }
 }
 
-// Bounded grid barrier on a monotonically increasing counter (release on arrival, acquire
-// while polling).  The outcome is uniform over the CTA: false means this CTA gave up and
-// recorded DOMINO_ERR_TIMEOUT.
-__device__ bool grid_barrier(unsigned* counter, unsigned target, int* status, volatile int* flag) {
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    red_release_add(counter, 1u);
-    int ok = 1;
-    const long long t0 = clock64();
-    while (ld_acquire_u32(counter) < target) {
-      if (clock64() - t0 > kWaitCycles) {
-        set_status(status, kStatusTimeout);
-        ok = 0;
-        break;
-      }
-    }
-    *flag = ok;
-  }
-  __syncthreads();
-  return *flag != 0;
+__device__ __forceinline__ uint32_t tagged(float h) {
+  const uint32_t b = static_cast<uint32_t>(__bfloat16_as_ushort(__float2bfloat16_rn(h)));
+  return (b << 16) | 1u;
+}
+
+// two tagged words -> packed bf16x2 (low element first)
+__device__ __forceinline__ uint32_t pack_hi_halves(uint32_t lo_word, uint32_t hi_word) {
+  return (lo_word >> 16) | (hi_word & 0xFFFF0000u);
 }
 
 __device__ __forceinline__ void cp_async16(void* smem_dst, const void* gmem_src) {
@@ -72,21 +81,23 @@ __device__ __forceinline__ void cp_async_wait_all() {
   asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
 }
 
-__device__ __forceinline__ float dot8_bf16(const uint4 w, const float4 h0, const float4 h1) {
-  const __nv_bfloat162* w2 = reinterpret_cast<const __nv_bfloat162*>(&w);
-  const float2 a = __bfloat1622float2(w2[0]);
-  const float2 b = __bfloat1622float2(w2[1]);
-  const float2 c = __bfloat1622float2(w2[2]);
-  const float2 d = __bfloat1622float2(w2[3]);
-  float s = a.x * h0.x;
-  s = fmaf(a.y, h0.y, s);
-  s = fmaf(b.x, h0.z, s);
-  s = fmaf(b.y, h0.w, s);
-  s = fmaf(c.x, h1.x, s);
-  s = fmaf(c.y, h1.y, s);
-  s = fmaf(d.x, h1.z, s);
-  s = fmaf(d.y, h1.w, s);
-  return s;
+__device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], const void* p) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(smem_u32(p)));
+}
+
+__device__ __forceinline__ void ldmatrix_x2(uint32_t (&r)[2], const void* p) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0,%1}, [%2];" : "=r"(r[0]), "=r"(r[1]) : "r"(smem_u32(p)));
+}
+
+// D (16x8, f32) += A (16x16 bf16, row-major) * B (16x8 bf16, column-major)
+__device__ __forceinline__ void mma_16816(float (&c)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
 }
 
 __device__ __forceinline__ float warp_sum(float v) {
@@ -99,137 +110,295 @@ __device__ __forceinline__ float bf_or0(const __nv_bfloat16* p, int i) {
   return p ? __bfloat162float(p[i]) : 0.f;
 }
 
-// Shared-memory layout of one GRU CTA (U hidden units, M = B*K rows, BG staged sequences):
-//   whh [3][U][Ds] bf16 | xs [M][3][U] f32 (input-gate sums + b_ih) | bh [3][U] f32 (b_hh)
-//   | hs [BG][Ds] f32 (h_{t-1}) | gs [BG][3][U] f32 (W_hh . h_{t-1}) | flag
+__device__ __forceinline__ float sigmoidf_(float x) { return 1.f / (1.f + expf(-x)); }
+
+// ---------------------------------------------------------------------------- smem layout
+// whh   [mt*16 rows][Ds + 8] bf16  this CTA's W_hh rows (gate g, unit jl) at row g*U + jl;
+//                                  rows past 3U are zero
+// hsm   [chunk][Ds + 8] bf16       h_{t-1} of up to 32 sequences (the MMA's n operand)
+// gsm   [mt*16][32] f32            W_hh . h_{t-1}
+// red   [16 tasks][16][8] f32      k-split partial tiles
+// hprev [bc][U] f32                this CTA's own previous states (fp32)
 struct GruSmem {
-  size_t whh, xs, bh, hs, gs, flag, total;
+  size_t whh, hsm, gsm, red, hprev, total;
+  int ldw, mt, chunk;
 };
 
-__host__ __device__ inline GruSmem gru_layout(int Ds, int U, int M, int BG) {
+__host__ __device__ inline GruSmem gru_layout(int Ds, int U, int bc) {
   GruSmem L;
+  L.ldw = Ds + 8;
+  L.mt = (3 * U + 15) / 16;
+  L.chunk = ((bc < kChunkSeqs ? bc : kChunkSeqs) + 7) / 8 * 8;  // staged sequences, whole n-tiles
   size_t o = 0;
-  L.whh = o; o += static_cast<size_t>(3) * U * Ds * 2;
-  L.xs = o;  o += static_cast<size_t>(M) * 3 * U * 4;
-  L.bh = o;  o += static_cast<size_t>(3) * U * 4;
-  o = (o + 15) & ~static_cast<size_t>(15);
-  L.hs = o;  o += static_cast<size_t>(BG) * Ds * 4;
-  L.gs = o;  o += static_cast<size_t>(BG) * 3 * U * 4;
-  L.flag = o; o += 16;
-  L.total = o;
+  L.whh = o;
+  o += static_cast<size_t>(L.mt) * 16 * L.ldw * 2;
+  L.hsm = o;
+  o += static_cast<size_t>(L.chunk) * L.ldw * 2;
+  L.gsm = o;
+  o += static_cast<size_t>(L.mt) * 16 * kChunkSeqs * 4;
+  L.red = o;
+  o += static_cast<size_t>(2 * kGruWarps) * 16 * 8 * 4;
+  L.hprev = o;
+  o += static_cast<size_t>(bc) * U * 4;
+  L.total = (o + 15) & ~static_cast<size_t>(15);
   return L;
 }
 
-__global__ void __launch_bounds__(kGruThreads) gru_kernel(const GruParams p, const int BG) {
-  extern __shared__ __align__(16) uint8_t gsm[];
+__global__ void __launch_bounds__(kGruThreads) gru_kernel(const GruParams p) {
+  extern __shared__ __align__(16) uint8_t gsmem[];
   const int U = p.units, Ds = p.Ds, K = p.K, B = p.B, R = p.R, H = p.H;
   const int M = B * K;
-  const int j0 = blockIdx.x * U;
-  const int Uc = min(U, Ds - j0);
-  const GruSmem L = gru_layout(Ds, U, M, BG);
-  __nv_bfloat16* whh = reinterpret_cast<__nv_bfloat16*>(gsm + L.whh);
-  float* xs = reinterpret_cast<float*>(gsm + L.xs);
-  float* bh = reinterpret_cast<float*>(gsm + L.bh);
-  float* hs = reinterpret_cast<float*>(gsm + L.hs);
-  float* gs = reinterpret_cast<float*>(gsm + L.gs);
-  volatile int* flag = reinterpret_cast<volatile int*>(gsm + L.flag);
+  const int cu = blockIdx.x % p.gu, cb = blockIdx.x / p.gu;
+  const int j0 = cu * U;
+  const int Uc = max(0, min(U, Ds - j0));
+  const int b0 = cb * p.bc;
+  const int nbc = max(0, min(p.bc, B - b0));  // sequences of this CTA
+  const GruSmem L = gru_layout(Ds, U, p.bc);
+  __nv_bfloat16* whh = reinterpret_cast<__nv_bfloat16*>(gsmem + L.whh);
+  __nv_bfloat16* hsm = reinterpret_cast<__nv_bfloat16*>(gsmem + L.hsm);
+  float* gsm = reinterpret_cast<float*>(gsmem + L.gsm);
+  float* red = reinterpret_cast<float*>(gsmem + L.red);
+  float* hprev = reinterpret_cast<float*>(gsmem + L.hprev);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  constexpr int kWarps = kGruThreads / 32;
+  const int ldw = L.ldw;
+  // the vocabulary GEMM that follows may start now: its first K segment does not read
+  // anything this kernel writes, and it waits for this grid before reading u
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
-  // this CTA's rows of W_hh (gate g, unit j0 + jl), copied asynchronously
+  // ---- W_hh rows of this CTA's units (asynchronous); zero rows past 3U and the state tile
   const int rowlen8 = Ds / 8;
   for (int e = tid; e < 3 * Uc * rowlen8; e += kGruThreads) {
-    const int c8 = e % rowlen8;
-    const int r = e / rowlen8;
+    const int c8 = e % rowlen8, r = e / rowlen8;
     const int g = r / Uc, jl = r % Uc;
-    cp_async16(whh + (static_cast<size_t>(g) * U + jl) * Ds + c8 * 8,
+    cp_async16(whh + static_cast<size_t>(g * U + jl) * ldw + c8 * 8,
                p.w_hh + (static_cast<size_t>(g) * Ds + j0 + jl) * Ds + c8 * 8);
   }
-  // input-gate sums for every row and this CTA's units: b_ih + sum over split-K partials
-  for (int e = tid; e < M * 3 * Uc; e += kGruThreads) {
-    const int jl = e % Uc;
-    const int g = (e / Uc) % 3;
-    const int m = e / (3 * Uc);
-    const int col = g * Ds + j0 + jl;
-    float a = bf_or0(p.b_ih, col);
-    for (int s = 0; s < p.xsplits; ++s) a += __ldg(p.xpart + (static_cast<size_t>(s) * M + m) * 3 * Ds + col);
-    xs[(static_cast<size_t>(m) * 3 + g) * U + jl] = a;
+  for (int e = tid; e < L.mt * 16 * (ldw / 8); e += kGruThreads) {
+    const int r = e / (ldw / 8);
+    const int jl = r % U;
+    if (r >= 3 * U || jl >= Uc) reinterpret_cast<uint4*>(whh)[e] = make_uint4(0, 0, 0, 0);
   }
-  for (int e = tid; e < 3 * Uc; e += kGruThreads) bh[(e / Uc) * U + e % Uc] = bf_or0(p.b_hh, (e / Uc) * Ds + j0 + e % Uc);
+  for (int r = tid; r < L.mt * 16; r += kGruThreads)  // padding columns Ds .. Ds+7 (k tail)
+    *reinterpret_cast<uint4*>(whh + static_cast<size_t>(r) * ldw + Ds) = make_uint4(0, 0, 0, 0);
+  for (int e = tid; e < L.chunk * (ldw / 8); e += kGruThreads) reinterpret_cast<uint4*>(hsm)[e] = make_uint4(0, 0, 0, 0);
+  // ---- input-gate sums b_ih + E . W_ih^T for this CTA's rows and units, spread over all
+  //      threads (made visible to the CTA by the barrier below)
+  const int xs_count = nbc * K * 3 * Uc;
+  for (int e0 = tid; e0 < xs_count; e0 += 4 * kGruThreads) {
+    float a[4];
+    size_t at[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int e = e0 + i * kGruThreads;
+      a[i] = 0.f;
+      at[i] = 0;
+      if (e < xs_count) {
+        const int jl = e % Uc, g = (e / Uc) % 3, bt = e / (3 * Uc);
+        const int col = g * Ds + j0 + jl;
+        const size_t m = static_cast<size_t>(b0) * K + bt;
+        at[i] = m * 3 * Ds + col;
+        a[i] = bf_or0(p.b_ih, col);
+      }
+    }
+    for (int s = 0; s < p.xsplits; ++s) {
+      const float* base = p.xpart + static_cast<size_t>(s) * M * 3 * Ds;
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (e0 + i * kGruThreads < xs_count) a[i] += __ldg(base + at[i]);
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      if (e0 + i * kGruThreads < xs_count) p.xs[at[i]] = a[i];
+  }
+  for (int e = tid; e < nbc * U; e += kGruThreads) hprev[e] = 0.f;
   cp_async_wait_all();
   __syncthreads();
 
-  for (int t = 0; t < K; ++t) {
-    for (int b0 = 0; b0 < B; b0 += BG) {
-      const int nb = min(BG, B - b0);
+  const int nk = (Ds + 15) / 16;  // a k tail of 8 reads the zero padding columns
+  bool ok = true;
+
+  for (int t = 0; t < K && ok; ++t) {
+    for (int c0 = 0; c0 < nbc; c0 += L.chunk) {
+      const int nb = min(L.chunk, nbc - c0);
+      const int nt_count = (nb + 7) / 8;
+      const int tiles = L.mt * nt_count;
+      int ks = 1;  // k-slices per tile, so that up to 16 warp tasks (two per warp) exist
+      while (tiles * ks * 2 <= 2 * kGruWarps && ks * 2 <= nk) ks *= 2;
       if (t > 0) {
-        // h_{t-1} of sequences b0 .. b0+nb-1 (written by every CTA in step t-1)
-        for (int e = tid; e < nb * (Ds / 4); e += kGruThreads) {
-          const int bb = e / (Ds / 4), c4 = e % (Ds / 4);
-          reinterpret_cast<float4*>(hs + static_cast<size_t>(bb) * Ds)[c4] = __ldcg(
-              reinterpret_cast<const float4*>(p.S + (static_cast<size_t>(b0 + bb) * K + (t - 1)) * Ds) + c4);
-        }
-        __syncthreads();
-        // W_hh[rows of this CTA] . h_{t-1}
-        for (int d = warp; d < 3 * Uc * nb; d += kWarps) {
-          const int r = d % (3 * Uc), bb = d / (3 * Uc);
-          const int g = r / Uc, jl = r % Uc;
-          const __nv_bfloat16* wrow = whh + (static_cast<size_t>(g) * U + jl) * Ds;
-          const float* hrow = hs + static_cast<size_t>(bb) * Ds;
-          float acc = 0.f;
-          for (int c = lane * 8; c < Ds; c += 256) {
-            const uint4 wv = *reinterpret_cast<const uint4*>(wrow + c);
-            const float4 h0 = *reinterpret_cast<const float4*>(hrow + c);
-            const float4 h1 = *reinterpret_cast<const float4*>(hrow + c + 4);
-            acc += dot8_bf16(wv, h0, h1);
+        // ---- h_{t-1} of this chunk's sequences, polled from the tagged rows
+        const int per_row = Ds / 4;
+        const int total = nb * per_row;
+        bool got = true;
+        for (int e0 = tid; e0 < total && got; e0 += 8 * kGruThreads) {
+          uint4 v[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {  // issue every load first, then check the flags
+            const int e = e0 + i * kGruThreads;
+            if (e < total) {
+              const size_t m = static_cast<size_t>(b0 + c0 + e / per_row) * K + (t - 1);
+              v[i] = ld_relaxed_v4(p.hx + m * Ds + (e % per_row) * 4);
+            }
           }
-          acc = warp_sum(acc);
-          if (lane == 0) gs[(bb * 3 + g) * U + jl] = acc;
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int e = e0 + i * kGruThreads;
+            if (e < total && got) {
+              const int bb = e / per_row, c4 = e % per_row;
+              if ((v[i].x & v[i].y & v[i].z & v[i].w & 1u) == 0u) {
+                const size_t m = static_cast<size_t>(b0 + c0 + bb) * K + (t - 1);
+                got = poll_v4(p.hx + m * Ds + c4 * 4, v[i]);
+              }
+              *reinterpret_cast<uint2*>(hsm + static_cast<size_t>(bb) * ldw + c4 * 4) =
+                  make_uint2(pack_hi_halves(v[i].x, v[i].y), pack_hi_halves(v[i].z, v[i].w));
+            }
+          }
+        }
+        if (__syncthreads_or(!got)) {
+          set_status(p.status, kStatusTimeout);
+          ok = false;
+          break;
+        }
+        // ---- g = W_hh[rows] . h_{t-1} on the tensor cores
+        // each warp takes two tasks at a time: two independent accumulator chains
+        const int ntasks = tiles * ks;
+        for (int tp = warp; tp < ntasks; tp += 2 * kGruWarps) {
+          const int tb = tp + kGruWarps;
+          const bool two = tb < ntasks;
+          const int tileA = tp % tiles, kslA = tp / tiles;
+          const int tileB = two ? tb % tiles : tileA, kslB = two ? tb / tiles : kslA;
+          const int kbA = kslA * (nk / ks), keA = (kslA == ks - 1) ? nk : kbA + nk / ks;
+          const int kbB = kslB * (nk / ks), keB = (kslB == ks - 1) ? nk : kbB + nk / ks;
+          float accA[4] = {0.f, 0.f, 0.f, 0.f}, accB[4] = {0.f, 0.f, 0.f, 0.f};
+          const __nv_bfloat16* arowA =
+              whh + static_cast<size_t>((tileA % L.mt) * 16 + (lane & 15)) * ldw + (lane >> 4) * 8;
+          const __nv_bfloat16* browA =
+              hsm + static_cast<size_t>((tileA / L.mt) * 8 + (lane & 7)) * ldw + ((lane >> 3) & 1) * 8;
+          const __nv_bfloat16* arowB =
+              whh + static_cast<size_t>((tileB % L.mt) * 16 + (lane & 15)) * ldw + (lane >> 4) * 8;
+          const __nv_bfloat16* browB =
+              hsm + static_cast<size_t>((tileB / L.mt) * 8 + (lane & 7)) * ldw + ((lane >> 3) & 1) * 8;
+          const int steps = max(keA - kbA, two ? keB - kbB : 0);
+          for (int i = 0; i < steps; ++i) {
+            if (kbA + i < keA) {
+              uint32_t a[4], b[2];
+              ldmatrix_x4(a, arowA + (kbA + i) * 16);
+              ldmatrix_x2(b, browA + (kbA + i) * 16);
+              mma_16816(accA, a, b);
+            }
+            if (two && kbB + i < keB) {
+              uint32_t a[4], b[2];
+              ldmatrix_x4(a, arowB + (kbB + i) * 16);
+              ldmatrix_x2(b, browB + (kbB + i) * 16);
+              mma_16816(accB, a, b);
+            }
+          }
+          const int g = lane >> 2, tq = lane & 3;
+          for (int w = 0; w < (two ? 2 : 1); ++w) {
+            const int task = w ? tb : tp;
+            const int tile = task % tiles;
+            const float* acc = w ? accB : accA;
+            float* out;
+            int ld;
+            if (ks == 1) {
+              out = gsm + static_cast<size_t>((tile % L.mt) * 16) * kChunkSeqs + (tile / L.mt) * 8;
+              ld = kChunkSeqs;
+            } else {
+              out = red + static_cast<size_t>(task) * 128;
+              ld = 8;
+            }
+            out[g * ld + 2 * tq] = acc[0];
+            out[g * ld + 2 * tq + 1] = acc[1];
+            out[(g + 8) * ld + 2 * tq] = acc[2];
+            out[(g + 8) * ld + 2 * tq + 1] = acc[3];
+          }
         }
         __syncthreads();
+        if (ks > 1) {
+          for (int e = tid; e < tiles * 128; e += kGruThreads) {
+            const int tile = e / 128, w = e % 128;
+            float s = 0.f;
+            for (int ksl = 0; ksl < ks; ++ksl) s += red[static_cast<size_t>(ksl * tiles + tile) * 128 + w];
+            const int mt = tile % L.mt, nt = tile / L.mt;
+            gsm[static_cast<size_t>(mt * 16 + w / 8) * kChunkSeqs + nt * 8 + (w % 8)] = s;
+          }
+          __syncthreads();
+        }
       }
-      // gates and the new state (torch.nn.GRU convention)
+      // ---- gates and the new state (torch.nn.GRU convention); publish the tagged state
       for (int e = tid; e < nb * Uc; e += kGruThreads) {
         const int bb = e / Uc, jl = e % Uc;
         const int j = j0 + jl;
-        const int m = (b0 + bb) * K + t;
-        const float* x = xs + static_cast<size_t>(m) * 3 * U;
-        float hr = bh[jl], hz = bh[U + jl], hn = bh[2 * U + jl];
-        float hprev = 0.f;
+        const int bl = c0 + bb;  // sequence index within this CTA
+        const size_t m = static_cast<size_t>(b0 + bl) * K + t;
+        const float* x = p.xs + m * 3 * Ds;
+        float hr = bf_or0(p.b_hh, j), hz = bf_or0(p.b_hh, Ds + j), hn = bf_or0(p.b_hh, 2 * Ds + j);
         if (t > 0) {
-          hr += gs[(bb * 3 + 0) * U + jl];
-          hz += gs[(bb * 3 + 1) * U + jl];
-          hn += gs[(bb * 3 + 2) * U + jl];
-          hprev = hs[static_cast<size_t>(bb) * Ds + j];
+          hr += gsm[static_cast<size_t>(jl) * kChunkSeqs + bb];
+          hz += gsm[static_cast<size_t>(U + jl) * kChunkSeqs + bb];
+          hn += gsm[static_cast<size_t>(2 * U + jl) * kChunkSeqs + bb];
         }
-        const float r = 1.f / (1.f + expf(-(x[jl] + hr)));
-        const float z = 1.f / (1.f + expf(-(x[U + jl] + hz)));
-        const float n = tanhf(x[2 * U + jl] + r * hn);
-        p.S[static_cast<size_t>(m) * Ds + j] = (1.f - z) * n + z * hprev;
+        const float hp = hprev[bl * U + jl];
+        const float r = sigmoidf_(x[j] + hr);
+        const float z = sigmoidf_(x[Ds + j] + hz);
+        const float n = tanhf(x[2 * Ds + j] + r * hn);
+        const float h = (1.f - z) * n + z * hp;
+        hprev[bl * U + jl] = h;
+        p.hx[m * Ds + j] = tagged(h);
+        if (p.s_out) p.s_out[m * Ds + j] = __float2bfloat16_rn(h);
       }
       __syncthreads();
     }
-    if (!grid_barrier(p.barrier, static_cast<unsigned>(gridDim.x) * (t + 1), p.status, flag)) return;
   }
+  if (!ok || p.u == nullptr) return;
 
-  // u[m, q] = SiLU(b1[q] + hidden_m . W1[q, :H] + S_m . W1[q, H:])
-  const int total_warps = gridDim.x * kWarps;
-  const int gw = blockIdx.x * kWarps + warp;
+  // ---- u[m, q] = SiLU(b1[q] + hidden_m . W1[q, :H] + S_m . W1[q, H:]) (small batches): the
+  //      hidden half arrives as split-K partial sums, the state half is a warp dot over the
+  //      tagged states (polled: other CTAs may still be publishing their last step)
+  const int total_warps = gridDim.x * kGruWarps;
+  const int gw = blockIdx.x * kGruWarps + warp;
   const int groups = max(1, total_warps / R);
   for (int pi = gw; pi < R * groups; pi += total_warps) {
     const int q = pi % R, mg = pi / R;
     const __nv_bfloat16* w1row = p.w1 + static_cast<size_t>(q) * (H + Ds) + H;
     const float bq = bf_or0(p.b1, q);
     for (int m = mg; m < M; m += groups) {
-      const float* srow = p.S + static_cast<size_t>(m) * Ds;
+      const uint32_t* srow = p.hx + static_cast<size_t>(m) * Ds;
       float acc = 0.f;
-      for (int c = lane * 8; c < Ds; c += 256) {
-        const uint4 wv = __ldg(reinterpret_cast<const uint4*>(w1row + c));
-        const float4 h0 = __ldcg(reinterpret_cast<const float4*>(srow + c));
-        const float4 h1 = __ldcg(reinterpret_cast<const float4*>(srow + c + 4));
-        acc += dot8_bf16(wv, h0, h1);
+      bool got = true;
+      for (int c0 = lane * 8; c0 < Ds && got; c0 += 4 * 256) {
+        uint4 wv[4], sv[8];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {  // issue every load of this slice first
+          const int c = c0 + i * 256;
+          if (c < Ds) {
+            wv[i] = __ldg(reinterpret_cast<const uint4*>(w1row + c));
+            sv[2 * i] = ld_relaxed_v4(srow + c);
+            sv[2 * i + 1] = ld_relaxed_v4(srow + c + 4);
+          }
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int c = c0 + i * 256;
+          if (c >= Ds || !got) continue;
+          for (int h = 0; h < 2; ++h) {
+            uint4& x = sv[2 * i + h];
+            if ((x.x & x.y & x.z & x.w & 1u) == 0u) got = got && poll_v4(srow + c + 4 * h, x);
+          }
+          const __nv_bfloat162* w2 = reinterpret_cast<const __nv_bfloat162*>(&wv[i]);
+          const uint32_t sw[8] = {sv[2 * i].x, sv[2 * i].y, sv[2 * i].z, sv[2 * i].w,
+                                  sv[2 * i + 1].x, sv[2 * i + 1].y, sv[2 * i + 1].z, sv[2 * i + 1].w};
+#pragma unroll
+          for (int q2 = 0; q2 < 4; ++q2) {
+            const float2 wf = __bfloat1622float2(w2[q2]);
+            acc = fmaf(wf.x, __uint_as_float(sw[2 * q2] & 0xFFFF0000u), acc);
+            acc = fmaf(wf.y, __uint_as_float(sw[2 * q2 + 1] & 0xFFFF0000u), acc);
+          }
+        }
       }
-      // the hidden half arrives as split-K partial sums; the lanes add them in parallel
+      if (__any_sync(0xffffffffu, !got)) {
+        if (lane == 0) set_status(p.status, kStatusTimeout);
+        return;
+      }
       for (int s = lane; s < p.usplits; s += 32) acc += __ldg(p.upart + (static_cast<size_t>(s) * M + m) * R + q);
       acc = warp_sum(acc);
       if (lane == 0) {
@@ -240,49 +409,61 @@ __global__ void __launch_bounds__(kGruThreads) gru_kernel(const GruParams p, con
   }
 }
 
-int gru_grid(int Ds, int num_sms, int* units) {
-  int G = Ds < 128 ? Ds : 128;
-  if (G > num_sms) G = num_sms;
-  int U = (Ds + G - 1) / G;
-  if (static_cast<size_t>(3) * U * Ds * 2 > 160 * 1024) {
-    G = Ds < num_sms ? Ds : num_sms;
-    U = (Ds + G - 1) / G;
+GruPlan gru_plan(int B, int Ds, int num_sms) {
+  GruPlan g{};
+  if (B <= 8) {
+    g.gu = Ds < 128 ? Ds : 128;
+    g.gb = 1;
+  } else {
+    g.gu = Ds < 64 ? Ds : 64;
+    g.gb = 2;
   }
-  G = (Ds + U - 1) / U;
-  *units = U;
-  return G;
+  while (g.gu * g.gb > num_sms && g.gu > 1) g.gu /= 2;
+  g.units = (Ds + g.gu - 1) / g.gu;
+  g.gu = (Ds + g.units - 1) / g.units;
+  g.bc = (B + g.gb - 1) / g.gb;
+  g.gb = (B + g.bc - 1) / g.bc;
+  const GruSmem L = gru_layout(Ds, g.units, g.bc);
+  g.smem = L.total <= 220 * 1024 ? L.total : 0;
+  return g;
 }
 
-static constexpr size_t kGruSmemBudget = 220 * 1024;
-
-static int gru_bg(int Ds, int U, int M, int B) {
-  int bg = B < 8 ? B : 8;
-  while (bg > 1 && gru_layout(Ds, U, M, bg).total > kGruSmemBudget) --bg;
-  return gru_layout(Ds, U, M, bg).total > kGruSmemBudget ? 0 : bg;
-}
-
-size_t gru_smem_bytes(int Ds, int units, int M, int B) {
-  const int bg = gru_bg(Ds, units, M, B);
-  return bg == 0 ? 0 : gru_layout(Ds, units, M, bg).total;
-}
-
-cudaError_t launch_gru(const GruParams& p, int grid, cudaStream_t stream) {
-  const int M = p.B * p.K;
-  const int bg = gru_bg(p.Ds, p.units, M, p.B);
-  if (bg == 0) return cudaErrorInvalidValue;
-  const size_t smem = gru_layout(p.Ds, p.units, M, bg).total;
+cudaError_t launch_gru(const GruParams& p, const GruPlan& plan, cudaStream_t stream) {
+  if (plan.smem == 0) return cudaErrorInvalidValue;
   static size_t attr_smem = 0;
-  if (smem > attr_smem) {
-    cudaError_t e = cudaFuncSetAttribute(gru_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (plan.smem > attr_smem) {
+    cudaError_t e = cudaFuncSetAttribute(gru_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(plan.smem));
     if (e != cudaSuccess) return e;
-    attr_smem = smem;
+    e = cudaFuncSetAttribute(gru_kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    if (e != cudaSuccess) return e;
+    attr_smem = plan.smem;
   }
   GruParams pp = p;
-  int bgv = bg;
-  void* args[] = {&pp, &bgv};
-  cudaError_t e = cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(gru_kernel), dim3(grid),
-                                              dim3(kGruThreads), args, smem, stream);
+  void* args[] = {&pp};
+  cudaError_t e = cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(gru_kernel),
+                                              dim3(plan.gu * plan.gb), dim3(kGruThreads), args, plan.smem, stream);
   if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------- u finalize
+__global__ void __launch_bounds__(256) u_finalize_kernel(const UFinalParams p) {
+  const size_t n = static_cast<size_t>(p.M) * p.R;
+  for (size_t e = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < n;
+       e += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const int q = static_cast<int>(e % p.R);
+    float a = bf_or0(p.b1, q);
+    for (int s = 0; s < p.splits; ++s) a += __ldg(p.part + static_cast<size_t>(s) * n + e);
+    p.u[e] = __float2bfloat16_rn(a / (1.f + expf(-a)));
+  }
+}
+
+cudaError_t launch_u_finalize(const UFinalParams& p, cudaStream_t stream) {
+  const size_t n = static_cast<size_t>(p.M) * p.R;
+  const size_t want = (n + 255) / 256;
+  const int blocks = static_cast<int>(want < 1024 ? want : 1024);
+  u_finalize_kernel<<<blocks, 256, 0, stream>>>(p);
   return cudaGetLastError();
 }
 

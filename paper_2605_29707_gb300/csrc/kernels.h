@@ -27,6 +27,9 @@ struct TcParams {
   // store mode: items (tok tile, w tile, split) round-robin over the CTAs
   int splits, kb_per_split, total_items;
   int w_evict_first;
+  int defer;      // softmax + swap only: first segment of every tile, then griddepcontrol.wait,
+                  // then the second segment (each tile keeps its own TMEM accumulator)
+  int tmem_cols;  // TMEM columns to allocate (power of two, 32..512)
   const __nv_bfloat16* bias;  // softmax: b2 [V] or nullptr
   float* out;                 // softmax: partial records [M][rec fields][nchunks]; store: [splits][M][ld_out]
   int ld_out;
@@ -38,21 +41,32 @@ constexpr int kSoftmaxRecWords(int kmax) { return 2 + 2 * kmax; }
 // Tensor maps in the order A1, B1, A2, B2 (A = 128-row operand, B = N-row operand).
 cudaError_t launch_tc_gemm(int mode, int bn, bool swap, int kmax, const CUtensorMap* maps,
                            const TcParams& p, int grid, cudaStream_t stream);
+// Deferred-segment vocabulary GEMM launched as a programmatic dependent of the GRU kernel
+// (bn 16 or 32; fewer pipeline stages so that its CTAs fit beside the GRU's on one SM).
+cudaError_t launch_tc_softmax_deferred(int bn, int kmax, const CUtensorMap* maps, const TcParams& p, int grid,
+                                       cudaStream_t stream);
+// Shared memory one deferred-mode CTA uses (for the co-residency budget).
+int tc_softmax_deferred_smem(int bn);
 
 // ---------------------------------------------------------------- gather / GRU
 struct GatherParams {
   const int32_t* ids;       // [M]
   const __nv_bfloat16* emb; // [V, H]
   __nv_bfloat16* E;         // [M, H] or nullptr (validate only)
-  int M, H, V;
+  uint32_t* hx;             // [M, Ds] tagged GRU states to clear, or nullptr
+  int M, H, V, Ds;
   int* status;
 };
 cudaError_t launch_gather(const GatherParams& p, cudaStream_t stream);
 
+// GRU recurrence.  CTA (cu, cb) of a gu x gb grid owns hidden units [cu*units, cu*units+units)
+// (gate rows r|z|n of each) for sequences [cb*bc, cb*bc+bc).  States travel between CTAs as
+// tagged words in hx: bf16 value in the high half, a non-zero flag in the low half, one row
+// per (sequence, position) written once per step, so a reader polls the data itself.
 struct GruParams {
   const float* xpart;  // [xsplits][M][3*Ds]  partial sums of E . W_ih^T
   int xsplits;
-  const float* upart;  // [usplits][M][R]     partial sums of hidden . W1[:, :H]^T
+  const float* upart;  // [usplits][M][R]     partial sums of hidden . W1[:, :H]^T (u phase only)
   int usplits;
   const __nv_bfloat16* w_hh;  // [3*Ds, Ds]
   const __nv_bfloat16* b_ih;  // [3*Ds] or nullptr
@@ -60,15 +74,28 @@ struct GruParams {
   const __nv_bfloat16* w1;    // [R, H + Ds]
   const __nv_bfloat16* b1;    // [R] or nullptr
   int B, K, H, Ds, R;
-  int units;                  // hidden units owned by one CTA
-  float* S;                   // [M][Ds] causal states (fp32)
-  __nv_bfloat16* u;           // [M][R] low-rank code
-  unsigned int* barrier;      // zeroed grid-barrier counter
+  int units, gu, gb, bc;      // grid shape: gu unit blocks x gb sequence groups of bc
+  float* xs;                  // [M][3*Ds] input-gate sums (scratch)
+  uint32_t* hx;               // [M][Ds] tagged states (cleared by the gather kernel)
+  __nv_bfloat16* s_out;       // [M][Ds] plain bf16 states, or nullptr
+  __nv_bfloat16* u;           // [M][R] low-rank code computed in-kernel, or nullptr
   int* status;
 };
-int gru_grid(int Ds, int num_sms, int* units);
-size_t gru_smem_bytes(int Ds, int units, int M, int B);  // 0 = does not fit
-cudaError_t launch_gru(const GruParams& p, int grid, cudaStream_t stream);
+struct GruPlan {
+  int units, gu, gb, bc;
+  size_t smem;  // 0 = unsupported
+};
+GruPlan gru_plan(int B, int Ds, int num_sms);
+cudaError_t launch_gru(const GruParams& p, const GruPlan& plan, cudaStream_t stream);
+
+// u = bf16(SiLU(b1 + sum over splits of part)) for the large-batch path.
+struct UFinalParams {
+  const float* part;  // [splits][M][R]
+  int splits, M, R;
+  const __nv_bfloat16* b1;
+  __nv_bfloat16* u;
+};
+cudaError_t launch_u_finalize(const UFinalParams& p, cudaStream_t stream);
 
 // ---------------------------------------------------------------- merge + tree
 struct TreeParams {

@@ -20,7 +20,7 @@
 
 namespace dm {
 
-template <int BN, bool SWAP, int MODE, int KMAX>
+template <int BN, bool SWAP, int MODE, int KMAX, int ST = 0>
 struct TcCfg {
   static constexpr int kABytes = 128 * 128;  // 128 rows x 64 bf16
   static constexpr int kBBytes = BN * 128;   // BN rows x 64 bf16
@@ -30,7 +30,7 @@ struct TcCfg {
   static constexpr int kTrBytes = (SWAP && MODE == kModeSoftmax) ? BN * kTrStride * 4 : 0;
   static constexpr int kBudget = 200 * 1024;
   static constexpr int kSt0 = (kBudget - kTrBytes) / kStageBytes;
-  static constexpr int kStages = kSt0 > 8 ? 8 : kSt0;
+  static constexpr int kStages = ST > 0 ? ST : (kSt0 > 8 ? 8 : kSt0);
   static constexpr int kTmemCols =
       (2 * BN <= 32) ? 32 : (2 * BN <= 64) ? 64 : (2 * BN <= 128) ? 128 : (2 * BN <= 256) ? 256 : 512;
   static constexpr int kBarBytes = 256;
@@ -175,12 +175,12 @@ __device__ __forceinline__ bool epi_any(bool pred) {
   return r != 0;
 }
 
-template <int BN, bool SWAP, int MODE, int KMAX>
+template <int BN, bool SWAP, int MODE, int KMAX, int ST>
 __global__ void __launch_bounds__(192, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
                    const __grid_constant__ CUtensorMap tmA2, const __grid_constant__ CUtensorMap tmB2,
                    const TcParams p) {
-  using C = TcCfg<BN, SWAP, MODE, KMAX>;
+  using C = TcCfg<BN, SWAP, MODE, KMAX, ST>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -221,7 +221,7 @@ __global__ void __launch_bounds__(192, 1)
     }
   }
   if (warp == 1) {
-    tmem_alloc(tmem_slot, C::kTmemCols);
+    tmem_alloc(tmem_slot, static_cast<uint32_t>(p.tmem_cols));
     tmem_relinquish();
   }
   tc_fence_before();
@@ -241,8 +241,16 @@ __global__ void __launch_bounds__(192, 1)
       int issued = 0;
       bool ok = true;
       TcItem it;
+      // Deferred mode streams the first K segment of every tile first; the second segment's
+      // activations (u) come from the preceding kernel, so they are loaded only after
+      // griddepcontrol.wait (the hardware's wait for the preceding grid to complete).
+      const int passes = p.defer ? 2 : 1;
+      for (int pass = 0; pass < passes && ok; ++pass) {
+      if (pass == 1) asm volatile("griddepcontrol.wait;" ::: "memory");
       for (int i = 0; ok && tc_get_item<MODE>(p, i, it); ++i) {
-        for (int kb = it.kb0; kb < it.kb1; ++kb) {
+        const int kb_lo = (p.defer && pass == 1) ? p.nkb1 : it.kb0;
+        const int kb_hi = (p.defer && pass == 0) ? p.nkb1 : it.kb1;
+        for (int kb = kb_lo; kb < kb_hi; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, p.status)) { ok = false; break; }
           mbar_arrive_expect_tx(&full[stage], C::kStageBytes);
           const bool seg2 = kb >= p.nkb1;
@@ -254,6 +262,7 @@ __global__ void __launch_bounds__(192, 1)
           ++issued;
           if (++stage == C::kStages) { stage = 0; phase ^= 1u; }
         }
+      }
       }
       // Let every load this thread issued land before the CTA can exit (each is the last
       // one on its stage; a completed phase of that parity returns at once).
@@ -276,13 +285,22 @@ __global__ void __launch_bounds__(192, 1)
       uint32_t phase = 0;
       bool ok = true;
       TcItem it;
+      const int passes = p.defer ? 2 : 1;
+      for (int pass = 0; pass < passes && ok; ++pass) {
       for (int i = 0; ok && tc_get_item<MODE>(p, i, it); ++i) {
         const int ab = i & 1;
         const uint32_t aph = (i >> 1) & 1;
-        if (!mbar_wait(&tempty[ab], aph ^ 1u, abort_flag, p.status)) break;
-        tc_fence_after();
-        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(ab * BN);
-        for (int kb = it.kb0; kb < it.kb1; ++kb) {
+        const bool last_pass = pass == passes - 1;
+        // the accumulator of item i: one of two alternating buffers, or (deferred mode) its own
+        // column block, which holds the first segment until the second one is added
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>((p.defer ? i : ab) * BN);
+        if (last_pass) {
+          if (!mbar_wait(&tempty[ab], aph ^ 1u, abort_flag, p.status)) break;
+          tc_fence_after();
+        }
+        const int kb_lo = (p.defer && pass == 1) ? p.nkb1 : it.kb0;
+        const int kb_hi = (p.defer && pass == 0) ? p.nkb1 : it.kb1;
+        for (int kb = kb_lo; kb < kb_hi; ++kb) {
           if (!mbar_wait(&full[stage], phase, abort_flag, p.status)) { ok = false; break; }
           tc_fence_after();
           const uint64_t da = smem_desc_sw128(smem_u32(sA + stage * C::kABytes));
@@ -295,7 +313,8 @@ __global__ void __launch_bounds__(192, 1)
           tc_commit(&empty[stage]);
           if (++stage == C::kStages) { stage = 0; phase ^= 1u; }
         }
-        if (ok) tc_commit(&tfull[ab]);
+        if (ok && last_pass) tc_commit(&tfull[ab]);
+      }
       }
     }
   } else {
@@ -314,7 +333,7 @@ __global__ void __launch_bounds__(192, 1)
       const bool ok = mbar_wait(&tfull[ab], aph, abort_flag, p.status);
       if (epi_any(!ok)) { aborted = true; break; }
       tc_fence_after();
-      const uint32_t tcol = tmem_base + lane_off + static_cast<uint32_t>(ab * BN);
+      const uint32_t tcol = tmem_base + lane_off + static_cast<uint32_t>((p.defer ? i : ab) * BN);
 
       if constexpr (MODE == kModeStore) {
         if constexpr (SWAP) {
@@ -443,21 +462,35 @@ __global__ void __launch_bounds__(192, 1)
     }
     __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tmem_base, C::kTmemCols);
+    tmem_dealloc(tmem_base, static_cast<uint32_t>(p.tmem_cols));
   }
 }
 
-template <int BN, bool SWAP, int MODE, int KMAX>
-cudaError_t launch_tc_instance(const CUtensorMap* maps, const TcParams& p, int grid, cudaStream_t stream) {
-  using C = TcCfg<BN, SWAP, MODE, KMAX>;
-  auto kern = tc_gemm_kernel<BN, SWAP, MODE, KMAX>;
+template <int BN, bool SWAP, int MODE, int KMAX, int ST = 0>
+cudaError_t launch_tc_instance(const CUtensorMap* maps, const TcParams& p, int grid, cudaStream_t stream,
+                               bool pdl = false) {
+  using C = TcCfg<BN, SWAP, MODE, KMAX, ST>;
+  auto kern = tc_gemm_kernel<BN, SWAP, MODE, KMAX, ST>;
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
     if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  kern<<<grid, 192, C::kSmemBytes, stream>>>(maps[0], maps[1], maps[2], maps[3], p);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(192);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, kern, maps[0], maps[1], maps[2], maps[3], p);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

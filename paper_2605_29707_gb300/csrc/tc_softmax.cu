@@ -15,4 +15,21 @@ cudaError_t launch_tc_softmax(int bn, bool swap, int kmax, const CUtensorMap* ma
   return cudaErrorInvalidValue;
 }
 
+// Deferred variants: 6 stages (BN 16) / 5 stages (BN 32) keep a CTA near 118 KB of shared
+// memory so that it fits on an SM next to a GRU CTA.
+cudaError_t launch_tc_softmax_deferred(int bn, int kmax, const CUtensorMap* maps, const TcParams& p, int grid,
+                                       cudaStream_t s) {
+  if (bn == 16 && kmax == 16) return launch_tc_instance<16, true, kModeSoftmax, 16, 6>(maps, p, grid, s, true);
+  if (bn == 16 && kmax == 32) return launch_tc_instance<16, true, kModeSoftmax, 32, 6>(maps, p, grid, s, true);
+  if (bn == 32 && kmax == 16) return launch_tc_instance<32, true, kModeSoftmax, 16, 5>(maps, p, grid, s, true);
+  if (bn == 32 && kmax == 32) return launch_tc_instance<32, true, kModeSoftmax, 32, 5>(maps, p, grid, s, true);
+  return cudaErrorInvalidValue;
+}
+
+int tc_softmax_deferred_smem(int bn) {
+  if (bn == 16) return TcCfg<16, true, kModeSoftmax, 16, 6>::kSmemBytes;
+  if (bn == 32) return TcCfg<32, true, kModeSoftmax, 16, 5>::kSmemBytes;
+  return 0;
+}
+
 }  // namespace dm
