@@ -324,12 +324,11 @@ def run_ours(args):
     if rc != 0:
         raise binding.DominoError(rc, "warm-up device status")
 
-    # ---- timed region: exactly K steps, per-kernel events on the launching stream
+    # ---- timed region: exactly K steps, CUDA events on the launching stream
     sampler = ClockSampler(local)
     sampler.start()
     barrier()
     torch.cuda.synchronize(device)
-    binding.domino_timing_begin(args.steps * launches)
     ev0 = torch.cuda.Event(enable_timing=True)
     ev1 = torch.cuda.Event(enable_timing=True)
     ev0.record(stream)
@@ -339,7 +338,6 @@ def run_ours(args):
     ev1.record(stream)
     torch.cuda.synchronize(device)
     barrier()
-    kern = binding.domino_timing_end()
     clocks = sampler.stop()
     if bad:
         raise RuntimeError("a timed step returned an error")
@@ -347,6 +345,19 @@ def run_ours(args):
     if rc != 0:
         raise binding.DominoError(rc, "timed device status")
     ms = ev0.elapsed_time(ev1)
+
+    # ---- second timed region: the same steps with an event pair around every kernel (the
+    #      per-kernel breakdown and the roofline).  Events between launches serialise the
+    #      GRU / vocabulary-GEMM overlap, so the step value comes from the region above.
+    k_steps = min(args.steps, 1000)
+    torch.cuda.synchronize(device)
+    binding.domino_timing_begin(k_steps * launches)
+    for _ in range(k_steps):
+        bad |= st.enqueue(hidden, ids, stream) != 0
+    torch.cuda.synchronize(device)
+    kern = binding.domino_timing_end()
+    if bad:
+        raise RuntimeError("a step of the per-kernel region returned an error")
     if world > 1:
         t = torch.tensor([ms], dtype=torch.float64, device=device)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
@@ -393,10 +404,11 @@ def run_ours(args):
     roof.update({"kernel": "vocab_gemm_softmax_topk", "traffic": traffic,
                  "algorithmic_bytes_per_launch": vw["bytes"], "algorithmic_flops_per_launch": vw["flops"],
                  "mean_launch_us": round(vk_mean * 1e3, 2), "launches": vk_n, "traffic_note": traffic_note,
+                 "timing": f"CUDA events around each launch, {k_steps} steps right after the timed region",
                  "share_of_step": round(vk_ms / max(1e-9, sum(v[0] for v in kern.values())), 4)})
     sw = step_work(c)
     step_roof = max(sw["bytes"] / (peaks["hbm_gbs"] * 1e9), sw["flops"] / (peaks["bf16_tflops_sustained"] * 1e12))
-    breakdown = {n: {"us_per_step": round(v[0] / args.steps * 1e3, 2), "launches": v[1]} for n, v in kern.items()}
+    breakdown = {n: {"us_per_step": round(v[0] / k_steps * 1e3, 2), "launches": v[1]} for n, v in kern.items()}
 
     line = {
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world, "steps": args.steps,

@@ -57,6 +57,7 @@ struct Plan {
   dm::GruPlan gru;
   bool u_in_gru;  // small M: u finished inside the GRU kernel; large M: W1 GEMM + finalize
   bool overlap;   // vocab GEMM launched as a programmatic dependent of the GRU (deferred W2)
+  int defer_tiles;  // leading tiles per CTA whose W2 segment waits for the GRU
   int tmem_cols;  // TMEM columns of the vocab GEMM
   // workspace layout (offsets in bytes)
   size_t ctrl_bytes;
@@ -164,10 +165,21 @@ int make_plan(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head
     // one SM (228 KB of shared memory, 1 KB reserved per CTA) and every tile of a CTA can keep
     // its own TMEM accumulator until u is ready.
     const int vsm = dm::tc_softmax_deferred_smem(p.bn);
-    p.overlap = p.u_in_gru && vsm > 0 && p.w_per_chunk * p.bn <= 512 &&
+    // The first D tiles of each CTA wait for u; the rest run whole, so their epilogues overlap
+    // the remaining weight stream.  D covers the GRU's expected time (12 us + K steps of
+    // 4.5 + 0.5 B us, generous for a GRU sharing its SMs with the stream) in tiles of
+    // 128 x (H + R) bf16 weights per CTA streamed at 6 TB/s; a short estimate only costs a
+    // wait at the checkpoint, never correctness.
+    {
+      const double t_tile_us = 128.0 * (H + R) * 2.0 * p.grid / 6.0e6;
+      const double t_gru_us = 12.0 + K * (4.5 + 0.5 * B);
+      int d = static_cast<int>(t_gru_us / t_tile_us) + 1;
+      p.defer_tiles = d < 1 ? 1 : (d > p.w_per_chunk ? p.w_per_chunk : d);
+    }
+    p.overlap = p.u_in_gru && vsm > 0 && (p.defer_tiles + 2) * p.bn <= 512 &&
                 static_cast<size_t>(vsm) + p.gru.smem + 2048 <= 228 * 1024;
   }
-  p.tmem_cols = pow2_at_least(p.overlap ? p.w_per_chunk * p.bn : 2 * p.bn, 32);
+  p.tmem_cols = pow2_at_least(p.overlap ? (p.defer_tiles + 2) * p.bn : 2 * p.bn, 32);
 
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -390,7 +402,7 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
     tp.tok_tiles = P.tok_tiles; tp.w_tiles = P.w_tiles;
     tp.nchunks = P.nchunks; tp.w_per_chunk = P.w_per_chunk;
     tp.w_evict_first = P.tok_tiles == 1 ? 1 : 0;
-    tp.defer = P.overlap ? 1 : 0;
+    tp.defer = P.overlap ? P.defer_tiles : 0;
     tp.tmem_cols = P.tmem_cols;
     tp.bias = hw ? static_cast<const __nv_bfloat16*>(hw->b2) : nullptr;
     tp.out = reinterpret_cast<float*>(ws + P.off_part);

@@ -27,8 +27,8 @@ struct TcParams {
   // store mode: items (tok tile, w tile, split) round-robin over the CTAs
   int splits, kb_per_split, total_items;
   int w_evict_first;
-  int defer;      // softmax + swap only: first segment of every tile, then griddepcontrol.wait,
-                  // then the second segment (each tile keeps its own TMEM accumulator)
+  int defer;      // softmax + swap only: number of leading tiles whose second segment waits for
+                  // the preceding grid (0 = off); see the producer in tc_gemm.cuh
   int tmem_cols;  // TMEM columns to allocate (power of two, 32..512)
   const __nv_bfloat16* bias;  // softmax: b2 [V] or nullptr
   float* out;                 // softmax: partial records [M][rec fields][nchunks]; store: [splits][M][ld_out]

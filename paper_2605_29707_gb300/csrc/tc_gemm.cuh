@@ -18,6 +18,10 @@
 #include "kernels.h"
 #include "ptx.cuh"
 
+#ifndef DOMINO_VOCAB_TRIGGER
+#define DOMINO_VOCAB_TRIGGER 1  // let the merge kernel launch while this grid runs
+#endif
+
 namespace dm {
 
 template <int BN, bool SWAP, int MODE, int KMAX, int ST = 0>
@@ -67,6 +71,16 @@ __device__ __forceinline__ bool tc_get_item(const TcParams& p, int i, TcItem& it
     it.kb1 = min(nkb, it.kb0 + p.kb_per_split);
     return true;
   }
+}
+
+// TMEM column of item i's accumulator: two alternating buffers; in deferred mode the first
+// p.defer tiles each keep their own column block (holding the first segment until the second
+// is added) and later tiles alternate between the two blocks after them.
+template <int BN>
+__device__ __forceinline__ uint32_t tc_acc_col(const TcParams& p, int i) {
+  if (!p.defer) return static_cast<uint32_t>((i & 1) * BN);
+  if (i < p.defer) return static_cast<uint32_t>(i * BN);
+  return static_cast<uint32_t>((p.defer + ((i - p.defer) & 1)) * BN);
 }
 
 // Running log-sum-exp state and top-KMAX list of one token over a stream of logits.
@@ -198,6 +212,9 @@ __global__ void __launch_bounds__(192, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  // a kernel launched as this grid's programmatic dependent may start now (it waits for this
+  // grid to complete before it reads anything this kernel writes)
+  if (DOMINO_VOCAB_TRIGGER) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
@@ -241,13 +258,15 @@ __global__ void __launch_bounds__(192, 1)
       int issued = 0;
       bool ok = true;
       TcItem it;
-      // Deferred mode streams the first K segment of every tile first; the second segment's
-      // activations (u) come from the preceding kernel, so they are loaded only after
-      // griddepcontrol.wait (the hardware's wait for the preceding grid to complete).
-      const int passes = p.defer ? 2 : 1;
+      // Deferred mode (p.defer = D > 0 tiles): pass 0 streams only the first K segment of tiles
+      // 0..D-1; the second segment's activations (u) come from the preceding kernel, so pass 1
+      // loads them only after griddepcontrol.wait (the hardware's wait for the preceding grid
+      // to complete) and adds the second segment to tiles 0..D-1; pass 2 runs tiles D.. whole.
+      const int passes = p.defer ? 3 : 1;
       for (int pass = 0; pass < passes && ok; ++pass) {
       if (pass == 1) asm volatile("griddepcontrol.wait;" ::: "memory");
-      for (int i = 0; ok && tc_get_item<MODE>(p, i, it); ++i) {
+      for (int i = (pass == 2 ? p.defer : 0); ok && tc_get_item<MODE>(p, i, it); ++i) {
+        if (pass < 2 && p.defer && i >= p.defer) break;
         const int kb_lo = (p.defer && pass == 1) ? p.nkb1 : it.kb0;
         const int kb_hi = (p.defer && pass == 0) ? p.nkb1 : it.kb1;
         for (int kb = kb_lo; kb < kb_hi; ++kb) {
@@ -285,15 +304,14 @@ __global__ void __launch_bounds__(192, 1)
       uint32_t phase = 0;
       bool ok = true;
       TcItem it;
-      const int passes = p.defer ? 2 : 1;
+      const int passes = p.defer ? 3 : 1;
       for (int pass = 0; pass < passes && ok; ++pass) {
-      for (int i = 0; ok && tc_get_item<MODE>(p, i, it); ++i) {
+      for (int i = (pass == 2 ? p.defer : 0); ok && tc_get_item<MODE>(p, i, it); ++i) {
+        if (pass < 2 && p.defer && i >= p.defer) break;
         const int ab = i & 1;
         const uint32_t aph = (i >> 1) & 1;
-        const bool last_pass = pass == passes - 1;
-        // the accumulator of item i: one of two alternating buffers, or (deferred mode) its own
-        // column block, which holds the first segment until the second one is added
-        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>((p.defer ? i : ab) * BN);
+        const bool last_pass = !p.defer || pass >= 1;  // passes that finish a tile
+        const uint32_t d_tmem = tmem_base + tc_acc_col<BN>(p, i);
         if (last_pass) {
           if (!mbar_wait(&tempty[ab], aph ^ 1u, abort_flag, p.status)) break;
           tc_fence_after();
@@ -333,7 +351,7 @@ __global__ void __launch_bounds__(192, 1)
       const bool ok = mbar_wait(&tfull[ab], aph, abort_flag, p.status);
       if (epi_any(!ok)) { aborted = true; break; }
       tc_fence_after();
-      const uint32_t tcol = tmem_base + lane_off + static_cast<uint32_t>((p.defer ? i : ab) * BN);
+      const uint32_t tcol = tmem_base + lane_off + tc_acc_col<BN>(p, i);
 
       if constexpr (MODE == kModeStore) {
         if constexpr (SWAP) {

@@ -18,6 +18,10 @@
 #include "kernels.h"
 #include "ptx.cuh"
 
+#ifndef DOMINO_TREE_PDL
+#define DOMINO_TREE_PDL 1  // launch the merge kernel as a programmatic dependent of the vocab GEMM
+#endif
+
 namespace dm {
 
 constexpr int kMergeThreads = 256;
@@ -62,15 +66,17 @@ struct TreeSlots {
   int j[kMaxN + 1];
 };
 
-// Best remaining child of slot s (one thread).
-__device__ __forceinline__ void refresh_slot(TreeSlots& S, int s, const float* lp, const int* ids, int K, int k) {
-  const int d = S.depth[s];
+// Best remaining child of slot s (one thread).  The caller passes the slot's depth d, score
+// and popped mask in registers; children of a slot have non-increasing scores, so the best
+// remaining one is the first unpopped child, or an unpopped child of exactly the same score
+// with a lower token id.
+__device__ __forceinline__ void refresh_slot(TreeSlots& S, int s, int d, float base, unsigned mask, const float* lp,
+                                             const int* ids, int K, int k) {
   if (d >= K) { S.hi[s] = 0u; return; }
   const unsigned all = (k == 32) ? 0xffffffffu : ((1u << k) - 1u);
-  const unsigned avail = ~S.mask[s] & all;
+  const unsigned avail = ~mask & all;
   if (avail == 0u) { S.hi[s] = 0u; return; }
   const int j0 = __ffs(avail) - 1;
-  const float base = S.score[s];
   const float* row_lp = lp + d * k;
   const int* row_id = ids + d * k;
   const float best_sc = base + row_lp[j0];
@@ -78,7 +84,7 @@ __device__ __forceinline__ void refresh_slot(TreeSlots& S, int s, const float* l
   for (int j = j0 + 1; j < k; ++j) {
     const float sc = base + row_lp[j];
     if (sc < best_sc) break;
-    if (!((S.mask[s] >> j) & 1u) && row_id[j] < best_tok) { best_j = j; best_tok = row_id[j]; }
+    if (!((mask >> j) & 1u) && row_id[j] < best_tok) { best_j = j; best_tok = row_id[j]; }
   }
   S.hi[s] = f32_ord(best_sc);
   S.lo[s] = ((0x3FFFFFu - static_cast<unsigned>(best_tok)) << 10) | (0x3FFu - static_cast<unsigned>(s));
@@ -90,9 +96,9 @@ __global__ void __launch_bounds__(kMergeThreads) merge_tree_kernel(const TreePar
   constexpr int F = 2 + 2 * KM;
   constexpr int kWarps = kMergeThreads / 32;
   __shared__ float s_mx[kWarps], s_se[kWarps];
-  __shared__ unsigned s_hi[kWarps], s_lo[kWarps];
-  __shared__ int s_src[kWarps];
-  __shared__ int s_win, s_last;
+  __shared__ int s_last;
+  __shared__ float s_cv[kWarps * kMaxTopk];
+  __shared__ int s_ci[kWarps * kMaxTopk];
   __shared__ float s_lp[kMaxK * kMaxTopk];
   __shared__ int s_id[kMaxK * kMaxTopk];
   __shared__ TreeSlots S;
@@ -101,6 +107,8 @@ __global__ void __launch_bounds__(kMergeThreads) merge_tree_kernel(const TreePar
   const int K = p.K, k = p.k, N = p.N, nch = p.nchunks;
   const int b = m / K;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  // launched as a programmatic dependent of the vocabulary GEMM: wait for its partials
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const float* base = p.partials + static_cast<size_t>(m) * F * nch;
   const int* ibase = reinterpret_cast<const int*>(base);
 
@@ -144,29 +152,38 @@ __global__ void __launch_bounds__(kMergeThreads) merge_tree_kernel(const TreePar
   for (int w = 0; w < kWarps; ++w) lse_merge(mx, se, s_mx[w], s_se[w]);
   const float lse = mx + logf(se);
 
-  // ------------------------------------------------------------ k best heads, one per round
+  // ------------------------------------------------------------ k best: per warp, then across warps
   for (int q = 0; q < k; ++q) {
     uint32_t mhi, mlo;
     int src;
     warp_argmax2(f32_ord(tv[0]), ~static_cast<uint32_t>(ti[0]), mhi, mlo, src);
-    if (lane == 0) { s_hi[warp] = mhi; s_lo[warp] = mlo; s_src[warp] = warp * 32 + src; }
-    __syncthreads();
-    if (warp == 0) {
-      const uint32_t h = lane < kWarps ? s_hi[lane] : 0u;
-      const uint32_t l = lane < kWarps ? s_lo[lane] : 0u;
-      uint32_t wh, wl;
-      int ws;
-      warp_argmax2(h, l, wh, wl, ws);
-      if (lane == 0) s_win = s_src[ws];
-    }
-    __syncthreads();
-    if (tid == s_win) {
-      p.topk_ids[static_cast<size_t>(m) * k + q] = ti[0];
-      p.topk_logp[static_cast<size_t>(m) * k + q] = tv[0] - lse;
+    const float val = __shfl_sync(0xffffffffu, tv[0], src);
+    const int id = __shfl_sync(0xffffffffu, ti[0], src);
+    if (lane == src) {
 #pragma unroll
       for (int i = 0; i + 1 < KM; ++i) { tv[i] = tv[i + 1]; ti[i] = ti[i + 1]; }
       tv[KM - 1] = -INFINITY;
       ti[KM - 1] = -1;
+    }
+    if (lane == 0) { s_cv[warp * kMaxTopk + q] = val; s_ci[warp * kMaxTopk + q] = id; }
+  }
+  __syncthreads();
+  if (warp == 0) {
+    int ptr = 0;  // lane w < kWarps walks warp w's sorted candidate list
+    for (int q = 0; q < k; ++q) {
+      uint32_t hi = 0u, lo = 0u;
+      if (lane < kWarps && ptr < k) {
+        hi = f32_ord(s_cv[lane * kMaxTopk + ptr]);
+        lo = ~static_cast<uint32_t>(s_ci[lane * kMaxTopk + ptr]);
+      }
+      uint32_t mhi, mlo;
+      int src;
+      warp_argmax2(hi, lo, mhi, mlo, src);
+      if (lane == src) {
+        p.topk_ids[static_cast<size_t>(m) * k + q] = s_ci[lane * kMaxTopk + ptr];
+        p.topk_logp[static_cast<size_t>(m) * k + q] = s_cv[lane * kMaxTopk + ptr] - lse;
+        ++ptr;
+      }
     }
   }
 
@@ -191,15 +208,15 @@ __global__ void __launch_bounds__(kMergeThreads) merge_tree_kernel(const TreePar
     S.score[0] = 0.f;
     S.depth[0] = 0;
     S.mask[0] = 0u;
-    refresh_slot(S, 0, s_lp, s_id, K, k);
+    refresh_slot(S, 0, 0, 0.f, 0u, s_lp, s_id, K, k);
   }
   __syncwarp();
   for (int i = 0; i < N; ++i) {
     uint32_t hi = 0u, lo = 0u;
     int sb = -1;
-    for (int s = lane; s <= i; s += 32) {
-      const uint32_t h = S.hi[s], l = S.lo[s];
-      if (h > hi || (h == hi && h != 0u && l > lo)) { hi = h; lo = l; sb = s; }
+    for (int s2 = lane; s2 <= i; s2 += 32) {
+      const uint32_t h = S.hi[s2], l = S.lo[s2];
+      if (h > hi || (h == hi && h != 0u && l > lo)) { hi = h; lo = l; sb = s2; }
     }
     uint32_t mhi, mlo;
     int src;
@@ -208,18 +225,20 @@ __global__ void __launch_bounds__(kMergeThreads) merge_tree_kernel(const TreePar
     if (lane == 0) {
       const int jj = S.j[s];
       const int d = S.depth[s];
+      const float base_s = S.score[s];
+      const unsigned mask_s = S.mask[s] | (1u << jj);
       const int tok = s_id[d * k + jj];
-      const float sc = S.score[s] + s_lp[d * k + jj];
+      const float sc = base_s + s_lp[d * k + jj];
       p.tree_parent[ob + i] = s - 1;
       p.tree_token[ob + i] = tok;
       p.tree_depth[ob + i] = d + 1;
       if (p.tree_score) p.tree_score[ob + i] = sc;
+      S.mask[s] = mask_s;
       S.score[i + 1] = sc;
       S.depth[i + 1] = d + 1;
       S.mask[i + 1] = 0u;
-      S.mask[s] |= 1u << jj;
-      refresh_slot(S, s, s_lp, s_id, K, k);
-      refresh_slot(S, i + 1, s_lp, s_id, K, k);
+      refresh_slot(S, s, d, base_s, mask_s, s_lp, s_id, K, k);
+      refresh_slot(S, i + 1, d + 1, sc, 0u, s_lp, s_id, K, k);
     }
     __syncwarp();
   }
@@ -227,10 +246,20 @@ __global__ void __launch_bounds__(kMergeThreads) merge_tree_kernel(const TreePar
 
 cudaError_t launch_merge_tree(const TreeParams& p, cudaStream_t stream) {
   if (p.K > kMaxK || p.k > kMaxTopk || p.N > kMaxN) return cudaErrorInvalidValue;
-  const int rows = p.B * p.K;
-  if (p.kmax == 16) merge_tree_kernel<16><<<rows, kMergeThreads, 0, stream>>>(p);
-  else if (p.kmax == 32) merge_tree_kernel<32><<<rows, kMergeThreads, 0, stream>>>(p);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.B * p.K);
+  cfg.blockDim = dim3(kMergeThreads);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = DOMINO_TREE_PDL ? 1 : 0;
+  cudaError_t e;
+  if (p.kmax == 16) e = cudaLaunchKernelEx(&cfg, merge_tree_kernel<16>, p);
+  else if (p.kmax == 32) e = cudaLaunchKernelEx(&cfg, merge_tree_kernel<32>, p);
   else return cudaErrorInvalidValue;
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
