@@ -13,11 +13,34 @@
 #include "kernels.h"
 #include "ptx.cuh"
 
+#ifndef DOMINO_GRU_BACKOFF_NS
+#define DOMINO_GRU_BACKOFF_NS 64  // pause between re-reads of a state word that is not ready
+#endif
+
 namespace dm {
 
+#ifdef DOMINO_GRU_TRACE
+__device__ unsigned long long g_gru_trace[2][64][8];  // [cta 0 / last][step][phase] globaltimer
+__device__ __forceinline__ void gru_trace(int step, int ph) {
+  const int w = blockIdx.x == 0 ? 0 : (blockIdx.x == gridDim.x - 1 ? 1 : -1);
+  if (w >= 0 && threadIdx.x == 0 && step < 64) {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    g_gru_trace[w][step][ph] = t;
+  }
+}
+#define GRU_TRACE(step, ph) gru_trace(step, ph)
+#else
+#define GRU_TRACE(step, ph)
+#endif
+
 constexpr int kGruThreads = 256;
+constexpr int kGatePairsPerThread = 4;  // (sequence, unit) gate evaluations per thread and chunk
 constexpr int kGruWarps = kGruThreads / 32;
 constexpr int kChunkSeqs = 32;  // sequences staged per MMA pass (4 n-tiles of 8)
+constexpr int kGsmLd = kChunkSeqs + 1;  // padded row stride of the W_hh . h tile (bank spread)
+constexpr int kChains = 4;              // independent mma accumulator chains per warp
+constexpr int kMmaTasks = kChains * 8;  // (tile, k-slice) tasks per MMA pass
 
 // ---------------------------------------------------------------------------- gather
 __global__ void __launch_bounds__(128) gather_kernel(const GatherParams p) {
@@ -57,6 +80,7 @@ __device__ __forceinline__ bool poll_v4(const uint32_t* p, uint4& v) {
   if ((v.x & v.y & v.z & v.w & 1u) != 0u) return true;
   const long long t0 = clock64();
   while (true) {
+    if (DOMINO_GRU_BACKOFF_NS > 0) __nanosleep(DOMINO_GRU_BACKOFF_NS);  // spare L2 while waiting
     v = ld_relaxed_v4(p);
     if ((v.x & v.y & v.z & v.w & 1u) != 0u) return true;
     if (clock64() - t0 > kWaitCycles) return false;
@@ -116,8 +140,8 @@ __device__ __forceinline__ float sigmoidf_(float x) { return 1.f / (1.f + expf(-
 // whh   [mt*16 rows][Ds + 8] bf16  this CTA's W_hh rows (gate g, unit jl) at row g*U + jl;
 //                                  rows past 3U are zero
 // hsm   [chunk][Ds + 8] bf16       h_{t-1} of up to 32 sequences (the MMA's n operand)
-// gsm   [mt*16][32] f32            W_hh . h_{t-1}
-// red   [16 tasks][16][8] f32      k-split partial tiles
+// gsm   [mt*16][33] f32            W_hh . h_{t-1} (padded rows)
+// red   [32 tasks][16][8] f32      k-split partial tiles
 // hprev [bc][U] f32                this CTA's own previous states (fp32)
 struct GruSmem {
   size_t whh, hsm, gsm, red, hprev, total;
@@ -135,9 +159,9 @@ __host__ __device__ inline GruSmem gru_layout(int Ds, int U, int bc) {
   L.hsm = o;
   o += static_cast<size_t>(L.chunk) * L.ldw * 2;
   L.gsm = o;
-  o += static_cast<size_t>(L.mt) * 16 * kChunkSeqs * 4;
+  o += static_cast<size_t>(L.mt) * 16 * kGsmLd * 4;
   L.red = o;
-  o += static_cast<size_t>(2 * kGruWarps) * 16 * 8 * 4;
+  o += static_cast<size_t>(kMmaTasks) * 16 * 8 * 4;
   L.hprev = o;
   o += static_cast<size_t>(bc) * U * 4;
   L.total = (o + 15) & ~static_cast<size_t>(15);
@@ -218,12 +242,30 @@ __global__ void __launch_bounds__(kGruThreads) gru_kernel(const GruParams p) {
   bool ok = true;
 
   for (int t = 0; t < K && ok; ++t) {
+    GRU_TRACE(t, 0);
     for (int c0 = 0; c0 < nbc; c0 += L.chunk) {
       const int nb = min(L.chunk, nbc - c0);
       const int nt_count = (nb + 7) / 8;
       const int tiles = L.mt * nt_count;
-      int ks = 1;  // k-slices per tile, so that up to 16 warp tasks (two per warp) exist
-      while (tiles * ks * 2 <= 2 * kGruWarps && ks * 2 <= nk) ks *= 2;
+      int ks = 1;  // k-slices per tile: up to kChains short independent chains per warp
+      while (tiles * ks * 2 <= kMmaTasks && ks * 2 <= nk) ks *= 2;
+      // gate inputs of this step (input-gate sums, b_hh) into registers before the wait
+      float gx[kGatePairsPerThread][3], gb[kGatePairsPerThread][3];
+#pragma unroll
+      for (int r = 0; r < kGatePairsPerThread; ++r) {
+        const int e = tid + r * kGruThreads;
+        if (e < nb * Uc) {
+          const int bb = e / Uc, jl = e % Uc;
+          const int j = j0 + jl;
+          const size_t m = static_cast<size_t>(b0 + c0 + bb) * K + t;
+          const float* x = p.xs + m * 3 * Ds;
+#pragma unroll
+          for (int g = 0; g < 3; ++g) {
+            gx[r][g] = x[g * Ds + j];
+            gb[r][g] = bf_or0(p.b_hh, g * Ds + j);
+          }
+        }
+      }
       if (t > 0) {
         // ---- h_{t-1} of this chunk's sequences, polled from the tagged rows
         const int per_row = Ds / 4;
@@ -258,89 +300,94 @@ __global__ void __launch_bounds__(kGruThreads) gru_kernel(const GruParams p) {
           ok = false;
           break;
         }
+        GRU_TRACE(t, 1);
         // ---- g = W_hh[rows] . h_{t-1} on the tensor cores
-        // each warp takes two tasks at a time: two independent accumulator chains
+        // each warp runs up to kChains (tile, k-slice) tasks at once: independent accumulator
+        // chains hide the latency of mma.sync
         const int ntasks = tiles * ks;
-        for (int tp = warp; tp < ntasks; tp += 2 * kGruWarps) {
-          const int tb = tp + kGruWarps;
-          const bool two = tb < ntasks;
-          const int tileA = tp % tiles, kslA = tp / tiles;
-          const int tileB = two ? tb % tiles : tileA, kslB = two ? tb / tiles : kslA;
-          const int kbA = kslA * (nk / ks), keA = (kslA == ks - 1) ? nk : kbA + nk / ks;
-          const int kbB = kslB * (nk / ks), keB = (kslB == ks - 1) ? nk : kbB + nk / ks;
-          float accA[4] = {0.f, 0.f, 0.f, 0.f}, accB[4] = {0.f, 0.f, 0.f, 0.f};
-          const __nv_bfloat16* arowA =
-              whh + static_cast<size_t>((tileA % L.mt) * 16 + (lane & 15)) * ldw + (lane >> 4) * 8;
-          const __nv_bfloat16* browA =
-              hsm + static_cast<size_t>((tileA / L.mt) * 8 + (lane & 7)) * ldw + ((lane >> 3) & 1) * 8;
-          const __nv_bfloat16* arowB =
-              whh + static_cast<size_t>((tileB % L.mt) * 16 + (lane & 15)) * ldw + (lane >> 4) * 8;
-          const __nv_bfloat16* browB =
-              hsm + static_cast<size_t>((tileB / L.mt) * 8 + (lane & 7)) * ldw + ((lane >> 3) & 1) * 8;
-          const int steps = max(keA - kbA, two ? keB - kbB : 0);
+        const int kper = nk / ks;
+        for (int t0 = warp; t0 < ntasks; t0 += kChains * kGruWarps) {
+          float acc[kChains][4];
+          const __nv_bfloat16* arow[kChains];
+          const __nv_bfloat16* brow[kChains];
+          int kbeg[kChains], kend[kChains];
+#pragma unroll
+          for (int c = 0; c < kChains; ++c) {
+            const int task = t0 + c * kGruWarps;
+            const int tile = task % tiles, ksl = task / tiles;
+            acc[c][0] = acc[c][1] = acc[c][2] = acc[c][3] = 0.f;
+            arow[c] = whh + static_cast<size_t>((tile % L.mt) * 16 + (lane & 15)) * ldw + (lane >> 4) * 8;
+            brow[c] = hsm + static_cast<size_t>((tile / L.mt) * 8 + (lane & 7)) * ldw + ((lane >> 3) & 1) * 8;
+            kbeg[c] = ksl * kper;
+            kend[c] = task < ntasks ? ((ksl == ks - 1) ? nk : kbeg[c] + kper) : kbeg[c];
+          }
+          const int steps = nk - (ks - 1) * kper;  // the longest slice
           for (int i = 0; i < steps; ++i) {
-            if (kbA + i < keA) {
-              uint32_t a[4], b[2];
-              ldmatrix_x4(a, arowA + (kbA + i) * 16);
-              ldmatrix_x2(b, browA + (kbA + i) * 16);
-              mma_16816(accA, a, b);
-            }
-            if (two && kbB + i < keB) {
-              uint32_t a[4], b[2];
-              ldmatrix_x4(a, arowB + (kbB + i) * 16);
-              ldmatrix_x2(b, browB + (kbB + i) * 16);
-              mma_16816(accB, a, b);
+#pragma unroll
+            for (int c = 0; c < kChains; ++c) {
+              if (kbeg[c] + i < kend[c]) {
+                uint32_t a[4], b[2];
+                ldmatrix_x4(a, arow[c] + (kbeg[c] + i) * 16);
+                ldmatrix_x2(b, brow[c] + (kbeg[c] + i) * 16);
+                mma_16816(acc[c], a, b);
+              }
             }
           }
           const int g = lane >> 2, tq = lane & 3;
-          for (int w = 0; w < (two ? 2 : 1); ++w) {
-            const int task = w ? tb : tp;
+#pragma unroll
+          for (int c = 0; c < kChains; ++c) {
+            const int task = t0 + c * kGruWarps;
+            if (task >= ntasks) continue;
             const int tile = task % tiles;
-            const float* acc = w ? accB : accA;
             float* out;
             int ld;
             if (ks == 1) {
-              out = gsm + static_cast<size_t>((tile % L.mt) * 16) * kChunkSeqs + (tile / L.mt) * 8;
-              ld = kChunkSeqs;
+              out = gsm + static_cast<size_t>((tile % L.mt) * 16) * kGsmLd + (tile / L.mt) * 8;
+              ld = kGsmLd;
             } else {
               out = red + static_cast<size_t>(task) * 128;
               ld = 8;
             }
-            out[g * ld + 2 * tq] = acc[0];
-            out[g * ld + 2 * tq + 1] = acc[1];
-            out[(g + 8) * ld + 2 * tq] = acc[2];
-            out[(g + 8) * ld + 2 * tq + 1] = acc[3];
+            out[g * ld + 2 * tq] = acc[c][0];
+            out[g * ld + 2 * tq + 1] = acc[c][1];
+            out[(g + 8) * ld + 2 * tq] = acc[c][2];
+            out[(g + 8) * ld + 2 * tq + 1] = acc[c][3];
           }
         }
+        GRU_TRACE(t, 4);
         __syncthreads();
+        GRU_TRACE(t, 5);
         if (ks > 1) {
           for (int e = tid; e < tiles * 128; e += kGruThreads) {
             const int tile = e / 128, w = e % 128;
             float s = 0.f;
             for (int ksl = 0; ksl < ks; ++ksl) s += red[static_cast<size_t>(ksl * tiles + tile) * 128 + w];
             const int mt = tile % L.mt, nt = tile / L.mt;
-            gsm[static_cast<size_t>(mt * 16 + w / 8) * kChunkSeqs + nt * 8 + (w % 8)] = s;
+            gsm[static_cast<size_t>(mt * 16 + w / 8) * kGsmLd + nt * 8 + (w % 8)] = s;
           }
           __syncthreads();
         }
       }
+      GRU_TRACE(t, 2);
       // ---- gates and the new state (torch.nn.GRU convention); publish the tagged state
-      for (int e = tid; e < nb * Uc; e += kGruThreads) {
+#pragma unroll
+      for (int rr = 0; rr < kGatePairsPerThread; ++rr) {
+        const int e = tid + rr * kGruThreads;
+        if (e >= nb * Uc) break;
         const int bb = e / Uc, jl = e % Uc;
         const int j = j0 + jl;
         const int bl = c0 + bb;  // sequence index within this CTA
         const size_t m = static_cast<size_t>(b0 + bl) * K + t;
-        const float* x = p.xs + m * 3 * Ds;
-        float hr = bf_or0(p.b_hh, j), hz = bf_or0(p.b_hh, Ds + j), hn = bf_or0(p.b_hh, 2 * Ds + j);
+        float hr = gb[rr][0], hz = gb[rr][1], hn = gb[rr][2];
         if (t > 0) {
-          hr += gsm[static_cast<size_t>(jl) * kChunkSeqs + bb];
-          hz += gsm[static_cast<size_t>(U + jl) * kChunkSeqs + bb];
-          hn += gsm[static_cast<size_t>(2 * U + jl) * kChunkSeqs + bb];
+          hr += gsm[static_cast<size_t>(jl) * kGsmLd + bb];
+          hz += gsm[static_cast<size_t>(U + jl) * kGsmLd + bb];
+          hn += gsm[static_cast<size_t>(2 * U + jl) * kGsmLd + bb];
         }
         const float hp = hprev[bl * U + jl];
-        const float r = sigmoidf_(x[j] + hr);
-        const float z = sigmoidf_(x[Ds + j] + hz);
-        const float n = tanhf(x[2 * Ds + j] + r * hn);
+        const float r = sigmoidf_(gx[rr][0] + hr);
+        const float z = sigmoidf_(gx[rr][1] + hz);
+        const float n = tanhf(gx[rr][2] + r * hn);
         const float h = (1.f - z) * n + z * hp;
         hprev[bl * U + jl] = h;
         p.hx[m * Ds + j] = tagged(h);
@@ -348,6 +395,7 @@ __global__ void __launch_bounds__(kGruThreads) gru_kernel(const GruParams p) {
       }
       __syncthreads();
     }
+    GRU_TRACE(t, 3);
   }
   if (!ok || p.u == nullptr) return;
 
@@ -425,6 +473,7 @@ GruPlan gru_plan(int B, int Ds, int num_sms) {
   g.gb = (B + g.bc - 1) / g.bc;
   const GruSmem L = gru_layout(Ds, g.units, g.bc);
   g.smem = L.total <= 220 * 1024 ? L.total : 0;
+  if (static_cast<long long>(L.chunk) * g.units > static_cast<long long>(kGatePairsPerThread) * kGruThreads) g.smem = 0;
   return g;
 }
 
@@ -468,3 +517,9 @@ cudaError_t launch_u_finalize(const UFinalParams& p, cudaStream_t stream) {
 }
 
 }  // namespace dm
+
+#ifdef DOMINO_GRU_TRACE
+extern "C" __attribute__((visibility("default"))) int domino_debug_gru_trace(unsigned long long* out) {
+  return cudaMemcpyFromSymbol(out, dm::g_gru_trace, sizeof(dm::g_gru_trace)) == cudaSuccess ? 0 : -3;
+}
+#endif
