@@ -164,7 +164,7 @@ int make_plan(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head
     // Overlap the GRU with the W_lm stream when a deferred-mode vocab CTA and a GRU CTA fit on
     // one SM (228 KB of shared memory, 1 KB reserved per CTA) and every tile of a CTA can keep
     // its own TMEM accumulator until u is ready.
-    const int vsm = dm::tc_softmax_deferred_smem(p.bn);
+    const int vsm = dm::tc_softmax_deferred_smem(p.bn, p.kmax);
     // The first D tiles of each CTA wait for u; the rest run whole, so their epilogues overlap
     // the remaining weight stream.  D covers the GRU's expected time (12 us + K steps of
     // 4.5 + 0.5 B us, generous for a GRU sharing its SMs with the stream) in tiles of

@@ -46,7 +46,7 @@ cudaError_t launch_tc_gemm(int mode, int bn, bool swap, int kmax, const CUtensor
 cudaError_t launch_tc_softmax_deferred(int bn, int kmax, const CUtensorMap* maps, const TcParams& p, int grid,
                                        cudaStream_t stream);
 // Shared memory one deferred-mode CTA uses (for the co-residency budget).
-int tc_softmax_deferred_smem(int bn);
+int tc_softmax_deferred_smem(int bn, int kmax);
 
 // ---------------------------------------------------------------- gather / GRU
 struct GatherParams {

@@ -38,10 +38,14 @@ struct TcCfg {
   static constexpr int kTmemCols =
       (2 * BN <= 32) ? 32 : (2 * BN <= 64) ? 64 : (2 * BN <= 128) ? 128 : (2 * BN <= 256) ? 256 : 512;
   static constexpr int kBarBytes = 256;
-  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kTrBytes + kBarBytes;
+  // per-thread scratch of one 32-value chunk (rare path of the normal orientation)
+  static constexpr int kListBytes = (MODE == kModeSoftmax && !SWAP) ? 128 * 32 * 4 : 0;
+  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kTrBytes + kListBytes + kBarBytes;
   static constexpr int kRec = 2 + 2 * KMAX;
   static_assert(kStages >= 2, "pipeline needs at least two stages");
-  static_assert(kSmemBytes > 116 * 1024, "one CTA per SM keeps TMEM allocation uncontended");
+  // two CTAs (each with 1 KB of reserved shared memory) never fit on one 228 KB SM, so TMEM
+  // allocation is never contended between CTAs of this kernel
+  static_assert(2 * (kSmemBytes + 1024) > 228 * 1024, "one CTA per SM keeps TMEM allocation uncontended");
   static_assert(BN % 16 == 0 && BN >= 16 && BN <= 256, "UMMA N for M = 128");
 };
 
@@ -175,6 +179,49 @@ struct OnlineTopK {
   }
 };
 
+// ---- streaming softmax/top-k of one epilogue thread ---------------------------------------
+// Running max, sum of exp and the top-KMAX list (value desc, id asc) live in registers.  The hot
+// path per chunk of values is branch-free: one chunk max, one rescale, one exp per value, and a
+// single compare of the chunk max with the list's last value.  Only when that compare passes
+// (rare once the list has filled) does a loop walk the chunk's values, read back from shared
+// memory, through the register insertion network, which is emitted once.  Values of one thread
+// arrive in increasing id order, so an equal value never displaces an earlier entry.
+template <int N, int KM>
+__device__ __forceinline__ void stream_chunk(const float (&r)[N], const float* sx, int sstride, int v0, int vstride,
+                                             int nvalid, float& mx, float& se, float (&tv)[KM], int (&ti)[KM]) {
+  float cm = -INFINITY;
+#pragma unroll
+  for (int j = 0; j < N; ++j) cm = fmaxf(cm, j < nvalid ? r[j] : -INFINITY);
+  if (cm > mx) {
+    se = (mx == -INFINITY) ? 0.f : se * __expf(mx - cm);
+    mx = cm;
+  }
+  if (mx == -INFINITY) return;
+  float sum = 0.f;
+#pragma unroll
+  for (int j = 0; j < N; ++j) sum += (j < nvalid) ? __expf(r[j] - mx) : 0.f;
+  se += sum;
+  if (cm > tv[KM - 1]) {
+    const int n = nvalid < N ? nvalid : N;
+#pragma unroll 1
+    for (int j = 0; j < n; ++j) {
+      float x = sx[j * sstride];
+      if (!(x > tv[KM - 1])) continue;
+      int id = v0 + j * vstride;
+#pragma unroll
+      for (int q = 0; q < KM; ++q) {
+        const bool sw = x > tv[q];
+        const float a = tv[q];
+        const int b = ti[q];
+        tv[q] = sw ? x : a;
+        ti[q] = sw ? id : b;
+        x = sw ? a : x;
+        id = sw ? b : id;
+      }
+    }
+  }
+}
+
 // Returns the OR of `pred` over the 128 epilogue threads (named barrier 1).
 __device__ __forceinline__ bool epi_any(bool pred) {
   uint32_t r;
@@ -189,8 +236,10 @@ __device__ __forceinline__ bool epi_any(bool pred) {
   return r != 0;
 }
 
+// Deferred variants (ST > 0) must fit their registers beside a GRU CTA on one SM: the bound of
+// two CTAs per SM caps them at 168 registers per thread.
 template <int BN, bool SWAP, int MODE, int KMAX, int ST>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(192, ST > 0 ? 2 : 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
                    const __grid_constant__ CUtensorMap tmA2, const __grid_constant__ CUtensorMap tmB2,
                    const TcParams p) {
@@ -201,7 +250,8 @@ __global__ void __launch_bounds__(192, 1)
   uint8_t* sA = smem;
   uint8_t* sB = smem + C::kStages * C::kABytes;
   float* tr = reinterpret_cast<float*>(sB + C::kStages * C::kBBytes);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(tr) + C::kTrBytes);
+  float* scratch = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(tr) + C::kTrBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(scratch) + C::kListBytes);
   uint64_t* full = bars;
   uint64_t* empty = bars + C::kStages;
   uint64_t* tfull = bars + 2 * C::kStages;
@@ -342,6 +392,7 @@ __global__ void __launch_bounds__(192, 1)
     const uint32_t lane_off = static_cast<uint32_t>(32 * q) << 16;
     OnlineTopK<KMAX> st;
     if (MODE == kModeSoftmax) st.init();
+    float* my_scratch = scratch + ep;
     bool aborted = false;
     TcItem it;
     it.tok = 0;
@@ -414,10 +465,17 @@ __global__ void __launch_bounds__(192, 1)
         const int sub = ep % C::kTPT;
         const int vbase = it.w * 128;
         const float* trow = tr + tt * C::kTrStride;
-#pragma unroll 4
-        for (int jj = 0; jj < BN; ++jj) {
-          const int vl = sub + C::kTPT * jj;
-          if (vbase + vl < p.rows_w) st.push(trow[vl], vbase + vl);
+        const int left = p.rows_w - vbase - sub;  // valid entries: sub + TPT * jj < rows_w - vbase
+        const int nvalid_all = left <= 0 ? 0 : (left + C::kTPT - 1) / C::kTPT;
+        constexpr int kSub = BN < 32 ? BN : 32;
+#pragma unroll 1
+        for (int j0 = 0; j0 < BN; j0 += kSub) {
+          float r[kSub];
+          const float* sx = trow + sub + C::kTPT * j0;
+#pragma unroll
+          for (int j = 0; j < kSub; ++j) r[j] = sx[C::kTPT * j];
+          stream_chunk<kSub, KMAX>(r, sx, C::kTPT, vbase + sub + C::kTPT * j0, C::kTPT, nvalid_all - j0, st.mx, st.se,
+                                   st.tv, st.ti);
         }
         named_bar_sync(1, 128);
       } else {
@@ -428,21 +486,23 @@ __global__ void __launch_bounds__(192, 1)
           tc_ld_x32(tcol + c0, r);
           tc_wait_ld();
           const int v0 = it.w * BN + c0;
-          if (v0 + 32 <= p.rows_w) {
-            if (p.bias != nullptr) {
+          const int nvalid = p.rows_w - v0;
+          if (p.bias != nullptr) {
 #pragma unroll
-              for (int j = 0; j < 32; ++j) st.push(r[j] + __bfloat162float(p.bias[v0 + j]), v0 + j);
-            } else {
+            for (int j = 0; j < 32; ++j)
+              if (j < nvalid) r[j] += __bfloat162float(p.bias[v0 + j]);
+          }
+          {
+            // the rare path re-reads the chunk from this thread's shared-memory scratch
+            float cm = -INFINITY;
 #pragma unroll
-              for (int j = 0; j < 32; ++j) st.push(r[j], v0 + j);
-            }
-          } else {
+            for (int j = 0; j < 32; ++j) cm = fmaxf(cm, j < nvalid ? r[j] : -INFINITY);
+            if (cm > st.tv[KMAX - 1]) {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
-              const int v = v0 + j;
-              if (v < p.rows_w) st.push(r[j] + (p.bias ? __bfloat162float(p.bias[v]) : 0.f), v);
+              for (int j = 0; j < 32; ++j) my_scratch[j * 128] = r[j];
             }
           }
+          stream_chunk<32, KMAX>(r, my_scratch, 128, v0, 1, nvalid, st.mx, st.se, st.tv, st.ti);
         }
         tc_fence_before();
         mbar_arrive(&tempty[ab]);
@@ -452,6 +512,7 @@ __global__ void __launch_bounds__(192, 1)
     if (MODE == kModeSoftmax && !aborted) {
       const int tok_tile = blockIdx.x % p.tok_tiles;
       const int chunk = blockIdx.x / p.tok_tiles;
+
       if constexpr (SWAP) {
 #pragma unroll
         for (int off = C::kTPT / 2; off >= 1; off >>= 1) st.merge_shfl_xor(off);

@@ -26,9 +26,11 @@ cudaError_t launch_tc_softmax_deferred(int bn, int kmax, const CUtensorMap* maps
   return cudaErrorInvalidValue;
 }
 
-int tc_softmax_deferred_smem(int bn) {
-  if (bn == 16) return TcCfg<16, true, kModeSoftmax, 16, 6>::kSmemBytes;
-  if (bn == 32) return TcCfg<32, true, kModeSoftmax, 16, 5>::kSmemBytes;
+int tc_softmax_deferred_smem(int bn, int kmax) {
+  if (bn == 16) return kmax <= 16 ? TcCfg<16, true, kModeSoftmax, 16, 6>::kSmemBytes
+                                  : TcCfg<16, true, kModeSoftmax, 32, 6>::kSmemBytes;
+  if (bn == 32) return kmax <= 16 ? TcCfg<32, true, kModeSoftmax, 16, 5>::kSmemBytes
+                                  : TcCfg<32, true, kModeSoftmax, 32, 5>::kSmemBytes;
   return 0;
 }
 
