@@ -39,8 +39,8 @@ constexpr int kGatePairsPerThread = 4;  // (sequence, unit) gate evaluations per
 constexpr int kGruWarps = kGruThreads / 32;
 constexpr int kChunkSeqs = 32;  // sequences staged per MMA pass (4 n-tiles of 8)
 constexpr int kGsmLd = kChunkSeqs + 1;  // padded row stride of the W_hh . h tile (bank spread)
-constexpr int kChains = 4;              // independent mma accumulator chains per warp
-constexpr int kMmaTasks = kChains * 8;  // (tile, k-slice) tasks per MMA pass
+constexpr int kMaxMt = 3;  // 16-row gate tiles per CTA (up to 16 units x 3 gates)
+constexpr int kMaxNt = 4;  // 8-sequence tiles per staged chunk
 
 // ---------------------------------------------------------------------------- gather
 __global__ void __launch_bounds__(128) gather_kernel(const GatherParams p) {
@@ -141,7 +141,7 @@ __device__ __forceinline__ float sigmoidf_(float x) { return 1.f / (1.f + expf(-
 //                                  rows past 3U are zero
 // hsm   [chunk][Ds + 8] bf16       h_{t-1} of up to 32 sequences (the MMA's n operand)
 // gsm   [mt*16][33] f32            W_hh . h_{t-1} (padded rows)
-// red   [32 tasks][16][8] f32      k-split partial tiles
+// red   [8 warps][tiles][16][8] f32  k-range partial tiles of each warp
 // hprev [bc][U] f32                this CTA's own previous states (fp32)
 struct GruSmem {
   size_t whh, hsm, gsm, red, hprev, total;
@@ -160,15 +160,17 @@ __host__ __device__ inline GruSmem gru_layout(int Ds, int U, int bc) {
   o += static_cast<size_t>(L.chunk) * L.ldw * 2;
   L.gsm = o;
   o += static_cast<size_t>(L.mt) * 16 * kGsmLd * 4;
-  L.red = o;
-  o += static_cast<size_t>(kMmaTasks) * 16 * 8 * 4;
+  L.red = o;  // [warp][tile][16][8] partials of each warp's k-range
+  o += static_cast<size_t>(kGruWarps) * L.mt * (L.chunk / 8) * 128 * 4;
   L.hprev = o;
   o += static_cast<size_t>(bc) * U * 4;
   L.total = (o + 15) & ~static_cast<size_t>(15);
   return L;
 }
 
-__global__ void __launch_bounds__(kGruThreads) gru_kernel(const GruParams p) {
+// At most 128 registers per thread (two CTAs' worth per SM), so that a GRU CTA and a vocabulary
+// GEMM CTA (at most 168 registers x 192 threads) fit in one SM's register file.
+__global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) {
   extern __shared__ __align__(16) uint8_t gsmem[];
   const int U = p.units, Ds = p.Ds, K = p.K, B = p.B, R = p.R, H = p.H;
   const int M = B * K;
@@ -247,8 +249,6 @@ __global__ void __launch_bounds__(kGruThreads) gru_kernel(const GruParams p) {
       const int nb = min(L.chunk, nbc - c0);
       const int nt_count = (nb + 7) / 8;
       const int tiles = L.mt * nt_count;
-      int ks = 1;  // k-slices per tile: up to kChains short independent chains per warp
-      while (tiles * ks * 2 <= kMmaTasks && ks * 2 <= nk) ks *= 2;
       // gate inputs of this step (input-gate sums, b_hh) into registers before the wait
       float gx[kGatePairsPerThread][3], gb[kGatePairsPerThread][3];
 #pragma unroll
@@ -267,106 +267,97 @@ __global__ void __launch_bounds__(kGruThreads) gru_kernel(const GruParams p) {
         }
       }
       if (t > 0) {
-        // ---- h_{t-1} of this chunk's sequences, polled from the tagged rows
-        const int per_row = Ds / 4;
-        const int total = nb * per_row;
+        // ---- each warp owns k-range [kw0, kw1) of W_hh . h_{t-1} (one k16 block is the state
+        //      of 16 consecutive units, i.e. of one or two writer CTAs): it polls exactly those
+        //      state words, stages them and multiplies them at once, so the tensor work on early
+        //      k-ranges overlaps the wait for late writers
+        const int kw0 = (nk * warp) / kGruWarps, kw1 = (nk * (warp + 1)) / kGruWarps;
+        const int q0 = kw0 * 4, q1 = min(kw1 * 4, Ds / 4);  // 4-word columns of the range
+        const int ncq = max(0, q1 - q0);
+        const int total = nb * ncq;
         bool got = true;
-        for (int e0 = tid; e0 < total && got; e0 += 8 * kGruThreads) {
+        for (int e0 = lane; e0 < total && got; e0 += 8 * 32) {
           uint4 v[8];
 #pragma unroll
           for (int i = 0; i < 8; ++i) {  // issue every load first, then check the flags
-            const int e = e0 + i * kGruThreads;
+            const int e = e0 + i * 32;
             if (e < total) {
-              const size_t m = static_cast<size_t>(b0 + c0 + e / per_row) * K + (t - 1);
-              v[i] = ld_relaxed_v4(p.hx + m * Ds + (e % per_row) * 4);
+              const size_t m = static_cast<size_t>(b0 + c0 + e / ncq) * K + (t - 1);
+              v[i] = ld_relaxed_v4(p.hx + m * Ds + (q0 + e % ncq) * 4);
             }
           }
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
-            const int e = e0 + i * kGruThreads;
+            const int e = e0 + i * 32;
             if (e < total && got) {
-              const int bb = e / per_row, c4 = e % per_row;
+              const int bb = e / ncq, cq = q0 + e % ncq;
               if ((v[i].x & v[i].y & v[i].z & v[i].w & 1u) == 0u) {
                 const size_t m = static_cast<size_t>(b0 + c0 + bb) * K + (t - 1);
-                got = poll_v4(p.hx + m * Ds + c4 * 4, v[i]);
+                got = poll_v4(p.hx + m * Ds + cq * 4, v[i]);
               }
-              *reinterpret_cast<uint2*>(hsm + static_cast<size_t>(bb) * ldw + c4 * 4) =
+              *reinterpret_cast<uint2*>(hsm + static_cast<size_t>(bb) * ldw + cq * 4) =
                   make_uint2(pack_hi_halves(v[i].x, v[i].y), pack_hi_halves(v[i].z, v[i].w));
             }
           }
         }
+        got = __all_sync(0xffffffffu, got);
+        __syncwarp();
+        if (got) {
+          float acc[kMaxMt][kMaxNt][4];
+#pragma unroll
+          for (int a = 0; a < kMaxMt; ++a)
+#pragma unroll
+            for (int b = 0; b < kMaxNt; ++b) acc[a][b][0] = acc[a][b][1] = acc[a][b][2] = acc[a][b][3] = 0.f;
+          const __nv_bfloat16* abase = whh + static_cast<size_t>(lane & 15) * ldw + (lane >> 4) * 8;
+          const __nv_bfloat16* bbase = hsm + static_cast<size_t>(lane & 7) * ldw + ((lane >> 3) & 1) * 8;
+          for (int kb = kw0; kb < kw1; ++kb) {
+            uint32_t bf[kMaxNt][2];
+#pragma unroll
+            for (int nt = 0; nt < kMaxNt; ++nt)
+              if (nt < nt_count) ldmatrix_x2(bf[nt], bbase + static_cast<size_t>(nt * 8) * ldw + kb * 16);
+#pragma unroll
+            for (int mt = 0; mt < kMaxMt; ++mt) {
+              if (mt >= L.mt) break;
+              uint32_t af[4];
+              ldmatrix_x4(af, abase + static_cast<size_t>(mt * 16) * ldw + kb * 16);
+#pragma unroll
+              for (int nt = 0; nt < kMaxNt; ++nt)
+                if (nt < nt_count) mma_16816(acc[mt][nt], af, bf[nt]);
+            }
+          }
+          const int g = lane >> 2, tq = lane & 3;
+#pragma unroll
+          for (int mt = 0; mt < kMaxMt; ++mt) {
+            if (mt >= L.mt) break;
+#pragma unroll
+            for (int nt = 0; nt < kMaxNt; ++nt) {
+              if (nt >= nt_count) continue;
+              float* out = red + (static_cast<size_t>(warp) * tiles + mt * nt_count + nt) * 128;
+              out[g * 8 + 2 * tq] = acc[mt][nt][0];
+              out[g * 8 + 2 * tq + 1] = acc[mt][nt][1];
+              out[(g + 8) * 8 + 2 * tq] = acc[mt][nt][2];
+              out[(g + 8) * 8 + 2 * tq + 1] = acc[mt][nt][3];
+            }
+          }
+        }
+        GRU_TRACE(t, 4);
         if (__syncthreads_or(!got)) {
           set_status(p.status, kStatusTimeout);
           ok = false;
           break;
         }
         GRU_TRACE(t, 1);
-        // ---- g = W_hh[rows] . h_{t-1} on the tensor cores
-        // each warp runs up to kChains (tile, k-slice) tasks at once: independent accumulator
-        // chains hide the latency of mma.sync
-        const int ntasks = tiles * ks;
-        const int kper = nk / ks;
-        for (int t0 = warp; t0 < ntasks; t0 += kChains * kGruWarps) {
-          float acc[kChains][4];
-          const __nv_bfloat16* arow[kChains];
-          const __nv_bfloat16* brow[kChains];
-          int kbeg[kChains], kend[kChains];
+        // ---- sum the eight k-range partials of every tile
+        for (int e = tid; e < tiles * 128; e += kGruThreads) {
+          const int tile = e / 128, w = e % 128;
+          float sum = 0.f;
 #pragma unroll
-          for (int c = 0; c < kChains; ++c) {
-            const int task = t0 + c * kGruWarps;
-            const int tile = task % tiles, ksl = task / tiles;
-            acc[c][0] = acc[c][1] = acc[c][2] = acc[c][3] = 0.f;
-            arow[c] = whh + static_cast<size_t>((tile % L.mt) * 16 + (lane & 15)) * ldw + (lane >> 4) * 8;
-            brow[c] = hsm + static_cast<size_t>((tile / L.mt) * 8 + (lane & 7)) * ldw + ((lane >> 3) & 1) * 8;
-            kbeg[c] = ksl * kper;
-            kend[c] = task < ntasks ? ((ksl == ks - 1) ? nk : kbeg[c] + kper) : kbeg[c];
-          }
-          const int steps = nk - (ks - 1) * kper;  // the longest slice
-          for (int i = 0; i < steps; ++i) {
-#pragma unroll
-            for (int c = 0; c < kChains; ++c) {
-              if (kbeg[c] + i < kend[c]) {
-                uint32_t a[4], b[2];
-                ldmatrix_x4(a, arow[c] + (kbeg[c] + i) * 16);
-                ldmatrix_x2(b, brow[c] + (kbeg[c] + i) * 16);
-                mma_16816(acc[c], a, b);
-              }
-            }
-          }
-          const int g = lane >> 2, tq = lane & 3;
-#pragma unroll
-          for (int c = 0; c < kChains; ++c) {
-            const int task = t0 + c * kGruWarps;
-            if (task >= ntasks) continue;
-            const int tile = task % tiles;
-            float* out;
-            int ld;
-            if (ks == 1) {
-              out = gsm + static_cast<size_t>((tile % L.mt) * 16) * kGsmLd + (tile / L.mt) * 8;
-              ld = kGsmLd;
-            } else {
-              out = red + static_cast<size_t>(task) * 128;
-              ld = 8;
-            }
-            out[g * ld + 2 * tq] = acc[c][0];
-            out[g * ld + 2 * tq + 1] = acc[c][1];
-            out[(g + 8) * ld + 2 * tq] = acc[c][2];
-            out[(g + 8) * ld + 2 * tq + 1] = acc[c][3];
-          }
+          for (int ww = 0; ww < kGruWarps; ++ww) sum += red[(static_cast<size_t>(ww) * tiles + tile) * 128 + w];
+          const int mt = tile / nt_count, nt = tile % nt_count;
+          gsm[static_cast<size_t>(mt * 16 + w / 8) * kGsmLd + nt * 8 + (w % 8)] = sum;
         }
-        GRU_TRACE(t, 4);
-        __syncthreads();
         GRU_TRACE(t, 5);
-        if (ks > 1) {
-          for (int e = tid; e < tiles * 128; e += kGruThreads) {
-            const int tile = e / 128, w = e % 128;
-            float s = 0.f;
-            for (int ksl = 0; ksl < ks; ++ksl) s += red[static_cast<size_t>(ksl * tiles + tile) * 128 + w];
-            const int mt = tile % L.mt, nt = tile / L.mt;
-            gsm[static_cast<size_t>(mt * 16 + w / 8) * kGsmLd + nt * 8 + (w % 8)] = s;
-          }
-          __syncthreads();
-        }
+        __syncthreads();
       }
       GRU_TRACE(t, 2);
       // ---- gates and the new state (torch.nn.GRU convention); publish the tagged state
@@ -459,21 +450,21 @@ __global__ void __launch_bounds__(kGruThreads) gru_kernel(const GruParams p) {
 
 GruPlan gru_plan(int B, int Ds, int num_sms) {
   GruPlan g{};
-  if (B <= 8) {
-    g.gu = Ds < 128 ? Ds : 128;
-    g.gb = 1;
-  } else {
-    g.gu = Ds < 64 ? Ds : 64;
-    g.gb = 2;
-  }
-  while (g.gu * g.gb > num_sms && g.gu > 1) g.gu /= 2;
-  g.units = (Ds + g.gu - 1) / g.gu;
+  // 8 units (2 gate tiles) per CTA for small batches, 16 (3 gate tiles) otherwise
+  g.units = B <= 8 ? 8 : 16;
   g.gu = (Ds + g.units - 1) / g.units;
+  if (g.gu > num_sms) {
+    g.units = 16;
+    g.gu = (Ds + g.units - 1) / g.units;
+    if (g.gu > num_sms) return g;  // smem == 0: unsupported
+  }
+  g.gb = B <= 8 ? 1 : (num_sms / g.gu >= 2 ? 2 : 1);
   g.bc = (B + g.gb - 1) / g.gb;
   g.gb = (B + g.bc - 1) / g.bc;
   const GruSmem L = gru_layout(Ds, g.units, g.bc);
   g.smem = L.total <= 220 * 1024 ? L.total : 0;
   if (static_cast<long long>(L.chunk) * g.units > static_cast<long long>(kGatePairsPerThread) * kGruThreads) g.smem = 0;
+  if (L.mt > kMaxMt || L.chunk / 8 > kMaxNt) g.smem = 0;
   return g;
 }
 
