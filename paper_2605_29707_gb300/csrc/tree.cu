@@ -2,17 +2,19 @@
 // then the best-first draft tree (the "Tree" cost of the paper's Fig. 1).
 //
 // Merge: one CTA per draft row (sequence b, position j).  Thread c reads chunk c's record
-// (running max, sum of exp, top-KMAX list; field-major, so the loads are coalesced), the CTA
-// reduces lse = max + log(sum) and extracts the k best (value desc, id asc) tokens; logp =
-// logit - lse.
+// (running max, sum of exp, the head of its top-KMAX list; field-major, so the loads are
+// coalesced).  The CTA reduces lse = max + log(sum); the k best (value desc, id asc) tokens
+// come from a bitonic merge of the chunks' sorted lists, first across the lanes of each warp
+// (butterfly), then across the warps.  logp = logit - lse.
 // Tree: the CTA that merges the last row of a sequence (atomic counter) selects N nodes
 // best-first with one warp.  The frontier is every child (from its position's top-k list) of
 // the anchor or of an already selected node that is not selected yet; the next node is the
 // frontier entry with the greatest (score, lower token id, lower parent index).  Each expanded
-// node ("slot") caches its best remaining child.  Children of a slot have non-increasing scores
-// (sorted log-probs plus the same parent score), so the best remaining child is the first
-// unselected one, or a lower-token child of exactly the same score; one lane refreshes a slot
-// by that short scan.
+// node ("slot") caches its best remaining child; after a pop only the popped slot and the new
+// node need a new best child.  A slot's children have non-increasing scores (its position's
+// sorted log-probs plus one parent score), so that child is the first unselected entry unless
+// a later unselected entry has exactly the same score and a lower token; every lane computes
+// it the same way, and one ballot finds such ties.
 #include <math.h>
 
 #include "kernels.h"
@@ -36,17 +38,61 @@ __device__ __forceinline__ void warp_argmax2(uint32_t hi, uint32_t lo, uint32_t&
   src = __ffs(ball) - 1;
 }
 
-template <int KM>
-__device__ __forceinline__ void insert_keyed(float (&tv)[KM], int (&ti)[KM], float x, int id) {
+// Total order of (logit, token) candidates: greater logit first, then lower token id.  Padding
+// entries carry (-inf, -1), which sorts after every real entry.
+__device__ __forceinline__ bool better(float a, int ia, float b, int ib) {
+  return a > b || (a == b && static_cast<unsigned>(ia) < static_cast<unsigned>(ib));
+}
+
+// Sort a bitonic sequence best-first (half-cleaners of decreasing span).
+template <int KK>
+__device__ __forceinline__ void bitonic_clean(float (&v)[KK], int (&id)[KK]) {
 #pragma unroll
-  for (int q = 0; q < KM; ++q) {
-    const bool sw = x > tv[q] || (x == tv[q] && (unsigned)id < (unsigned)ti[q]);
-    const float a = tv[q];
-    const int b = ti[q];
-    tv[q] = sw ? x : a;
-    ti[q] = sw ? id : b;
-    x = sw ? a : x;
-    id = sw ? b : id;
+  for (int h = KK / 2; h > 0; h >>= 1) {
+#pragma unroll
+    for (int q = 0; q < KK; ++q) {
+      if ((q & h) == 0) {
+        const int r = q + h;
+        const bool keep = better(v[q], id[q], v[r], id[r]);
+        const float a = v[q], b = v[r];
+        const int ia = id[q], ib = id[r];
+        v[q] = keep ? a : b;
+        id[q] = keep ? ia : ib;
+        v[r] = keep ? b : a;
+        id[r] = keep ? ib : ia;
+      }
+    }
+  }
+}
+
+// (v, id) <- best KK of the union of two best-first lists: the half-cleaner of a ++ reverse(b)
+// keeps the KK best as a bitonic sequence, which bitonic_clean sorts.
+template <int KK>
+__device__ __forceinline__ void merge_lists(float (&v)[KK], int (&id)[KK], const float (&w)[KK], const int (&iw)[KK]) {
+#pragma unroll
+  for (int q = 0; q < KK; ++q) {
+    const float b = w[KK - 1 - q];
+    const int ib = iw[KK - 1 - q];
+    const bool keep = better(v[q], id[q], b, ib);
+    v[q] = keep ? v[q] : b;
+    id[q] = keep ? id[q] : ib;
+  }
+  bitonic_clean<KK>(v, id);
+}
+
+// Butterfly over lanes l ^ o for o = span/2 .. 1: every lane of each span-wide group ends with
+// the best KK entries of the group's lists.
+template <int KK>
+__device__ __forceinline__ void butterfly_lists(float (&v)[KK], int (&id)[KK], int span) {
+  for (int o = span >> 1; o; o >>= 1) {
+    float w[KK];
+    int iw[KK];
+#pragma unroll
+    for (int q = 0; q < KK; ++q) {
+      w[q] = __shfl_xor_sync(0xffffffffu, v[q], o);
+      iw[q] = __shfl_xor_sync(0xffffffffu, id[q], o);
+    }
+    merge_lists<KK>(v, id, w, iw);
   }
 }
 
@@ -57,48 +103,118 @@ __device__ __forceinline__ void lse_merge(float& mx, float& se, float om, float 
   mx = nm;
 }
 
+// Tree slots.  Slot 0 is the anchor, slot i + 1 the i-th selected node.  Slot s belongs to
+// lane s % 32 of the tree warp: slots 0..31 live in that lane's registers, later ones in these
+// arrays, which only the owner lane reads and writes.
 struct TreeSlots {
   float score[kMaxN + 1];
   int depth[kMaxN + 1];
-  unsigned mask[kMaxN + 1];
-  unsigned hi[kMaxN + 1];
-  unsigned lo[kMaxN + 1];
-  int j[kMaxN + 1];
+  unsigned mask[kMaxN + 1];  // children already selected (bit j: entry j of the top-k list)
+  unsigned hi[kMaxN + 1];    // cached best child: f32_ord(score), 0 when the slot has none left
+  unsigned lo[kMaxN + 1];    // (0x3FFFFF - token) << 10 | (0x3FF - slot): lower token, then slot
+  int j[kMaxN + 1];          // the cached child's index in its position's top-k list
+  int parent[kMaxN + 1];
+  int token[kMaxN + 1];
 };
 
-// Best remaining child of slot s (one thread).  The caller passes the slot's depth d, score
-// and popped mask in registers; children of a slot have non-increasing scores, so the best
-// remaining one is the first unpopped child, or an unpopped child of exactly the same score
-// with a lower token id.
-__device__ __forceinline__ void refresh_slot(TreeSlots& S, int s, int d, float base, unsigned mask, const float* lp,
-                                             const int* ids, int K, int k) {
-  if (d >= K) { S.hi[s] = 0u; return; }
-  const unsigned all = (k == 32) ? 0xffffffffu : ((1u << k) - 1u);
-  const unsigned avail = ~mask & all;
-  if (avail == 0u) { S.hi[s] = 0u; return; }
-  const int j0 = __ffs(avail) - 1;
-  const float* row_lp = lp + d * k;
-  const int* row_id = ids + d * k;
-  const float best_sc = base + row_lp[j0];
-  int best_j = j0, best_tok = row_id[j0];
-  for (int j = j0 + 1; j < k; ++j) {
-    const float sc = base + row_lp[j];
-    if (sc < best_sc) break;
-    if (!((mask >> j) & 1u) && row_id[j] < best_tok) { best_j = j; best_tok = row_id[j]; }
+struct SlotState {
+  float score;
+  int depth;
+  unsigned mask;
+  uint32_t hi, lo;
+  int j, parent, token;
+};
+
+__device__ __forceinline__ void slot_put(TreeSlots& S, SlotState& reg, int slot, const SlotState& v) {
+  if (slot < 32) {
+    reg = v;
+  } else {
+    S.score[slot] = v.score;
+    S.depth[slot] = v.depth;
+    S.mask[slot] = v.mask;
+    S.hi[slot] = v.hi;
+    S.lo[slot] = v.lo;
+    S.j[slot] = v.j;
+    S.parent[slot] = v.parent;
+    S.token[slot] = v.token;
   }
-  S.hi[s] = f32_ord(best_sc);
-  S.lo[s] = ((0x3FFFFFu - static_cast<unsigned>(best_tok)) << 10) | (0x3FFu - static_cast<unsigned>(s));
-  S.j[s] = best_j;
 }
 
-template <int KM>
+__device__ __forceinline__ SlotState slot_get(const TreeSlots& S, const SlotState& reg, int slot) {
+  if (slot < 32) return reg;
+  SlotState v;
+  v.score = S.score[slot];
+  v.depth = S.depth[slot];
+  v.mask = S.mask[slot];
+  v.hi = S.hi[slot];
+  v.lo = S.lo[slot];
+  v.j = S.j[slot];
+  v.parent = S.parent[slot];
+  v.token = S.token[slot];
+  return v;
+}
+
+// Cached best child of a slot from its first unselected entry j0 (score s0) and the entries
+// that tie it (bit mask `ties`): the lowest token among them.  (0, 0) when j0 < 0.
+__device__ __forceinline__ void child_key(int j0, float s0, unsigned ties, const int* row_ids, int slot,
+                                          uint32_t& hi, uint32_t& lo, int& jb) {
+  hi = 0u;
+  lo = 0u;
+  jb = 0;
+  if (j0 < 0) return;
+  int tb = row_ids[j0];
+  jb = j0;
+  for (unsigned t = ties; t; t &= t - 1u) {  // rare: an exact tie in fp32
+    const int j = __ffs(t) - 1;
+    const int tt = row_ids[j];
+    if (tt < tb) { tb = tt; jb = j; }
+  }
+  hi = f32_ord(s0);
+  lo = ((0x3FFFFFu - static_cast<unsigned>(tb)) << 10) | (0x3FFu - static_cast<unsigned>(slot));
+}
+
+// Best remaining children of two slots a and b (available-entry masks av*, 0 for none; rows
+// r* of the top-k lists, clamped to a loaded row; parent scores b*), identical on every lane.
+// The tie test runs one entry per lane: half a warp per slot when k <= 16.
+__device__ __forceinline__ void best_children(const float* lp, const int* ids, int k, int lane, int ra, float ba,
+                                              unsigned ava, int sa, int rb, float bb, unsigned avb, int sb,
+                                              uint32_t& ha, uint32_t& la, int& ja, uint32_t& hb, uint32_t& lb,
+                                              int& jb) {
+  const float* pa = lp + ra * k;
+  const float* pb = lp + rb * k;
+  const int a0 = ava ? __ffs(ava) - 1 : -1;
+  const int b0 = avb ? __ffs(avb) - 1 : -1;
+  const float sa0 = ba + pa[a0 < 0 ? 0 : a0];
+  const float sb0 = bb + pb[b0 < 0 ? 0 : b0];
+  unsigned ta, tb;
+  if (k <= 16) {
+    const bool up = lane >= 16;
+    const int j = lane & 15;
+    const float x = (up ? bb : ba) + (up ? pb : pa)[j];  // j < 16 <= row stride bound of the array
+    const unsigned av = up ? avb : ava;
+    const int j0 = up ? b0 : a0;
+    const bool tie = j0 >= 0 && j > j0 && ((av >> j) & 1u) && x == (up ? sb0 : sa0);
+    const unsigned t = __ballot_sync(0xffffffffu, tie);
+    ta = t & 0xffffu;
+    tb = t >> 16;
+  } else {
+    const float xa = ba + pa[lane], xb = bb + pb[lane];
+    ta = __ballot_sync(0xffffffffu, a0 >= 0 && lane > a0 && ((ava >> lane) & 1u) && xa == sa0);
+    tb = __ballot_sync(0xffffffffu, b0 >= 0 && lane > b0 && ((avb >> lane) & 1u) && xb == sb0);
+  }
+  child_key(a0, sa0, ta, ids + ra * k, sa, ha, la, ja);
+  child_key(b0, sb0, tb, ids + rb * k, sb, hb, lb, jb);
+}
+
+template <int KM, int KK>
 __global__ void __launch_bounds__(kMergeThreads) merge_tree_kernel(const TreeParams p) {
   constexpr int F = 2 + 2 * KM;
   constexpr int kWarps = kMergeThreads / 32;
+  static_assert(KK <= KM && kWarps <= 32, "list and warp counts");
   __shared__ float s_mx[kWarps], s_se[kWarps];
   __shared__ int s_last;
-  __shared__ float s_cv[kWarps * kMaxTopk];
-  __shared__ int s_ci[kWarps * kMaxTopk];
+  __shared__ float s_cv[kWarps * KK];
+  __shared__ int s_ci[kWarps * KK];
   __shared__ float s_lp[kMaxK * kMaxTopk];
   __shared__ int s_id[kMaxK * kMaxTopk];
   __shared__ TreeSlots S;
@@ -113,27 +229,27 @@ __global__ void __launch_bounds__(kMergeThreads) merge_tree_kernel(const TreePar
   const int* ibase = reinterpret_cast<const int*>(base);
 
   // ------------------------------------------------------------ this thread's chunks
+  // Only the first k entries of each chunk's (sorted) list can reach the row's top k.
   float mx = -INFINITY, se = 0.f;
-  float tv[KM];
-  int ti[KM];
+  float tv[KK];
+  int ti[KK];
 #pragma unroll
-  for (int q = 0; q < KM; ++q) { tv[q] = -INFINITY; ti[q] = -1; }
+  for (int q = 0; q < KK; ++q) { tv[q] = -INFINITY; ti[q] = -1; }
   for (int c = tid; c < nch; c += kMergeThreads) {
     const float cm = __ldg(base + c), cs = __ldg(base + nch + c);
-    float v[KM];
-    int id[KM];
+    float v[KK];
+    int id[KK];
 #pragma unroll
-    for (int q = 0; q < KM; ++q) {
-      v[q] = __ldg(base + (2 + q) * nch + c);
-      id[q] = __ldg(ibase + (2 + KM + q) * nch + c);
+    for (int q = 0; q < KK; ++q) {
+      v[q] = q < k ? __ldg(base + (2 + q) * nch + c) : -INFINITY;
+      id[q] = q < k ? __ldg(ibase + (2 + KM + q) * nch + c) : -1;
     }
     lse_merge(mx, se, cm, cs);
     if (c == tid) {
 #pragma unroll
-      for (int q = 0; q < KM; ++q) { tv[q] = v[q]; ti[q] = id[q]; }
+      for (int q = 0; q < KK; ++q) { tv[q] = v[q]; ti[q] = id[q]; }
     } else {
-#pragma unroll
-      for (int q = 0; q < KM; ++q) insert_keyed<KM>(tv, ti, v[q], id[q]);
+      merge_lists<KK>(tv, ti, v, id);
     }
   }
 
@@ -145,44 +261,34 @@ __global__ void __launch_bounds__(kMergeThreads) merge_tree_kernel(const TreePar
     lse_merge(mx, se, om, os);
   }
   if (lane == 0) { s_mx[warp] = mx; s_se[warp] = se; }
-  __syncthreads();
-  mx = -INFINITY;
-  se = 0.f;
-#pragma unroll
-  for (int w = 0; w < kWarps; ++w) lse_merge(mx, se, s_mx[w], s_se[w]);
-  const float lse = mx + logf(se);
 
   // ------------------------------------------------------------ k best: per warp, then across warps
-  for (int q = 0; q < k; ++q) {
-    uint32_t mhi, mlo;
-    int src;
-    warp_argmax2(f32_ord(tv[0]), ~static_cast<uint32_t>(ti[0]), mhi, mlo, src);
-    const float val = __shfl_sync(0xffffffffu, tv[0], src);
-    const int id = __shfl_sync(0xffffffffu, ti[0], src);
-    if (lane == src) {
+  butterfly_lists<KK>(tv, ti, 32);
+  if (lane == 0) {
 #pragma unroll
-      for (int i = 0; i + 1 < KM; ++i) { tv[i] = tv[i + 1]; ti[i] = ti[i + 1]; }
-      tv[KM - 1] = -INFINITY;
-      ti[KM - 1] = -1;
-    }
-    if (lane == 0) { s_cv[warp * kMaxTopk + q] = val; s_ci[warp * kMaxTopk + q] = id; }
+    for (int q = 0; q < KK; ++q) { s_cv[warp * KK + q] = tv[q]; s_ci[warp * KK + q] = ti[q]; }
   }
   __syncthreads();
   if (warp == 0) {
-    int ptr = 0;  // lane w < kWarps walks warp w's sorted candidate list
-    for (int q = 0; q < k; ++q) {
-      uint32_t hi = 0u, lo = 0u;
-      if (lane < kWarps && ptr < k) {
-        hi = f32_ord(s_cv[lane * kMaxTopk + ptr]);
-        lo = ~static_cast<uint32_t>(s_ci[lane * kMaxTopk + ptr]);
-      }
-      uint32_t mhi, mlo;
-      int src;
-      warp_argmax2(hi, lo, mhi, mlo, src);
-      if (lane == src) {
-        p.topk_ids[static_cast<size_t>(m) * k + q] = s_ci[lane * kMaxTopk + ptr];
-        p.topk_logp[static_cast<size_t>(m) * k + q] = s_cv[lane * kMaxTopk + ptr] - lse;
-        ++ptr;
+    mx = -INFINITY;
+    se = 0.f;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) lse_merge(mx, se, s_mx[w], s_se[w]);
+    const float lse = mx + logf(se);
+    const int src = lane < kWarps ? lane : 0;
+#pragma unroll
+    for (int q = 0; q < KK; ++q) {
+      tv[q] = lane < kWarps ? s_cv[src * KK + q] : -INFINITY;
+      ti[q] = lane < kWarps ? s_ci[src * KK + q] : -1;
+    }
+    butterfly_lists<KK>(tv, ti, kWarps);
+    if (lane == 0) {
+#pragma unroll
+      for (int q = 0; q < KK; ++q) {
+        if (q < k) {
+          p.topk_ids[static_cast<size_t>(m) * k + q] = ti[q];
+          p.topk_logp[static_cast<size_t>(m) * k + q] = tv[q] - lse;
+        }
       }
     }
   }
@@ -203,49 +309,101 @@ __global__ void __launch_bounds__(kMergeThreads) merge_tree_kernel(const TreePar
   if (warp != 0) return;
 
   // ------------------------------------------------------------ tree (warp 0)
+  // Row reads below stay inside s_lp / s_id: rows are clamped to K - 1 and entries to
+  // j < max(k, 16) <= 32, and (K - 1) * k + 31 < kMaxK * kMaxTopk; what a clamped read returns
+  // is discarded by the masks.
   const size_t ob = static_cast<size_t>(b) * N;
-  if (lane == 0) {
-    S.score[0] = 0.f;
-    S.depth[0] = 0;
-    S.mask[0] = 0u;
-    refresh_slot(S, 0, 0, 0.f, 0u, s_lp, s_id, K, k);
+  const unsigned all = (k == 32) ? 0xffffffffu : ((1u << k) - 1u);
+  SlotState mine;  // slot `lane`
+  mine.hi = 0u;
+  mine.lo = 0u;
+  {
+    uint32_t ha, la, hb, lb;
+    int ja, jb;
+    best_children(s_lp, s_id, k, lane, 0, 0.f, all, 0, 0, 0.f, 0u, 0, ha, la, ja, hb, lb, jb);
+    if (lane == 0) {
+      mine.score = 0.f;
+      mine.depth = 0;
+      mine.mask = 0u;
+      mine.hi = ha;
+      mine.lo = la;
+      mine.j = ja;
+      mine.parent = -1;
+      mine.token = -1;
+    }
   }
-  __syncwarp();
+  int n_sel = 0;
   for (int i = 0; i < N; ++i) {
+    // best cached child over this lane's slots, with that slot's state
     uint32_t hi = 0u, lo = 0u;
     int sb = -1;
-    for (int s2 = lane; s2 <= i; s2 += 32) {
+    SlotState w;
+    w.depth = 0;
+    w.score = 0.f;
+    w.mask = 0u;
+    w.j = 0;
+    if (lane <= i && mine.hi != 0u) { hi = mine.hi; lo = mine.lo; sb = lane; w = mine; }
+    for (int s2 = lane + 32; s2 <= i; s2 += 32) {
       const uint32_t h = S.hi[s2], l = S.lo[s2];
-      if (h > hi || (h == hi && h != 0u && l > lo)) { hi = h; lo = l; sb = s2; }
+      if (h > hi || (h == hi && h != 0u && l > lo)) {
+        hi = h;
+        lo = l;
+        sb = s2;
+        w = slot_get(S, mine, s2);
+      }
     }
     uint32_t mhi, mlo;
     int src;
     warp_argmax2(hi, lo, mhi, mlo, src);
+    if (mhi == 0u) break;  // no frontier left (the host keeps N within the tree's capacity)
     const int s = __shfl_sync(0xffffffffu, sb, src);
-    if (lane == 0) {
-      const int jj = S.j[s];
-      const int d = S.depth[s];
-      const float base_s = S.score[s];
-      const unsigned mask_s = S.mask[s] | (1u << jj);
-      const int tok = s_id[d * k + jj];
-      const float sc = base_s + s_lp[d * k + jj];
-      p.tree_parent[ob + i] = s - 1;
-      p.tree_token[ob + i] = tok;
-      p.tree_depth[ob + i] = d + 1;
-      if (p.tree_score) p.tree_score[ob + i] = sc;
-      S.mask[s] = mask_s;
-      S.score[i + 1] = sc;
-      S.depth[i + 1] = d + 1;
-      S.mask[i + 1] = 0u;
-      refresh_slot(S, s, d, base_s, mask_s, s_lp, s_id, K, k);
-      refresh_slot(S, i + 1, d + 1, sc, 0u, s_lp, s_id, K, k);
+    const int jj = __shfl_sync(0xffffffffu, w.j, src);
+    const int d = __shfl_sync(0xffffffffu, w.depth, src);
+    const float base_s = __shfl_sync(0xffffffffu, w.score, src);
+    const unsigned mask_s = __shfl_sync(0xffffffffu, w.mask, src) | (1u << jj);
+    const int tok = s_id[d * k + jj];
+    const float sc = base_s + s_lp[d * k + jj];
+    // new best children of the popped slot s (row d) and of the new node i + 1 (row d + 1)
+    const int rn = d + 1 < K ? d + 1 : K - 1;
+    uint32_t ha, la, hb, lb;
+    int ja, jb;
+    best_children(s_lp, s_id, k, lane, d, base_s, ~mask_s & all, s, rn, sc, d + 1 < K ? all : 0u, i + 1, ha, la,
+                  ja, hb, lb, jb);
+    if (lane == src) {
+      w.mask = mask_s;
+      w.hi = ha;
+      w.lo = la;
+      w.j = ja;
+      slot_put(S, mine, s, w);
     }
-    __syncwarp();
+    if (lane == ((i + 1) & 31)) {
+      SlotState v;
+      v.score = sc;
+      v.depth = d + 1;
+      v.mask = 0u;
+      v.hi = hb;
+      v.lo = lb;
+      v.j = jb;
+      v.parent = s - 1;
+      v.token = tok;
+      slot_put(S, mine, i + 1, v);
+    }
+    n_sel = i + 1;
+  }
+  // each owner writes its nodes: output i is slot i + 1
+  for (int sl = lane; sl <= n_sel; sl += 32) {
+    if (sl == 0) continue;
+    const SlotState v = slot_get(S, mine, sl);
+    const int i = sl - 1;
+    p.tree_parent[ob + i] = v.parent;
+    p.tree_token[ob + i] = v.token;
+    p.tree_depth[ob + i] = v.depth;
+    if (p.tree_score) p.tree_score[ob + i] = v.score;
   }
 }
 
 cudaError_t launch_merge_tree(const TreeParams& p, cudaStream_t stream) {
-  if (p.K > kMaxK || p.k > kMaxTopk || p.N > kMaxN) return cudaErrorInvalidValue;
+  if (p.K > kMaxK || p.k > kMaxTopk || p.k > p.kmax || p.N > kMaxN) return cudaErrorInvalidValue;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.B * p.K);
   cfg.blockDim = dim3(kMergeThreads);
@@ -256,9 +414,11 @@ cudaError_t launch_merge_tree(const TreeParams& p, cudaStream_t stream) {
   cfg.attrs = attr;
   cfg.numAttrs = DOMINO_TREE_PDL ? 1 : 0;
   cudaError_t e;
-  if (p.kmax == 16) e = cudaLaunchKernelEx(&cfg, merge_tree_kernel<16>, p);
-  else if (p.kmax == 32) e = cudaLaunchKernelEx(&cfg, merge_tree_kernel<32>, p);
-  else return cudaErrorInvalidValue;
+  if (p.kmax == 32) e = cudaLaunchKernelEx(&cfg, merge_tree_kernel<32, 32>, p);
+  else if (p.kmax != 16) return cudaErrorInvalidValue;
+  else if (p.k <= 4) e = cudaLaunchKernelEx(&cfg, merge_tree_kernel<16, 4>, p);
+  else if (p.k <= 8) e = cudaLaunchKernelEx(&cfg, merge_tree_kernel<16, 8>, p);
+  else e = cudaLaunchKernelEx(&cfg, merge_tree_kernel<16, 16>, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
