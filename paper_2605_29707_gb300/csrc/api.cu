@@ -54,6 +54,7 @@ struct Plan {
   bool swap;
   int bn, kmax, rec, tok_tiles, w_tiles, nchunks, w_per_chunk, grid;
   StorePlan xg, ug;
+  bool chain;  // head kernels launched as a programmatic-dependent chain (small M with overlap)
   dm::GruPlan gru;
   bool u_in_gru;  // small M: u finished inside the GRU kernel; large M: W1 GEMM + finalize
   bool overlap;   // vocab GEMM launched as a programmatic dependent of the GRU (deferred W2)
@@ -178,6 +179,11 @@ int make_plan(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head
     }
     p.overlap = p.u_in_gru && vsm > 0 && (p.defer_tiles + 2) * p.bn <= 512 &&
                 static_cast<size_t>(vsm) + p.gru.smem + 2048 <= 228 * 1024;
+    // With the overlap, chain the whole head: the gather, both projection GEMMs and the GRU
+    // each let the next kernel launch early, so that the GRU's CTAs (and with them the
+    // vocabulary stream) start while the projections still run.
+    p.chain = p.overlap && p.xg.swap && p.ug.swap && dm::tc_store_chained_smem(p.xg.bn) > 0 &&
+              dm::tc_store_chained_smem(p.ug.bn) > 0;
   }
   p.tmem_cols = pow2_at_least(p.overlap ? (p.defer_tiles + 2) * p.bn : 2 * p.bn, 32);
 
@@ -316,8 +322,10 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
       tp.tmem_cols = pow2_at_least(2 * g.bn, 32);
       tp.out = xpart; tp.ld_out = 3 * Ds;
       tp.status = status;
+      tp.pdl_wait = P.chain ? 1 : 0;  // E comes from the gather
       ts = timing_open(DOMINO_KERNEL_GRU_INPUT, st);
-      rc = cuda_rc(dm::launch_tc_gemm(dm::kModeStore, g.bn, g.swap, 16, maps, tp, g.grid, st));
+      rc = cuda_rc(P.chain ? dm::launch_tc_store_chained(g.bn, maps, tp, g.grid, st)
+                           : dm::launch_tc_gemm(dm::kModeStore, g.bn, g.swap, 16, maps, tp, g.grid, st));
       timing_close(ts, st);
       if (rc) return rc;
     }
@@ -345,8 +353,11 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
       tp.tmem_cols = pow2_at_least(2 * g.bn, 32);
       tp.out = upart; tp.ld_out = R;
       tp.status = status;
+      const bool chained = P.chain && !both;
+      tp.pdl_wait = chained ? 2 : 0;  // reads nothing the X GEMM writes; completes after it
       const int slot = timing_open(DOMINO_KERNEL_W1_HIDDEN, st);
-      const int r = cuda_rc(dm::launch_tc_gemm(dm::kModeStore, g.bn, g.swap, 16, maps, tp, g.grid, st));
+      const int r = cuda_rc(chained ? dm::launch_tc_store_chained(g.bn, maps, tp, g.grid, st)
+                                    : dm::launch_tc_gemm(dm::kModeStore, g.bn, g.swap, 16, maps, tp, g.grid, st));
       timing_close(slot, st);
       return r;
     };
@@ -370,7 +381,7 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
     gr.u = P.u_in_gru ? u : nullptr;
     gr.status = status;
     ts = timing_open(DOMINO_KERNEL_GRU, st);
-    rc = cuda_rc(dm::launch_gru(gr, P.gru, st));
+    rc = cuda_rc(dm::launch_gru(gr, P.gru, st, P.chain));
     timing_close(ts, st);
     if (rc) return rc;
     if (!P.u_in_gru) {

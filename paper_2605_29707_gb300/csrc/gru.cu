@@ -44,6 +44,9 @@ constexpr int kMaxNt = 4;  // 8-sequence tiles per staged chunk
 
 // ---------------------------------------------------------------------------- gather
 __global__ void __launch_bounds__(128) gather_kernel(const GatherParams p) {
+  // the input projection launched after this kernel may start its setup now; it waits for
+  // this grid before it reads E
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int m = blockIdx.x;
   const int id = p.ids[m];
   const bool ok = id >= 0 && id < p.V;
@@ -207,6 +210,10 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
   for (int r = tid; r < L.mt * 16; r += kGruThreads)  // padding columns Ds .. Ds+7 (k tail)
     *reinterpret_cast<uint4*>(whh + static_cast<size_t>(r) * ldw + Ds) = make_uint4(0, 0, 0, 0);
   for (int e = tid; e < L.chunk * (ldw / 8); e += kGruThreads) reinterpret_cast<uint4*>(hsm)[e] = make_uint4(0, 0, 0, 0);
+  // Launched as a programmatic dependent of the projection GEMMs: everything below reads
+  // what they (and, through their own waits, the gather) wrote -- X partials, u partials and
+  // the cleared state words.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   // ---- input-gate sums b_ih + E . W_ih^T for this CTA's rows and units, spread over all
   //      threads (made visible to the CTA by the barrier below)
   const int xs_count = nbc * K * 3 * Uc;
@@ -468,7 +475,7 @@ GruPlan gru_plan(int B, int Ds, int num_sms) {
   return g;
 }
 
-cudaError_t launch_gru(const GruParams& p, const GruPlan& plan, cudaStream_t stream) {
+cudaError_t launch_gru(const GruParams& p, const GruPlan& plan, cudaStream_t stream, bool pdl) {
   if (plan.smem == 0) return cudaErrorInvalidValue;
   static size_t attr_smem = 0;
   if (plan.smem > attr_smem) {
@@ -479,10 +486,27 @@ cudaError_t launch_gru(const GruParams& p, const GruPlan& plan, cudaStream_t str
     if (e != cudaSuccess) return e;
     attr_smem = plan.smem;
   }
-  GruParams pp = p;
-  void* args[] = {&pp};
-  cudaError_t e = cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(gru_kernel),
-                                              dim3(plan.gu * plan.gb), dim3(kGruThreads), args, plan.smem, stream);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(plan.gu * plan.gb);
+  cfg.blockDim = dim3(kGruThreads);
+  cfg.dynamicSmemBytes = plan.smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeCooperative;  // every CTA resident at once (state exchange)
+  attr[0].val.cooperative = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  // A runtime that refuses the pair gets the cooperative launch alone from then on.
+  static bool pdl_refused = false;
+  cfg.numAttrs = (pdl && !pdl_refused) ? 2 : 1;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, gru_kernel, p);
+  if (e != cudaSuccess && cfg.numAttrs == 2) {
+    (void)cudaGetLastError();
+    pdl_refused = true;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, gru_kernel, p);
+  }
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

@@ -29,6 +29,8 @@ struct TcParams {
   int w_evict_first;
   int defer;      // softmax + swap only: number of leading tiles whose second segment waits for
                   // the preceding grid (0 = off); see the producer in tc_gemm.cuh
+  int pdl_wait;   // launched as a programmatic dependent: 1 = wait for the preceding grid before
+                  // the first load, 2 = after the last load (0 = no wait)
   int tmem_cols;  // TMEM columns to allocate (power of two, 32..512)
   const __nv_bfloat16* bias;  // softmax: b2 [V] or nullptr
   float* out;                 // softmax: partial records [M][rec fields][nchunks]; store: [splits][M][ld_out]
@@ -47,6 +49,12 @@ cudaError_t launch_tc_softmax_deferred(int bn, int kmax, const CUtensorMap* maps
                                        cudaStream_t stream);
 // Shared memory one deferred-mode CTA uses (for the co-residency budget).
 int tc_softmax_deferred_smem(int bn, int kmax);
+// Small-M (swap, bn 16..128) store-mode GEMM with four pipeline stages, launched as a
+// programmatic dependent of the preceding kernel (p.pdl_wait says where it waits for it).
+cudaError_t launch_tc_store_chained(int bn, const CUtensorMap* maps, const TcParams& p, int grid,
+                                   cudaStream_t stream);
+// Shared memory one such CTA uses.
+int tc_store_chained_smem(int bn);
 
 // ---------------------------------------------------------------- gather / GRU
 struct GatherParams {
@@ -86,7 +94,9 @@ struct GruPlan {
   size_t smem;  // 0 = unsupported
 };
 GruPlan gru_plan(int B, int Ds, int num_sms);
-cudaError_t launch_gru(const GruParams& p, const GruPlan& plan, cudaStream_t stream);
+// Cooperative launch; with pdl, also as a programmatic dependent of the preceding kernel (the
+// kernel waits for that grid before it reads the projections).
+cudaError_t launch_gru(const GruParams& p, const GruPlan& plan, cudaStream_t stream, bool pdl);
 
 // u = bf16(SiLU(b1 + sum over splits of part)) for the large-batch path.
 struct UFinalParams {

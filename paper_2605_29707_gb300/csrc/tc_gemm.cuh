@@ -43,9 +43,11 @@ struct TcCfg {
   static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kTrBytes + kListBytes + kBarBytes;
   static constexpr int kRec = 2 + 2 * KMAX;
   static_assert(kStages >= 2, "pipeline needs at least two stages");
-  // two CTAs (each with 1 KB of reserved shared memory) never fit on one 228 KB SM, so TMEM
-  // allocation is never contended between CTAs of this kernel
-  static_assert(2 * (kSmemBytes + 1024) > 228 * 1024, "one CTA per SM keeps TMEM allocation uncontended");
+  // CTAs of this kernel that fit on one 228 KB SM (1 KB of shared memory reserved per CTA)
+  // never hold more than the SM's 512 TMEM columns between them.  (Across kernels, see the
+  // trigger after the allocation in the kernel body.)
+  static constexpr int kPerSm = (228 * 1024) / (kSmemBytes + 1024);
+  static_assert(kPerSm <= 1 || kPerSm * kTmemCols <= 512, "co-resident CTAs fit in TMEM");
   static_assert(BN % 16 == 0 && BN >= 16 && BN <= 256, "UMMA N for M = 128");
 };
 
@@ -262,9 +264,6 @@ __global__ void __launch_bounds__(192, ST > 0 ? 2 : 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  // a kernel launched as this grid's programmatic dependent may start now (it waits for this
-  // grid to complete before it reads anything this kernel writes)
-  if (DOMINO_VOCAB_TRIGGER) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
@@ -295,6 +294,11 @@ __global__ void __launch_bounds__(192, ST > 0 ? 2 : 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  // A kernel launched as this grid's programmatic dependent may start now: it waits for this
+  // grid to complete before it reads anything this kernel writes.  The trigger comes after the
+  // TMEM allocation, so a dependent that allocates TMEM on this SM can only wait for columns
+  // this CTA frees when it ends, never the other way round.
+  if (DOMINO_VOCAB_TRIGGER) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
@@ -312,6 +316,9 @@ __global__ void __launch_bounds__(192, ST > 0 ? 2 : 1)
       // 0..D-1; the second segment's activations (u) come from the preceding kernel, so pass 1
       // loads them only after griddepcontrol.wait (the hardware's wait for the preceding grid
       // to complete) and adds the second segment to tiles 0..D-1; pass 2 runs tiles D.. whole.
+      // Chained launch: the preceding grid wrote this kernel's token operand (pdl_wait = 1), or
+      // wrote nothing it reads but must complete before this grid does (pdl_wait = 2).
+      if (p.pdl_wait == 1) asm volatile("griddepcontrol.wait;" ::: "memory");
       const int passes = p.defer ? 3 : 1;
       for (int pass = 0; pass < passes && ok; ++pass) {
       if (pass == 1) asm volatile("griddepcontrol.wait;" ::: "memory");
@@ -333,6 +340,7 @@ __global__ void __launch_bounds__(192, ST > 0 ? 2 : 1)
         }
       }
       }
+      if (p.pdl_wait == 2) asm volatile("griddepcontrol.wait;" ::: "memory");
       // Let every load this thread issued land before the CTA can exit (each is the last
       // one on its stage; a completed phase of that parity returns at once).
       const int outstanding = issued < C::kStages ? issued : C::kStages;

@@ -16,6 +16,24 @@ static cudaError_t launch_tc_store(int bn, bool swap, const CUtensorMap* maps, c
   return cudaErrorInvalidValue;
 }
 
+cudaError_t launch_tc_store_chained(int bn, const CUtensorMap* maps, const TcParams& p, int grid, cudaStream_t s) {
+#define DM_STC(BN) \
+  if (bn == BN) return launch_tc_instance<BN, true, kModeStore, 16, 4>(maps, p, grid, s, true);
+  DM_STC(16) DM_STC(32) DM_STC(64) DM_STC(128)
+#undef DM_STC
+  return cudaErrorInvalidValue;
+}
+
+int tc_store_chained_smem(int bn) {
+  switch (bn) {
+    case 16: return TcCfg<16, true, kModeStore, 16, 4>::kSmemBytes;
+    case 32: return TcCfg<32, true, kModeStore, 16, 4>::kSmemBytes;
+    case 64: return TcCfg<64, true, kModeStore, 16, 4>::kSmemBytes;
+    case 128: return TcCfg<128, true, kModeStore, 16, 4>::kSmemBytes;
+    default: return 0;
+  }
+}
+
 cudaError_t launch_tc_gemm(int mode, int bn, bool swap, int kmax, const CUtensorMap* maps, const TcParams& p,
                            int grid, cudaStream_t stream) {
   if (mode == kModeSoftmax) return launch_tc_softmax(bn, swap, kmax, maps, p, grid, stream);
