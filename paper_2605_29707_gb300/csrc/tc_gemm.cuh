@@ -17,6 +17,7 @@
 
 #include "kernels.h"
 #include "ptx.cuh"
+#include "topk.cuh"
 
 #ifndef DOMINO_VOCAB_TRIGGER
 #define DOMINO_VOCAB_TRIGGER 1  // let the merge kernel launch while this grid runs
@@ -126,23 +127,6 @@ struct OnlineTopK {
     }
   }
 
-  // Keyed insert (value desc, then id asc) for merging lists from other streams.
-  __device__ __forceinline__ void insert_keyed(float x, int id) {
-    const bool better_than_last =
-        x > tv[KM - 1] || (x == tv[KM - 1] && (unsigned)id < (unsigned)ti[KM - 1]);
-    if (!better_than_last) return;
-#pragma unroll
-    for (int q = 0; q < KM; ++q) {
-      const bool sw = x > tv[q] || (x == tv[q] && (unsigned)id < (unsigned)ti[q]);
-      const float a = tv[q];
-      const int b = ti[q];
-      tv[q] = sw ? x : a;
-      ti[q] = sw ? id : b;
-      x = sw ? a : x;
-      id = sw ? b : id;
-    }
-  }
-
   __device__ __forceinline__ void merge_lse(float omx, float ose) {
     const float m = fmaxf(mx, omx);
     if (m == -INFINITY) return;
@@ -152,7 +136,8 @@ struct OnlineTopK {
     se = a + b;
   }
 
-  // Merge with the state held by lane (laneid ^ offset).
+  // Merge with the state held by lane (laneid ^ offset): both lanes end with the same state
+  // (the best KM of the two lists by a bitonic merge).
   __device__ __forceinline__ void merge_shfl_xor(int offset) {
     const float omx = __shfl_xor_sync(0xffffffffu, mx, offset);
     const float ose = __shfl_xor_sync(0xffffffffu, se, offset);
@@ -164,8 +149,7 @@ struct OnlineTopK {
       oi[q] = __shfl_xor_sync(0xffffffffu, ti[q], offset);
     }
     merge_lse(omx, ose);
-#pragma unroll
-    for (int q = 0; q < KM; ++q) insert_keyed(ov[q], oi[q]);
+    merge_lists<KM>(tv, ti, ov, oi);
   }
 
   // Partial records are stored field-major: field f of chunk c at base[f * stride + c], so a
