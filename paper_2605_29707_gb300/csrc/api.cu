@@ -16,6 +16,7 @@
 #include <stdint.h>
 #include <string.h>
 
+#include <cmath>
 #include <mutex>
 #include <vector>
 
@@ -166,16 +167,19 @@ int make_plan(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head
     // one SM (228 KB of shared memory, 1 KB reserved per CTA) and every tile of a CTA can keep
     // its own TMEM accumulator until u is ready.
     const int vsm = dm::tc_softmax_deferred_smem(p.bn, p.kmax);
-    // The first D tiles of each CTA wait for u; the rest run whole, so their epilogues overlap
-    // the remaining weight stream.  D covers the GRU's expected time (12 us + K steps of
-    // 4.5 + 0.5 B us, generous for a GRU sharing its SMs with the stream) in tiles of
-    // 128 x (H + R) bf16 weights per CTA streamed at 6 TB/s; a short estimate only costs a
-    // wait at the checkpoint, never correctness.
+    // The first D tiles of each CTA wait for u; the rest run whole.  Pass 0 streams only the
+    // W_lm segment of those D tiles (128 x H bf16 per CTA and tile, about 6.6 TB/s over the
+    // grid), so D covers the GRU's expected time (12 us + K steps of 4.5 + 0.5 B us, generous
+    // for a GRU sharing its SMs with the stream) in such tile waves, plus one.  A deferred tile
+    // never waits for the epilogue, so a larger D costs only TMEM columns ((D+2) x BN <= 512)
+    // and a later epilogue; a short estimate costs a wait at the checkpoint, never correctness.
     {
-      const double t_tile_us = 128.0 * (H + R) * 2.0 * p.grid / 6.0e6;
+      const double t_seg1_us = 128.0 * H * 2.0 * p.grid / 6.6e6;
       const double t_gru_us = 12.0 + K * (4.5 + 0.5 * B);
-      int d = static_cast<int>(t_gru_us / t_tile_us) + 1;
-      p.defer_tiles = d < 1 ? 1 : (d > p.w_per_chunk ? p.w_per_chunk : d);
+      int d = static_cast<int>(std::ceil(t_gru_us / t_seg1_us)) + 1;
+      int dmax = p.w_per_chunk < dm::kMaxDefer ? p.w_per_chunk : dm::kMaxDefer;
+      if (512 / p.bn - 2 < dmax) dmax = 512 / p.bn - 2;
+      p.defer_tiles = d < 1 ? 1 : (d > dmax ? dmax : d);
     }
     p.overlap = p.u_in_gru && vsm > 0 && (p.defer_tiles + 2) * p.bn <= 512 &&
                 static_cast<size_t>(vsm) + p.gru.smem + 2048 <= 228 * 1024;

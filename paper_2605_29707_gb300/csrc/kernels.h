@@ -10,6 +10,10 @@ namespace dm {
 
 enum TcMode { kModeSoftmax = 0, kModeStore = 1 };
 
+// Most deferred tiles one CTA of the vocabulary GEMM can hold (each has its own completion
+// barrier in shared memory).
+constexpr int kMaxDefer = 32;
+
 // One tcgen05 GEMM launch: acc[tok, w] = sum over two K segments of
 //   seg1: X1[tok, :] . W1[w, :]      (k blocks 0 .. nkb1-1)
 //   seg2: X2[tok, :] . W2[w, :]      (k blocks nkb1 .. nkb1+nkb2-1)

@@ -38,7 +38,7 @@ struct TcCfg {
   static constexpr int kStages = ST > 0 ? ST : (kSt0 > 8 ? 8 : kSt0);
   static constexpr int kTmemCols =
       (2 * BN <= 32) ? 32 : (2 * BN <= 64) ? 64 : (2 * BN <= 128) ? 128 : (2 * BN <= 256) ? 256 : 512;
-  static constexpr int kBarBytes = 256;
+  static constexpr int kBarBytes = 512;  // ring, accumulator and per-deferred-tile barriers
   // per-thread scratch of one 32-value chunk (rare path of the normal orientation)
   static constexpr int kListBytes = (MODE == kModeSoftmax && !SWAP) ? 128 * 32 * 4 : 0;
   static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kTrBytes + kListBytes + kBarBytes;
@@ -169,9 +169,12 @@ struct OnlineTopK {
 // Running max, sum of exp and the top-KMAX list (value desc, id asc) live in registers.  The hot
 // path per chunk of values is branch-free: one chunk max, one rescale, one exp per value, and a
 // single compare of the chunk max with the list's last value.  Only when that compare passes
-// (rare once the list has filled) does a loop walk the chunk's values, read back from shared
-// memory, through the register insertion network, which is emitted once.  Values of one thread
-// arrive in increasing id order, so an equal value never displaces an earlier entry.
+// (rare once the list has filled) does the chunk join the list.  A 16-value chunk and a 16-entry
+// list (the small-batch swap orientation) are merged by a bitonic sort of the chunk and a
+// bitonic merge, a short dependency chain; wider chunks or lists walk the chunk's values, read
+// back from shared memory, through the register insertion network, which is emitted once (the
+// unrolled networks cost more than they save there).  Values of one thread arrive in increasing
+// id order, so an equal value never displaces an earlier entry.
 template <int N, int KM>
 __device__ __forceinline__ void stream_chunk(const float (&r)[N], const float* sx, int sstride, int v0, int vstride,
                                              int nvalid, float& mx, float& se, float (&tv)[KM], int (&ti)[KM]) {
@@ -188,6 +191,19 @@ __device__ __forceinline__ void stream_chunk(const float (&r)[N], const float* s
   for (int j = 0; j < N; ++j) sum += (j < nvalid) ? __expf(r[j] - mx) : 0.f;
   se += sum;
   if (cm > tv[KM - 1]) {
+    if constexpr (N == 16 && KM == 16) {
+      float c[16];
+      int ci[16];
+#pragma unroll
+      for (int q = 0; q < 16; ++q) {
+        const bool in = q < nvalid;
+        c[q] = in ? r[q] : -INFINITY;
+        ci[q] = in ? v0 + q * vstride : -1;
+      }
+      bitonic_sort<16>(c, ci);
+      merge_lists<16>(tv, ti, c, ci);
+      return;
+    }
     const int n = nvalid < N ? nvalid : N;
 #pragma unroll 1
     for (int j = 0; j < n; ++j) {
@@ -242,7 +258,8 @@ __global__ void __launch_bounds__(192, ST > 0 ? 2 : 1)
   uint64_t* empty = bars + C::kStages;
   uint64_t* tfull = bars + 2 * C::kStages;
   uint64_t* tempty = tfull + 2;
-  uint64_t* drain = tempty + 2;
+  uint64_t* tdone = tempty + 2;  // deferred tile i < p.defer: its accumulator is complete
+  uint64_t* drain = tdone + kMaxDefer;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
@@ -258,6 +275,7 @@ __global__ void __launch_bounds__(192, ST > 0 ? 2 : 1)
       mbar_init(&tfull[a], 1);
       mbar_init(&tempty[a], 128);
     }
+    for (int d = 0; d < kMaxDefer; ++d) mbar_init(&tdone[d], 1);
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
@@ -350,11 +368,15 @@ __global__ void __launch_bounds__(192, ST > 0 ? 2 : 1)
       for (int pass = 0; pass < passes && ok; ++pass) {
       for (int i = (pass == 2 ? p.defer : 0); ok && tc_get_item<MODE>(p, i, it); ++i) {
         if (pass < 2 && p.defer && i >= p.defer) break;
-        const int ab = i & 1;
-        const uint32_t aph = (i >> 1) & 1;
+        // A deferred tile (i < p.defer) keeps its own TMEM block and signals its own barrier,
+        // so it never waits for the epilogue; later tiles take turns on two blocks.
+        const bool own = p.defer && i < p.defer;
+        const int jd = own ? 0 : i - p.defer;
+        const int ab = jd & 1;
+        const uint32_t aph = (jd >> 1) & 1;
         const bool last_pass = !p.defer || pass >= 1;  // passes that finish a tile
         const uint32_t d_tmem = tmem_base + tc_acc_col<BN>(p, i);
-        if (last_pass) {
+        if (last_pass && !own) {
           if (!mbar_wait(&tempty[ab], aph ^ 1u, abort_flag, p.status)) break;
           tc_fence_after();
         }
@@ -373,7 +395,7 @@ __global__ void __launch_bounds__(192, ST > 0 ? 2 : 1)
           tc_commit(&empty[stage]);
           if (++stage == C::kStages) { stage = 0; phase ^= 1u; }
         }
-        if (ok && last_pass) tc_commit(&tfull[ab]);
+        if (ok && last_pass) tc_commit(own ? &tdone[i] : &tfull[ab]);
       }
       }
     }
@@ -389,9 +411,12 @@ __global__ void __launch_bounds__(192, ST > 0 ? 2 : 1)
     TcItem it;
     it.tok = 0;
     for (int i = 0; tc_get_item<MODE>(p, i, it); ++i) {
-      const int ab = i & 1;
-      const uint32_t aph = (i >> 1) & 1;
-      const bool ok = mbar_wait(&tfull[ab], aph, abort_flag, p.status);
+      const bool own = p.defer && i < p.defer;
+      const int jd = own ? 0 : i - p.defer;
+      const int ab = jd & 1;
+      const uint32_t aph = (jd >> 1) & 1;
+      const bool ok = own ? mbar_wait(&tdone[i], 0u, abort_flag, p.status)
+                          : mbar_wait(&tfull[ab], aph, abort_flag, p.status);
       if (epi_any(!ok)) { aborted = true; break; }
       tc_fence_after();
       const uint32_t tcol = tmem_base + lane_off + tc_acc_col<BN>(p, i);
@@ -451,7 +476,7 @@ __global__ void __launch_bounds__(192, ST > 0 ? 2 : 1)
           for (int j = 0; j < (BN < 32 ? 16 : 32); ++j) tr[(c0 + j) * C::kTrStride + vrow] = r[j] + bv;
         }
         tc_fence_before();
-        mbar_arrive(&tempty[ab]);
+        if (!own) mbar_arrive(&tempty[ab]);  // a deferred tile's block is never reused
         named_bar_sync(1, 128);
         const int tt = ep / C::kTPT;
         const int sub = ep % C::kTPT;

@@ -19,6 +19,7 @@ cudaError_t launch_tc_softmax(int bn, bool swap, int kmax, const CUtensorMap* ma
 // memory so that it fits on an SM next to a GRU CTA.
 cudaError_t launch_tc_softmax_deferred(int bn, int kmax, const CUtensorMap* maps, const TcParams& p, int grid,
                                        cudaStream_t s) {
+  if (p.defer < 1 || p.defer > kMaxDefer) return cudaErrorInvalidValue;
   if (bn == 16 && kmax == 16) return launch_tc_instance<16, true, kModeSoftmax, 16, 6>(maps, p, grid, s, true);
   if (bn == 16 && kmax == 32) return launch_tc_instance<16, true, kModeSoftmax, 32, 6>(maps, p, grid, s, true);
   if (bn == 32 && kmax == 16) return launch_tc_instance<32, true, kModeSoftmax, 16, 5>(maps, p, grid, s, true);

@@ -46,4 +46,31 @@ __device__ __forceinline__ void merge_lists(float (&v)[KK], int (&id)[KK], const
   bitonic_clean<KK>(v, id);
 }
 
+// Sort KK candidates best-first (bitonic sorting network, depth log2(KK)(log2(KK)+1)/2).
+template <int KK>
+__device__ __forceinline__ void bitonic_sort(float (&v)[KK], int (&id)[KK]) {
+#pragma unroll
+  for (int size = 2; size <= KK; size <<= 1) {
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+#pragma unroll
+      for (int q = 0; q < KK; ++q) {
+        const int r = q ^ stride;
+        if (r > q) {
+          // blocks with (q & size) == 0 end best-first, the others worst-first; the last
+          // pass (size == KK) leaves the whole array best-first
+          const bool q_better = better(v[q], id[q], v[r], id[r]);
+          const bool sw = ((q & size) == 0) ? !q_better : q_better;
+          const float a = v[q], b = v[r];
+          const int ia = id[q], ib = id[r];
+          v[q] = sw ? b : a;
+          id[q] = sw ? ib : ia;
+          v[r] = sw ? a : b;
+          id[r] = sw ? ia : ib;
+        }
+      }
+    }
+  }
+}
+
 }  // namespace dm
