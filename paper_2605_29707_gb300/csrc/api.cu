@@ -55,6 +55,7 @@ struct Plan {
   bool swap;
   int bn, kmax, rec, tok_tiles, w_tiles, nchunks, w_per_chunk, grid;
   StorePlan xg, ug;
+  int mcast;   // vocab GEMM, tokens on M: CTAs per cluster sharing each weight box (1 = off)
   bool chain;  // head kernels launched as a programmatic-dependent chain (small M with overlap)
   dm::GruPlan gru;
   bool u_in_gru;  // small M: u finished inside the GRU kernel; large M: W1 GEMM + finalize
@@ -155,6 +156,10 @@ int make_plan(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head
   p.w_per_chunk = ceil_div(p.w_tiles, per_tok);
   p.nchunks = ceil_div(p.w_tiles, p.w_per_chunk);
   p.grid = p.tok_tiles * p.nchunks;
+  // Tokens on M: pairs of CTAs with consecutive token tiles of one vocabulary chunk share each
+  // weight box by TMA multicast (halving the weight traffic from L2; clusters of two still
+  // cover every SM).
+  p.mcast = (!p.swap && p.tok_tiles % 2 == 0) ? 2 : 1;
 
   if (head) {
     p.u_in_gru = p.swap;
@@ -255,11 +260,12 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, u
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 // Maps for one GEMM: activations X [M, inner] (row stride xs) and weights W [rows_w, inner]
-// (row stride ws), in A/B order for the orientation.
+// (row stride ws), in A/B order for the orientation.  With weight multicast (tokens on M) each
+// CTA of a cluster loads 1/mcast of the weight box, so that map's box is bn / mcast rows high.
 bool gemm_maps(CUtensorMap* a, CUtensorMap* b, bool swap, int bn, const void* X, int M, int inner, int xs,
-               const void* W, int rows_w, int ws) {
+               const void* W, int rows_w, int ws, int mcast = 1) {
   if (swap) return make_map(a, W, inner, rows_w, ws, 128) && make_map(b, X, inner, M, xs, bn);
-  return make_map(a, X, inner, M, xs, 128) && make_map(b, W, inner, rows_w, ws, bn);
+  return make_map(a, X, inner, M, xs, 128) && make_map(b, W, inner, rows_w, ws, bn / (mcast > 1 ? mcast : 1));
 }
 
 int cuda_rc(cudaError_t e) { return e == cudaSuccess ? DOMINO_OK : DOMINO_ERR_CUDA; }
@@ -404,9 +410,9 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
     const dm::TcParams base{};
     TcParams tp = base;
     CUtensorMap maps[4];
-    if (!gemm_maps(&maps[0], &maps[1], P.swap, P.bn, hidden, M, H, H, w_lm, V, H)) return DOMINO_ERR_CUDA;
+    if (!gemm_maps(&maps[0], &maps[1], P.swap, P.bn, hidden, M, H, H, w_lm, V, H, P.mcast)) return DOMINO_ERR_CUDA;
     if (P.head) {
-      if (!gemm_maps(&maps[2], &maps[3], P.swap, P.bn, u, M, R, R, hw->w2, V, R)) return DOMINO_ERR_CUDA;
+      if (!gemm_maps(&maps[2], &maps[3], P.swap, P.bn, u, M, R, R, hw->w2, V, R, P.mcast)) return DOMINO_ERR_CUDA;
     } else {
       maps[2] = maps[0];
       maps[3] = maps[1];
@@ -418,6 +424,7 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
     tp.nchunks = P.nchunks; tp.w_per_chunk = P.w_per_chunk;
     tp.w_evict_first = P.tok_tiles == 1 ? 1 : 0;
     tp.defer = P.overlap ? P.defer_tiles : 0;
+    tp.mcast = P.mcast;
     tp.tmem_cols = P.tmem_cols;
     tp.bias = hw ? static_cast<const __nv_bfloat16*>(hw->b2) : nullptr;
     tp.out = reinterpret_cast<float*>(ws + P.off_part);

@@ -35,6 +35,9 @@ struct TcParams {
                   // the preceding grid (0 = off); see the producer in tc_gemm.cuh
   int pdl_wait;   // launched as a programmatic dependent: 1 = wait for the preceding grid before
                   // the first load, 2 = after the last load (0 = no wait)
+  int mcast;      // tokens-on-M orientation: CTAs per cluster sharing each weight box by TMA
+                  // multicast (1 = off; 2 or 4, dividing tok_tiles); the weight maps' box is
+                  // BN / mcast rows high
   int tmem_cols;  // TMEM columns to allocate (power of two, 32..512)
   const __nv_bfloat16* bias;  // softmax: b2 [V] or nullptr
   float* out;                 // softmax: partial records [M][rec fields][nchunks]; store: [splits][M][ld_out]

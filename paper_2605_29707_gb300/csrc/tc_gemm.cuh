@@ -44,6 +44,7 @@ struct TcCfg {
   static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kTrBytes + kListBytes + kBarBytes;
   static constexpr int kRec = 2 + 2 * KMAX;
   static_assert(kStages >= 2, "pipeline needs at least two stages");
+  static_assert(kSmemBytes <= 227 * 1024, "one CTA's dynamic shared memory limit");
   // CTAs of this kernel that fit on one 228 KB SM (1 KB of shared memory reserved per CTA)
   // never hold more than the SM's 512 TMEM columns between them.  (Across kernels, see the
   // trigger after the allocation in the kernel body.)
@@ -269,7 +270,7 @@ __global__ void __launch_bounds__(192, ST > 0 ? 2 : 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], p.mcast > 1 ? p.mcast : 1);  // every CTA of a multicast cluster releases it
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
@@ -296,6 +297,12 @@ __global__ void __launch_bounds__(192, ST > 0 ? 2 : 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  // Weight multicast (p.mcast > 1, tokens-on-M orientation): the CTAs of a cluster hold
+  // consecutive token tiles of one vocabulary chunk and stream the same weight tiles; each loads
+  // 1/mcast of every weight box into all of them.  No CTA may multicast before every CTA of the
+  // cluster has initialised its barriers.
+  const uint16_t mc_mask = static_cast<uint16_t>((1u << (p.mcast > 1 ? p.mcast : 1)) - 1u);
+  if (p.mcast > 1) cluster_sync();
   // A kernel launched as this grid's programmatic dependent may start now: it waits for this
   // grid to complete before it reads anything this kernel writes.  The trigger comes after the
   // TMEM allocation, so a dependent that allocates TMEM on this SM can only wait for columns
@@ -336,7 +343,15 @@ __global__ void __launch_bounds__(192, ST > 0 ? 2 : 1)
           const int ay = SWAP ? it.w * 128 : it.tok * 128;
           const int by = SWAP ? it.tok * BN : it.w * BN;
           tma_load_2d(sA + stage * C::kABytes, seg2 ? &tmA2 : &tmA1, &full[stage], kx, ay, polA);
-          tma_load_2d(sB + stage * C::kBBytes, seg2 ? &tmB2 : &tmB1, &full[stage], kx, by, polB);
+          if (!SWAP && p.mcast > 1) {
+            // this CTA's BN / mcast rows of the weight box (the map's box is that high)
+            const int part = static_cast<int>(cluster_ctarank());
+            const int rows = BN / p.mcast;
+            tma_load_2d_multicast(sB + stage * C::kBBytes + part * rows * 128, seg2 ? &tmB2 : &tmB1, &full[stage],
+                                  kx, by + part * rows, mc_mask, polB);
+          } else {
+            tma_load_2d(sB + stage * C::kBBytes, seg2 ? &tmB2 : &tmB1, &full[stage], kx, by, polB);
+          }
           ++issued;
           if (++stage == C::kStages) { stage = 0; phase ^= 1u; }
         }
@@ -344,14 +359,16 @@ __global__ void __launch_bounds__(192, ST > 0 ? 2 : 1)
       }
       if (p.pdl_wait == 2) asm volatile("griddepcontrol.wait;" ::: "memory");
       // Let every load this thread issued land before the CTA can exit (each is the last
-      // one on its stage; a completed phase of that parity returns at once).
+      // one on its stage; a completed phase of that parity returns at once).  With multicast,
+      // wait until every CTA of the cluster has consumed them (the stage's release).
       const int outstanding = issued < C::kStages ? issued : C::kStages;
       for (int j = 1; j <= outstanding; ++j) {
         int s = stage - j;
         uint32_t ph = phase;
         if (s < 0) { s += C::kStages; ph ^= 1u; }
+        uint64_t* last = p.mcast > 1 ? &empty[s] : &full[s];
         const long long t0 = clock64();
-        while (!mbar_try_wait(&full[s], ph)) {
+        while (!mbar_try_wait(last, ph)) {
           if (clock64() - t0 > kWaitCycles) { set_status(p.status, kStatusTimeout); break; }
         }
       }
@@ -392,7 +409,8 @@ __global__ void __launch_bounds__(192, ST > 0 ? 2 : 1)
             tc_mma_bf16(d_tmem, da + static_cast<uint64_t>(2 * kk), db + static_cast<uint64_t>(2 * kk),
                         kIdesc, (kb > it.kb0 || kk > 0) ? 1u : 0u);
           }
-          tc_commit(&empty[stage]);
+          if (p.mcast > 1) tc_commit_multicast(&empty[stage], mc_mask);  // release it in every CTA
+          else tc_commit(&empty[stage]);
           if (++stage == C::kStages) { stage = 0; phase ^= 1u; }
         }
         if (ok && last_pass) tc_commit(own ? &tdone[i] : &tfull[ab]);
@@ -547,6 +565,7 @@ __global__ void __launch_bounds__(192, ST > 0 ? 2 : 1)
   // ------------------------------------------------------------ teardown
   tc_fence_before();
   __syncthreads();
+  if (p.mcast > 1) cluster_sync();  // no CTA leaves while a peer may still write into it
   if (warp == 1) {
     if (lane == 0) {
       // every MMA this thread issued must be finished before the TMEM is released
@@ -583,8 +602,21 @@ cudaError_t launch_tc_instance(const CUtensorMap* maps, const TcParams& p, int g
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
+  cudaLaunchAttribute attrs[2];
+  int na = 0;
+  if (pdl) attrs[na++] = attr[0];
+  if (p.mcast > 1) {
+    if (SWAP || MODE != kModeSoftmax || p.mcast > 8 || p.tok_tiles % p.mcast != 0 || grid % p.mcast != 0 ||
+        BN % (8 * p.mcast) != 0)
+      return cudaErrorInvalidValue;
+    attrs[na].id = cudaLaunchAttributeClusterDimension;
+    attrs[na].val.clusterDim.x = p.mcast;
+    attrs[na].val.clusterDim.y = 1;
+    attrs[na].val.clusterDim.z = 1;
+    ++na;
+  }
+  cfg.attrs = attrs;
+  cfg.numAttrs = na;
   cudaError_t e = cudaLaunchKernelEx(&cfg, kern, maps[0], maps[1], maps[2], maps[3], p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
