@@ -140,7 +140,7 @@ def vocab_plan(cfg, num_sms):
     per_tok = max(1, num_sms // tok_tiles)
     wpc = -(-w_tiles // per_tok)
     nchunks = -(-w_tiles // wpc)
-    kmax = 16 if cfg.k <= 16 else 32
+    kmax = 8 if cfg.k <= 8 else (16 if cfg.k <= 16 else 32)
     return dict(swap=swap, bn=bn, nchunks=nchunks, rec_words=2 + 2 * kmax, grid=tok_tiles * nchunks)
 
 

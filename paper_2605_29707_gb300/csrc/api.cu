@@ -147,7 +147,8 @@ int make_plan(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head
   const int M = p.M;
 
   choose_orientation(M, &p.swap, &p.bn);
-  p.kmax = k <= 16 ? 16 : 32;
+  // top-k list length per (token, CTA): the merge reads only the first k entries
+  p.kmax = k <= 8 ? 8 : (k <= 16 ? 16 : 32);
   p.rec = dm::kSoftmaxRecWords(p.kmax);
   p.tok_tiles = p.swap ? ceil_div(M, p.bn) : ceil_div(M, 128);
   p.w_tiles = p.swap ? ceil_div(V, 128) : ceil_div(V, p.bn);

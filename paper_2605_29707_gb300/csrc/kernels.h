@@ -56,6 +56,12 @@ cudaError_t launch_tc_softmax_deferred(int bn, int kmax, const CUtensorMap* maps
                                        cudaStream_t stream);
 // Shared memory one deferred-mode CTA uses (for the co-residency budget).
 int tc_softmax_deferred_smem(int bn, int kmax);
+// The same three for 8-entry top-k lists (kmax = 8; tc_softmax_k8.cu).
+cudaError_t launch_tc_softmax_k8(int bn, bool swap, const CUtensorMap* maps, const TcParams& p, int grid,
+                                 cudaStream_t stream);
+cudaError_t launch_tc_softmax_deferred_k8(int bn, const CUtensorMap* maps, const TcParams& p, int grid,
+                                          cudaStream_t stream);
+int tc_softmax_deferred_smem_k8(int bn);
 // Small-M (swap, bn 16..128) store-mode GEMM with four pipeline stages, launched as a
 // programmatic dependent of the preceding kernel (p.pdl_wait says where it waits for it).
 cudaError_t launch_tc_store_chained(int bn, const CUtensorMap* maps, const TcParams& p, int grid,

@@ -170,9 +170,9 @@ struct OnlineTopK {
 // Running max, sum of exp and the top-KMAX list (value desc, id asc) live in registers.  The hot
 // path per chunk of values is branch-free: one chunk max, one rescale, one exp per value, and a
 // single compare of the chunk max with the list's last value.  Only when that compare passes
-// (rare once the list has filled) does the chunk join the list.  A 16-value chunk and a 16-entry
-// list (the small-batch swap orientation) are merged by a bitonic sort of the chunk and a
-// bitonic merge, a short dependency chain; wider chunks or lists walk the chunk's values, read
+// (rare once the list has filled) does the chunk join the list.  A 16-value chunk and a list of
+// at most 16 entries (the small-batch swap orientation) are merged by a bitonic sort of the chunk
+// and a bitonic merge, a short dependency chain; wider chunks or lists walk the chunk's values, read
 // back from shared memory, through the register insertion network, which is emitted once (the
 // unrolled networks cost more than they save there).  Values of one thread arrive in increasing
 // id order, so an equal value never displaces an earlier entry.
@@ -192,7 +192,7 @@ __device__ __forceinline__ void stream_chunk(const float (&r)[N], const float* s
   for (int j = 0; j < N; ++j) sum += (j < nvalid) ? __expf(r[j] - mx) : 0.f;
   se += sum;
   if (cm > tv[KM - 1]) {
-    if constexpr (N == 16 && KM == 16) {
+    if constexpr (N == 16 && KM <= 16) {
       float c[16];
       int ci[16];
 #pragma unroll
@@ -202,7 +202,11 @@ __device__ __forceinline__ void stream_chunk(const float (&r)[N], const float* s
         ci[q] = in ? v0 + q * vstride : -1;
       }
       bitonic_sort<16>(c, ci);
-      merge_lists<16>(tv, ti, c, ci);
+      float h[KM];
+      int hi[KM];
+#pragma unroll
+      for (int q = 0; q < KM; ++q) { h[q] = c[q]; hi[q] = ci[q]; }
+      merge_lists<KM>(tv, ti, h, hi);
       return;
     }
     const int n = nvalid < N ? nvalid : N;

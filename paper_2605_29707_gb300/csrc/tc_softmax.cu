@@ -6,6 +6,7 @@ namespace dm {
 
 cudaError_t launch_tc_softmax(int bn, bool swap, int kmax, const CUtensorMap* maps, const TcParams& p,
                               int grid, cudaStream_t s) {
+  if (kmax == 8) return launch_tc_softmax_k8(bn, swap, maps, p, grid, s);
 #define DM_SM(BN, SW, KM)                                                              \
   if (bn == BN && swap == SW && kmax == KM)                                            \
     return launch_tc_instance<BN, SW, kModeSoftmax, KM>(maps, p, grid, s);
@@ -20,6 +21,7 @@ cudaError_t launch_tc_softmax(int bn, bool swap, int kmax, const CUtensorMap* ma
 cudaError_t launch_tc_softmax_deferred(int bn, int kmax, const CUtensorMap* maps, const TcParams& p, int grid,
                                        cudaStream_t s) {
   if (p.defer < 1 || p.defer > kMaxDefer) return cudaErrorInvalidValue;
+  if (kmax == 8) return launch_tc_softmax_deferred_k8(bn, maps, p, grid, s);
   if (bn == 16 && kmax == 16) return launch_tc_instance<16, true, kModeSoftmax, 16, 6>(maps, p, grid, s, true);
   if (bn == 16 && kmax == 32) return launch_tc_instance<16, true, kModeSoftmax, 32, 6>(maps, p, grid, s, true);
   if (bn == 32 && kmax == 16) return launch_tc_instance<32, true, kModeSoftmax, 16, 5>(maps, p, grid, s, true);
@@ -28,6 +30,7 @@ cudaError_t launch_tc_softmax_deferred(int bn, int kmax, const CUtensorMap* maps
 }
 
 int tc_softmax_deferred_smem(int bn, int kmax) {
+  if (kmax == 8) return tc_softmax_deferred_smem_k8(bn);
   if (bn == 16) return kmax <= 16 ? TcCfg<16, true, kModeSoftmax, 16, 6>::kSmemBytes
                                   : TcCfg<16, true, kModeSoftmax, 32, 6>::kSmemBytes;
   if (bn == 32) return kmax <= 16 ? TcCfg<32, true, kModeSoftmax, 16, 5>::kSmemBytes

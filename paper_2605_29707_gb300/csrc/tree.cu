@@ -374,6 +374,8 @@ cudaError_t launch_merge_tree(const TreeParams& p, cudaStream_t stream) {
   cfg.numAttrs = DOMINO_TREE_PDL ? 1 : 0;
   cudaError_t e;
   if (p.kmax == 32) e = cudaLaunchKernelEx(&cfg, merge_tree_kernel<32, 32>, p);
+  else if (p.kmax == 8) e = p.k <= 4 ? cudaLaunchKernelEx(&cfg, merge_tree_kernel<8, 4>, p)
+                                     : cudaLaunchKernelEx(&cfg, merge_tree_kernel<8, 8>, p);
   else if (p.kmax != 16) return cudaErrorInvalidValue;
   else if (p.k <= 4) e = cudaLaunchKernelEx(&cfg, merge_tree_kernel<16, 4>, p);
   else if (p.k <= 8) e = cudaLaunchKernelEx(&cfg, merge_tree_kernel<16, 8>, p);
