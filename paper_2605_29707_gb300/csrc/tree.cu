@@ -27,7 +27,11 @@
 
 namespace dm {
 
-constexpr int kMergeThreads = 256;
+// Threads per merge CTA: 256, or 64 when a row has at most 64 chunk records and lists of at most
+// 16 entries (tokens-on-M launches, where the rows are many and 256-thread CTAs at their register
+// use would need several waves).
+constexpr int kMergeThreadsWide = 256;
+constexpr int kMergeThreadsNarrow = 64;
 constexpr int kMaxK = 64;
 constexpr int kMaxTopk = 32;
 constexpr int kMaxN = 256;
@@ -165,10 +169,10 @@ __device__ __forceinline__ void best_children(const float* lp, const int* ids, i
   child_key(b0, sb0, tb, ids + rb * k, sb, hb, lb, jb);
 }
 
-template <int KM, int KK>
-__global__ void __launch_bounds__(kMergeThreads) merge_tree_kernel(const TreeParams p) {
+template <int KM, int KK, int NT>
+__global__ void __launch_bounds__(NT, NT == kMergeThreadsNarrow ? 8 : 1) merge_tree_kernel(const TreeParams p) {
   constexpr int F = 2 + 2 * KM;
-  constexpr int kWarps = kMergeThreads / 32;
+  constexpr int kWarps = NT / 32;
   static_assert(KK <= KM && kWarps <= 32, "list and warp counts");
   __shared__ float s_mx[kWarps], s_se[kWarps];
   __shared__ int s_last;
@@ -194,7 +198,7 @@ __global__ void __launch_bounds__(kMergeThreads) merge_tree_kernel(const TreePar
   int ti[KK];
 #pragma unroll
   for (int q = 0; q < KK; ++q) { tv[q] = -INFINITY; ti[q] = -1; }
-  for (int c = tid; c < nch; c += kMergeThreads) {
+  for (int c = tid; c < nch; c += NT) {
     const float cm = __ldg(base + c), cs = __ldg(base + nch + c);
     float v[KK];
     int id[KK];
@@ -260,7 +264,7 @@ __global__ void __launch_bounds__(kMergeThreads) merge_tree_kernel(const TreePar
   if (!s_last) return;
   __threadfence();
   const size_t rows = static_cast<size_t>(b) * K * k;
-  for (int e = tid; e < K * k; e += kMergeThreads) {
+  for (int e = tid; e < K * k; e += NT) {
     s_id[e] = __ldcg(p.topk_ids + rows + e);
     s_lp[e] = __ldcg(p.topk_logp + rows + e);
   }
@@ -361,25 +365,34 @@ __global__ void __launch_bounds__(kMergeThreads) merge_tree_kernel(const TreePar
   }
 }
 
+template <int NT>
+static cudaError_t launch_merge_nt(cudaLaunchConfig_t& cfg, const TreeParams& p) {
+  cfg.blockDim = dim3(NT);
+  if constexpr (NT == kMergeThreadsWide) {
+    if (p.kmax == 32) return cudaLaunchKernelEx(&cfg, merge_tree_kernel<32, 32, NT>, p);
+  }
+  if (p.kmax == 8)
+    return p.k <= 4 ? cudaLaunchKernelEx(&cfg, merge_tree_kernel<8, 4, NT>, p)
+                    : cudaLaunchKernelEx(&cfg, merge_tree_kernel<8, 8, NT>, p);
+  if (p.kmax != 16) return cudaErrorInvalidValue;
+  if (p.k <= 4) return cudaLaunchKernelEx(&cfg, merge_tree_kernel<16, 4, NT>, p);
+  if (p.k <= 8) return cudaLaunchKernelEx(&cfg, merge_tree_kernel<16, 8, NT>, p);
+  return cudaLaunchKernelEx(&cfg, merge_tree_kernel<16, 16, NT>, p);
+}
+
 cudaError_t launch_merge_tree(const TreeParams& p, cudaStream_t stream) {
   if (p.K > kMaxK || p.k > kMaxTopk || p.k > p.kmax || p.N > kMaxN) return cudaErrorInvalidValue;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.B * p.K);
-  cfg.blockDim = dim3(kMergeThreads);
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = DOMINO_TREE_PDL ? 1 : 0;
-  cudaError_t e;
-  if (p.kmax == 32) e = cudaLaunchKernelEx(&cfg, merge_tree_kernel<32, 32>, p);
-  else if (p.kmax == 8) e = p.k <= 4 ? cudaLaunchKernelEx(&cfg, merge_tree_kernel<8, 4>, p)
-                                     : cudaLaunchKernelEx(&cfg, merge_tree_kernel<8, 8>, p);
-  else if (p.kmax != 16) return cudaErrorInvalidValue;
-  else if (p.k <= 4) e = cudaLaunchKernelEx(&cfg, merge_tree_kernel<16, 4>, p);
-  else if (p.k <= 8) e = cudaLaunchKernelEx(&cfg, merge_tree_kernel<16, 8>, p);
-  else e = cudaLaunchKernelEx(&cfg, merge_tree_kernel<16, 16>, p);
+  // 32-entry lists keep the wide CTA (their registers do not fit the narrow one's budget)
+  const bool narrow = p.nchunks <= kMergeThreadsNarrow && p.kmax <= 16;
+  const cudaError_t e = narrow ? launch_merge_nt<kMergeThreadsNarrow>(cfg, p) : launch_merge_nt<kMergeThreadsWide>(cfg, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
