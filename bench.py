@@ -288,6 +288,53 @@ def config_dict(c, world):
 
 
 # ---------------------------------------------------------------------------- our arm
+def time_steps(st, hidden, ids, stream, n, warmup):
+    """Mean device time (us) of n back-to-back steps on `stream` after `warmup` untimed ones."""
+    import torch
+    for _ in range(max(3, warmup)):
+        st.enqueue(hidden, ids, stream)
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(n):
+        rc = st.enqueue(hidden, ids, stream)
+        if rc != 0:
+            raise RuntimeError(f"step returned {rc}")
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / n * 1e3
+
+
+def graph_replay(st, hidden, ids, device, n, blocks_per_step):
+    """Capture one step in a CUDA graph and time n replays; on a capture failure, say why."""
+    import torch
+    try:
+        s = torch.cuda.Stream(device)
+        g = torch.cuda.CUDAGraph()
+        torch.cuda.synchronize()
+        with torch.cuda.graph(g, stream=s):
+            rc = st.enqueue(hidden, ids, s)
+        if rc != 0:
+            return {"error": f"capture: step returned {rc}"}
+        for _ in range(3):
+            g.replay()
+        torch.cuda.synchronize()
+        cur = torch.cuda.current_stream(device)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(cur)
+        for _ in range(n):
+            g.replay()
+        e1.record(cur)
+        torch.cuda.synchronize()
+        us = e0.elapsed_time(e1) / n * 1e3
+        return {"us_per_step": round(us, 2), "value": round(blocks_per_step * 1e6 / us, 3), "replays": n}
+    except Exception as e:  # noqa: BLE001 -- reported, not fatal
+        torch.cuda.synchronize()
+        return {"error": str(e).splitlines()[0][:200]}
+
+
 def run_ours(args):
     import numpy as np
     import torch
@@ -393,6 +440,18 @@ def run_ours(args):
     h2d = M * c.H * 2 + M * 4
     d2h = M * c.k * 8 + c.B * c.N * 16 + 4
 
+    # ---- Domino-head overhead: the same workload with the correction branch off (R = 0, the
+    #      paper's "w/o Domino head" base distribution), same device weights
+    head_overhead = None
+    if st.head_on:
+        st_off = DraftStep(st.w, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=device, head_on=False)
+        us_off = time_steps(st_off, hidden, ids, stream, min(args.steps, 1000), args.warmup)
+        us_on = ms_step * 1e3
+        head_overhead = {"us_head_off": round(us_off, 2), "us_head_on": round(us_on, 2),
+                         "overhead_us": round(us_on - us_off, 2), "overhead_pct": round(100.0 * (us_on / us_off - 1.0), 2),
+                         "note": "head off = W_lm projection + softmax/top-k + tree only (R = 0)"}
+        del st_off
+
     # ---- roofline of the dominant kernel, measured in the timed region
     peaks = load_peaks()
     dominant = max(kern, key=lambda n: kern[n][0])
@@ -423,7 +482,11 @@ def run_ours(args):
         "e2e": {"value": round(e2e_value, 3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "steps": n_e2e, "api": "domino_draft_step_host (synchronous per step)"},
         "gpu_launches": args.steps * launches, "clocks": clocks,
+        "head_overhead": head_overhead,
     }
+    # ---- last: the same step replayed from a CUDA graph (one captured step, replayed back to
+    #      back); a failed capture is reported in the line, after everything else was measured
+    line["graph_replay"] = graph_replay(st, hidden, ids, device, min(args.steps, 1000), c.B * world)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, args.cpu_seconds)
     if rank == 0:
