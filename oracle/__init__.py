@@ -54,6 +54,7 @@ def _load():
         _lib.oracle_topk.argtypes = [P, I, I, I, P, P]
         _lib.oracle_tree.argtypes = [P, P, I, I, I, P, P, P, P]
         _lib.oracle_draft_step.argtypes = [P] * 12 + [I] * 8 + [P, I] + [P] * 8 + [I]
+        _lib.oracle_verify_greedy.argtypes = [P, I, I, P, P, P, P, P, P]
         _lib.oracle_max_threads.restype = I
         for name in ("oracle_embed", "oracle_gru", "oracle_lowrank", "oracle_logits",
                      "oracle_log_softmax", "oracle_topk", "oracle_tree", "oracle_draft_step"):
@@ -167,6 +168,22 @@ def tree(topk_ids, topk_logp, N):
     _check(_load().oracle_tree(_p(topk_ids), _p(topk_logp), K, k, N, _p(par), _p(tok), _p(dep),
                                _p(sc)), "oracle_tree")
     return par, tok, dep, sc
+
+
+def verify_greedy(target, parent, token):
+    """Greedy tree verification of one sequence: target fp32 [N+1, V], parent/token [N].
+    Returns (row_argmax [N+1], accepted nodes [n_acc], bonus token)."""
+    target = np.ascontiguousarray(target, np.float32)
+    parent = _i32(parent); token = _i32(token)
+    N = parent.shape[0]
+    V = target.shape[1]
+    if target.shape[0] != N + 1:
+        raise OracleError(-1, "oracle_verify_greedy: target must have N + 1 rows")
+    ra = np.empty(N + 1, np.int32); nodes = np.empty(max(N, 1), np.int32)
+    n = np.zeros(1, np.int32); bonus = np.zeros(1, np.int32)
+    _check(_load().oracle_verify_greedy(_p(target), N, V, _p(parent), _p(token), _p(ra), _p(nodes), _p(n),
+                                        _p(bonus)), "oracle_verify_greedy")
+    return ra, nodes[: int(n[0])].copy(), int(bonus[0])
 
 
 def draft_step(w, hidden, prefix_ids, k, N, seqs=None, want_logp_full=False, nthreads=0):

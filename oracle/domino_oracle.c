@@ -14,6 +14,7 @@
  *                  L_i = L_base_i + dL_i                          -> oracle_logits (sum)
  *   Fig. 3 caption: tokens are drawn from the final logits        -> oracle_log_softmax
  *   Fig. 1 caption: the "Tree" construction cost                  -> oracle_topk, oracle_tree
+ *   section 3.1, verification of the draft (the step after it)     -> oracle_verify_greedy
  * Readings of points the paper leaves open (GRU gate convention, which ids feed which
  * position, tree tie-breaks) are listed in the design notes; the comments below state the
  * reading each function implements.
@@ -314,4 +315,36 @@ int oracle_draft_step(const uint16_t* hidden, const int32_t* prefix_ids, const u
   }
   free(hid); free(E); free(S); free(u); free(z); free(lp); free(ls);
   return rc;
+}
+
+/* O8: greedy verification of one tree (section 3.1, "accepts the longest valid prefix"). */
+int oracle_verify_greedy(const float* target, int N, int V, const int32_t* parent, const int32_t* token,
+                         int32_t* row_argmax, int32_t* nodes, int32_t* n_acc, int32_t* bonus) {
+  if (!target || !row_argmax || !nodes || !n_acc || !bonus || N < 0 || V <= 0) return ORACLE_ERR_ARG;
+  if (N > 0 && (!parent || !token)) return ORACLE_ERR_ARG;
+  for (int i = 0; i < N; ++i)
+    if (parent[i] < -1 || parent[i] >= i) return ORACLE_ERR_ARG;
+  for (int r = 0; r <= N; ++r) {
+    const float* row = target + (long)r * V;
+    int best = 0;
+    for (int v = 1; v < V; ++v)
+      if (row[v] > row[best]) best = v; /* strict: an equal value keeps the lower id */
+    row_argmax[r] = best;
+  }
+  for (int i = 0; i < N; ++i) nodes[i] = -1;
+  int cur = -1, n = 0;
+  for (;;) {
+    const int a = row_argmax[cur + 1];
+    int next = -1;
+    for (int c = 0; c < N; ++c)
+      if (parent[c] == cur && token[c] == a) { next = c; break; }
+    if (next < 0) {
+      *bonus = a;
+      break;
+    }
+    nodes[n++] = next;
+    cur = next;
+  }
+  *n_acc = n;
+  return 0;
 }

@@ -95,6 +95,22 @@ int oracle_draft_step(const uint16_t* hidden, const int32_t* prefix_ids, const u
                       int32_t* tree_parent, int32_t* tree_token, int32_t* tree_depth,
                       double* tree_score, int nthreads);
 
+/* O8, the step after the draft (section 3.1: the target model evaluates the draft in one pass
+ * and "accepts the longest valid prefix"; tau counts the accepted tokens plus the bonus token
+ * the target produces).  Greedy verification of one draft tree at temperature 0, where a draft
+ * token is valid when it equals the target's most likely next token:
+ *   parent/token [N]: the tree (parent -1 = the anchor, otherwise an earlier node), as from
+ *     oracle_tree; target [N+1, V] fp32: the target's next-token logits after the anchor
+ *     (row 0) and after each node i (row i+1).
+ *   Walk from the anchor: a = the argmax of the current node's row (equal values: the lowest
+ *   id); if a child of the current node carries token a (several: the lowest node index),
+ *   accept it and continue from it; otherwise stop.
+ * Outputs: row_argmax [N+1]; nodes [N] = the accepted nodes in order, -1 after the last;
+ *   n_acc = their number; bonus = the last argmax (the target's own next token). tau =
+ *   n_acc + 1.  The comparisons are on the given fp32 values, exactly. */
+int oracle_verify_greedy(const float* target, int N, int V, const int32_t* parent, const int32_t* token,
+                         int32_t* row_argmax, int32_t* nodes, int32_t* n_acc, int32_t* bonus);
+
 /* Number of OpenMP threads the oracle would use for nthreads <= 0 (all available). */
 int oracle_max_threads(void);
 

@@ -266,3 +266,58 @@ def custom_config(name="custom", **kw) -> Config:
     base = dict(B=1, K=4, H=256, V=4096, k=4, N=8, seed=0)
     base.update(kw)
     return Config(name, **base)
+
+
+# ---------------------------------------------------------------------------- verification inputs
+@dataclasses.dataclass
+class VerifyCase:
+    """Synthetic inputs of greedy tree verification: a draft tree per sequence and the target's
+    next-token logits after the anchor (row 0) and after each node (row i + 1)."""
+    parent: np.ndarray  # int32 [B, N]
+    token: np.ndarray   # int32 [B, N]
+    target: np.ndarray  # float32 [B, N + 1, V]
+
+
+def random_tree(N: int, V: int, key: tuple, chain: bool = False):
+    """A valid draft tree of N nodes: parent[i] in [-1, i) (the previous node for a chain),
+    tokens in [0, V) distinct among the children of one node."""
+    g = torch.Generator().manual_seed(_key_seed(*key))
+    parent = np.empty(N, np.int32)
+    token = np.empty(N, np.int32)
+    used = {}
+    for i in range(N):
+        p = i - 1 if chain else int(torch.randint(-1, i, (1,), generator=g)) if i > 0 else -1
+        parent[i] = p
+        taken = used.setdefault(p, set())
+        while True:
+            t = int(torch.randint(0, V, (1,), generator=g))
+            if t not in taken:
+                break
+        taken.add(t)
+        token[i] = t
+    return parent, token
+
+
+def make_verify_case(B: int, N: int, V: int, seed: int, p_plant: float = 0.7, chain: bool = False,
+                     trees=None) -> VerifyCase:
+    """Target logits ~ N(0, 1) fp32; with probability p_plant the row after a node (or after the
+    anchor) gets one of that node's children's tokens raised to the row maximum + 1, so that
+    accepted paths of every length occur.  `trees` ([B] pairs of parent/token) replaces the
+    random trees, e.g. with trees a draft step produced."""
+    parent = np.empty((B, N), np.int32)
+    token = np.empty((B, N), np.int32)
+    target = np.empty((B, N + 1, V), np.float32)
+    for b in range(B):
+        if trees is not None:
+            parent[b], token[b] = trees[b]
+        else:
+            parent[b], token[b] = random_tree(N, V, (seed, "verify-tree", b), chain=chain)
+        t = normal_f32((N + 1, V), (seed, "verify-target", b)).numpy()
+        u = uniform01(2 * (N + 1), (seed, "verify-plant", b))
+        for r in range(N + 1):
+            kids = [c for c in range(N) if parent[b, c] == r - 1]
+            if kids and u[2 * r] < p_plant:
+                c = kids[min(len(kids) - 1, int(u[2 * r + 1] * len(kids)))]
+                t[r, token[b, c]] = t[r].max() + 1.0
+        target[b] = t
+    return VerifyCase(parent, token, target)

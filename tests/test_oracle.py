@@ -369,3 +369,77 @@ def test_parameter_count_matches_paper_56M():
     hidden = rand_bf16(rng, (1, 2, H), 1.0)
     out = oracle.draft_step(w, hidden, np.array([[1, 2]], np.int32), 2, 3)
     assert out["topk_ids"].shape == (1, 2, 2)
+
+
+# ---------------------------------------------------------------------------- O8 tree verification
+def _golden(name):
+    with open(os.path.join(os.path.dirname(__file__), "golden", name)) as f:
+        return json.load(f)
+
+
+def test_verify_hand_case_a():
+    """Hand-worked greedy verification (section 3.1): tie at the anchor, a negative row, a leaf stop."""
+    g = _golden("verify_case_a.json")
+    ra, nodes, bonus = oracle.verify_greedy(np.array(g["target"], np.float32), g["parent"], g["token"])
+    assert ra.tolist() == g["expect_row_argmax"]
+    assert nodes.tolist() == g["expect_nodes"]
+    assert bonus == g["expect_bonus"]
+    assert len(nodes) + 1 == g["expect_tau"]
+
+
+def _brute_force_accepted(target, parent, token):
+    """Every path from the anchor whose tokens all equal numpy's argmax (first occurrence) of the
+    parent's row; the accepted path is the longest such path (each step has one candidate)."""
+    N = len(parent)
+    am = np.argmax(target, axis=1)
+    best = []
+    for end in range(N):
+        path, c = [], end
+        while c != -1:
+            path.append(c)
+            c = int(parent[c])
+        path.reverse()
+        ok = all(token[n] == am[(parent[n] + 1)] for n in path)
+        if ok and len(path) > len(best):
+            best = path
+    last = best[-1] if best else -1
+    return am, best, int(am[last + 1])
+
+
+@pytest.mark.parametrize("seed,N,V,chain,p", [(1, 12, 300, False, 0.7), (2, 20, 50, False, 0.9),
+                                               (3, 16, 1000, True, 0.8), (4, 1, 7, False, 1.0),
+                                               (5, 30, 64, False, 0.5)])
+def test_verify_matches_brute_force(seed, N, V, chain, p):
+    from paper_2605_29707_gb300 import inputs
+    c = inputs.make_verify_case(2, N, V, seed, p_plant=p, chain=chain)
+    for b in range(2):
+        ra, nodes, bonus = oracle.verify_greedy(c.target[b], c.parent[b], c.token[b])
+        am, best, bb = _brute_force_accepted(c.target[b], c.parent[b], c.token[b])
+        assert ra.tolist() == am.tolist()
+        assert nodes.tolist() == best
+        assert bonus == bb
+        # stop rule: no child of the last accepted node carries the bonus token
+        last = nodes[-1] if len(nodes) else -1
+        assert not any(c.parent[b, i] == last and c.token[b, i] == bonus for i in range(N))
+
+
+def test_verify_special_cases():
+    # no nodes: tau = 1, bonus = argmax after the anchor
+    t = np.array([[0.0, 3.0, 3.0, -1.0]], np.float32)
+    ra, nodes, bonus = oracle.verify_greedy(t, np.zeros(0, np.int32), np.zeros(0, np.int32))
+    assert ra.tolist() == [1] and len(nodes) == 0 and bonus == 1
+    # a chain whose every row points at the next token: all N accepted, tau = N + 1
+    N, V = 6, 10
+    parent = np.arange(-1, N - 1, dtype=np.int32)
+    token = np.array([(3 * i + 1) % V for i in range(N)], np.int32)
+    t = np.zeros((N + 1, V), np.float32)
+    for r in range(N):
+        t[r, token[r]] = 1.0
+    t[N, 9] = 2.0
+    ra, nodes, bonus = oracle.verify_greedy(t, parent, token)
+    assert nodes.tolist() == list(range(N)) and bonus == 9
+    # invalid parent (not an earlier node)
+    with pytest.raises(oracle.OracleError):
+        oracle.verify_greedy(np.zeros((3, 4), np.float32), np.array([-1, 1], np.int32), np.array([0, 1], np.int32))
+    with pytest.raises(oracle.OracleError):
+        oracle.verify_greedy(np.zeros((2, 4), np.float32), np.array([-1, 0], np.int32), np.array([0, 1], np.int32))
