@@ -306,6 +306,42 @@ def time_steps(st, hidden, ids, stream, n, warmup):
     return e0.elapsed_time(e1) / n * 1e3
 
 
+def verify_timing(st, c, device, stream, reps=200):
+    import torch
+    from paper_2605_29707_gb300 import binding, inputs
+    torch.cuda.synchronize()
+    trees = [(st.tree_parent.view(c.B, c.N)[b].cpu().numpy(), st.tree_token.view(c.B, c.N)[b].cpu().numpy())
+             for b in range(c.B)]
+    case = inputs.make_verify_case(c.B, c.N, c.V, 97, p_plant=0.8, trees=trees)
+    t = torch.from_numpy(case.target).to(device)
+    par = st.tree_parent.view(c.B, c.N)
+    tok = st.tree_token.view(c.B, c.N)
+    ra = torch.empty((c.B, c.N + 1), dtype=torch.int32, device=device)
+    nodes = torch.empty((c.B, c.N), dtype=torch.int32, device=device)
+    cnt = torch.empty(c.B, dtype=torch.int32, device=device)
+    bon = torch.empty(c.B, dtype=torch.int32, device=device)
+
+    def run():
+        rc = binding.domino_verify_tree_greedy(t, par, tok, c.B, c.N, c.V, ra, nodes, cnt, bon, stream)
+        if rc != 0:
+            raise RuntimeError(f"domino_verify_tree_greedy returned {rc}")
+    for _ in range(3):
+        run()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(reps):
+        run()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    us = e0.elapsed_time(e1) / reps * 1e3
+    nbytes = c.B * (c.N + 1) * c.V * 4
+    return {"us": round(us, 2), "logits_bytes": nbytes, "GB_per_s": round(nbytes / (us * 1e-6) / 1e9, 1),
+            "tau_mean": round(float(cnt.float().mean().item()) + 1.0, 3),
+            "note": "synthetic target logits (planted argmaxes); tau is a mechanics check, not a quality number"}
+
+
 def graph_replay(st, hidden, ids, device, n, blocks_per_step):
     """Capture one step in a CUDA graph and time n replays; on a capture failure, say why."""
     import torch
@@ -452,6 +488,10 @@ def run_ours(args):
                          "note": "head off = W_lm projection + softmax/top-k + tree only (R = 0)"}
         del st_off
 
+    # ---- the step after the draft: greedy verification of this step's trees against synthetic
+    #      target logits [B, N+1, V] fp32 (timing only; parity is in the tests)
+    verify = verify_timing(st, c, device, stream) if c.B <= 4 else None
+
     # ---- roofline of the dominant kernel, measured in the timed region
     peaks = load_peaks()
     dominant = max(kern, key=lambda n: kern[n][0])
@@ -482,7 +522,7 @@ def run_ours(args):
         "e2e": {"value": round(e2e_value, 3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "steps": n_e2e, "api": "domino_draft_step_host (synchronous per step)"},
         "gpu_launches": args.steps * launches, "clocks": clocks,
-        "head_overhead": head_overhead,
+        "head_overhead": head_overhead, "tree_verify": verify,
     }
     # ---- last: the same step replayed from a CUDA graph (one captured step, replayed back to
     #      back); a failed capture is reported in the line, after everything else was measured

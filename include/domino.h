@@ -144,6 +144,26 @@ DOMINO_API int domino_abi_version(void);
  * R > 0), so a caller can count device work. */
 DOMINO_API int domino_launches_per_step(int B, int K, int H, int V, int Ds, int R, int k, int N);
 
+/* Greedy verification of draft trees against the target model's logits: the step after the
+ * draft.  Section 3.1: the target evaluates the draft in one pass and accepts the longest valid
+ * prefix; tau counts the accepted tokens plus the bonus token the target produces.  At
+ * temperature 0 a draft token is valid when it equals the target's most likely next token.
+ * For each sequence b, from the anchor: a = argmax of the current node's row (equal values: the
+ * lowest id); if a child of the current node carries token a (several: the lowest node index),
+ * accept it and continue from it; otherwise stop, and a is the bonus token.
+ *   target_logits: device fp32 [B, N + 1, V]: the target's next-token logits after the anchor
+ *     (row 0) and after tree node i (row i + 1).  Finite values (NaN is not ordered).
+ *   tree_parent / tree_token: device int32 [B, N] as domino_draft_step writes them (parent -1 =
+ *     the anchor, otherwise an earlier node); may be NULL when N = 0.
+ * Outputs (device int32): row_argmax [B, N + 1]; accepted_nodes [B, N] = the accepted nodes in
+ *   order, -1 after the last; accepted_count [B] (tau = accepted_count + 1); bonus_token [B].
+ * Two kernels on `stream`; no workspace.  Returns DOMINO_OK once enqueued, or a negative code
+ * (bad sizes or pointers) with nothing enqueued. */
+DOMINO_API int domino_verify_tree_greedy(const float* target_logits, const int32_t* tree_parent,
+                                         const int32_t* tree_token, int B, int N, int V, int32_t* row_argmax,
+                                         int32_t* accepted_nodes, int32_t* accepted_count,
+                                         int32_t* bonus_token, void* stream);
+
 /* Draft step for callers that cannot allocate device memory.  Some callers cannot call
  * cudaMalloc or any allocator at all: code running inside a host framework that owns every
  * allocation, a plugin loaded into a process whose memory pool is fixed up front, or a

@@ -24,7 +24,7 @@ DOMINO_ERR_BAD_TOKEN = -5
 SYMBOLS = ("domino_workspace_bytes", "domino_draft_step", "domino_workspace_bytes_host",
            "domino_draft_step_host", "domino_check_status", "domino_status_string",
            "domino_abi_version", "domino_launches_per_step", "domino_timing_begin", "domino_timing_end",
-           "domino_draft_step_static_scratch")
+           "domino_draft_step_static_scratch", "domino_verify_tree_greedy")
 
 DOMINO_STATIC_SCRATCH_BYTES = 16 << 20
 
@@ -80,6 +80,8 @@ def load():
     lib.domino_draft_step_static_scratch.argtypes = [P, P, P, ctypes.POINTER(domino_head_weights)] + [I] * 6 + \
         [P] * 6 + [P, P]
     lib.domino_draft_step_static_scratch.restype = I
+    lib.domino_verify_tree_greedy.argtypes = [P, P, P, I, I, I, P, P, P, P, P]
+    lib.domino_verify_tree_greedy.restype = I
     _lib = lib
     return lib
 
@@ -178,3 +180,11 @@ def domino_draft_step_static_scratch(hidden, prefix_ids, w_lm, head, B, K, H, V,
         _addr(hidden), _addr(prefix_ids), _addr(w_lm), h, B, K, H, V, k, N, _addr(topk_ids), _addr(topk_logp),
         _addr(tree_parent), _addr(tree_token), _addr(tree_depth), _addr(tree_score), _addr(device_status),
         _stream(stream)))
+
+
+def domino_verify_tree_greedy(target_logits, tree_parent, tree_token, B, N, V, row_argmax, accepted_nodes,
+                              accepted_count, bonus_token, stream=None) -> int:
+    """Greedy verification of B draft trees against the target's fp32 logits [B, N+1, V] (device)."""
+    return int(load().domino_verify_tree_greedy(_addr(target_logits), _addr(tree_parent), _addr(tree_token), B, N, V,
+                                                _addr(row_argmax), _addr(accepted_nodes), _addr(accepted_count),
+                                                _addr(bonus_token), _stream(stream)))

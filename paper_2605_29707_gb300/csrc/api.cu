@@ -604,6 +604,18 @@ int domino_timing_end(float* total_ms, int* launches, int nkinds) {
   return DOMINO_OK;
 }
 
+int domino_verify_tree_greedy(const float* target_logits, const int32_t* tree_parent, const int32_t* tree_token,
+                              int B, int N, int V, int32_t* row_argmax, int32_t* accepted_nodes,
+                              int32_t* accepted_count, int32_t* bonus_token, void* stream) {
+  if (B < 1 || N < 0 || V < 1 || N > (1 << 20)) return DOMINO_ERR_INVALID_ARG;
+  if (static_cast<long long>(B) * (N + 1) > 0x7fffffffLL) return DOMINO_ERR_INVALID_ARG;
+  if (!target_logits || !row_argmax || !accepted_count || !bonus_token) return DOMINO_ERR_INVALID_ARG;
+  if (N > 0 && (!tree_parent || !tree_token || !accepted_nodes)) return DOMINO_ERR_INVALID_ARG;
+  return cuda_rc(dm::launch_verify_greedy(target_logits, tree_parent, tree_token, B, N, V, row_argmax,
+                                          accepted_nodes, accepted_count, bonus_token,
+                                          static_cast<cudaStream_t>(stream)));
+}
+
 int domino_launches_per_step(int B, int K, int H, int V, int Ds, int R, int k, int N) {
   (void)H; (void)V; (void)Ds; (void)k; (void)N;
   if (R <= 0) return 3;  // gather (id check), vocab GEMM, merge + tree

@@ -135,4 +135,9 @@ struct TreeParams {
 };
 cudaError_t launch_merge_tree(const TreeParams& p, cudaStream_t stream);
 
+// ---------------------------------------------------------------- tree verification (verify.cu)
+cudaError_t launch_verify_greedy(const float* logits, const int32_t* parent, const int32_t* token, int B, int N,
+                                 int V, int32_t* row_argmax, int32_t* nodes, int32_t* count, int32_t* bonus,
+                                 cudaStream_t stream);
+
 }  // namespace dm

@@ -65,3 +65,16 @@ def test_launch_count_query():
     _lib()
     assert binding.domino_launches_per_step(1, 16, 4096, 151936, 1024, 256, 8, 16) == 6
     assert binding.domino_launches_per_step(1, 16, 4096, 151936, 0, 0, 8, 16) == 3
+
+
+def test_verify_rejects_bad_arguments_before_launch():
+    """Argument errors of domino_verify_tree_greedy come back before anything is enqueued."""
+    f = binding.domino_verify_tree_greedy
+    bad = binding.DOMINO_ERR_INVALID_ARG
+    one = 1  # a non-null stand-in; never dereferenced because validation fails first
+    assert f(one, one, one, 0, 4, 10, one, one, one, one) == bad        # B < 1
+    assert f(one, one, one, 1, -1, 10, one, one, one, one) == bad       # N < 0
+    assert f(one, one, one, 1, 4, 0, one, one, one, one) == bad         # V < 1
+    assert f(None, one, one, 1, 4, 10, one, one, one, one) == bad       # no logits
+    assert f(one, None, one, 1, 4, 10, one, one, one, one) == bad       # N > 0 without a tree
+    assert f(one, one, one, 1, 4, 10, one, None, one, one) == bad       # no accepted_nodes
