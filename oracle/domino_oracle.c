@@ -15,6 +15,7 @@
  *   Fig. 3 caption: tokens are drawn from the final logits        -> oracle_log_softmax
  *   Fig. 1 caption: the "Tree" construction cost                  -> oracle_topk, oracle_tree
  *   section 3.1, verification of the draft (the step after it)     -> oracle_verify_greedy
+ *   section 4.1.2 / Fig. 3, tokens chosen and fed back one by one   -> oracle_rollout_greedy
  * Readings of points the paper leaves open (GRU gate convention, which ids feed which
  * position, tree tie-breaks) are listed in the design notes; the comments below state the
  * reading each function implements.
@@ -347,4 +348,60 @@ int oracle_verify_greedy(const float* target, int N, int V, const int32_t* paren
   }
   *n_acc = n;
   return 0;
+}
+
+/* O9: the greedy sequential draft loop.  Each position is computed from scratch out of the
+ * primitives above (the GRU re-run over the whole prefix chosen so far), so the only new step is
+ * the feedback: the argmax of position j becomes the input of position j + 1. */
+int oracle_rollout_greedy(const uint16_t* hidden, const int32_t* anchors, const uint16_t* w_lm,
+                          const uint16_t* emb, const uint16_t* w_ih, const uint16_t* w_hh,
+                          const uint16_t* b_ih, const uint16_t* b_hh, const uint16_t* w1,
+                          const uint16_t* b1, const uint16_t* w2, const uint16_t* b2, int B, int K,
+                          int H, int V, int Ds, int R, const int32_t* seqs, int nseq, int32_t* tokens,
+                          double* logp, int nthreads) {
+  if (!hidden || !anchors || !w_lm || !tokens || !logp) return ORACLE_ERR_ARG;
+  if (B <= 0 || K <= 0 || H <= 0 || V <= 0 || R < 0) return ORACLE_ERR_ARG;
+  const int use_head = (w2 != NULL && R > 0);
+  if (use_head && (!emb || !w_ih || !w_hh || !w1 || Ds <= 0)) return ORACLE_ERR_ARG;
+  if (!seqs) nseq = B;
+  if (nseq <= 0) return ORACLE_ERR_ARG;
+
+  int32_t* ids = (int32_t*)malloc((size_t)(K + 1) * sizeof(int32_t));
+  double* hid = (double*)malloc((size_t)H * sizeof(double));
+  double* E = (double*)malloc((size_t)K * H * sizeof(double));
+  double* S = use_head ? (double*)malloc((size_t)K * Ds * sizeof(double)) : NULL;
+  double* u = use_head ? (double*)malloc((size_t)R * sizeof(double)) : NULL;
+  double* z = (double*)malloc((size_t)V * sizeof(double));
+  double* lp = (double*)malloc((size_t)V * sizeof(double));
+  double ls;
+  int rc = 0;
+  if (!ids || !hid || !E || !z || !lp || (use_head && (!S || !u))) rc = ORACLE_ERR_ARG;
+
+  for (int si = 0; si < nseq && rc == 0; ++si) {
+    const int b = seqs ? seqs[si] : si;
+    if (b < 0 || b >= B) { rc = ORACLE_ERR_ARG; break; }
+    ids[0] = anchors[b];
+    if (ids[0] < 0 || ids[0] >= V) { rc = ORACLE_ERR_TOKEN; break; }
+    for (int j = 0; j < K && rc == 0; ++j) {
+      for (int c = 0; c < H; ++c) hid[c] = bf(hidden, ((long)b * K + j) * H + c);
+      if (use_head) {
+        /* the causal encoder over the prefix t_0 .. t_j chosen so far */
+        rc = oracle_embed(emb, V, H, ids, j + 1, E);
+        if (!rc) rc = oracle_gru(E, j + 1, H, Ds, w_ih, w_hh, b_ih, b_hh, S);
+        if (!rc) rc = oracle_lowrank(hid, S + (long)j * Ds, 1, H, Ds, R, w1, b1, u);
+        if (rc) break;
+      }
+      rc = oracle_logits(hid, u, 1, H, V, use_head ? R : 0, w_lm, use_head ? w2 : NULL, b2, z, nthreads);
+      if (!rc) rc = oracle_log_softmax(z, 1, V, lp, &ls);
+      if (rc) break;
+      int best = 0;
+      for (int v = 1; v < V; ++v)
+        if (z[v] > z[best]) best = v; /* strict: an equal value keeps the lower id */
+      ids[j + 1] = best;
+      tokens[(long)si * K + j] = best;
+      logp[(long)si * K + j] = lp[best];
+    }
+  }
+  free(ids); free(hid); free(E); free(S); free(u); free(z); free(lp);
+  return rc;
 }

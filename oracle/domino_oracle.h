@@ -111,6 +111,21 @@ int oracle_draft_step(const uint16_t* hidden, const int32_t* prefix_ids, const u
 int oracle_verify_greedy(const float* target, int N, int V, const int32_t* parent, const int32_t* token,
                          int32_t* row_argmax, int32_t* nodes, int32_t* n_acc, int32_t* bonus);
 
+/* O9, the sequential draft loop at inference (section 4.1.2 and Fig. 3: each draft token is
+ * chosen from the final logits and is the causal encoder's next input), greedy: per sequence,
+ * t_0 = anchors[b]; for j = 0..K-1: S_j = the GRU state after E_0..E_j with E_i = emb[t_i];
+ * u_j = SiLU(W1 [hidden_j ; S_j] + b1); L_j = W_lm hidden_j + W2 u_j + b2; t_{j+1} = argmax L_j
+ * (equal values: the lowest id); logp_j = log-softmax(L_j)[t_{j+1}].  With the correction branch
+ * off (w2 NULL or R = 0) L_j = W_lm hidden_j + b2.
+ * Outputs for the sequences in seqs (as in oracle_draft_step): tokens [nseq, K] = t_1..t_K,
+ * logp [nseq, K]. */
+int oracle_rollout_greedy(const uint16_t* hidden, const int32_t* anchors, const uint16_t* w_lm,
+                          const uint16_t* emb, const uint16_t* w_ih, const uint16_t* w_hh,
+                          const uint16_t* b_ih, const uint16_t* b_hh, const uint16_t* w1,
+                          const uint16_t* b1, const uint16_t* w2, const uint16_t* b2, int B, int K,
+                          int H, int V, int Ds, int R, const int32_t* seqs, int nseq, int32_t* tokens,
+                          double* logp, int nthreads);
+
 /* Number of OpenMP threads the oracle would use for nthreads <= 0 (all available). */
 int oracle_max_threads(void);
 

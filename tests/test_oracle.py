@@ -443,3 +443,56 @@ def test_verify_special_cases():
         oracle.verify_greedy(np.zeros((3, 4), np.float32), np.array([-1, 1], np.int32), np.array([0, 1], np.int32))
     with pytest.raises(oracle.OracleError):
         oracle.verify_greedy(np.zeros((2, 4), np.float32), np.array([-1, 0], np.int32), np.array([0, 1], np.int32))
+
+
+# ---------------------------------------------------------------------------- O9 greedy rollout
+def test_rollout_hand_case_c():
+    """Hand-worked greedy rollout (section 4.1.2 / Fig. 3) from hand case C's numbers."""
+    g = load("hand_case_c.json")
+    r = load("rollout_case_c.json")
+    w = {n: bf16(g[n]) for n in ("w_lm", "emb", "w_ih", "w_hh", "b_ih", "b_hh", "w1", "b1", "w2", "b2")}
+    hidden = bf16(g["hidden"]).reshape(1, g["K"], g["H"])
+    tokens, logp = oracle.rollout_greedy(w, hidden, np.array([r["anchor"]], np.int32))
+    assert tokens[0].tolist() == r["expect_tokens"]
+    assert logp[0] == pytest.approx(r["expect_logp"], abs=r["tolerance"])
+
+
+def _small_weights(rng, V, H, Ds, R, biases):
+    w = {"w_lm": rand_bf16(rng, (V, H), 0.3), "emb": rand_bf16(rng, (V, H), 0.5),
+         "w_ih": rand_bf16(rng, (3 * Ds, H), 0.3), "w_hh": rand_bf16(rng, (3 * Ds, Ds), 0.3),
+         "w1": rand_bf16(rng, (R, H + Ds), 0.3), "w2": rand_bf16(rng, (V, R), 0.8)}
+    if biases:
+        for n, m in (("b_ih", 3 * Ds), ("b_hh", 3 * Ds), ("b1", R), ("b2", V)):
+            w[n] = rand_bf16(rng, (m,), 0.2)
+    return w
+
+
+@pytest.mark.parametrize("B,K,V,H,Ds,R,biases", [(2, 5, 40, 16, 6, 4, False), (3, 7, 13, 8, 3, 2, True),
+                                                 (1, 6, 200, 24, 8, 8, True)])
+def test_rollout_is_the_fixed_point_of_the_teacher_forced_step(B, K, V, H, Ds, R, biases):
+    """The draft step fed the rollout's own tokens as its prefix has, at every position, the
+    rollout's token as its argmax and the rollout's log-probability for it."""
+    rng = np.random.default_rng(B * 100 + K)
+    w = _small_weights(rng, V, H, Ds, R, biases)
+    hidden = rand_bf16(rng, (B, K, H), 1.0)
+    anchors = rng.integers(0, V, B).astype(np.int32)
+    tokens, logp = oracle.rollout_greedy(w, hidden, anchors)
+    prefix = np.concatenate([anchors[:, None], tokens[:, :-1]], axis=1).astype(np.int32)
+    ref = oracle.draft_step(w, hidden, prefix, 1, 1, want_logp_full=True)
+    for b in range(B):
+        for j in range(K):
+            row = ref["logp_full"][b, j]
+            assert int(np.argmax(row)) == tokens[b, j]
+            assert logp[b, j] == pytest.approx(row[tokens[b, j]], abs=1e-12)
+
+
+def test_rollout_head_off_is_the_base_argmax_and_rejects_bad_anchors():
+    rng = np.random.default_rng(7)
+    V, H, K = 30, 12, 4
+    w = {"w_lm": rand_bf16(rng, (V, H), 0.4)}
+    hidden = rand_bf16(rng, (2, K, H), 1.0)
+    tokens, logp = oracle.rollout_greedy(w, hidden, np.array([3, 4], np.int32))
+    z = np.einsum("bkh,vh->bkv", to_f64(hidden), to_f64(w["w_lm"]))
+    assert tokens.tolist() == np.argmax(z, axis=2).tolist()
+    with pytest.raises(oracle.OracleError):
+        oracle.rollout_greedy(w, hidden, np.array([3, V], np.int32))
