@@ -507,7 +507,8 @@ def run_ours(args):
                  "share_of_step": round(vk_ms / max(1e-9, sum(v[0] for v in kern.values())), 4)})
     sw = step_work(c)
     step_roof = max(sw["bytes"] / (peaks["hbm_gbs"] * 1e9), sw["flops"] / (peaks["bf16_tflops_sustained"] * 1e12))
-    breakdown = {n: {"us_per_step": round(v[0] / k_steps * 1e3, 2), "launches": v[1]} for n, v in kern.items()}
+    breakdown = {n: {"us_per_step": round(v[0] / k_steps * 1e3, 2), "launches": v[1]} for n, v in kern.items()
+                 if v[1] > 0}
 
     line = {
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world, "steps": args.steps,

@@ -164,6 +164,32 @@ DOMINO_API int domino_verify_tree_greedy(const float* target_logits, const int32
                                          int32_t* accepted_nodes, int32_t* accepted_count,
                                          int32_t* bonus_token, void* stream);
 
+/* The greedy sequential draft loop, the paper's inference loop (section 4.1.2 and Fig. 3: each
+ * draft token is chosen from the final logits and becomes the causal encoder's next input), as
+ * a variant of domino_draft_step for callers that do not have the prefix:
+ *   t_0 = anchors[b]; for j = 0..K-1: S_j = the GRU state after emb[t_0..t_j];
+ *   u_j = SiLU(W1 [hidden_j ; S_j] + b1); L_j = W_lm hidden_j + W2 u_j + b2;
+ *   t_{j+1} = argmax L_j (equal values: the lowest id); logp_j = log-softmax(L_j)[t_{j+1}].
+ * With the correction branch off (head NULL, R = 0 or w2 NULL) L_j = W_lm hidden_j + b2.
+ *   hidden [B, K, H] bf16, anchors [B] int32, w_lm [V, H] bf16, head as for domino_draft_step,
+ *   all device pointers, 16-byte aligned.  B <= 8 (a latency path; batches use
+ *   domino_draft_step); H, d_s and r multiples of 8; r <= 8192; one CTA of the step kernel
+ *   (one per SM) holds in shared memory a 64 KB ring of W2 rows, u of every sequence (4 B r)
+ *   and its share of the base logits (4 B ceil(V / SMs) rows, rounded up to whole W2 chunks),
+ *   which must total at most 227 KB (else DOMINO_ERR_INVALID_ARG; B = 8, r = 256 and
+ *   V = 151936 take 104 KB).
+ * Outputs (device): tokens int32 [B, K] = t_1 .. t_K; logp fp32 [B, K].
+ * workspace: device memory of domino_rollout_workspace_bytes(...) bytes (16-byte aligned);
+ * its first int32 receives the device status (DOMINO_OK, DOMINO_ERR_BAD_TOKEN,
+ * DOMINO_ERR_TIMEOUT; domino_check_status reads it).  Two kernels on `stream` (a tensor-core
+ * GEMM for W_lm hidden_j of every position, then one cooperative kernel for the K steps).
+ * Returns DOMINO_OK once enqueued, or a negative code with nothing enqueued. */
+DOMINO_API size_t domino_rollout_workspace_bytes(int B, int K, int H, int V, int Ds, int R);
+DOMINO_API int domino_rollout_greedy(const void* hidden, const int32_t* anchors, const void* w_lm,
+                                     const domino_head_weights* head, int B, int K, int H, int V,
+                                     int32_t* tokens, float* logp, void* workspace, size_t workspace_bytes,
+                                     void* stream);
+
 /* Draft step for callers that cannot allocate device memory.  Some callers cannot call
  * cudaMalloc or any allocator at all: code running inside a host framework that owns every
  * allocation, a plugin loaded into a process whose memory pool is fixed up front, or a
@@ -211,7 +237,10 @@ enum domino_kernel_kind {
                                      M <= 128) */
   DOMINO_KERNEL_VOCAB = 4,        /* [hidden | u] . [W_lm | W2]^T with online softmax / top-k */
   DOMINO_KERNEL_TREE = 5,         /* merge to log-probs and top-k; best-first tree */
-  DOMINO_KERNEL_KINDS = 6
+  DOMINO_KERNEL_ROLLOUT_BASE = 6, /* domino_rollout_greedy: W_lm hidden_j of every position */
+  DOMINO_KERNEL_ROLLOUT = 7,      /* domino_rollout_greedy: the K sequential steps */
+  DOMINO_KERNEL_VERIFY = 8,       /* domino_verify_tree_greedy: row argmax and tree walk */
+  DOMINO_KERNEL_KINDS = 9
 };
 DOMINO_API int domino_timing_begin(int max_launches);
 DOMINO_API int domino_timing_end(float* total_ms, int* launches, int nkinds);

@@ -24,11 +24,13 @@ DOMINO_ERR_BAD_TOKEN = -5
 SYMBOLS = ("domino_workspace_bytes", "domino_draft_step", "domino_workspace_bytes_host",
            "domino_draft_step_host", "domino_check_status", "domino_status_string",
            "domino_abi_version", "domino_launches_per_step", "domino_timing_begin", "domino_timing_end",
-           "domino_draft_step_static_scratch", "domino_verify_tree_greedy")
+           "domino_draft_step_static_scratch", "domino_verify_tree_greedy", "domino_rollout_workspace_bytes",
+           "domino_rollout_greedy")
 
 DOMINO_STATIC_SCRATCH_BYTES = 16 << 20
 
-KERNEL_KINDS = ("gather", "gru_input_proj", "w1_hidden_proj", "gru", "vocab_gemm_softmax_topk", "merge_tree")
+KERNEL_KINDS = ("gather", "gru_input_proj", "w1_hidden_proj", "gru", "vocab_gemm_softmax_topk", "merge_tree",
+                "rollout_base_gemm", "rollout_steps", "tree_verify")
 
 
 class domino_head_weights(ctypes.Structure):
@@ -82,6 +84,11 @@ def load():
     lib.domino_draft_step_static_scratch.restype = I
     lib.domino_verify_tree_greedy.argtypes = [P, P, P, I, I, I, P, P, P, P, P]
     lib.domino_verify_tree_greedy.restype = I
+    lib.domino_rollout_workspace_bytes.argtypes = [I] * 6
+    lib.domino_rollout_workspace_bytes.restype = ctypes.c_size_t
+    lib.domino_rollout_greedy.argtypes = [P, P, P, ctypes.POINTER(domino_head_weights)] + [I] * 4 + [P, P, P,
+                                                                                               ctypes.c_size_t, P]
+    lib.domino_rollout_greedy.restype = I
     _lib = lib
     return lib
 
@@ -188,3 +195,16 @@ def domino_verify_tree_greedy(target_logits, tree_parent, tree_token, B, N, V, r
     return int(load().domino_verify_tree_greedy(_addr(target_logits), _addr(tree_parent), _addr(tree_token), B, N, V,
                                                 _addr(row_argmax), _addr(accepted_nodes), _addr(accepted_count),
                                                 _addr(bonus_token), _stream(stream)))
+
+
+def domino_rollout_workspace_bytes(B, K, H, V, Ds, R) -> int:
+    return int(load().domino_rollout_workspace_bytes(B, K, H, V, Ds, R))
+
+
+def domino_rollout_greedy(hidden, anchors, w_lm, head, B, K, H, V, tokens, logp, workspace, workspace_bytes,
+                          stream=None) -> int:
+    """Greedy sequential draft loop: tokens t_1..t_K [B, K] and their log-probabilities (device)."""
+    h = ctypes.byref(head) if head is not None else None
+    return int(load().domino_rollout_greedy(_addr(hidden), _addr(anchors), _addr(w_lm), h, B, K, H, V,
+                                            _addr(tokens), _addr(logp), _addr(workspace), int(workspace_bytes),
+                                            _stream(stream)))

@@ -611,9 +611,138 @@ int domino_verify_tree_greedy(const float* target_logits, const int32_t* tree_pa
   if (static_cast<long long>(B) * (N + 1) > 0x7fffffffLL) return DOMINO_ERR_INVALID_ARG;
   if (!target_logits || !row_argmax || !accepted_count || !bonus_token) return DOMINO_ERR_INVALID_ARG;
   if (N > 0 && (!tree_parent || !tree_token || !accepted_nodes)) return DOMINO_ERR_INVALID_ARG;
-  return cuda_rc(dm::launch_verify_greedy(target_logits, tree_parent, tree_token, B, N, V, row_argmax,
-                                          accepted_nodes, accepted_count, bonus_token,
-                                          static_cast<cudaStream_t>(stream)));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int ts = timing_open(DOMINO_KERNEL_VERIFY, st);
+  const int rc = cuda_rc(dm::launch_verify_greedy(target_logits, tree_parent, tree_token, B, N, V, row_argmax,
+                                                  accepted_nodes, accepted_count, bonus_token, st));
+  timing_close(ts, st);
+  return rc;
+}
+
+// ---------------------------------------------------------------- greedy rollout
+namespace {
+struct RollPlan {
+  int B, K, H, V, Ds, R, M, grid;
+  bool head;
+  StorePlan g;  // base-logit GEMM, no split
+  size_t off_h, off_u, off_part, off_base, clear_bytes, total;
+};
+
+int make_roll_plan(int B, int K, int H, int V, int Ds, int R, bool head, RollPlan* P) {
+  if (B < 1 || B > dm::kRollMaxB || K < 1 || H < 8 || (H & 7) || V < 1) return DOMINO_ERR_INVALID_ARG;
+  // head on: a W2 row must fit one 16 KB stage of the rollout's ring
+  if (head && (Ds < 8 || (Ds & 7) || R < 8 || (R & 7) || R > 8192)) return DOMINO_ERR_INVALID_ARG;
+  if (static_cast<long long>(B) * K * V > (1LL << 33)) return DOMINO_ERR_UNSUPPORTED;
+  int sms = 0, major = 0, minor = 0;
+  int rc = device_sms(&sms, &major, &minor);
+  if (rc != DOMINO_OK) return rc;
+  if (major != 10 || minor != 3) return DOMINO_ERR_UNSUPPORTED;
+  RollPlan& p = *P;
+  p.B = B; p.K = K; p.H = H; p.V = V; p.head = head;
+  p.Ds = head ? Ds : 0;
+  p.R = head ? R : 0;
+  p.M = B * K;
+  p.grid = sms;  // one CTA per SM, all resident (cooperative launch)
+  // the ring, u and the CTA's rows of base logits must fit one CTA's shared memory
+  if (dm::rollout_smem_bytes(B, V, p.R, head, sms) > dm::kRollMaxSmem) return DOMINO_ERR_INVALID_ARG;
+  p.g = plan_store(p.M, V, ceil_div(H, 64), sms);
+  // one split: the GEMM writes finished logits
+  p.g.splits = 1;
+  p.g.kb_per_split = p.g.nkb;
+  p.g.total_items = p.g.tok_tiles * p.g.w_tiles;
+  p.g.grid = p.g.total_items < sms ? p.g.total_items : sms;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off = align_up(off + bytes);
+    return o;
+  };
+  take(256);  // status (offset 0, as for domino_check_status) and the grid barrier counter
+  p.off_h = take(static_cast<size_t>(2) * B * (p.Ds > 0 ? p.Ds : 1) * 4);
+  p.clear_bytes = off;
+  p.off_u = take(static_cast<size_t>(B) * (p.R > 0 ? p.R : 1) * 4);
+  p.off_part = take(static_cast<size_t>(p.grid) * dm::kRollMaxB * 16);
+  p.off_base = take(static_cast<size_t>(p.M) * V * 4);
+  p.total = off;
+  return DOMINO_OK;
+}
+}  // namespace
+
+size_t domino_rollout_workspace_bytes(int B, int K, int H, int V, int Ds, int R) {
+  RollPlan P;
+  if (make_roll_plan(B, K, H, V, Ds, R, R > 0, &P) != DOMINO_OK) return 0;
+  return P.total;
+}
+
+int domino_rollout_greedy(const void* hidden, const int32_t* anchors, const void* w_lm,
+                          const domino_head_weights* head, int B, int K, int H, int V, int32_t* tokens,
+                          float* logp, void* workspace, size_t workspace_bytes, void* stream) {
+  const bool hd = head_active(head);
+  if (!hidden || !anchors || !w_lm || !tokens || !logp || !workspace) return DOMINO_ERR_INVALID_ARG;
+  if (hd && (!head->emb || !head->w_ih || !head->w_hh || !head->w1)) return DOMINO_ERR_INVALID_ARG;
+  if (!aligned16(hidden) || !aligned16(w_lm)) return DOMINO_ERR_INVALID_ARG;
+  if (hd && (!aligned16(head->w2) || !aligned16(head->w1) || !aligned16(head->w_ih) || !aligned16(head->w_hh) ||
+             !aligned16(head->emb)))
+    return DOMINO_ERR_INVALID_ARG;
+  RollPlan P;
+  int rc = make_roll_plan(B, K, H, V, hd ? head->Ds : 0, hd ? head->R : 0, hd, &P);
+  if (rc) return rc;
+  if (workspace_bytes < P.total) return DOMINO_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  if (cudaMemsetAsync(ws, 0, P.clear_bytes, st) != cudaSuccess) return DOMINO_ERR_CUDA;
+  int* status = reinterpret_cast<int*>(ws);
+  float* base = reinterpret_cast<float*>(ws + P.off_base);
+  // base logits W_lm hidden_j for every position (tensor cores, fp32 out)
+  {
+    const dm::TcParams b0{};
+    TcParams tp = b0;
+    const StorePlan& g = P.g;
+    CUtensorMap maps[4];
+    if (!gemm_maps(&maps[0], &maps[1], g.swap, g.bn, hidden, P.M, H, H, w_lm, V, H)) return DOMINO_ERR_CUDA;
+    maps[2] = maps[0];
+    maps[3] = maps[1];
+    tp.nkb1 = g.nkb; tp.nkb2 = 0;
+    tp.rows_tok = P.M; tp.rows_w = V;
+    tp.tok_tiles = g.tok_tiles; tp.w_tiles = g.w_tiles;
+    tp.splits = 1; tp.kb_per_split = g.kb_per_split; tp.total_items = g.total_items;
+    tp.w_evict_first = 1;
+    tp.tmem_cols = pow2_at_least(2 * g.bn, 32);
+    tp.out = base; tp.ld_out = V;
+    tp.status = status;
+    const int ts = timing_open(DOMINO_KERNEL_ROLLOUT_BASE, st);
+    rc = cuda_rc(dm::launch_tc_gemm(dm::kModeStore, g.bn, g.swap, 16, maps, tp, g.grid, st));
+    timing_close(ts, st);
+    if (rc) return rc;
+  }
+  dm::RolloutParams rp{};
+  rp.hidden = static_cast<const __nv_bfloat16*>(hidden);
+  rp.anchors = anchors;
+  if (hd) {
+    rp.emb = static_cast<const __nv_bfloat16*>(head->emb);
+    rp.w_ih = static_cast<const __nv_bfloat16*>(head->w_ih);
+    rp.w_hh = static_cast<const __nv_bfloat16*>(head->w_hh);
+    rp.b_ih = static_cast<const __nv_bfloat16*>(head->b_ih);
+    rp.b_hh = static_cast<const __nv_bfloat16*>(head->b_hh);
+    rp.w1 = static_cast<const __nv_bfloat16*>(head->w1);
+    rp.b1 = static_cast<const __nv_bfloat16*>(head->b1);
+    rp.w2 = static_cast<const __nv_bfloat16*>(head->w2);
+  }
+  rp.b2 = head ? static_cast<const __nv_bfloat16*>(head->b2) : nullptr;
+  rp.head = hd ? 1 : 0;
+  rp.B = B; rp.K = K; rp.H = H; rp.V = V; rp.Ds = P.Ds; rp.R = P.R;
+  rp.base = base;
+  rp.h = reinterpret_cast<float*>(ws + P.off_h);
+  rp.u = reinterpret_cast<float*>(ws + P.off_u);
+  rp.partials = reinterpret_cast<float*>(ws + P.off_part);
+  rp.barrier = reinterpret_cast<unsigned*>(ws + 64);
+  rp.tokens = tokens;
+  rp.logp = logp;
+  rp.status = status;
+  const int ts = timing_open(DOMINO_KERNEL_ROLLOUT, st);
+  rc = cuda_rc(dm::launch_rollout(rp, P.grid, st));
+  timing_close(ts, st);
+  return rc;
 }
 
 int domino_launches_per_step(int B, int K, int H, int V, int Ds, int R, int k, int N) {

@@ -135,6 +135,29 @@ struct TreeParams {
 };
 cudaError_t launch_merge_tree(const TreeParams& p, cudaStream_t stream);
 
+// ---------------------------------------------------------------- greedy rollout (rollout.cu)
+constexpr int kRollMaxB = 8;  // sequences per rollout launch
+struct RolloutParams {
+  const __nv_bfloat16* hidden;  // [B, K, H]
+  const int32_t* anchors;       // [B]
+  const __nv_bfloat16 *emb, *w_ih, *w_hh, *b_ih, *b_hh, *w1, *b1, *w2, *b2;  // b* may be null
+  int head;                     // correction branch on (R > 0 and W2 given)
+  int B, K, H, V, Ds, R;
+  const float* base;            // [B*K, V] W_lm hidden (fp32, from the store-mode GEMM)
+  float* h;                     // [2][B][Ds] GRU states (cleared: h_{-1} = 0)
+  float* u;                     // [B][R]
+  float* partials;              // [grid][kRollMaxB] float4 (max, sum exp, argmax bits, 0)
+  unsigned* barrier;            // grid barrier counter (cleared)
+  int32_t* tokens;              // [B, K] t_1 .. t_K
+  float* logp;                  // [B, K]
+  int* status;
+};
+// dynamic shared memory of one rollout CTA: the W2 ring (head on), u of every sequence and this
+// CTA's rows of base logits + b2; at most kRollMaxSmem
+constexpr size_t kRollMaxSmem = 227 * 1024;
+size_t rollout_smem_bytes(int B, int V, int R, bool head, int grid);
+cudaError_t launch_rollout(const RolloutParams& p, int grid, cudaStream_t stream);
+
 // ---------------------------------------------------------------- tree verification (verify.cu)
 cudaError_t launch_verify_greedy(const float* logits, const int32_t* parent, const int32_t* token, int B, int N,
                                  int V, int32_t* row_argmax, int32_t* nodes, int32_t* count, int32_t* bonus,

@@ -78,3 +78,13 @@ def test_verify_rejects_bad_arguments_before_launch():
     assert f(None, one, one, 1, 4, 10, one, one, one, one) == bad       # no logits
     assert f(one, None, one, 1, 4, 10, one, one, one, one) == bad       # N > 0 without a tree
     assert f(one, one, one, 1, 4, 10, one, None, one, one) == bad       # no accepted_nodes
+
+
+def test_rollout_rejects_bad_sizes_before_any_device_work():
+    f = binding.domino_rollout_workspace_bytes
+    assert f(0, 4, 256, 100, 64, 64) == 0       # B < 1
+    assert f(9, 4, 256, 100, 64, 64) == 0       # B above the rollout's 8
+    assert f(1, 4, 250, 100, 64, 64) == 0       # H not a multiple of 8
+    assert f(1, 4, 256, 100, 60, 64) == 0       # d_s not a multiple of 8
+    assert binding.domino_rollout_greedy(None, None, None, None, 1, 4, 256, 100, None, None, None, 0) == \
+        binding.DOMINO_ERR_INVALID_ARG
