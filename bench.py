@@ -342,6 +342,54 @@ def verify_timing(st, c, device, stream, reps=200):
             "note": "synthetic target logits (planted argmaxes); tau is a mechanics check, not a quality number"}
 
 
+def rollout_timing(st, wl, c, hidden, device, stream, reps=50):
+    """The greedy sequential draft loop (domino_rollout_greedy) on this workload's weights and
+    hidden states: device time per block of K tokens, split into the base-logit GEMM and the
+    cooperative step kernel (per-kernel CUDA events of the library's timing hooks)."""
+    import numpy as np
+    import torch
+    from paper_2605_29707_gb300 import binding
+    if c.B > 8 or not st.head_on:
+        return None
+    anchors = torch.from_numpy(np.ascontiguousarray(wl.prefix_ids[:, 0])).to(device)
+    nb = binding.domino_rollout_workspace_bytes(c.B, c.K, c.H, c.V, c.Ds, c.R)
+    ws = torch.empty(nb, dtype=torch.uint8, device=device)
+    tok = torch.empty((c.B, c.K), dtype=torch.int32, device=device)
+    lp = torch.empty((c.B, c.K), dtype=torch.float32, device=device)
+
+    def run():
+        rc = binding.domino_rollout_greedy(hidden, anchors, st.w["w_lm"], st.head, c.B, c.K, c.H, c.V, tok, lp,
+                                           ws, nb, stream)
+        if rc != 0:
+            raise RuntimeError(f"domino_rollout_greedy returned {rc}")
+    for _ in range(3):
+        run()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(reps):
+        run()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    us = e0.elapsed_time(e1) / reps * 1e3
+    binding.domino_timing_begin(4 * reps)
+    for _ in range(reps):
+        run()
+    torch.cuda.synchronize()
+    kern = binding.domino_timing_end()
+    status = binding.domino_check_status(ws, stream)
+    split = {n: round(v[0] / max(1, v[1]) * 1e3, 2) for n, v in kern.items() if v[1] > 0}
+    # bytes the loop streams per block when nothing stays in L2 across steps: W_lm once, then
+    # every step the GRU weights, W1 and W2
+    head_step = 2 * (3 * c.Ds * c.H + 3 * c.Ds * c.Ds + c.R * (c.H + c.Ds) + c.V * c.R)
+    streamed = 2 * c.V * c.H + c.K * head_step
+    return {"us_per_block": round(us, 2), "draft_tokens_per_s": round(c.B * c.K / (us * 1e-6), 1),
+            "us_per_kernel": split, "status": status, "streamed_bytes_per_block": streamed,
+            "streamed_GB_per_s": round(streamed / (us * 1e-6) / 1e9, 1),
+            "note": "B sequences x K greedy draft tokens, each fed back; timing only (parity is in the tests)"}
+
+
 def graph_replay(st, hidden, ids, device, n, blocks_per_step):
     """Capture one step in a CUDA graph and time n replays; on a capture failure, say why."""
     import torch
@@ -491,6 +539,8 @@ def run_ours(args):
     # ---- the step after the draft: greedy verification of this step's trees against synthetic
     #      target logits [B, N+1, V] fp32 (timing only; parity is in the tests)
     verify = verify_timing(st, c, device, stream) if c.B <= 4 else None
+    # ---- the sequential draft loop (the paper's inference loop) on the same weights
+    rollout = rollout_timing(st, wl, c, hidden, device, stream)
 
     # ---- roofline of the dominant kernel, measured in the timed region
     peaks = load_peaks()
@@ -523,7 +573,7 @@ def run_ours(args):
         "e2e": {"value": round(e2e_value, 3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "steps": n_e2e, "api": "domino_draft_step_host (synchronous per step)"},
         "gpu_launches": args.steps * launches, "clocks": clocks,
-        "head_overhead": head_overhead, "tree_verify": verify,
+        "head_overhead": head_overhead, "tree_verify": verify, "rollout_greedy": rollout,
     }
     # ---- last: the same step replayed from a CUDA graph (one captured step, replayed back to
     #      back); a failed capture is reported in the line, after everything else was measured

@@ -36,6 +36,21 @@ __device__ __forceinline__ void bf8(const __nv_bfloat16* p, float (&f)[8]) {
   }
 }
 
+// 8 bf16 of global memory with an L2 eviction-priority hint
+__device__ __forceinline__ void bf8_hint(const __nv_bfloat16* p, float (&f)[8], uint64_t pol) {
+  uint4 v;
+  asm("ld.global.nc.L2::cache_hint.v4.u32 {%0, %1, %2, %3}, [%4], %5;"
+      : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+      : "l"(p), "l"(pol));
+  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 t = __bfloat1622float2(h[i]);
+    f[2 * i] = t.x;
+    f[2 * i + 1] = t.y;
+  }
+}
+
 // 8 bf16 of shared memory (16-byte aligned) to fp32
 __device__ __forceinline__ void bf8_smem(const __nv_bfloat16* p, float (&f)[8]) {
   const uint4 v = *reinterpret_cast<const uint4*>(p);
@@ -247,7 +262,9 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
     //      every compute warp has released the chunk g - kW2Stages held there
     const long long n_loads = p.head ? static_cast<long long>(K) * nch : 0;
     if (lane == 0 && n_loads > 0) {
-      const uint64_t pol_keep = l2_policy_evict_last();
+      // W2 (r x V, the largest operand) streams through L2 at first-eviction priority so that
+      // the GRU and W1 weights of phases A and B, re-read every step, stay in L2
+      const uint64_t pol_w2 = l2_policy_evict_first();
       long long g = 0;
       for (; g < n_loads; ++g) {
         const int sidx = static_cast<int>(g % kW2Stages);
@@ -259,7 +276,7 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
         const uint32_t bytes = static_cast<uint32_t>(rows) * R * 2;
         mbar_arrive_expect_tx(&s_full[sidx], bytes);
         bulk_load(s_ring + sidx * kW2StageBytes, p.w2 + static_cast<size_t>(c) * ch * R, bytes, &s_full[sidx],
-                  pol_keep);
+                  pol_w2);
       }
       // the CTA leaves only once its copies in flight have landed (bounded)
       for (long long q = g > kW2Stages ? g - kW2Stages : 0; q < g; ++q) {
@@ -279,6 +296,7 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
   const int my_r = my_idx / KB, my_b = my_idx % KB;
   const bool my_rep = (lane & ((32 >> kLogN) - 1)) == 0;  // one lane per value pushes it
 
+  const uint64_t pol_ab = l2_policy_evict_normal();
   unsigned nbar = 0;
   for (int j = 0; j < K; ++j) {
     const float* hprev = p.h + static_cast<size_t>((j + 1) & 1) * B * Ds;  // h_{j-1} (zeros at j = 0)
@@ -293,9 +311,9 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
           for (int c = lane * 8; c < H; c += 256) {
             float xv[8], wr[8], wz[8], wn[8];
             bf8(x + c, xv);
-            bf8(p.w_ih + static_cast<size_t>(q) * H + c, wr);
-            bf8(p.w_ih + static_cast<size_t>(Ds + q) * H + c, wz);
-            bf8(p.w_ih + static_cast<size_t>(2 * Ds + q) * H + c, wn);
+            bf8_hint(p.w_ih + static_cast<size_t>(q) * H + c, wr, pol_ab);
+            bf8_hint(p.w_ih + static_cast<size_t>(Ds + q) * H + c, wz, pol_ab);
+            bf8_hint(p.w_ih + static_cast<size_t>(2 * Ds + q) * H + c, wn, pol_ab);
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
               ar += wr[e] * xv[e];
@@ -307,9 +325,9 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
 #pragma unroll 4
           for (int c = lane * 8; c < Ds; c += 256) {
             float wr[8], wz[8], wn[8];
-            bf8(p.w_hh + static_cast<size_t>(q) * Ds + c, wr);
-            bf8(p.w_hh + static_cast<size_t>(Ds + q) * Ds + c, wz);
-            bf8(p.w_hh + static_cast<size_t>(2 * Ds + q) * Ds + c, wn);
+            bf8_hint(p.w_hh + static_cast<size_t>(q) * Ds + c, wr, pol_ab);
+            bf8_hint(p.w_hh + static_cast<size_t>(Ds + q) * Ds + c, wz, pol_ab);
+            bf8_hint(p.w_hh + static_cast<size_t>(2 * Ds + q) * Ds + c, wn, pol_ab);
             // written by other CTAs in this launch: read through L2, never a stale L1 line
             const float4 h0 = __ldcg(reinterpret_cast<const float4*>(hp + c));
             const float4 h1 = __ldcg(reinterpret_cast<const float4*>(hp + c + 4));
@@ -346,7 +364,7 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
 #pragma unroll 4
           for (int c = lane * 8; c < H; c += 256) {
             float wv[8], xv[8];
-            bf8(w + c, wv);
+            bf8_hint(w + c, wv, pol_ab);
             bf8(hid + c, xv);
 #pragma unroll
             for (int e = 0; e < 8; ++e) acc += wv[e] * xv[e];
@@ -354,7 +372,7 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
 #pragma unroll 4
           for (int c = lane * 8; c < Ds; c += 256) {
             float wv[8];
-            bf8(w + H + c, wv);
+            bf8_hint(w + H + c, wv, pol_ab);
             const float4 h0 = __ldcg(reinterpret_cast<const float4*>(hc + c));
             const float4 h1 = __ldcg(reinterpret_cast<const float4*>(hc + c + 4));
             const float hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
