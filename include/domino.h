@@ -173,11 +173,14 @@ DOMINO_API int domino_verify_tree_greedy(const float* target_logits, const int32
  * With the correction branch off (head NULL, R = 0 or w2 NULL) L_j = W_lm hidden_j + b2.
  *   hidden [B, K, H] bf16, anchors [B] int32, w_lm [V, H] bf16, head as for domino_draft_step,
  *   all device pointers, 16-byte aligned.  B <= 8 (a latency path; batches use
- *   domino_draft_step); H, d_s and r multiples of 8; r <= 8192; one CTA of the step kernel
- *   (one per SM) holds in shared memory a 64 KB ring of W2 rows, u of every sequence (4 B r)
- *   and its share of the base logits (4 B ceil(V / SMs) rows, rounded up to whole W2 chunks),
- *   which must total at most 227 KB (else DOMINO_ERR_INVALID_ARG; B = 8, r = 256 and
- *   V = 151936 take 104 KB).
+ *   domino_draft_step); H, d_s and r multiples of 8; r <= 8192.  The step kernel runs one CTA
+ *   per SM; a CTA's shared memory (at most 225 KB) holds u of every sequence (4 B r) and its
+ *   share of the base logits (4 B ceil(V / SMs) rows), plus, for r <= 256, as many of its W2
+ *   rows as fit (its first 512 W2 rows live in the tensor memory, all of it, of the SM for the
+ *   whole call), or,
+ *   for r > 256, a 96 KB ring W2 streams through every step (those shares rounded up to whole
+ *   ring chunks).  Sizes whose u and base-logit share alone exceed 225 KB return
+ *   DOMINO_ERR_INVALID_ARG.
  * Outputs (device): tokens int32 [B, K] = t_1 .. t_K; logp fp32 [B, K].
  * workspace: device memory of domino_rollout_workspace_bytes(...) bytes (16-byte aligned);
  * its first int32 receives the device status (DOMINO_OK, DOMINO_ERR_BAD_TOKEN,

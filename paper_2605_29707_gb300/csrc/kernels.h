@@ -143,6 +143,7 @@ struct RolloutParams {
   const __nv_bfloat16 *emb, *w_ih, *w_hh, *b_ih, *b_hh, *w1, *b1, *w2, *b2;  // b* may be null
   int head;                     // correction branch on (R > 0 and W2 given)
   int B, K, H, V, Ds, R;
+  int smem_rows;                // set by launch_rollout: W2 rows a CTA keeps in shared memory
   const float* base;            // [B*K, V] W_lm hidden (fp32, from the store-mode GEMM)
   float* h;                     // [2][B][Ds] GRU states (cleared: h_{-1} = 0)
   float* u;                     // [B][R]
@@ -152,9 +153,10 @@ struct RolloutParams {
   float* logp;                  // [B, K]
   int* status;
 };
-// dynamic shared memory of one rollout CTA: the W2 ring (head on), u of every sequence and this
-// CTA's rows of base logits + b2; at most kRollMaxSmem
-constexpr size_t kRollMaxSmem = 227 * 1024;
+// dynamic shared memory of one rollout CTA (the resident W2 rows or the W2 ring, u of every
+// sequence and this CTA's rows of base logits + b2): at most kRollMaxSmem, the 227 KB a CTA may
+// hold less 2 KB for the kernels' static shared memory
+constexpr size_t kRollMaxSmem = 225 * 1024;
 size_t rollout_smem_bytes(int B, int V, int R, bool head, int grid);
 cudaError_t launch_rollout(const RolloutParams& p, int grid, cudaStream_t stream);
 

@@ -1,14 +1,20 @@
 // rollout.cu -- the greedy sequential draft loop (section 4.1.2 and Fig. 3: at inference each
 // draft token is chosen from the final logits L_j = L_base_j + W2 u_j + b2 and becomes the
 // causal encoder's next input).  The base logits W_lm hidden_j of every position come first from
-// the tensor-core GEMM (store mode, fp32); this persistent cooperative kernel then runs the K
+// the tensor-core GEMM (store mode, fp32); a persistent cooperative kernel then runs the K
 // dependent steps, each in three phases separated by grid barriers:
 //   A  GRU step: h_j = GRU(emb[t_j], h_{j-1}), one warp per hidden unit (torch.nn.GRU gates);
 //   B  u_j = SiLU(W1 [hidden_j ; h_j] + b1), one warp per rank row;
-//   C  L_j = base_j + W2 u_j + b2, each lane owning vocabulary rows, with a running max, sum of
-//      exp and argmax (equal values: the lowest id) per sequence, reduced per CTA;
+//   C  L_j = base_j + W2 u_j + b2 over the CTA's slice of the vocabulary, with a running max,
+//      sum of exp and argmax (equal values: the lowest id) per sequence, reduced per CTA;
 // after the third barrier every CTA combines the per-CTA partials itself (the same result
 // everywhere), so t_{j+1} needs no fourth barrier.  Every wait is bounded.
+//
+// W2 (V x r bf16, 78 MB at the Qwen3 vocabulary) is the operand phase C reads every step.  With
+// r <= 256 the resident kernel keeps each CTA's slice of it on chip for the whole block: 512
+// rows in the SM's tensor memory (used as storage: written once with tcgen05.st, read with
+// tcgen05.ld), as many rows as fit in shared memory, and the few rows left read through L2.
+// Wider r uses the streamed kernel, which feeds W2 through a shared-memory ring every step.
 #include <math.h>
 
 #include "kernels.h"
@@ -16,17 +22,21 @@
 
 namespace dm {
 
-constexpr int kRollThreads = 256;                 // the compute warps
+constexpr int kRollThreads = 256;                   // the compute warps
 constexpr int kRollWarps = kRollThreads / 32;
-constexpr int kRollThreadsAll = kRollThreads + 32;  // + one warp streaming W2 into shared memory
+constexpr int kRollThreadsAll = kRollThreads + 32;  // streamed kernel: + one warp feeding the W2 ring
 constexpr int kW2Stages = 6;                        // shared-memory ring of W2 chunks
 constexpr int kW2StageBytes = 16 * 1024;            // one chunk: kW2StageBytes / (2 r) rows of W2
 constexpr int kRowsPerPass = 4;                     // W2 rows one warp takes at a time
+constexpr int kResidentMaxR = 256;                  // r one lane's 8 columns x 32 lanes cover
+constexpr int kTmemCols = 512;                      // the whole tensor memory of an SM
+// W2 rows in tensor memory: lane quarter q (warps q and q + 4) holds rows 128 q .. 128 q + 127,
+// TMEM lane 32 q + l holding columns 8 l .. 8 l + 7 of each (4 32-bit columns per row)
+constexpr int kTmemRows = 4 * (kTmemCols / 4);
 
 __device__ __forceinline__ float bf2f(__nv_bfloat16 x) { return __bfloat162float(x); }
 
-__device__ __forceinline__ void bf8(const __nv_bfloat16* p, float (&f)[8]) {
-  const uint4 v = __ldg(reinterpret_cast<const uint4*>(p));
+__device__ __forceinline__ void unpack8(const uint4& v, float (&f)[8]) {
   const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
@@ -36,47 +46,49 @@ __device__ __forceinline__ void bf8(const __nv_bfloat16* p, float (&f)[8]) {
   }
 }
 
-// 8 bf16 of global memory with an L2 eviction-priority hint
-__device__ __forceinline__ void bf8_hint(const __nv_bfloat16* p, float (&f)[8], uint64_t pol) {
+__device__ __forceinline__ void bf8(const __nv_bfloat16* p, float (&f)[8]) {
+  unpack8(__ldg(reinterpret_cast<const uint4*>(p)), f);
+}
+
+// 16 bytes of global memory with an L2 eviction-priority hint
+__device__ __forceinline__ uint4 ld16_hint(const void* p, uint64_t pol) {
   uint4 v;
   asm("ld.global.nc.L2::cache_hint.v4.u32 {%0, %1, %2, %3}, [%4], %5;"
       : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
       : "l"(p), "l"(pol));
-  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const float2 t = __bfloat1622float2(h[i]);
-    f[2 * i] = t.x;
-    f[2 * i + 1] = t.y;
-  }
+  return v;
 }
 
-// 8 bf16 of shared memory (16-byte aligned) to fp32
-__device__ __forceinline__ void bf8_smem(const __nv_bfloat16* p, float (&f)[8]) {
-  const uint4 v = *reinterpret_cast<const uint4*>(p);
-  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const float2 t = __bfloat1622float2(h[i]);
-    f[2 * i] = t.x;
-    f[2 * i + 1] = t.y;
-  }
+__device__ __forceinline__ void bf8_hint(const __nv_bfloat16* p, float (&f)[8], uint64_t pol) {
+  unpack8(ld16_hint(p, pol), f);
 }
 
-// Columns cc .. cc + 7 of the pass's rows r0 .. r0 + 3 of a W2 chunk in shared memory (rows
-// past the chunk's end read as zero).
+// Columns cc .. cc + 7 of rows r0 .. r0 + 3 of a row-major W2 block in shared memory (rows past
+// `rows` read as zero).
 __device__ __forceinline__ void load_rows(const __nv_bfloat16* sw, int r0, int rows, int R, int cc,
                                           float (&wv)[kRowsPerPass][8]) {
 #pragma unroll
   for (int r = 0; r < kRowsPerPass; ++r) {
     if (r0 + r < rows) {
-      bf8_smem(sw + static_cast<size_t>(r0 + r) * R + cc, wv[r]);
+      unpack8(*reinterpret_cast<const uint4*>(sw + static_cast<size_t>(r0 + r) * R + cc), wv[r]);
     } else {
 #pragma unroll
       for (int e = 0; e < 8; ++e) wv[r][e] = 0.f;
     }
   }
 }
+
+// tensor memory: each thread of the warp writes 16 consecutive 32-bit columns of its lane
+__device__ __forceinline__ void tc_st_x16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+      "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
+}
+
+__device__ __forceinline__ void tc_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
 __device__ __forceinline__ float warp_sum(float x) {
 #pragma unroll
@@ -114,8 +126,8 @@ struct ReduceScatter<1, O> {
 
 __host__ __device__ constexpr int ilog2(int n) { return n <= 1 ? 0 : 1 + ilog2(n / 2); }
 
-// Rows of the vocabulary one CTA covers: a contiguous run of chunks of `ch` rows (ch = the rows
-// of W2 in one ring stage with the head on, 1024 without it).
+// Streamed kernel: rows of the vocabulary one CTA covers, a contiguous run of chunks of `ch`
+// rows (ch = the rows of W2 in one ring stage with the head on, 1024 without it).
 __host__ __device__ inline int rollout_chunk_rows(int R, int head) {
   return head ? max(1, kW2StageBytes / (2 * R)) : 1024;
 }
@@ -160,7 +172,7 @@ __device__ __forceinline__ void lse_merge(Lse& a, const Lse& b) {
   a.i = i;
 }
 
-// Barrier of the compute warps only (the streaming warp runs on its own).
+// Barrier of the compute warps only (the streamed kernel's feeding warp runs on its own).
 __device__ __forceinline__ void compute_sync() {
   asm volatile("bar.sync 1, %0;" ::"n"(kRollThreads) : "memory");
 }
@@ -213,11 +225,408 @@ __device__ bool grid_barrier(unsigned* ctr, unsigned n, int* status, volatile in
   return *fail == 0;
 }
 
-// KB: sequences the phase-C arithmetic is laid out for (B <= KB; the extra ones compute on
-// zeros and are never read).
+// ---- phase A: h_j = GRU(emb[t_j], h_{j-1}) (torch.nn.GRU: gates r|z|n, r multiplies
+//      W_hn h + b_hn), one warp per hidden unit q, every sequence
+__device__ __forceinline__ void gru_phase(const RolloutParams& p, const int* s_tok, const float* hprev, float* hcur,
+                                          int gw, int nwarps, int lane, uint64_t pol) {
+  const int B = p.B, H = p.H, Ds = p.Ds;
+  for (int q = gw; q < Ds; q += nwarps) {
+    for (int b = 0; b < B; ++b) {
+      const __nv_bfloat16* x = p.emb + static_cast<size_t>(s_tok[b]) * H;
+      float ar = 0.f, az = 0.f, an = 0.f, hr = 0.f, hz = 0.f, hn = 0.f;
+#pragma unroll 4
+      for (int c = lane * 8; c < H; c += 256) {
+        float xv[8], wr[8], wz[8], wn[8];
+        bf8(x + c, xv);
+        bf8_hint(p.w_ih + static_cast<size_t>(q) * H + c, wr, pol);
+        bf8_hint(p.w_ih + static_cast<size_t>(Ds + q) * H + c, wz, pol);
+        bf8_hint(p.w_ih + static_cast<size_t>(2 * Ds + q) * H + c, wn, pol);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          ar += wr[e] * xv[e];
+          az += wz[e] * xv[e];
+          an += wn[e] * xv[e];
+        }
+      }
+      const float* hp = hprev + static_cast<size_t>(b) * Ds;
+#pragma unroll 4
+      for (int c = lane * 8; c < Ds; c += 256) {
+        float wr[8], wz[8], wn[8];
+        bf8_hint(p.w_hh + static_cast<size_t>(q) * Ds + c, wr, pol);
+        bf8_hint(p.w_hh + static_cast<size_t>(Ds + q) * Ds + c, wz, pol);
+        bf8_hint(p.w_hh + static_cast<size_t>(2 * Ds + q) * Ds + c, wn, pol);
+        // written by other CTAs in this launch: read through L2, never a stale L1 line
+        const float4 h0 = __ldcg(reinterpret_cast<const float4*>(hp + c));
+        const float4 h1 = __ldcg(reinterpret_cast<const float4*>(hp + c + 4));
+        const float hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          hr += wr[e] * hv[e];
+          hz += wz[e] * hv[e];
+          hn += wn[e] * hv[e];
+        }
+      }
+      ar = warp_sum(ar); az = warp_sum(az); an = warp_sum(an);
+      hr = warp_sum(hr); hz = warp_sum(hz); hn = warp_sum(hn);
+      if (lane == 0) {
+        const float bir = p.b_ih ? bf2f(p.b_ih[q]) : 0.f, biz = p.b_ih ? bf2f(p.b_ih[Ds + q]) : 0.f;
+        const float bin = p.b_ih ? bf2f(p.b_ih[2 * Ds + q]) : 0.f;
+        const float bhr = p.b_hh ? bf2f(p.b_hh[q]) : 0.f, bhz = p.b_hh ? bf2f(p.b_hh[Ds + q]) : 0.f;
+        const float bhn = p.b_hh ? bf2f(p.b_hh[2 * Ds + q]) : 0.f;
+        const float r = 1.f / (1.f + expf(-(ar + bir + hr + bhr)));
+        const float z = 1.f / (1.f + expf(-(az + biz + hz + bhz)));
+        const float n = tanhf(an + bin + r * (hn + bhn));
+        hcur[static_cast<size_t>(b) * Ds + q] = (1.f - z) * n + z * __ldcg(hp + q);
+      }
+    }
+  }
+}
+
+// ---- phase B: u_j = SiLU(W1 [hidden_j ; h_j] + b1), one warp per rank row q, every sequence
+__device__ __forceinline__ void u_phase(const RolloutParams& p, int j, const float* hcur, int gw, int nwarps,
+                                        int lane, uint64_t pol) {
+  const int B = p.B, K = p.K, H = p.H, Ds = p.Ds, R = p.R;
+  for (int q = gw; q < R; q += nwarps) {
+    const __nv_bfloat16* w = p.w1 + static_cast<size_t>(q) * (H + Ds);
+    for (int b = 0; b < B; ++b) {
+      const __nv_bfloat16* hid = p.hidden + (static_cast<size_t>(b) * K + j) * H;
+      const float* hc = hcur + static_cast<size_t>(b) * Ds;
+      float acc = 0.f;
+#pragma unroll 4
+      for (int c = lane * 8; c < H; c += 256) {
+        float wv[8], xv[8];
+        bf8_hint(w + c, wv, pol);
+        bf8(hid + c, xv);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc += wv[e] * xv[e];
+      }
+#pragma unroll 4
+      for (int c = lane * 8; c < Ds; c += 256) {
+        float wv[8];
+        bf8_hint(w + H + c, wv, pol);
+        const float4 h0 = __ldcg(reinterpret_cast<const float4*>(hc + c));
+        const float4 h1 = __ldcg(reinterpret_cast<const float4*>(hc + c + 4));
+        const float hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc += wv[e] * hv[e];
+      }
+      acc = warp_sum(acc);
+      if (lane == 0) {
+        const float a = acc + (p.b1 ? bf2f(p.b1[q]) : 0.f);
+        p.u[static_cast<size_t>(b) * R + q] = a / (1.f + expf(-a));
+      }
+    }
+  }
+}
+
+// ---- phase C, one pass of a warp: 4 rows x KB sequences.  A lane holds 8 consecutive columns
+//      of each row (wv) and of u (ur); the 4 KB dot products are summed over the warp by a
+//      reduce-scatter, after which lane `role.idx` holds row role.r of sequence role.b.
+struct PassRole {
+  int r, b;
+  bool rep;  // the one lane of those holding the same value that pushes it
+};
+
+template <int KB>
+__device__ __forceinline__ PassRole pass_role(int lane) {
+  constexpr int kN = kRowsPerPass * KB;
+  constexpr int kLogN = ilog2(kN);
+  static_assert((1 << kLogN) == kN && kN <= 32, "rows x sequences per pass must be a power of two <= 32");
+  const int idx = lane >> (5 - kLogN);
+  PassRole role;
+  role.r = idx / KB;
+  role.b = idx % KB;
+  role.rep = (lane & ((32 >> kLogN) - 1)) == 0;
+  return role;
+}
+
+template <int KB>
+__device__ __forceinline__ void pass_fma(const float (&wv)[kRowsPerPass][8], const float (&uv)[KB][8],
+                                         float (&dot)[kRowsPerPass * KB]) {
+#pragma unroll
+  for (int r = 0; r < kRowsPerPass; ++r)
+#pragma unroll
+    for (int b = 0; b < KB; ++b)
+#pragma unroll
+      for (int e = 0; e < 8; ++e) dot[r * KB + b] += wv[r][e] * uv[b][e];
+}
+
+// Sums the pass over the warp and pushes row (row0 + role.r) of sequence role.b: CTA-local
+// row index row0 (for the staged base logits), vocabulary id vid0 + role.r, nvalid rows valid.
+template <int KB>
+__device__ __forceinline__ void pass_push(const float (&dot)[kRowsPerPass * KB], const PassRole& role, int nvalid,
+                                          int row0, int vid0, const float* s_base, int rows_cta, int B, Lse& mine) {
+  const float d = ReduceScatter<kRowsPerPass * KB, 16>::run(dot);
+  if (role.rep && role.r < nvalid && role.b < B)
+    lse_push(mine, s_base[role.b * rows_cta + row0 + role.r] + d, vid0 + role.r);
+}
+
+// The end of a step, shared by both kernels: per-CTA partials, grid barrier, every CTA's
+// combine (thread c loads CTA c's partials, then the same block reduction in every CTA, so all
+// reach the same t_{j+1}), the outputs.  Returns false if the barrier gave up.
+template <int KB>
+__device__ __forceinline__ bool finish_step(const RolloutParams& p, int j, Lse (&st)[KB], Lse (*s_red)[kRollMaxB],
+                                            int* s_tok, unsigned& nbar, volatile int* s_fail) {
+  const int B = p.B, K = p.K, tid = threadIdx.x;
+  block_reduce(st, s_red, B);
+  if (tid < B) {
+    Lse a = s_red[0][tid];
+    for (int w = 1; w < kRollWarps; ++w) lse_merge(a, s_red[w][tid]);
+    float4* out = reinterpret_cast<float4*>(p.partials) + static_cast<size_t>(blockIdx.x) * kRollMaxB + tid;
+    *out = make_float4(a.m, a.s, __int_as_float(a.i), 0.f);
+  }
+  if (!grid_barrier(p.barrier, nbar++, p.status, s_fail)) return false;
+#pragma unroll
+  for (int b = 0; b < KB; ++b) st[b] = lse_empty();
+  for (int c = tid; c < static_cast<int>(gridDim.x); c += kRollThreads) {
+#pragma unroll
+    for (int b = 0; b < KB; ++b) {
+      if (b < B) {
+        const float4 f = __ldcg(reinterpret_cast<const float4*>(p.partials) + static_cast<size_t>(c) * kRollMaxB + b);
+        Lse t;
+        t.m = f.x; t.s = f.y; t.i = __float_as_int(f.z);
+        lse_merge(st[b], t);
+      }
+    }
+  }
+  block_reduce(st, s_red, B);
+  if (tid < B) {
+    Lse a = s_red[0][tid];
+    for (int w = 1; w < kRollWarps; ++w) lse_merge(a, s_red[w][tid]);
+    const int tok = a.i == 0x7fffffff ? 0 : a.i;
+    s_tok[tid] = tok;
+    if (blockIdx.x == 0) {
+      p.tokens[static_cast<size_t>(tid) * K + j] = tok;
+      p.logp[static_cast<size_t>(tid) * K + j] = -logf(a.s);  // the argmax's logit is the max
+    }
+  }
+  compute_sync();
+  return true;
+}
+
+// Base logits + b2 of step j for this CTA's rows [r_lo, r_lo + r_n), staged in shared memory.
+__device__ __forceinline__ void stage_base(const RolloutParams& p, int j, int r_lo, int r_n, int rows_cta,
+                                           float* s_base) {
+  const int B = p.B, K = p.K, V = p.V;
+  for (int e = threadIdx.x; e < B * r_n; e += kRollThreads) {
+    const int b = e / r_n, r = e - b * r_n;
+    s_base[b * rows_cta + r] = __ldcg(p.base + (static_cast<size_t>(b) * K + j) * V + r_lo + r) +
+                               (p.b2 ? bf2f(p.b2[r_lo + r]) : 0.f);
+  }
+}
+
+// ---- phase C, resident kernel: a pass covers 32 / KB rows x KB sequences, so that after the
+//      reduce-scatter every lane holds one finished dot product (row lane / KB, sequence
+//      lane % KB); rows come in groups of up to 8, each a 16-byte load per lane.
+template <int KB>
+struct WidePass {
+  static constexpr int kRows = 32 / KB;
+  static constexpr int kGroup = kRows < 8 ? kRows : 8;
+};
+
+template <int KB, int G>
+__device__ __forceinline__ void group_fma(const uint4 (&raw)[G], int r_in_pass, const float (&ur)[KB][8],
+                                          float (&dot)[32]) {
+#pragma unroll
+  for (int r = 0; r < G; ++r) {
+    float w[8];
+    unpack8(raw[r], w);
+#pragma unroll
+    for (int b = 0; b < KB; ++b)
+#pragma unroll
+      for (int e = 0; e < 8; ++e) dot[(r_in_pass + r) * KB + b] += w[e] * ur[b][e];
+  }
+}
+
+template <int KB>
+__device__ __forceinline__ void wide_push(const float (&dot)[32], int lane, int nvalid, int row0, int vid0,
+                                          const float* s_base, int rows_cta, int B, Lse& mine) {
+  const float d = ReduceScatter<32, 16>::run(dot);
+  const int r = lane / KB, b = lane % KB;
+  if (r < nvalid && b < B) lse_push(mine, s_base[b * rows_cta + row0 + r] + d, vid0 + r);
+}
+
+// ================================================================ resident kernel (r <= 256)
+__host__ __device__ inline int resident_rows_per_cta(int V, int grid) { return (V + grid - 1) / grid; }
+
+template <int KB>
+__global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const RolloutParams p) {
+  const int B = p.B, K = p.K, V = p.V, R = p.R;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int nwarps = gridDim.x * kRollWarps;
+  const int gw = blockIdx.x * kRollWarps + warp;
+  // this CTA's rows: [r_lo, r_lo + r_n); the first n_t in tensor memory, the next n_s in
+  // shared memory, the last n_g read from global memory (L2) every step
+  const int rows_cta = resident_rows_per_cta(V, gridDim.x);
+  const int r_lo = min(V, static_cast<int>(blockIdx.x) * rows_cta);
+  const int r_n = min(V, r_lo + rows_cta) - r_lo;
+  const int n_t = min(r_n, kTmemRows);
+  const int n_s = min(r_n - n_t, p.smem_rows);
+  const int n_g = r_n - n_t - n_s;
+  extern __shared__ __align__(128) uint8_t s_dyn[];
+  __nv_bfloat16* s_w2 = reinterpret_cast<__nv_bfloat16*>(s_dyn);                      // [smem_rows][R]
+  float* s_u = reinterpret_cast<float*>(s_dyn + static_cast<size_t>(p.smem_rows) * R * 2);  // [B][R]
+  float* s_base = s_u + B * R;                                                          // [B][rows_cta]
+  __shared__ __align__(8) uint64_t s_fill;  // the shared-memory rows landed
+  __shared__ uint32_t s_tmem;
+  __shared__ int s_tok[kRollMaxB];
+  __shared__ Lse s_red[kRollWarps][kRollMaxB];
+  __shared__ int s_fail;
+  if (tid == 0) {
+    s_fail = 0;
+    mbar_init(&s_fill, 1);
+    fence_mbar_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(&s_tmem, kTmemCols);
+    tmem_relinquish();
+  }
+  if (tid < B) s_tok[tid] = p.anchors[tid];
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tbase = s_tmem;
+  bool tokens_ok = true;
+  for (int b = 0; b < B; ++b)
+    if (s_tok[b] < 0 || s_tok[b] >= V) tokens_ok = false;  // the same ids in every CTA
+  bool fill_issued = false;
+  if (!tokens_ok) {
+    if (tid == 0) set_status(p.status, kStatusBadToken);
+  } else {
+    // ---- fill: shared-memory rows by bulk copies (one barrier, pieces of at most 64 KB)
+    if (tid == 0) {
+      const uint32_t bytes = static_cast<uint32_t>(n_s) * R * 2;
+      mbar_arrive_expect_tx(&s_fill, bytes);
+      const uint8_t* src = reinterpret_cast<const uint8_t*>(p.w2 + static_cast<size_t>(r_lo + n_t) * R);
+      for (uint32_t off = 0; off < bytes; off += 64 * 1024) {
+        const uint32_t n = min(bytes - off, 64u * 1024u);
+        bulk_load(reinterpret_cast<uint8_t*>(s_w2) + off, src + off, n, &s_fill, l2_policy_evict_first());
+      }
+    }
+    fill_issued = true;
+    // ---- fill: tensor-memory rows.  Warp w writes lane quarter q = w % 4, rows 64 (w / 4) ..
+    //      64 (w / 4) + 63 of the quarter's 128, 4 rows (16 columns) per store.
+    const int q = warp & 3, half = warp >> 2;
+    const uint32_t tq = tbase + (static_cast<uint32_t>(32 * q) << 16);
+    const uint64_t pol_once = l2_policy_evict_first();
+#pragma unroll 1
+    for (int g0 = 0; g0 < 64; g0 += 32) {
+      uint4 v[32];  // 8 groups of 4 rows in flight
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const int row = 128 * q + 64 * half + g0 + i;  // CTA-local
+        v[i] = (row < n_t && lane * 8 < R)
+                   ? ld16_hint(p.w2 + static_cast<size_t>(r_lo + row) * R + lane * 8, pol_once)
+                   : make_uint4(0, 0, 0, 0);
+      }
+#pragma unroll
+      for (int gi = 0; gi < 8; ++gi) {
+        const uint32_t r[16] = {v[4 * gi].x,     v[4 * gi].y,     v[4 * gi].z,     v[4 * gi].w,
+                                v[4 * gi + 1].x, v[4 * gi + 1].y, v[4 * gi + 1].z, v[4 * gi + 1].w,
+                                v[4 * gi + 2].x, v[4 * gi + 2].y, v[4 * gi + 2].z, v[4 * gi + 2].w,
+                                v[4 * gi + 3].x, v[4 * gi + 3].y, v[4 * gi + 3].z, v[4 * gi + 3].w};
+        tc_st_x16(tq + static_cast<uint32_t>(4 * (64 * half + g0 + 4 * gi)), r);
+      }
+    }
+    tc_wait_st();  // a warp reads back only what it wrote itself
+
+    constexpr int kRows = WidePass<KB>::kRows, kGroup = WidePass<KB>::kGroup;
+    const uint64_t pol_ab = l2_policy_evict_normal();
+    const uint64_t pol_rest = l2_policy_evict_last();
+    const int n_sg = n_s + n_g;  // rows past tensor memory: shared memory first, then L2
+    unsigned nbar = 0;
+    for (int j = 0; j < K; ++j) {
+      const float* hprev = p.h + static_cast<size_t>((j + 1) & 1) * B * p.Ds;  // h_{j-1} (zeros at j = 0)
+      float* hcur = p.h + static_cast<size_t>(j & 1) * B * p.Ds;
+      gru_phase(p, s_tok, hprev, hcur, gw, nwarps, lane, pol_ab);
+      if (!grid_barrier(p.barrier, nbar++, p.status, &s_fail)) break;
+      u_phase(p, j, hcur, gw, nwarps, lane, pol_ab);
+      if (!grid_barrier(p.barrier, nbar++, p.status, &s_fail)) break;
+      for (int e = tid; e < B * R; e += kRollThreads) s_u[e] = __ldcg(p.u + e);
+      stage_base(p, j, r_lo, r_n, rows_cta, s_base);
+      compute_sync();
+      float ur[KB][8];  // u at this lane's 8 columns (zero past r)
+#pragma unroll
+      for (int b = 0; b < KB; ++b)
+#pragma unroll
+        for (int e = 0; e < 8; ++e) ur[b][e] = (b < B && lane * 8 < R) ? s_u[b * R + lane * 8 + e] : 0.f;
+      Lse mine = lse_empty();
+      // rows in tensor memory: this warp's 64 rows of its lane quarter, 8 rows (32 columns) a load
+      for (int rho0 = 64 * half; rho0 < 64 * half + 64; rho0 += kRows) {
+        const int row0 = 128 * q + rho0;
+        if (row0 >= n_t) break;
+        float dot[32] = {};
+#pragma unroll
+        for (int g = 0; g < kRows; g += kGroup) {
+          uint4 raw[kGroup];
+          if (kGroup == 8) {
+            float t[32];
+            tc_ld_x32(tq + static_cast<uint32_t>(4 * (rho0 + g)), t);
+            tc_wait_ld();
+#pragma unroll
+            for (int r = 0; r < kGroup; ++r)
+              raw[r] = make_uint4(__float_as_uint(t[4 * r]), __float_as_uint(t[4 * r + 1]),
+                                  __float_as_uint(t[4 * r + 2]), __float_as_uint(t[4 * r + 3]));
+          } else {
+            float t[16];
+            tc_ld_x16(tq + static_cast<uint32_t>(4 * (rho0 + g)), t);
+            tc_wait_ld();
+#pragma unroll
+            for (int r = 0; r < kGroup; ++r)
+              raw[r] = make_uint4(__float_as_uint(t[4 * r]), __float_as_uint(t[4 * r + 1]),
+                                  __float_as_uint(t[4 * r + 2]), __float_as_uint(t[4 * r + 3]));
+          }
+          group_fma<KB, kGroup>(raw, g, ur, dot);
+        }
+        wide_push<KB>(dot, lane, n_t - row0, row0, r_lo + row0, s_base, rows_cta, B, mine);
+      }
+      // rows past tensor memory: shared memory (landed before the first step's phase C) then L2
+      if (j == 0 && n_s > 0) mbar_wait(&s_fill, 0, &s_fail, p.status);
+      if (!s_fail) {
+        for (int r0 = warp * kRows; r0 < n_sg; r0 += kRollWarps * kRows) {
+          float dot[32] = {};
+#pragma unroll
+          for (int g = 0; g < kRows; g += kGroup) {
+            uint4 raw[kGroup];
+#pragma unroll
+            for (int r = 0; r < kGroup; ++r) {
+              const int row = r0 + g + r;
+              if (row < n_s && lane * 8 < R)
+                raw[r] = *reinterpret_cast<const uint4*>(s_w2 + static_cast<size_t>(row) * R + lane * 8);
+              else if (row < n_sg && lane * 8 < R)
+                raw[r] = ld16_hint(p.w2 + static_cast<size_t>(r_lo + n_t + row) * R + lane * 8, pol_rest);
+              else
+                raw[r] = make_uint4(0, 0, 0, 0);
+            }
+            group_fma<KB, kGroup>(raw, g, ur, dot);
+          }
+          wide_push<KB>(dot, lane, n_sg - r0, n_t + r0, r_lo + n_t + r0, s_base, rows_cta, B, mine);
+        }
+      }
+      Lse st[KB];
+#pragma unroll
+      for (int b = 0; b < KB; ++b) st[b] = (b == lane % KB) ? mine : lse_empty();
+      if (!finish_step<KB>(p, j, st, s_red, s_tok, nbar, &s_fail)) break;
+    }
+  }
+  // ---- teardown: the shared-memory fill has landed (bounded), tensor memory is released
+  if (tid == 0 && fill_issued && n_s > 0) {
+    const long long t0 = clock64();
+    while (!mbar_try_wait(&s_fill, 0))
+      if (clock64() - t0 > kWaitCycles) break;
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tbase, kTmemCols);
+  }
+}
+
+// ================================================================ streamed kernel (any r)
 template <int KB>
 __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const RolloutParams p) {
-  const int B = p.B, K = p.K, H = p.H, V = p.V, Ds = p.Ds, R = p.R;
+  const int B = p.B, K = p.K, V = p.V, R = p.R;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nwarps = gridDim.x * kRollWarps;
   const int gw = blockIdx.x * kRollWarps + warp;
@@ -258,12 +667,12 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
     }
 
   if (warp == kRollWarps) {
-    // ---- streaming warp: chunk g of the stream (step g / nch) into stage g % kW2Stages once
+    // ---- feeding warp: chunk g of the stream (step g / nch) into stage g % kW2Stages once
     //      every compute warp has released the chunk g - kW2Stages held there
     const long long n_loads = p.head ? static_cast<long long>(K) * nch : 0;
     if (lane == 0 && n_loads > 0) {
-      // W2 (r x V, the largest operand) streams through L2 at first-eviction priority so that
-      // the GRU and W1 weights of phases A and B, re-read every step, stay in L2
+      // W2 streams through L2 at first-eviction priority so that the GRU and W1 weights of
+      // phases A and B, re-read every step, stay in L2
       const uint64_t pol_w2 = l2_policy_evict_first();
       long long g = 0;
       for (; g < n_loads; ++g) {
@@ -288,122 +697,28 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
     return;
   }
 
-  // phase-C lane roles: value (r, b) of a pass lands on lanes with idx = r * KB + b
-  constexpr int kN = kRowsPerPass * KB;
-  constexpr int kLogN = ilog2(kN);
-  static_assert((1 << kLogN) == kN && kN <= 32, "rows x sequences per pass must be a power of two <= 32");
-  const int my_idx = lane >> (5 - kLogN);
-  const int my_r = my_idx / KB, my_b = my_idx % KB;
-  const bool my_rep = (lane & ((32 >> kLogN) - 1)) == 0;  // one lane per value pushes it
-
+  const PassRole role = pass_role<KB>(lane);
   const uint64_t pol_ab = l2_policy_evict_normal();
   unsigned nbar = 0;
   for (int j = 0; j < K; ++j) {
-    const float* hprev = p.h + static_cast<size_t>((j + 1) & 1) * B * Ds;  // h_{j-1} (zeros at j = 0)
-    float* hcur = p.h + static_cast<size_t>(j & 1) * B * Ds;
+    const float* hprev = p.h + static_cast<size_t>((j + 1) & 1) * B * p.Ds;  // h_{j-1} (zeros at j = 0)
+    float* hcur = p.h + static_cast<size_t>(j & 1) * B * p.Ds;
     if (p.head) {
-      // ---- A: GRU step (torch.nn.GRU: gates r|z|n, r multiplies W_hn h + b_hn)
-      for (int q = gw; q < Ds; q += nwarps) {
-        for (int b = 0; b < B; ++b) {
-          const __nv_bfloat16* x = p.emb + static_cast<size_t>(s_tok[b]) * H;
-          float ar = 0.f, az = 0.f, an = 0.f, hr = 0.f, hz = 0.f, hn = 0.f;
-#pragma unroll 4
-          for (int c = lane * 8; c < H; c += 256) {
-            float xv[8], wr[8], wz[8], wn[8];
-            bf8(x + c, xv);
-            bf8_hint(p.w_ih + static_cast<size_t>(q) * H + c, wr, pol_ab);
-            bf8_hint(p.w_ih + static_cast<size_t>(Ds + q) * H + c, wz, pol_ab);
-            bf8_hint(p.w_ih + static_cast<size_t>(2 * Ds + q) * H + c, wn, pol_ab);
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              ar += wr[e] * xv[e];
-              az += wz[e] * xv[e];
-              an += wn[e] * xv[e];
-            }
-          }
-          const float* hp = hprev + static_cast<size_t>(b) * Ds;
-#pragma unroll 4
-          for (int c = lane * 8; c < Ds; c += 256) {
-            float wr[8], wz[8], wn[8];
-            bf8_hint(p.w_hh + static_cast<size_t>(q) * Ds + c, wr, pol_ab);
-            bf8_hint(p.w_hh + static_cast<size_t>(Ds + q) * Ds + c, wz, pol_ab);
-            bf8_hint(p.w_hh + static_cast<size_t>(2 * Ds + q) * Ds + c, wn, pol_ab);
-            // written by other CTAs in this launch: read through L2, never a stale L1 line
-            const float4 h0 = __ldcg(reinterpret_cast<const float4*>(hp + c));
-            const float4 h1 = __ldcg(reinterpret_cast<const float4*>(hp + c + 4));
-            const float hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-              hr += wr[e] * hv[e];
-              hz += wz[e] * hv[e];
-              hn += wn[e] * hv[e];
-            }
-          }
-          ar = warp_sum(ar); az = warp_sum(az); an = warp_sum(an);
-          hr = warp_sum(hr); hz = warp_sum(hz); hn = warp_sum(hn);
-          if (lane == 0) {
-            const float bir = p.b_ih ? bf2f(p.b_ih[q]) : 0.f, biz = p.b_ih ? bf2f(p.b_ih[Ds + q]) : 0.f;
-            const float bin = p.b_ih ? bf2f(p.b_ih[2 * Ds + q]) : 0.f;
-            const float bhr = p.b_hh ? bf2f(p.b_hh[q]) : 0.f, bhz = p.b_hh ? bf2f(p.b_hh[Ds + q]) : 0.f;
-            const float bhn = p.b_hh ? bf2f(p.b_hh[2 * Ds + q]) : 0.f;
-            const float r = 1.f / (1.f + expf(-(ar + bir + hr + bhr)));
-            const float z = 1.f / (1.f + expf(-(az + biz + hz + bhz)));
-            const float n = tanhf(an + bin + r * (hn + bhn));
-            hcur[static_cast<size_t>(b) * Ds + q] = (1.f - z) * n + z * __ldcg(hp + q);
-          }
-        }
-      }
+      gru_phase(p, s_tok, hprev, hcur, gw, nwarps, lane, pol_ab);
       if (!grid_barrier(p.barrier, nbar++, p.status, &s_fail)) return;
-      // ---- B: u_j = SiLU(W1 [hidden_j ; h_j] + b1)
-      for (int q = gw; q < R; q += nwarps) {
-        const __nv_bfloat16* w = p.w1 + static_cast<size_t>(q) * (H + Ds);
-        for (int b = 0; b < B; ++b) {
-          const __nv_bfloat16* hid = p.hidden + (static_cast<size_t>(b) * K + j) * H;
-          const float* hc = hcur + static_cast<size_t>(b) * Ds;
-          float acc = 0.f;
-#pragma unroll 4
-          for (int c = lane * 8; c < H; c += 256) {
-            float wv[8], xv[8];
-            bf8_hint(w + c, wv, pol_ab);
-            bf8(hid + c, xv);
-#pragma unroll
-            for (int e = 0; e < 8; ++e) acc += wv[e] * xv[e];
-          }
-#pragma unroll 4
-          for (int c = lane * 8; c < Ds; c += 256) {
-            float wv[8];
-            bf8_hint(w + H + c, wv, pol_ab);
-            const float4 h0 = __ldcg(reinterpret_cast<const float4*>(hc + c));
-            const float4 h1 = __ldcg(reinterpret_cast<const float4*>(hc + c + 4));
-            const float hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
-#pragma unroll
-            for (int e = 0; e < 8; ++e) acc += wv[e] * hv[e];
-          }
-          acc = warp_sum(acc);
-          if (lane == 0) {
-            const float a = acc + (p.b1 ? bf2f(p.b1[q]) : 0.f);
-            p.u[static_cast<size_t>(b) * R + q] = a / (1.f + expf(-a));
-          }
-        }
-      }
+      u_phase(p, j, hcur, gw, nwarps, lane, pol_ab);
       if (!grid_barrier(p.barrier, nbar++, p.status, &s_fail)) return;
       for (int e = tid; e < B * R; e += kRollThreads) s_u[e] = __ldcg(p.u + e);
     }
     // ---- C: L_j = base_j + W2 u_j + b2 over this CTA's rows; running max / sum exp / argmax
-    for (int e = tid; e < B * r_n; e += kRollThreads) {
-      const int b = e / r_n, r = e - b * r_n;
-      s_base[b * rows_cta + r] = __ldcg(p.base + (static_cast<size_t>(b) * K + j) * V + r_lo + r) +
-                                 (p.b2 ? bf2f(p.b2[r_lo + r]) : 0.f);
-    }
+    stage_base(p, j, r_lo, r_n, rows_cta, s_base);
     compute_sync();
     Lse st[KB];
 #pragma unroll
     for (int b = 0; b < KB; ++b) st[b] = lse_empty();
     if (p.head) {
       // W2 rows arrive chunk by chunk in the ring; warp w takes rows 4w .. 4w + 3, 4w + 32, ...
-      // of a chunk, a lane holding 8 consecutive columns of each (one 16-byte load per row); the
-      // 4 x KB dot products of a pass are summed over the warp by a reduce-scatter, after which
-      // lane my_idx holds row my_r of sequence my_b.
+      // of a chunk
       float ur[KB][8];  // u at this lane's first 8 columns
 #pragma unroll
       for (int b = 0; b < KB; ++b)
@@ -418,53 +733,39 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
         const int rows = min(ch, V - c * ch);
         const __nv_bfloat16* sw = reinterpret_cast<const __nv_bfloat16*>(s_ring + sidx * kW2StageBytes);
         for (int r0 = warp * kRowsPerPass; r0 < rows; r0 += kRollWarps * kRowsPerPass) {
-          float dot[kN];
-#pragma unroll
-          for (int v = 0; v < kN; ++v) dot[v] = 0.f;
+          float dot[kRowsPerPass * KB] = {};
           // columns lane*8 .. +8 against u held in registers, then (r > 256) the rest from shared memory
           if (lane * 8 < R) {
             float wv[kRowsPerPass][8];
             load_rows(sw, r0, rows, R, lane * 8, wv);
-#pragma unroll
-            for (int r = 0; r < kRowsPerPass; ++r)
-#pragma unroll
-              for (int b = 0; b < KB; ++b)
-#pragma unroll
-                for (int e = 0; e < 8; ++e) dot[r * KB + b] += wv[r][e] * ur[b][e];
+            pass_fma<KB>(wv, ur, dot);
           }
           for (int cc = lane * 8 + 256; cc < R; cc += 256) {
             float wv[kRowsPerPass][8];
             load_rows(sw, r0, rows, R, cc, wv);
+            float uv[KB][8];
 #pragma unroll
             for (int b = 0; b < KB; ++b) {
-              float uv[8];
               if (b < B) {
                 const float4 u0 = *reinterpret_cast<const float4*>(s_u + b * R + cc);
                 const float4 u1 = *reinterpret_cast<const float4*>(s_u + b * R + cc + 4);
-                uv[0] = u0.x; uv[1] = u0.y; uv[2] = u0.z; uv[3] = u0.w;
-                uv[4] = u1.x; uv[5] = u1.y; uv[6] = u1.z; uv[7] = u1.w;
+                uv[b][0] = u0.x; uv[b][1] = u0.y; uv[b][2] = u0.z; uv[b][3] = u0.w;
+                uv[b][4] = u1.x; uv[b][5] = u1.y; uv[b][6] = u1.z; uv[b][7] = u1.w;
               } else {
 #pragma unroll
-                for (int e = 0; e < 8; ++e) uv[e] = 0.f;
+                for (int e = 0; e < 8; ++e) uv[b][e] = 0.f;
               }
-#pragma unroll
-              for (int r = 0; r < kRowsPerPass; ++r)
-#pragma unroll
-                for (int e = 0; e < 8; ++e) dot[r * KB + b] += wv[r][e] * uv[e];
             }
+            pass_fma<KB>(wv, uv, dot);
           }
-          const float d = ReduceScatter<kN, 16>::run(dot);
-          if (my_rep && r0 + my_r < rows && my_b < B) {
-            const int v = c * ch + r0 + my_r;
-            lse_push(mine, s_base[my_b * rows_cta + (v - r_lo)] + d, v);
-          }
+          pass_push<KB>(dot, role, rows - r0, i * ch + r0, c * ch + r0, s_base, rows_cta, B, mine);
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&s_empty[sidx]);  // this warp is done with the stage
       }
 #pragma unroll
       for (int b = 0; b < KB; ++b)
-        if (b == my_b) st[b] = mine;
+        if (b == role.b) st[b] = mine;
     } else {
       for (int r = tid; r < r_n; r += kRollThreads) {
 #pragma unroll
@@ -472,75 +773,72 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
           if (b < B) lse_push(st[b], s_base[b * rows_cta + r], r_lo + r);
       }
     }
-    block_reduce(st, s_red, B);
-    if (tid < B) {
-      Lse a = s_red[0][tid];
-      for (int w = 1; w < kRollWarps; ++w) lse_merge(a, s_red[w][tid]);
-      float4* out = reinterpret_cast<float4*>(p.partials) + static_cast<size_t>(blockIdx.x) * kRollMaxB + tid;
-      *out = make_float4(a.m, a.s, __int_as_float(a.i), 0.f);
-    }
-    if (!grid_barrier(p.barrier, nbar++, p.status, &s_fail)) return;
-    // ---- every CTA: combine the partials (thread c loads CTA c's, then the same block reduction;
-    //      every CTA reduces in the same order, so all reach the same t_{j+1}), choose t_{j+1}
-#pragma unroll
-    for (int b = 0; b < KB; ++b) st[b] = lse_empty();
-    for (int c = tid; c < static_cast<int>(gridDim.x); c += kRollThreads) {
-#pragma unroll
-      for (int b = 0; b < KB; ++b) {
-        if (b < B) {
-          const float4 f = __ldcg(reinterpret_cast<const float4*>(p.partials) + static_cast<size_t>(c) * kRollMaxB + b);
-          Lse t;
-          t.m = f.x; t.s = f.y; t.i = __float_as_int(f.z);
-          lse_merge(st[b], t);
-        }
-      }
-    }
-    block_reduce(st, s_red, B);
-    if (tid < B) {
-      Lse a = s_red[0][tid];
-      for (int w = 1; w < kRollWarps; ++w) lse_merge(a, s_red[w][tid]);
-      const int tok = a.i == 0x7fffffff ? 0 : a.i;
-      s_tok[tid] = tok;
-      if (blockIdx.x == 0) {
-        p.tokens[static_cast<size_t>(tid) * K + j] = tok;
-        p.logp[static_cast<size_t>(tid) * K + j] = -logf(a.s);  // the argmax's logit is the max
-      }
-    }
-    compute_sync();
+    if (!finish_step<KB>(p, j, st, s_red, s_tok, nbar, &s_fail)) return;
   }
 }
 
+// ================================================================ launch
+static bool use_resident(const RolloutParams& p) { return p.head && p.R <= kResidentMaxR; }
+
+// Resident kernel: shared-memory W2 rows that fit beside u and the staged base logits.
+static int resident_smem_rows(int B, int V, int R, int grid) {
+  const int rows_cta = resident_rows_per_cta(V, grid);
+  const long long fixed = static_cast<long long>(B) * R * 4 + static_cast<long long>(B) * rows_cta * 4;
+  const long long avail = static_cast<long long>(kRollMaxSmem) - fixed;
+  if (avail < 0) return -1;
+  const long long fit = (avail / (2LL * R)) & ~3LL;
+  const long long want = rows_cta > kTmemRows ? rows_cta - kTmemRows : 0;
+  return static_cast<int>(fit < want ? fit : want);
+}
+
 size_t rollout_smem_bytes(int B, int V, int R, bool head, int grid) {
+  if (head && R <= kResidentMaxR) {
+    const int ns = resident_smem_rows(B, V, R, grid);
+    if (ns < 0) return kRollMaxSmem + 1;
+    return static_cast<size_t>(ns) * R * 2 + static_cast<size_t>(B) * R * 4 +
+           static_cast<size_t>(B) * resident_rows_per_cta(V, grid) * 4;
+  }
   return (head ? static_cast<size_t>(kW2Stages) * kW2StageBytes : 0) +
          static_cast<size_t>(B) * (head ? R : 0) * sizeof(float) +
          static_cast<size_t>(B) * rollout_rows_per_cta(V, R, head, grid) * sizeof(float);
 }
 
-template <int KB>
-static cudaError_t launch_rollout_kb(const RolloutParams& p, int grid, size_t smem, cudaStream_t stream) {
-  static size_t attr_smem = 0;
+template <typename Kern>
+static cudaError_t launch_coop(Kern kern, size_t& attr_smem, const RolloutParams& p, int grid, int threads,
+                               size_t smem, cudaStream_t stream) {
   if (smem > 48 * 1024 && smem > attr_smem) {
-    cudaError_t e = cudaFuncSetAttribute(rollout_kernel<KB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     attr_smem = smem;
   }
   RolloutParams pp = p;
   void* args[] = {&pp};
-  cudaError_t e = cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(rollout_kernel<KB>), dim3(grid),
-                                              dim3(kRollThreadsAll), args, smem, stream);
+  cudaError_t e = cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(kern), dim3(grid), dim3(threads), args,
+                                              smem, stream);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
+}
+
+template <int KB>
+static cudaError_t launch_rollout_kb(const RolloutParams& p, int grid, size_t smem, cudaStream_t stream) {
+  if (use_resident(p)) {
+    static size_t attr = 0;
+    return launch_coop(rollout_resident_kernel<KB>, attr, p, grid, kRollThreads, smem, stream);
+  }
+  static size_t attr = 0;
+  return launch_coop(rollout_kernel<KB>, attr, p, grid, kRollThreadsAll, smem, stream);
 }
 
 cudaError_t launch_rollout(const RolloutParams& p, int grid, cudaStream_t stream) {
   if (p.B < 1 || p.B > kRollMaxB || grid < 1) return cudaErrorInvalidValue;
   const size_t smem = rollout_smem_bytes(p.B, p.V, p.R, p.head, grid);
   if (smem > kRollMaxSmem) return cudaErrorInvalidValue;
-  if (p.B <= 1) return launch_rollout_kb<1>(p, grid, smem, stream);
-  if (p.B <= 2) return launch_rollout_kb<2>(p, grid, smem, stream);
-  if (p.B <= 4) return launch_rollout_kb<4>(p, grid, smem, stream);
-  return launch_rollout_kb<8>(p, grid, smem, stream);
+  RolloutParams pp = p;
+  pp.smem_rows = use_resident(p) ? resident_smem_rows(p.B, p.V, p.R, grid) : 0;
+  if (p.B <= 1) return launch_rollout_kb<1>(pp, grid, smem, stream);
+  if (p.B <= 2) return launch_rollout_kb<2>(pp, grid, smem, stream);
+  if (p.B <= 4) return launch_rollout_kb<4>(pp, grid, smem, stream);
+  return launch_rollout_kb<8>(pp, grid, smem, stream);
 }
 
 }  // namespace dm

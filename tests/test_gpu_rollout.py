@@ -84,6 +84,12 @@ def _check(wl, head_on=True):
     inputs.custom_config("roll-b3", B=3, K=8, H=512, V=3000, Ds=64, R=64, seed=21, biases=True),
     inputs.custom_config("roll-b8", B=8, K=5, H=256, V=1000, Ds=32, R=16, seed=22),
     inputs.custom_config("roll-k1", B=2, K=1, H=128, V=777, Ds=16, R=8, seed=23),
+    # r > 256: W2 streamed through the shared-memory ring every step
+    inputs.custom_config("roll-wide", B=2, K=4, H=256, V=2500, Ds=32, R=512, seed=26, biases=True),
+    # r = 256 at a vocabulary past 152 x 1024 rows: every CTA's slice spans tensor memory, shared
+    # memory and rows read through L2, with a ragged last slice
+    inputs.custom_config("roll-tiers", B=8, K=3, H=256, V=167001, Ds=32, R=256, seed=27),
+    inputs.custom_config("roll-tiers-b1", B=1, K=4, H=256, V=160003, Ds=32, R=256, seed=28, biases=True),
 ])
 def test_rollout_matches_oracle(cfg):
     _check(inputs.make_workload(cfg))
