@@ -90,6 +90,14 @@ __device__ __forceinline__ void tc_st_x16(uint32_t taddr, const uint32_t (&r)[16
 
 __device__ __forceinline__ void tc_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
+// 4-byte asynchronous copy global -> shared (completes at cp_async_wait_all)
+__device__ __forceinline__ void cp_async4(void* dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_all;" ::: "memory");
+}
+
 __device__ __forceinline__ float warp_sum(float x) {
 #pragma unroll
   for (int o = 16; o; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
@@ -205,8 +213,9 @@ __device__ __forceinline__ void block_reduce(Lse (&st)[NB], Lse (*red)[kRollMaxB
 __device__ bool grid_barrier(unsigned* ctr, unsigned n, int* status, volatile int* fail) {
   compute_sync();
   if (threadIdx.x == 0) {
-    __threadfence();
-    atomicAdd(ctr, 1u);
+    // release at GPU scope: every write the CTA made before the barrier above is visible to a
+    // CTA that acquires the counter's new value
+    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
     const unsigned target = (n + 1) * gridDim.x;
     const long long t0 = clock64();
     while (true) {
@@ -440,10 +449,10 @@ __device__ __forceinline__ void group_fma(const uint4 (&raw)[G], int r_in_pass, 
 
 template <int KB>
 __device__ __forceinline__ void wide_push(const float (&dot)[32], int lane, int nvalid, int row0, int vid0,
-                                          const float* s_base, int rows_cta, int B, Lse& mine) {
+                                          const float* s_base, const float* s_b2, int rows_cta, int B, Lse& mine) {
   const float d = ReduceScatter<32, 16>::run(dot);
   const int r = lane / KB, b = lane % KB;
-  if (r < nvalid && b < B) lse_push(mine, s_base[b * rows_cta + row0 + r] + d, vid0 + r);
+  if (r < nvalid && b < B) lse_push(mine, s_base[b * rows_cta + row0 + r] + s_b2[row0 + r] + d, vid0 + r);
 }
 
 // ================================================================ resident kernel (r <= 256)
@@ -467,6 +476,7 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
   __nv_bfloat16* s_w2 = reinterpret_cast<__nv_bfloat16*>(s_dyn);                      // [smem_rows][R]
   float* s_u = reinterpret_cast<float*>(s_dyn + static_cast<size_t>(p.smem_rows) * R * 2);  // [B][R]
   float* s_base = s_u + B * R;                                                          // [B][rows_cta]
+  float* s_b2 = s_base + B * rows_cta;                                                  // [rows_cta]
   __shared__ __align__(8) uint64_t s_fill;  // the shared-memory rows landed
   __shared__ uint32_t s_tmem;
   __shared__ int s_tok[kRollMaxB];
@@ -529,21 +539,26 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
       }
     }
     tc_wait_st();  // a warp reads back only what it wrote itself
+    for (int r = tid; r < r_n; r += kRollThreads) s_b2[r] = p.b2 ? bf2f(p.b2[r_lo + r]) : 0.f;
 
     constexpr int kRows = WidePass<KB>::kRows, kGroup = WidePass<KB>::kGroup;
     const uint64_t pol_ab = l2_policy_evict_normal();
     const uint64_t pol_rest = l2_policy_evict_last();
-    const int n_sg = n_s + n_g;  // rows past tensor memory: shared memory first, then L2
-    unsigned nbar = 0;
+      unsigned nbar = 0;
     for (int j = 0; j < K; ++j) {
       const float* hprev = p.h + static_cast<size_t>((j + 1) & 1) * B * p.Ds;  // h_{j-1} (zeros at j = 0)
       float* hcur = p.h + static_cast<size_t>(j & 1) * B * p.Ds;
+      // this step's base logits for the CTA's rows: asynchronous copies that land during A and B
+      for (int e = tid; e < B * r_n; e += kRollThreads) {
+        const int b = e / r_n, r = e - b * r_n;
+        cp_async4(s_base + b * rows_cta + r, p.base + (static_cast<size_t>(b) * K + j) * V + r_lo + r);
+      }
       gru_phase(p, s_tok, hprev, hcur, gw, nwarps, lane, pol_ab);
       if (!grid_barrier(p.barrier, nbar++, p.status, &s_fail)) break;
       u_phase(p, j, hcur, gw, nwarps, lane, pol_ab);
       if (!grid_barrier(p.barrier, nbar++, p.status, &s_fail)) break;
       for (int e = tid; e < B * R; e += kRollThreads) s_u[e] = __ldcg(p.u + e);
-      stage_base(p, j, r_lo, r_n, rows_cta, s_base);
+      cp_async_wait_all();
       compute_sync();
       float ur[KB][8];  // u at this lane's 8 columns (zero past r)
 #pragma unroll
@@ -551,6 +566,19 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
 #pragma unroll
         for (int e = 0; e < 8; ++e) ur[b][e] = (b < B && lane * 8 < R) ? s_u[b * R + lane * 8 + e] : 0.f;
       Lse mine = lse_empty();
+      // rows read through L2 first (the longest latency): one group of rows per warp at a time
+      for (int r0 = warp * kGroup; r0 < n_g; r0 += kRollWarps * kGroup) {
+        uint4 raw[kGroup];
+#pragma unroll
+        for (int r = 0; r < kGroup; ++r)
+          raw[r] = (r0 + r < n_g && lane * 8 < R)
+                       ? ld16_hint(p.w2 + static_cast<size_t>(r_lo + n_t + n_s + r0 + r) * R + lane * 8, pol_rest)
+                       : make_uint4(0, 0, 0, 0);
+        float dot[32] = {};
+        group_fma<KB, kGroup>(raw, 0, ur, dot);
+        wide_push<KB>(dot, lane, min(kGroup, n_g - r0), n_t + n_s + r0, r_lo + n_t + n_s + r0, s_base, s_b2,
+                      rows_cta, B, mine);
+      }
       // rows in tensor memory: this warp's 64 rows of its lane quarter, 8 rows (32 columns) a load
       for (int rho0 = 64 * half; rho0 < 64 * half + 64; rho0 += kRows) {
         const int row0 = 128 * q + rho0;
@@ -578,29 +606,24 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
           }
           group_fma<KB, kGroup>(raw, g, ur, dot);
         }
-        wide_push<KB>(dot, lane, n_t - row0, row0, r_lo + row0, s_base, rows_cta, B, mine);
+        wide_push<KB>(dot, lane, n_t - row0, row0, r_lo + row0, s_base, s_b2, rows_cta, B, mine);
       }
-      // rows past tensor memory: shared memory (landed before the first step's phase C) then L2
+      // rows in shared memory (landed before the first step's phase C)
       if (j == 0 && n_s > 0) mbar_wait(&s_fill, 0, &s_fail, p.status);
       if (!s_fail) {
-        for (int r0 = warp * kRows; r0 < n_sg; r0 += kRollWarps * kRows) {
+        for (int r0 = warp * kRows; r0 < n_s; r0 += kRollWarps * kRows) {
           float dot[32] = {};
 #pragma unroll
           for (int g = 0; g < kRows; g += kGroup) {
             uint4 raw[kGroup];
 #pragma unroll
-            for (int r = 0; r < kGroup; ++r) {
-              const int row = r0 + g + r;
-              if (row < n_s && lane * 8 < R)
-                raw[r] = *reinterpret_cast<const uint4*>(s_w2 + static_cast<size_t>(row) * R + lane * 8);
-              else if (row < n_sg && lane * 8 < R)
-                raw[r] = ld16_hint(p.w2 + static_cast<size_t>(r_lo + n_t + row) * R + lane * 8, pol_rest);
-              else
-                raw[r] = make_uint4(0, 0, 0, 0);
-            }
+            for (int r = 0; r < kGroup; ++r)
+              raw[r] = (r0 + g + r < n_s && lane * 8 < R)
+                           ? *reinterpret_cast<const uint4*>(s_w2 + static_cast<size_t>(r0 + g + r) * R + lane * 8)
+                           : make_uint4(0, 0, 0, 0);
             group_fma<KB, kGroup>(raw, g, ur, dot);
           }
-          wide_push<KB>(dot, lane, n_sg - r0, n_t + r0, r_lo + n_t + r0, s_base, rows_cta, B, mine);
+          wide_push<KB>(dot, lane, n_s - r0, n_t + r0, r_lo + n_t + r0, s_base, s_b2, rows_cta, B, mine);
         }
       }
       Lse st[KB];
@@ -609,7 +632,9 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
       if (!finish_step<KB>(p, j, st, s_red, s_tok, nbar, &s_fail)) break;
     }
   }
-  // ---- teardown: the shared-memory fill has landed (bounded), tensor memory is released
+  // ---- teardown: the asynchronous copies have landed (the fill: bounded), tensor memory is
+  //      released
+  cp_async_wait_all();
   if (tid == 0 && fill_issued && n_s > 0) {
     const long long t0 = clock64();
     while (!mbar_try_wait(&s_fill, 0))
@@ -783,7 +808,7 @@ static bool use_resident(const RolloutParams& p) { return p.head && p.R <= kResi
 // Resident kernel: shared-memory W2 rows that fit beside u and the staged base logits.
 static int resident_smem_rows(int B, int V, int R, int grid) {
   const int rows_cta = resident_rows_per_cta(V, grid);
-  const long long fixed = static_cast<long long>(B) * R * 4 + static_cast<long long>(B) * rows_cta * 4;
+  const long long fixed = static_cast<long long>(B) * R * 4 + static_cast<long long>(B + 1) * rows_cta * 4;
   const long long avail = static_cast<long long>(kRollMaxSmem) - fixed;
   if (avail < 0) return -1;
   const long long fit = (avail / (2LL * R)) & ~3LL;
@@ -796,7 +821,7 @@ size_t rollout_smem_bytes(int B, int V, int R, bool head, int grid) {
     const int ns = resident_smem_rows(B, V, R, grid);
     if (ns < 0) return kRollMaxSmem + 1;
     return static_cast<size_t>(ns) * R * 2 + static_cast<size_t>(B) * R * 4 +
-           static_cast<size_t>(B) * resident_rows_per_cta(V, grid) * 4;
+           static_cast<size_t>(B + 1) * resident_rows_per_cta(V, grid) * 4;
   }
   return (head ? static_cast<size_t>(kW2Stages) * kW2StageBytes : 0) +
          static_cast<size_t>(B) * (head ? R : 0) * sizeof(float) +
