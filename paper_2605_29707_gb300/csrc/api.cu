@@ -57,13 +57,15 @@ struct Plan {
   StorePlan xg, ug;
   int mcast;   // vocab GEMM, tokens on M: CTAs per cluster sharing each weight box (1 = off)
   bool chain;  // head kernels launched as a programmatic-dependent chain (small M with overlap)
+  bool fused;  // chain path whose GRU computes E . W_ih^T and hidden . W1[:, :H] itself (no
+               // gather and no projection GEMMs; the step's first kernel is the GRU)
   dm::GruPlan gru;
   bool u_in_gru;  // small M: u finished inside the GRU kernel; large M: W1 GEMM + finalize
   bool overlap;   // vocab GEMM launched as a programmatic dependent of the GRU (deferred W2)
   int defer_tiles;  // leading tiles per CTA whose W2 segment waits for the GRU
   int tmem_cols;  // TMEM columns of the vocab GEMM
   // workspace layout (offsets in bytes)
-  size_t ctrl_bytes;
+  size_t ctrl_bytes, clear_bytes;  // clear_bytes from off_ctrl: the control words (+ hx, fused)
   size_t off_ctrl, off_E, off_xpart, off_upart, off_xs, off_hx, off_S, off_u, off_part, dev_total;
   size_t off_hid, off_ids, off_tid, off_tlp, off_tpar, off_ttok, off_tdep, off_tsc, host_total;
 };
@@ -194,6 +196,14 @@ int make_plan(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head
     // vocabulary stream) start while the projections still run.
     p.chain = p.overlap && p.xg.swap && p.ug.swap && dm::tc_store_chained_smem(p.xg.bn) > 0 &&
               dm::tc_store_chained_smem(p.ug.bn) > 0;
+    // Fused projections: 8 units per GRU CTA (one MMA n-tile per gate) and every warp's u pairs
+    // (rank row, position) within the kernel's shared-memory slots.
+    if (p.chain && p.gru.units == 8) {
+      const int total_warps = p.gru.gu * p.gru.gb * 8;
+      const int groups = total_warps / R > 1 ? total_warps / R : 1;
+      const long long pairs = static_cast<long long>(ceil_div(R * groups, total_warps)) * ceil_div(M, groups);
+      p.fused = pairs <= dm::kGruMaxUPairs;
+    }
   }
   p.tmem_cols = pow2_at_least(p.overlap ? (p.defer_tiles + 2) * p.bn : 2 * p.bn, 32);
 
@@ -205,12 +215,14 @@ int make_plan(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head
   };
   p.ctrl_bytes = align_up(256 + static_cast<size_t>(B) * 4);
   p.off_ctrl = take(p.ctrl_bytes);
+  p.clear_bytes = p.ctrl_bytes;
   if (head) {
+    p.off_hx = take(static_cast<size_t>(M) * Ds * 4);  // right after the control words: one clear
+    if (p.fused) p.clear_bytes = p.off_hx + static_cast<size_t>(M) * Ds * 4 - p.off_ctrl;
     p.off_E = take(static_cast<size_t>(M) * H * 2);
     p.off_xpart = take(static_cast<size_t>(p.xg.splits) * M * 3 * Ds * 4);
     p.off_upart = take(static_cast<size_t>(p.ug.splits) * M * R * 4);
     p.off_xs = take(static_cast<size_t>(M) * 3 * Ds * 4);
-    p.off_hx = take(static_cast<size_t>(M) * Ds * 4);
     p.off_S = take(static_cast<size_t>(M) * Ds * 2);
     p.off_u = take(static_cast<size_t>(M) * R * 2);
   }
@@ -301,15 +313,18 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
   int* status = reinterpret_cast<int*>(ws + P.off_ctrl);
   unsigned* barrier = reinterpret_cast<unsigned*>(ws + P.off_ctrl + 64);
   unsigned* seq_done = reinterpret_cast<unsigned*>(ws + P.off_ctrl + 256);
-  if (cudaMemsetAsync(ws + P.off_ctrl, 0, P.ctrl_bytes, st) != cudaSuccess) return DOMINO_ERR_CUDA;
+  if (cudaMemsetAsync(ws + P.off_ctrl, 0, P.clear_bytes, st) != cudaSuccess) return DOMINO_ERR_CUDA;
 
   __nv_bfloat16* E = P.head ? reinterpret_cast<__nv_bfloat16*>(ws + P.off_E) : nullptr;
   uint32_t* hx = P.head ? reinterpret_cast<uint32_t*>(ws + P.off_hx) : nullptr;
-  dm::GatherParams gp{ids, P.head ? static_cast<const __nv_bfloat16*>(hw->emb) : nullptr, E, hx, M, H, V, Ds, status};
-  int ts = timing_open(DOMINO_KERNEL_GATHER, st);
-  int rc = cuda_rc(dm::launch_gather(gp, st));
-  timing_close(ts, st);
-  if (rc) return rc;
+  int ts = -1, rc = DOMINO_OK;
+  if (!P.fused) {
+    dm::GatherParams gp{ids, P.head ? static_cast<const __nv_bfloat16*>(hw->emb) : nullptr, E, hx, M, H, V, Ds, status};
+    ts = timing_open(DOMINO_KERNEL_GATHER, st);
+    rc = cuda_rc(dm::launch_gather(gp, st));
+    timing_close(ts, st);
+    if (rc) return rc;
+  }
 
   __nv_bfloat16* u = nullptr;
   if (P.head) {
@@ -317,7 +332,7 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
     float* upart = reinterpret_cast<float*>(ws + P.off_upart);
     u = reinterpret_cast<__nv_bfloat16*>(ws + P.off_u);
     // X partials: E [M, H] . W_ih [3Ds, H]^T
-    {
+    if (!P.fused) {
       const dm::TcParams base{};
       TcParams tp = base;
       const StorePlan& g = P.xg;
@@ -372,7 +387,7 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
       timing_close(slot, st);
       return r;
     };
-    if (P.u_in_gru) {
+    if (P.u_in_gru && !P.fused) {
       rc = w1_gemm(false);
       if (rc) return rc;
     }
@@ -391,8 +406,15 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
     gr.s_out = P.u_in_gru ? nullptr : S;
     gr.u = P.u_in_gru ? u : nullptr;
     gr.status = status;
+    if (P.fused) {
+      gr.ids = ids;
+      gr.emb = static_cast<const __nv_bfloat16*>(hw->emb);
+      gr.w_ih = static_cast<const __nv_bfloat16*>(hw->w_ih);
+      gr.hidden = static_cast<const __nv_bfloat16*>(hidden);
+      gr.V = V;
+    }
     ts = timing_open(DOMINO_KERNEL_GRU, st);
-    rc = cuda_rc(dm::launch_gru(gr, P.gru, st, P.chain));
+    rc = cuda_rc(dm::launch_gru(gr, P.gru, st, P.chain && !P.fused));
     timing_close(ts, st);
     if (rc) return rc;
     if (!P.u_in_gru) {

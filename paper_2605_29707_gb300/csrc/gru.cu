@@ -171,6 +171,120 @@ __host__ __device__ inline GruSmem gru_layout(int Ds, int U, int bc) {
   return L;
 }
 
+// ---------------------------------------------------------------------------- fused projections
+__device__ __forceinline__ void ldg_words8(const __nv_bfloat16* row, int k0, int H, bool valid, uint32_t (&w)[8]) {
+  // elements k0 .. k0 + 15 of a row (two 16-byte halves; zero past H or for an invalid row)
+  const uint4 lo = (valid && k0 < H) ? __ldg(reinterpret_cast<const uint4*>(row + k0)) : make_uint4(0, 0, 0, 0);
+  const uint4 hi = (valid && k0 + 8 < H) ? __ldg(reinterpret_cast<const uint4*>(row + k0 + 8)) : make_uint4(0, 0, 0, 0);
+  w[0] = lo.x; w[1] = lo.y; w[2] = lo.z; w[3] = lo.w;
+  w[4] = hi.x; w[5] = hi.y; w[6] = hi.z; w[7] = hi.w;
+}
+
+// Small batches, u computed in-kernel: this CTA's input-gate sums xs = b_ih + E . W_ih^T for its
+// units (E = emb rows of the prefix ids, which are checked here) on the tensor cores, and the
+// hidden half of u, hidden_m . W1[q, :H], for the (q, m) pairs each warp finalises after the
+// recurrence.  The MMA (m16n8k16, positions on M, the 3 x 8 gate rows of the units on N) sums k
+// in an order of its own: in each 64-element chunk, lane l = 4 g + t loads elements
+// 16 t .. 16 t + 15 of its A rows (g, g + 8) and B row (g), and MMA step s of the chunk takes
+// words 2 s and 2 s + 1 of those, the same columns in A and B.  The warps split k; their partial
+// tiles meet in `red` (one 16 x 8 tile per warp at a time).
+__device__ void fused_projections(const GruParams& p, int j0, int Uc, int b0, int nbc, float* red,
+                                  float (*s_uh)[kGruMaxUPairs]) {
+  const int H = p.H, Ds = p.Ds, K = p.K, R = p.R, M = p.B * p.K;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, t = lane & 3;
+  for (int m = tid; m < M; m += kGruThreads) {
+    const int id = p.ids[m];
+    if (id < 0 || id >= p.V) set_status(p.status, kStatusBadToken);
+  }
+  const int rows = nbc * K;  // this CTA's positions: m = b0 * K + r
+  const int nchunk = (H + 63) / 64;
+  const int c_lo = (nchunk * warp) / kGruWarps, c_hi = (nchunk * (warp + 1)) / kGruWarps;
+  // B rows of n-tile nt: gate nt, unit g (8 units per CTA on this path)
+  const __nv_bfloat16* brow[3];
+  bool bvalid[3];
+#pragma unroll
+  for (int nt = 0; nt < 3; ++nt) {
+    bvalid[nt] = g < Uc;
+    brow[nt] = p.w_ih + static_cast<size_t>(nt * Ds + j0 + (g < Uc ? g : 0)) * H;
+  }
+  for (int mt = 0; mt * 16 < rows; ++mt) {
+    const int ra = mt * 16 + g, rb = ra + 8;
+    const int ida = ra < rows ? p.ids[b0 * K + ra] : 0, idb = rb < rows ? p.ids[b0 * K + rb] : 0;
+    const bool va = ra < rows && ida >= 0 && ida < p.V, vb = rb < rows && idb >= 0 && idb < p.V;
+    const __nv_bfloat16* arow = p.emb + static_cast<size_t>(va ? ida : 0) * H;
+    const __nv_bfloat16* brow2 = p.emb + static_cast<size_t>(vb ? idb : 0) * H;
+    float acc[3][4];
+#pragma unroll
+    for (int nt = 0; nt < 3; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
+    for (int c = c_lo; c < c_hi; ++c) {
+      const int k0 = c * 64 + 16 * t;
+      uint32_t wa[8], wb[8], wn[3][8];
+      ldg_words8(arow, k0, H, va, wa);
+      ldg_words8(brow2, k0, H, vb, wb);
+#pragma unroll
+      for (int nt = 0; nt < 3; ++nt) ldg_words8(brow[nt], k0, H, bvalid[nt], wn[nt]);
+#pragma unroll
+      for (int st = 0; st < 4; ++st) {
+        const uint32_t a[4] = {wa[2 * st], wb[2 * st], wa[2 * st + 1], wb[2 * st + 1]};
+#pragma unroll
+        for (int nt = 0; nt < 3; ++nt) {
+          const uint32_t b[2] = {wn[nt][2 * st], wn[nt][2 * st + 1]};
+          mma_16816(acc[nt], a, b);
+        }
+      }
+    }
+    // sum the warps' tiles, one gate (n-tile) at a time: entry (row, col) of the 16 x 8 tile
+#pragma unroll
+    for (int nt = 0; nt < 3; ++nt) {
+      float* out = red + warp * 128;
+      out[g * 8 + 2 * t] = acc[nt][0];
+      out[g * 8 + 2 * t + 1] = acc[nt][1];
+      out[(g + 8) * 8 + 2 * t] = acc[nt][2];
+      out[(g + 8) * 8 + 2 * t + 1] = acc[nt][3];
+      __syncthreads();
+      if (tid < 128) {
+        const int row = tid / 8, jl = tid % 8, r = mt * 16 + row;
+        if (r < rows && jl < Uc) {
+          float sum = bf_or0(p.b_ih, nt * Ds + j0 + jl);
+#pragma unroll
+          for (int w = 0; w < kGruWarps; ++w) sum += red[w * 128 + tid];
+          p.xs[static_cast<size_t>(b0 * K + r) * 3 * Ds + nt * Ds + j0 + jl] = sum;
+        }
+      }
+      __syncthreads();
+    }
+  }
+  // hidden halves of u for this warp's (q, m) pairs, in the tail's order
+  const int total_warps = gridDim.x * kGruWarps;
+  const int gw = blockIdx.x * kGruWarps + warp;
+  const int groups = max(1, total_warps / R);
+  int np = 0;
+  for (int pi = gw; pi < R * groups; pi += total_warps) {
+    const int q = pi % R, mg = pi / R;
+    const __nv_bfloat16* w1row = p.w1 + static_cast<size_t>(q) * (H + Ds);
+    for (int m = mg; m < M; m += groups, ++np) {
+      const __nv_bfloat16* hrow = p.hidden + static_cast<size_t>(m) * H;
+      float acc = 0.f;
+#pragma unroll 4
+      for (int c = lane * 8; c < H; c += 256) {
+        const uint4 wv = __ldg(reinterpret_cast<const uint4*>(w1row + c));
+        const uint4 hv = __ldg(reinterpret_cast<const uint4*>(hrow + c));
+        const __nv_bfloat162* w2 = reinterpret_cast<const __nv_bfloat162*>(&wv);
+        const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&hv);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float2 wf = __bfloat1622float2(w2[i]), hf = __bfloat1622float2(h2[i]);
+          acc = fmaf(wf.x, hf.x, acc);
+          acc = fmaf(wf.y, hf.y, acc);
+        }
+      }
+      acc = warp_sum(acc);
+      if (lane == 0 && np < kGruMaxUPairs) s_uh[warp][np] = acc;
+    }
+  }
+}
+
 // At most 128 registers per thread (two CTAs' worth per SM), so that a GRU CTA and a vocabulary
 // GEMM CTA (at most 168 registers x 192 threads) fit in one SM's register file.
 __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) {
@@ -210,6 +324,10 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
   for (int r = tid; r < L.mt * 16; r += kGruThreads)  // padding columns Ds .. Ds+7 (k tail)
     *reinterpret_cast<uint4*>(whh + static_cast<size_t>(r) * ldw + Ds) = make_uint4(0, 0, 0, 0);
   for (int e = tid; e < L.chunk * (ldw / 8); e += kGruThreads) reinterpret_cast<uint4*>(hsm)[e] = make_uint4(0, 0, 0, 0);
+  __shared__ float s_uh[kGruWarps][kGruMaxUPairs];  // fused: hidden halves of this warp's u pairs
+  if (p.ids != nullptr) {
+    fused_projections(p, j0, Uc, b0, nbc, red, s_uh);
+  } else {
   // Launched as a programmatic dependent of the projection GEMMs: everything below reads
   // what they (and, through their own waits, the gather) wrote -- X partials, u partials and
   // the cleared state words.
@@ -242,6 +360,7 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
 #pragma unroll
     for (int i = 0; i < 4; ++i)
       if (e0 + i * kGruThreads < xs_count) p.xs[at[i]] = a[i];
+  }
   }
   for (int e = tid; e < nbc * U; e += kGruThreads) hprev[e] = 0.f;
   cp_async_wait_all();
@@ -403,6 +522,7 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
   const int total_warps = gridDim.x * kGruWarps;
   const int gw = blockIdx.x * kGruWarps + warp;
   const int groups = max(1, total_warps / R);
+  int np = 0;  // this warp's pair counter (the fused prologue's order)
   for (int pi = gw; pi < R * groups; pi += total_warps) {
     const int q = pi % R, mg = pi / R;
     const __nv_bfloat16* w1row = p.w1 + static_cast<size_t>(q) * (H + Ds) + H;
@@ -445,7 +565,12 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
         if (lane == 0) set_status(p.status, kStatusTimeout);
         return;
       }
-      for (int s = lane; s < p.usplits; s += 32) acc += __ldg(p.upart + (static_cast<size_t>(s) * M + m) * R + q);
+      if (p.ids != nullptr) {
+        if (lane == 0 && np < kGruMaxUPairs) acc += s_uh[warp][np];
+        ++np;
+      } else {
+        for (int s = lane; s < p.usplits; s += 32) acc += __ldg(p.upart + (static_cast<size_t>(s) * M + m) * R + q);
+      }
       acc = warp_sum(acc);
       if (lane == 0) {
         const float a = acc + bq;

@@ -97,11 +97,22 @@ struct GruParams {
   int B, K, H, Ds, R;
   int units, gu, gb, bc;      // grid shape: gu unit blocks x gb sequence groups of bc
   float* xs;                  // [M][3*Ds] input-gate sums (scratch)
-  uint32_t* hx;               // [M][Ds] tagged states (cleared by the gather kernel)
+  uint32_t* hx;               // [M][Ds] tagged states (cleared before the launch)
   __nv_bfloat16* s_out;       // [M][Ds] plain bf16 states, or nullptr
   __nv_bfloat16* u;           // [M][R] low-rank code computed in-kernel, or nullptr
   int* status;
+  // Fused projections (small batches, u computed in-kernel): with ids set, the kernel computes
+  // its own input-gate sums E . W_ih^T (E = emb rows of ids, checked against V) and the hidden
+  // half of u, and xpart / upart are unused; hx must arrive cleared.
+  const int32_t* ids;         // [M] or nullptr
+  const __nv_bfloat16* emb;   // [V, H]
+  const __nv_bfloat16* w_ih;  // [3*Ds, H]
+  const __nv_bfloat16* hidden;  // [M, H]
+  int V;
 };
+// Largest number of (rank row, position) pairs of u one warp finalises for which the fused
+// projections apply (their hidden halves wait in shared memory).
+constexpr int kGruMaxUPairs = 8;
 struct GruPlan {
   int units, gu, gb, bc;
   size_t smem;  // 0 = unsupported
