@@ -141,7 +141,10 @@ DOMINO_API const char* domino_status_string(int status);
 DOMINO_API int domino_abi_version(void);
 
 /* Number of kernel launches one domino_draft_step makes for these sizes (head on when
- * R > 0), so a caller can count device work. */
+ * R > 0), so a caller can count device work: the plan of the current device (of a 152-SM GB300
+ * when no device is visible).  3 with the head off, 3 for small batches whose GRU computes its
+ * own projections (B <= 2 at K = 16), 6 for other batches of at most 128 positions, 7 above;
+ * a negative code for sizes domino_draft_step would reject. */
 DOMINO_API int domino_launches_per_step(int B, int K, int H, int V, int Ds, int R, int k, int N);
 
 /* Greedy verification of draft trees against the target model's logits: the step after the

@@ -131,13 +131,8 @@ int check_sizes(int B, int K, int H, int V, int Ds, int R, int k, int N, bool he
   return DOMINO_OK;
 }
 
-int make_plan(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head, Plan* P) {
-  int rc = check_sizes(B, K, H, V, Ds, R, k, N, head);
-  if (rc != DOMINO_OK) return rc;
-  int sms = 0, major = 0, minor = 0;
-  rc = device_sms(&sms, &major, &minor);
-  if (rc != DOMINO_OK) return rc;
-  if (major != 10 || minor != 3) return DOMINO_ERR_UNSUPPORTED;
+// The plan for a GPU with `sms` SMs (sizes already checked).
+int make_plan_sms(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head, int sms, Plan* P) {
   Plan& p = *P;
   memset(&p, 0, sizeof p);
   p.B = B; p.K = K; p.H = H; p.V = V; p.k = k; p.N = N;
@@ -238,6 +233,16 @@ int make_plan(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head
   p.off_tsc = take(static_cast<size_t>(B) * N * 4);
   p.host_total = off;
   return DOMINO_OK;
+}
+
+int make_plan(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head, Plan* P) {
+  int rc = check_sizes(B, K, H, V, Ds, R, k, N, head);
+  if (rc != DOMINO_OK) return rc;
+  int sms = 0, major = 0, minor = 0;
+  rc = device_sms(&sms, &major, &minor);
+  if (rc != DOMINO_OK) return rc;
+  if (major != 10 || minor != 3) return DOMINO_ERR_UNSUPPORTED;
+  return make_plan_sms(B, K, H, V, Ds, R, k, N, head, sms, P);
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -768,11 +773,19 @@ int domino_rollout_greedy(const void* hidden, const int32_t* anchors, const void
 }
 
 int domino_launches_per_step(int B, int K, int H, int V, int Ds, int R, int k, int N) {
-  (void)H; (void)V; (void)Ds; (void)k; (void)N;
-  if (R <= 0) return 3;  // gather (id check), vocab GEMM, merge + tree
-  // small M: gather, X GEMM, W1-hidden GEMM, GRU (+u), vocab GEMM, merge + tree;
-  // large M: gather, X GEMM, GRU, W1 GEMM, u finalize, vocab GEMM, merge + tree
-  return static_cast<long long>(B) * K <= 128 ? 6 : 7;
+  const bool head = R > 0;
+  if (check_sizes(B, K, H, V, Ds, R, k, N, head) != DOMINO_OK) return -1;
+  if (!head) return 3;  // gather (id check), vocab GEMM, merge + tree
+  // the plan of this device, or of a 152-SM GB300 when none is visible
+  int sms = 0, major = 0, minor = 0;
+  if (device_sms(&sms, &major, &minor) != DOMINO_OK || sms <= 0) sms = 152;
+  Plan P;
+  if (make_plan_sms(B, K, H, V, Ds, R, k, N, head, sms, &P) != DOMINO_OK) return -1;
+  // fused small M: GRU (+ its projections and u), vocab GEMM, merge + tree; other small M:
+  // gather, X GEMM, W1-hidden GEMM, GRU (+u), vocab GEMM, merge + tree; large M: gather, X GEMM,
+  // GRU, W1 GEMM, u finalize, vocab GEMM, merge + tree
+  if (P.fused) return 3;
+  return P.u_in_gru ? 6 : 7;
 }
 
 }  // extern "C"

@@ -63,8 +63,14 @@ def test_null_pointers_rejected_before_any_cuda_call():
 
 def test_launch_count_query():
     _lib()
-    assert binding.domino_launches_per_step(1, 16, 4096, 151936, 1024, 256, 8, 16) == 6
+    # B = 1: the GRU (with its own projections), the vocab GEMM, merge + tree
+    assert binding.domino_launches_per_step(1, 16, 4096, 151936, 1024, 256, 8, 16) == 3
+    # B = 4 (M = 64, no overlap): gather, X GEMM, W1-hidden GEMM, GRU, vocab GEMM, merge + tree
+    assert binding.domino_launches_per_step(4, 16, 4096, 151936, 1024, 256, 8, 16) == 6
+    # B = 32 (tokens on M): gather, X GEMM, GRU, W1 GEMM, u finalize, vocab GEMM, merge + tree
+    assert binding.domino_launches_per_step(32, 16, 4096, 151936, 1024, 256, 8, 16) == 7
     assert binding.domino_launches_per_step(1, 16, 4096, 151936, 0, 0, 8, 16) == 3
+    assert binding.domino_launches_per_step(0, 16, 4096, 151936, 1024, 256, 8, 16) < 0
 
 
 def test_verify_rejects_bad_arguments_before_launch():
