@@ -57,6 +57,9 @@ SMALL = {
     "normal-ragged": dict(B=9, K=31, H=200, V=2049, Ds=72, R=40, k=3, N=7, seed=16, biases=True),
     "k1-chain": dict(B=2, K=6, H=64, V=700, Ds=32, R=16, k=1, N=6, seed=17),
     "K1": dict(B=5, K=1, H=64, V=900, Ds=32, R=16, k=6, N=6, seed=18),
+    # the GRU computes its own projections (three launches): H not a multiple of 64 (a short last
+    # k chunk), 32 GRU CTAs, four u pairs per warp
+    "fused-ragged": dict(B=2, K=7, H=328, V=5000, Ds=256, R=64, k=5, N=12, seed=19, biases=True),
 }
 
 
@@ -100,9 +103,12 @@ def test_deterministic_and_host_entry_point_matches():
     np.testing.assert_array_equal(host["tree_score"].numpy().reshape(out1["tree_score"].shape), out1["tree_score"])
 
 
-def test_bad_token_reported_by_device_status():
-    wl = inputs.make_workload(inputs.custom_config("bad", B=1, K=4, H=64, V=500, Ds=32, R=16, k=2, N=3, seed=23))
+# the GRU's own id check (3 launches) and the gather kernel's (6 launches)
+@pytest.mark.parametrize("B,K,expect", [(1, 4, 3), (4, 16, 6)])
+def test_bad_token_reported_by_device_status(B, K, expect):
+    wl = inputs.make_workload(inputs.custom_config("bad", B=B, K=K, H=64, V=500, Ds=32, R=16, k=2, N=3, seed=23))
     c = wl.cfg
+    assert binding.domino_launches_per_step(c.B, c.K, c.H, c.V, c.Ds, c.R, c.k, c.N) == expect
     st = DraftStep(wl.weights, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=_dev())
     hidden = torch.from_numpy(wl.hidden.view(np.int16)).view(torch.bfloat16).to(_dev())
     ids = torch.from_numpy(wl.prefix_ids).to(_dev())
