@@ -169,6 +169,82 @@ __device__ __forceinline__ void best_children(const float* lp, const int* ids, i
   child_key(b0, sb0, tb, ids + rb * k, sb, hb, lb, jb);
 }
 
+// Best remaining child of a slot, computed by its owner lane: the first available entry j0 of
+// row `row` (a best-first top-k list) and, among the available entries whose score
+// parent + logp ties it exactly in fp32, the lowest token (scores fall along the row, so the
+// scan stops at the first lower one).  The key is child_key's; (0, 0) when nothing is available.
+__device__ __forceinline__ void own_best_child(const float* lp, const int* ids, int k, int row, float parent,
+                                               unsigned avail, int slot, uint32_t& hi, uint32_t& lo, int& jb) {
+  hi = 0u;
+  lo = 0u;
+  jb = 0;
+  if (avail == 0u) return;
+  const int j0 = __ffs(avail) - 1;
+  const float* pl = lp + row * k;
+  const int* pi = ids + row * k;
+  const float s0 = parent + pl[j0];
+  int tb = pi[j0];
+  jb = j0;
+  for (int j = j0 + 1; j < k; ++j) {
+    if (parent + pl[j] != s0) break;
+    if (((avail >> j) & 1u) && pi[j] < tb) { tb = pi[j]; jb = j; }
+  }
+  hi = f32_ord(s0);
+  lo = ((0x3FFFFFu - static_cast<unsigned>(tb)) << 10) | (0x3FFu - static_cast<unsigned>(slot));
+}
+
+__device__ __forceinline__ float f32_from_ord(uint32_t o) {
+  return __uint_as_float((o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o);
+}
+
+// The best-first tree for N <= 31 (every slot in its own lane's registers): the same selection,
+// keys and tie rules as the general warp version below, with a short dependency chain per pop.
+// The popped child's score and token come out of the winning key itself; only the parent's depth
+// crosses lanes; the two slots that change (the popped one and the new node) each compute their
+// next best child in their own lane, on the same instruction path.
+__device__ void tree_lanes(const float* lp, const int* ids, int K, int k, int N, unsigned all, int lane,
+                           int32_t* tpar, int32_t* ttok, int32_t* tdep, float* tsc) {
+  // slot `lane`: score, depth, mask of selected entries, cached best child (hi, lo, j), and the
+  // node it is (parent index, token)
+  float score = 0.f;
+  int depth = 0, j = 0, par = -1, tok = -1;
+  unsigned mask = 0u;
+  uint32_t hi = 0u, lo = 0u;
+  own_best_child(lp, ids, k, 0, 0.f, lane == 0 ? all : 0u, 0, hi, lo, j);
+  int n_sel = 0;
+  for (int i = 0; i < N; ++i) {
+    const bool live = lane <= i;
+    const uint32_t mhi = __reduce_max_sync(0xffffffffu, live ? hi : 0u);
+    if (mhi == 0u) break;  // no frontier left (the host keeps N within the tree's capacity)
+    const uint32_t mlo = __reduce_max_sync(0xffffffffu, (live && hi == mhi) ? lo : 0u);
+    const int src = __ffs(__ballot_sync(0xffffffffu, live && hi == mhi && lo == mlo)) - 1;
+    const int d = __shfl_sync(0xffffffffu, depth, src);
+    const float sc = f32_from_ord(mhi);
+    const int t = static_cast<int>(0x3FFFFFu - (mlo >> 10));
+    const bool is_new = lane == i + 1, is_src = lane == src;
+    if (is_new) {
+      score = sc;
+      depth = d + 1;
+      mask = 0u;
+      par = src - 1;
+      tok = t;
+    }
+    if (is_src) mask |= 1u << j;
+    // the two changed slots: the new node's children come from row d + 1 (none past the last
+    // position), the popped slot's from its own row without the entries taken
+    const int row = is_new ? (d + 1 < K ? d + 1 : K - 1) : depth;
+    const unsigned avail = is_new ? (d + 1 < K ? all : 0u) : (~mask & all);
+    if (is_new || is_src) own_best_child(lp, ids, k, row, score, avail, lane, hi, lo, j);
+    n_sel = i + 1;
+  }
+  if (lane >= 1 && lane <= n_sel) {  // node lane - 1
+    tpar[lane - 1] = par;
+    ttok[lane - 1] = tok;
+    tdep[lane - 1] = depth;
+    if (tsc) tsc[lane - 1] = score;
+  }
+}
+
 template <int KM, int KK, int NT>
 __global__ void __launch_bounds__(NT, NT == kMergeThreadsNarrow ? 8 : 1) merge_tree_kernel(const TreeParams p) {
   constexpr int F = 2 + 2 * KM;
@@ -270,6 +346,12 @@ __global__ void __launch_bounds__(NT, NT == kMergeThreadsNarrow ? 8 : 1) merge_t
   }
   __syncthreads();
   if (warp != 0) return;
+  if (N <= 31) {
+    const size_t ob1 = static_cast<size_t>(b) * N;
+    tree_lanes(s_lp, s_id, K, k, N, (k == 32) ? 0xffffffffu : ((1u << k) - 1u), lane, p.tree_parent + ob1,
+               p.tree_token + ob1, p.tree_depth + ob1, p.tree_score ? p.tree_score + ob1 : nullptr);
+    return;
+  }
 
   // ------------------------------------------------------------ tree (warp 0)
   // Row reads below stay inside s_lp / s_id: rows are clamped to K - 1 and entries to
