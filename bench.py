@@ -525,7 +525,10 @@ def run_ours(args):
         t_e2e = float(t.item())
     e2e_value = world * c.B * n_e2e / t_e2e
     h2d = M * c.H * 2 + M * 4
-    d2h = M * c.k * 8 + c.B * c.N * 16 + 4
+    # the host entry point reads its outputs (top-k ids and log-probs, the four tree arrays) and a
+    # copy of the status in one copy of the workspace region that holds them (256-byte aligned)
+    al = lambda n: (n + 255) // 256 * 256
+    d2h = 2 * al(M * c.k * 4) + 4 * al(c.B * c.N * 4) + 4
 
     # ---- Domino-head overhead: the same workload with the correction branch off (R = 0, the
     #      paper's "w/o Domino head" base distribution), same device weights

@@ -115,11 +115,13 @@ DOMINO_API int domino_draft_step(const void* hidden, const int32_t* prefix_ids, 
                       void* workspace, size_t workspace_bytes, void* stream);
 
 /* The same step with the per-step inputs and the outputs in HOST memory (pinned memory
- * recommended) and the weights on the device.  hidden / prefix_ids are copied into the
- * workspace, the step runs, the outputs are copied back, and the call synchronises the
- * stream before returning.  The workspace must hold
- * domino_workspace_bytes_host(...) bytes.  Returns DOMINO_OK or the first error, including
- * device-side errors (it calls domino_check_status itself). */
+ * recommended for the inputs) and the weights on the device.  hidden / prefix_ids are copied
+ * into the workspace, the step runs, and every output plus the device status come back in one
+ * copy into a pinned staging buffer the library allocates on first use and keeps for the
+ * process (calls from several threads take turns on it), from which they are copied to the
+ * caller's buffers; the call synchronises the stream before returning.  The workspace must
+ * hold domino_workspace_bytes_host(...) bytes.  Returns DOMINO_OK or the first error,
+ * including device-side errors (bad prefix id, timeout). */
 DOMINO_API size_t domino_workspace_bytes_host(int B, int K, int H, int V, int Ds, int R, int k, int N);
 DOMINO_API int domino_draft_step_host(const void* hidden_host, const int32_t* prefix_ids_host,
                            const void* w_lm, const domino_head_weights* head, int B, int K,

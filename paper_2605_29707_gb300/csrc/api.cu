@@ -67,7 +67,7 @@ struct Plan {
   // workspace layout (offsets in bytes)
   size_t ctrl_bytes, clear_bytes;  // clear_bytes from off_ctrl: the control words (+ hx, fused)
   size_t off_ctrl, off_E, off_xpart, off_upart, off_xs, off_hx, off_S, off_u, off_part, dev_total;
-  size_t off_hid, off_ids, off_tid, off_tlp, off_tpar, off_ttok, off_tdep, off_tsc, host_total;
+  size_t off_hid, off_ids, off_tid, off_tlp, off_tpar, off_ttok, off_tdep, off_tsc, off_ostat, host_total;
 };
 
 // Orientation: up to 128 tokens ride on the MMA's N dimension (weights fill the 128-row
@@ -231,6 +231,7 @@ int make_plan_sms(int B, int K, int H, int V, int Ds, int R, int k, int N, bool 
   p.off_ttok = take(static_cast<size_t>(B) * N * 4);
   p.off_tdep = take(static_cast<size_t>(B) * N * 4);
   p.off_tsc = take(static_cast<size_t>(B) * N * 4);
+  p.off_ostat = take(4);  // the status copy: the host entry point reads [off_tid, off_ostat + 4) at once
   p.host_total = off;
   return DOMINO_OK;
 }
@@ -288,6 +289,25 @@ bool gemm_maps(CUtensorMap* a, CUtensorMap* b, bool swap, int bn, const void* X,
 
 int cuda_rc(cudaError_t e) { return e == cudaSuccess ? DOMINO_OK : DOMINO_ERR_CUDA; }
 
+// ---------------------------------------------------------------- host staging
+// Pinned host buffer the host entry point copies a step's outputs into (one copy), grown on
+// demand and kept for the process; callers hold g_stage_mu while they use it.
+std::mutex g_stage_mu;
+uint8_t* g_stage = nullptr;
+size_t g_stage_bytes = 0;
+
+uint8_t* stage_buffer(size_t bytes) {
+  if (bytes <= g_stage_bytes) return g_stage;
+  if (g_stage) cudaFreeHost(g_stage);
+  g_stage = nullptr;
+  g_stage_bytes = 0;
+  void* p = nullptr;
+  if (cudaHostAlloc(&p, bytes, cudaHostAllocDefault) != cudaSuccess) return nullptr;
+  g_stage = static_cast<uint8_t*>(p);
+  g_stage_bytes = bytes;
+  return g_stage;
+}
+
 // ---------------------------------------------------------------- per-kernel timing
 struct Timing {
   bool on = false;
@@ -313,7 +333,7 @@ void timing_close(int slot, cudaStream_t st) {
 
 int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* w_lm, const domino_head_weights* hw,
              int32_t* topk_ids, float* topk_logp, int32_t* tpar, int32_t* ttok, int32_t* tdep, float* tsc,
-             uint8_t* ws, cudaStream_t st) {
+             uint8_t* ws, cudaStream_t st, int32_t* status_out = nullptr) {
   const int M = P.M, H = P.H, V = P.V, Ds = P.Ds, R = P.R;
   int* status = reinterpret_cast<int*>(ws + P.off_ctrl);
   unsigned* barrier = reinterpret_cast<unsigned*>(ws + P.off_ctrl + 64);
@@ -474,6 +494,8 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
   tr.B = P.B; tr.K = P.K; tr.k = P.k; tr.N = P.N;
   tr.topk_ids = topk_ids; tr.topk_logp = topk_logp;
   tr.tree_parent = tpar; tr.tree_token = ttok; tr.tree_depth = tdep; tr.tree_score = tsc;
+  tr.status = status;
+  tr.status_out = status_out;
   ts = timing_open(DOMINO_KERNEL_TREE, st);
   rc = cuda_rc(dm::launch_merge_tree(tr, st));
   timing_close(ts, st);
@@ -557,18 +579,26 @@ int domino_draft_step_host(const void* hidden_host, const int32_t* prefix_ids_ho
   int32_t* d_tok = reinterpret_cast<int32_t*>(ws + P.off_ttok);
   int32_t* d_dep = reinterpret_cast<int32_t*>(ws + P.off_tdep);
   float* d_sc = reinterpret_cast<float*>(ws + P.off_tsc);
-  rc = run_step(P, d_hid, d_ids, w_lm, head, d_tid, d_tlp, d_par, d_tok, d_dep, d_sc, ws, st);
+  int32_t* d_ostat = reinterpret_cast<int32_t*>(ws + P.off_ostat);
+  rc = run_step(P, d_hid, d_ids, w_lm, head, d_tid, d_tlp, d_par, d_tok, d_dep, d_sc, ws, st, d_ostat);
   if (rc) return rc;
+  // every output and the status in one copy, through a pinned staging buffer of this library
+  const size_t lo = P.off_tid, bytes = P.off_ostat + 4 - lo;
+  std::lock_guard<std::mutex> lock(g_stage_mu);
+  uint8_t* h = stage_buffer(bytes);
+  if (!h) return DOMINO_ERR_CUDA;
+  if (cudaMemcpyAsync(h, ws + lo, bytes, cudaMemcpyDeviceToHost, st) != cudaSuccess) return DOMINO_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return DOMINO_ERR_CUDA;
   const size_t BN = static_cast<size_t>(P.B) * N;
-  cudaError_t e = cudaSuccess;
-  e = e ? e : cudaMemcpyAsync(topk_ids_host, d_tid, M * k * 4, cudaMemcpyDeviceToHost, st);
-  e = e ? e : cudaMemcpyAsync(topk_logp_host, d_tlp, M * k * 4, cudaMemcpyDeviceToHost, st);
-  e = e ? e : cudaMemcpyAsync(tree_parent_host, d_par, BN * 4, cudaMemcpyDeviceToHost, st);
-  e = e ? e : cudaMemcpyAsync(tree_token_host, d_tok, BN * 4, cudaMemcpyDeviceToHost, st);
-  e = e ? e : cudaMemcpyAsync(tree_depth_host, d_dep, BN * 4, cudaMemcpyDeviceToHost, st);
-  if (tree_score_host) e = e ? e : cudaMemcpyAsync(tree_score_host, d_sc, BN * 4, cudaMemcpyDeviceToHost, st);
-  if (e != cudaSuccess) return DOMINO_ERR_CUDA;
-  return domino_check_status(workspace, stream);
+  memcpy(topk_ids_host, h + (P.off_tid - lo), M * k * 4);
+  memcpy(topk_logp_host, h + (P.off_tlp - lo), M * k * 4);
+  memcpy(tree_parent_host, h + (P.off_tpar - lo), BN * 4);
+  memcpy(tree_token_host, h + (P.off_ttok - lo), BN * 4);
+  memcpy(tree_depth_host, h + (P.off_tdep - lo), BN * 4);
+  if (tree_score_host) memcpy(tree_score_host, h + (P.off_tsc - lo), BN * 4);
+  int32_t status = 0;
+  memcpy(&status, h + (P.off_ostat - lo), 4);
+  return status;
 }
 
 int domino_check_status(const void* workspace, void* stream) {

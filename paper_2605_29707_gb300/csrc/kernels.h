@@ -143,6 +143,8 @@ struct TreeParams {
   int32_t* tree_token;
   int32_t* tree_depth;
   float* tree_score;      // or nullptr
+  const int* status;      // the step's device status word
+  int32_t* status_out;    // or nullptr: a copy of it beside the outputs, made once the step is done
 };
 cudaError_t launch_merge_tree(const TreeParams& p, cudaStream_t stream);
 

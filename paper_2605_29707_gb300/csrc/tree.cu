@@ -264,6 +264,8 @@ __global__ void __launch_bounds__(NT, NT == kMergeThreadsNarrow ? 8 : 1) merge_t
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   // launched as a programmatic dependent of the vocabulary GEMM: wait for its partials
   asm volatile("griddepcontrol.wait;" ::: "memory");
+  // every earlier kernel of the step has completed: its status is final
+  if (m == 0 && tid == 0 && p.status_out) *p.status_out = *p.status;
   const float* base = p.partials + static_cast<size_t>(m) * F * nch;
   const int* ibase = reinterpret_cast<const int*>(base);
 
