@@ -56,6 +56,7 @@ def _load():
         _lib.oracle_draft_step.argtypes = [P] * 12 + [I] * 8 + [P, I] + [P] * 8 + [I]
         _lib.oracle_verify_greedy.argtypes = [P, I, I, P, P, P, P, P, P]
         _lib.oracle_rollout_greedy.argtypes = [P] * 12 + [I] * 6 + [P, I, P, P, I]
+        _lib.oracle_rollout_sample.argtypes = [P] * 13 + [I] * 6 + [P, I, P, P, I]
         _lib.oracle_max_threads.restype = I
         for name in ("oracle_embed", "oracle_gru", "oracle_lowrank", "oracle_logits",
                      "oracle_log_softmax", "oracle_topk", "oracle_tree", "oracle_draft_step"):
@@ -208,6 +209,31 @@ def rollout_greedy(w, hidden, anchors, seqs=None, nthreads=0):
                                          _p(g("b_ih")), _p(g("b_hh")), _p(g("w1")), _p(g("b1")), _p(w2),
                                          _p(g("b2")), B, K, H, V, Ds, R, _p(sq), nseq, _p(tokens), _p(logp),
                                          nthreads), "oracle_rollout_greedy")
+    return tokens, logp
+
+
+def rollout_sample(w, hidden, anchors, uniforms, seqs=None, nthreads=0):
+    """Sampled sequential draft loop: ``uniforms`` float32 [B, K] in [0, 1), the caller's random
+    draws (one per sequence and step).  Otherwise as rollout_greedy."""
+    hidden = _u16(hidden)
+    B, K, H = hidden.shape
+    anchors = _i32(anchors)
+    uni = np.ascontiguousarray(uniforms, dtype=np.float32).reshape(B, K)
+    g = lambda n: _u16(w[n]) if w.get(n) is not None else None  # noqa: E731
+    w_lm = g("w_lm")
+    V = w_lm.shape[0]
+    w2 = g("w2")
+    R = w2.shape[1] if w2 is not None else 0
+    w_hh = g("w_hh")
+    Ds = w_hh.shape[1] if w_hh is not None else 0
+    sq = None if seqs is None else _i32(seqs)
+    nseq = B if sq is None else sq.shape[0]
+    tokens = np.empty((nseq, K), np.int32)
+    logp = np.empty((nseq, K), np.float64)
+    _check(_load().oracle_rollout_sample(_p(hidden), _p(anchors), _p(uni), _p(w_lm), _p(g("emb")), _p(g("w_ih")),
+                                         _p(w_hh), _p(g("b_ih")), _p(g("b_hh")), _p(g("w1")), _p(g("b1")), _p(w2),
+                                         _p(g("b2")), B, K, H, V, Ds, R, _p(sq), nseq, _p(tokens), _p(logp),
+                                         nthreads), "oracle_rollout_sample")
     return tokens, logp
 
 

@@ -15,7 +15,8 @@
  *   Fig. 3 caption: tokens are drawn from the final logits        -> oracle_log_softmax
  *   Fig. 1 caption: the "Tree" construction cost                  -> oracle_topk, oracle_tree
  *   section 3.1, verification of the draft (the step after it)     -> oracle_verify_greedy
- *   section 4.1.2 / Fig. 3, tokens chosen and fed back one by one   -> oracle_rollout_greedy
+ *   section 4.1.2 / Fig. 3, tokens chosen and fed back one by one   -> oracle_rollout_greedy,
+ *                                                                       oracle_rollout_sample
  * Readings of points the paper leaves open (GRU gate convention, which ids feed which
  * position, tree tie-breaks) are listed in the design notes; the comments below state the
  * reading each function implements.
@@ -353,12 +354,13 @@ int oracle_verify_greedy(const float* target, int N, int V, const int32_t* paren
 /* O9: the greedy sequential draft loop.  Each position is computed from scratch out of the
  * primitives above (the GRU re-run over the whole prefix chosen so far), so the only new step is
  * the feedback: the argmax of position j becomes the input of position j + 1. */
-int oracle_rollout_greedy(const uint16_t* hidden, const int32_t* anchors, const uint16_t* w_lm,
-                          const uint16_t* emb, const uint16_t* w_ih, const uint16_t* w_hh,
-                          const uint16_t* b_ih, const uint16_t* b_hh, const uint16_t* w1,
-                          const uint16_t* b1, const uint16_t* w2, const uint16_t* b2, int B, int K,
-                          int H, int V, int Ds, int R, const int32_t* seqs, int nseq, int32_t* tokens,
-                          double* logp, int nthreads) {
+/* The draft loop of section 4.1.2 / Fig. 3 for both selection rules: with `uniforms` NULL the
+ * greedy choice (O9), otherwise the sampled one (O10). */
+static int rollout(const uint16_t* hidden, const int32_t* anchors, const float* uniforms, const uint16_t* w_lm,
+                   const uint16_t* emb, const uint16_t* w_ih, const uint16_t* w_hh, const uint16_t* b_ih,
+                   const uint16_t* b_hh, const uint16_t* w1, const uint16_t* b1, const uint16_t* w2,
+                   const uint16_t* b2, int B, int K, int H, int V, int Ds, int R, const int32_t* seqs, int nseq,
+                   int32_t* tokens, double* logp, int nthreads) {
   if (!hidden || !anchors || !w_lm || !tokens || !logp) return ORACLE_ERR_ARG;
   if (B <= 0 || K <= 0 || H <= 0 || V <= 0 || R < 0) return ORACLE_ERR_ARG;
   const int use_head = (w2 != NULL && R > 0);
@@ -395,8 +397,24 @@ int oracle_rollout_greedy(const uint16_t* hidden, const int32_t* anchors, const 
       if (!rc) rc = oracle_log_softmax(z, 1, V, lp, &ls);
       if (rc) break;
       int best = 0;
-      for (int v = 1; v < V; ++v)
-        if (z[v] > z[best]) best = v; /* strict: an equal value keeps the lower id */
+      if (!uniforms) {
+        for (int v = 1; v < V; ++v)
+          if (z[v] > z[best]) best = v; /* strict: an equal value keeps the lower id */
+      } else {
+        /* O10: the first id whose cumulative probability (in id order) exceeds the uniform;
+         * a uniform at or past the total (rounding) takes the last id of non-zero mass */
+        const double uu = (double)uniforms[(long)b * K + j];
+        double cdf = 0.0;
+        int last = 0;
+        best = -1;
+        for (int v = 0; v < V; ++v) {
+          const double pv = exp(lp[v]);
+          if (pv > 0.0) last = v;
+          cdf += pv;
+          if (cdf > uu) { best = v; break; }
+        }
+        if (best < 0) best = last;
+      }
       ids[j + 1] = best;
       tokens[(long)si * K + j] = best;
       logp[(long)si * K + j] = lp[best];
@@ -404,4 +422,27 @@ int oracle_rollout_greedy(const uint16_t* hidden, const int32_t* anchors, const 
   }
   free(ids); free(hid); free(E); free(S); free(u); free(z); free(lp);
   return rc;
+}
+
+int oracle_rollout_greedy(const uint16_t* hidden, const int32_t* anchors, const uint16_t* w_lm,
+                          const uint16_t* emb, const uint16_t* w_ih, const uint16_t* w_hh,
+                          const uint16_t* b_ih, const uint16_t* b_hh, const uint16_t* w1,
+                          const uint16_t* b1, const uint16_t* w2, const uint16_t* b2, int B, int K,
+                          int H, int V, int Ds, int R, const int32_t* seqs, int nseq, int32_t* tokens,
+                          double* logp, int nthreads) {
+  return rollout(hidden, anchors, NULL, w_lm, emb, w_ih, w_hh, b_ih, b_hh, w1, b1, w2, b2, B, K, H, V, Ds, R, seqs,
+                 nseq, tokens, logp, nthreads);
+}
+
+int oracle_rollout_sample(const uint16_t* hidden, const int32_t* anchors, const float* uniforms,
+                          const uint16_t* w_lm, const uint16_t* emb, const uint16_t* w_ih,
+                          const uint16_t* w_hh, const uint16_t* b_ih, const uint16_t* b_hh,
+                          const uint16_t* w1, const uint16_t* b1, const uint16_t* w2, const uint16_t* b2,
+                          int B, int K, int H, int V, int Ds, int R, const int32_t* seqs, int nseq,
+                          int32_t* tokens, double* logp, int nthreads) {
+  if (!uniforms) return ORACLE_ERR_ARG;
+  for (long i = 0; i < (long)B * K; ++i)
+    if (!(uniforms[i] >= 0.0f && uniforms[i] < 1.0f)) return ORACLE_ERR_ARG;
+  return rollout(hidden, anchors, uniforms, w_lm, emb, w_ih, w_hh, b_ih, b_hh, w1, b1, w2, b2, B, K, H, V, Ds, R,
+                 seqs, nseq, tokens, logp, nthreads);
 }

@@ -126,6 +126,19 @@ int oracle_rollout_greedy(const uint16_t* hidden, const int32_t* anchors, const 
                           int H, int V, int Ds, int R, const int32_t* seqs, int nseq, int32_t* tokens,
                           double* logp, int nthreads);
 
+/* O10, the same loop with each token sampled from the final distribution (section 4.1.2: "each
+ * draft token is sampled from the final logits"): with u_j = uniforms[b * K + j] in [0, 1)
+ * (the caller's random draws), t_{j+1} = the first id v whose cumulative probability
+ * sum_{v' <= v} softmax(L_j)[v'] (in id order) exceeds u_j; a u_j at or past the rounded total
+ * takes the last id of non-zero probability.  logp_j = log-softmax(L_j)[t_{j+1}].  Returns
+ * ORACLE_ERR_ARG for a uniform outside [0, 1). */
+int oracle_rollout_sample(const uint16_t* hidden, const int32_t* anchors, const float* uniforms,
+                          const uint16_t* w_lm, const uint16_t* emb, const uint16_t* w_ih,
+                          const uint16_t* w_hh, const uint16_t* b_ih, const uint16_t* b_hh,
+                          const uint16_t* w1, const uint16_t* b1, const uint16_t* w2, const uint16_t* b2,
+                          int B, int K, int H, int V, int Ds, int R, const int32_t* seqs, int nseq,
+                          int32_t* tokens, double* logp, int nthreads);
+
 /* Number of OpenMP threads the oracle would use for nthreads <= 0 (all available). */
 int oracle_max_threads(void);
 

@@ -457,6 +457,33 @@ def test_rollout_hand_case_c():
     assert logp[0] == pytest.approx(r["expect_logp"], abs=r["tolerance"])
 
 
+def test_rollout_sample_hand_case_c():
+    """Hand-worked sampled rollout (section 4.1.2 / Fig. 3) from hand case C's distributions:
+    inverse-CDF choices in id order for given uniforms."""
+    g = load("hand_case_c.json")
+    r = load("rollout_sample_case_c.json")
+    w = {n: bf16(g[n]) for n in ("w_lm", "emb", "w_ih", "w_hh", "b_ih", "b_hh", "w1", "b1", "w2", "b2")}
+    hidden = bf16(g["hidden"]).reshape(1, g["K"], g["H"])
+    for case in r["cases"]:
+        uni = np.array([case["uniforms"]], np.float32)
+        tokens, logp = oracle.rollout_sample(w, hidden, np.array([r["anchor"]], np.int32), uni)
+        if "expect_tokens" in case:
+            assert tokens[0].tolist() == case["expect_tokens"]
+            assert logp[0] == pytest.approx(case["expect_logp"], abs=r["tolerance"])
+        else:
+            assert int(tokens[0, 0]) == case["expect_first"]
+            assert logp[0, 0] == pytest.approx(case["expect_first_logp"], abs=r["tolerance"])
+
+
+def test_rollout_sample_rejects_uniforms_outside_unit_interval():
+    g = load("hand_case_c.json")
+    w = {n: bf16(g[n]) for n in ("w_lm", "emb", "w_ih", "w_hh", "b_ih", "b_hh", "w1", "b1", "w2", "b2")}
+    hidden = bf16(g["hidden"]).reshape(1, g["K"], g["H"])
+    for bad in (1.0, -0.25, np.nan):
+        with pytest.raises(RuntimeError):
+            oracle.rollout_sample(w, hidden, np.array([2], np.int32), np.array([[0.5, bad]], np.float32))
+
+
 def _small_weights(rng, V, H, Ds, R, biases):
     w = {"w_lm": rand_bf16(rng, (V, H), 0.3), "emb": rand_bf16(rng, (V, H), 0.5),
          "w_ih": rand_bf16(rng, (3 * Ds, H), 0.3), "w_hh": rand_bf16(rng, (3 * Ds, Ds), 0.3),
@@ -484,6 +511,33 @@ def test_rollout_is_the_fixed_point_of_the_teacher_forced_step(B, K, V, H, Ds, R
             row = ref["logp_full"][b, j]
             assert int(np.argmax(row)) == tokens[b, j]
             assert logp[b, j] == pytest.approx(row[tokens[b, j]], abs=1e-12)
+
+
+@pytest.mark.parametrize("B,K,V,H,Ds,R,biases", [(2, 5, 40, 16, 6, 4, False), (3, 7, 13, 8, 3, 2, True)])
+def test_rollout_sample_follows_the_teacher_forced_step(B, K, V, H, Ds, R, biases):
+    """Fed the sampled tokens as its prefix, the (pinned) draft step gives, at every position, a
+    distribution whose cumulative interval of the sampled token holds that step's uniform, and
+    the sampled token's log-probability; uniforms near 0 and near 1 pick the first and the last
+    id of non-zero probability."""
+    rng = np.random.default_rng(B * 1000 + K)
+    w = _small_weights(rng, V, H, Ds, R, biases)
+    hidden = rand_bf16(rng, (B, K, H), 1.0)
+    anchors = rng.integers(0, V, B).astype(np.int32)
+    uni = rng.random((B, K), dtype=np.float32)
+    uni[0, 0] = 0.0
+    uni[-1, -1] = np.float32(1.0) - np.float32(2 ** -24)
+    tokens, logp = oracle.rollout_sample(w, hidden, anchors, uni)
+    prefix = np.concatenate([anchors[:, None], tokens[:, :-1]], axis=1).astype(np.int32)
+    ref = oracle.draft_step(w, hidden, prefix, 1, 1, want_logp_full=True)
+    for b in range(B):
+        for j in range(K):
+            p = np.exp(ref["logp_full"][b, j])
+            t = int(tokens[b, j])
+            lo, hi = float(np.sum(p[:t])), float(np.sum(p[: t + 1]))
+            assert lo - 1e-12 <= uni[b, j] < hi + 1e-12, (b, j, t, lo, float(uni[b, j]), hi)
+            assert logp[b, j] == pytest.approx(ref["logp_full"][b, j, t], abs=1e-12)
+    assert int(tokens[0, 0]) == 0
+    assert int(tokens[-1, -1]) == int(np.nonzero(np.exp(ref["logp_full"][B - 1, K - 1]) > 0)[0][-1])
 
 
 def test_rollout_head_off_is_the_base_argmax_and_rejects_bad_anchors():
