@@ -193,6 +193,19 @@ DOMINO_API int domino_verify_tree_greedy(const float* target_logits, const int32
  * GEMM for W_lm hidden_j of every position, then one cooperative kernel for the K steps).
  * Returns DOMINO_OK once enqueued, or a negative code with nothing enqueued. */
 DOMINO_API size_t domino_rollout_workspace_bytes(int B, int K, int H, int V, int Ds, int R);
+
+/* The same loop with every draft token SAMPLED from the final distribution (section 4.1.2: each
+ * draft token is sampled from the final logits; temperature 1): with u = uniforms[b * K + j],
+ * the caller's random draws in [0, 1) (device float [B, K]; values outside are clamped to it),
+ * t_{j+1} = the first id v whose cumulative probability sum_{v' <= v} softmax(L_j)[v'], in id
+ * order, exceeds u (computed in fp32: where u falls within rounding of a boundary either
+ * neighbour may be chosen); logp_j = log-softmax(L_j)[t_{j+1}].  Arguments, outputs, workspace
+ * (domino_rollout_workspace_bytes) and errors as domino_rollout_greedy; uniforms NULL or not
+ * 4-byte aligned: DOMINO_ERR_INVALID_ARG.  One grid barrier per step more than the greedy loop. */
+DOMINO_API int domino_rollout_sample(const void* hidden, const int32_t* anchors, const float* uniforms,
+                                     const void* w_lm, const domino_head_weights* head, int B, int K, int H,
+                                     int V, int32_t* tokens, float* logp, void* workspace,
+                                     size_t workspace_bytes, void* stream);
 DOMINO_API int domino_rollout_greedy(const void* hidden, const int32_t* anchors, const void* w_lm,
                                      const domino_head_weights* head, int B, int K, int H, int V,
                                      int32_t* tokens, float* logp, void* workspace, size_t workspace_bytes,

@@ -25,7 +25,7 @@ SYMBOLS = ("domino_workspace_bytes", "domino_draft_step", "domino_workspace_byte
            "domino_draft_step_host", "domino_check_status", "domino_status_string",
            "domino_abi_version", "domino_launches_per_step", "domino_timing_begin", "domino_timing_end",
            "domino_draft_step_static_scratch", "domino_verify_tree_greedy", "domino_rollout_workspace_bytes",
-           "domino_rollout_greedy")
+           "domino_rollout_greedy", "domino_rollout_sample")
 
 DOMINO_STATIC_SCRATCH_BYTES = 16 << 20
 
@@ -89,6 +89,9 @@ def load():
     lib.domino_rollout_greedy.argtypes = [P, P, P, ctypes.POINTER(domino_head_weights)] + [I] * 4 + [P, P, P,
                                                                                                ctypes.c_size_t, P]
     lib.domino_rollout_greedy.restype = I
+    lib.domino_rollout_sample.argtypes = [P, P, P, P, ctypes.POINTER(domino_head_weights)] + [I] * 4 + [
+        P, P, P, ctypes.c_size_t, P]
+    lib.domino_rollout_sample.restype = I
     _lib = lib
     return lib
 
@@ -207,4 +210,13 @@ def domino_rollout_greedy(hidden, anchors, w_lm, head, B, K, H, V, tokens, logp,
     h = ctypes.byref(head) if head is not None else None
     return int(load().domino_rollout_greedy(_addr(hidden), _addr(anchors), _addr(w_lm), h, B, K, H, V,
                                             _addr(tokens), _addr(logp), _addr(workspace), int(workspace_bytes),
+                                            _stream(stream)))
+
+
+def domino_rollout_sample(hidden, anchors, uniforms, w_lm, head, B, K, H, V, tokens, logp, workspace,
+                          workspace_bytes, stream=None) -> int:
+    """Sampled sequential draft loop: ``uniforms`` device float32 [B, K] in [0, 1)."""
+    h = ctypes.byref(head) if head is not None else None
+    return int(load().domino_rollout_sample(_addr(hidden), _addr(anchors), _addr(uniforms), _addr(w_lm), h, B, K, H,
+                                            V, _addr(tokens), _addr(logp), _addr(workspace), int(workspace_bytes),
                                             _stream(stream)))

@@ -682,7 +682,7 @@ struct RollPlan {
   int B, K, H, V, Ds, R, M, grid;
   bool head;
   StorePlan g;  // base-logit GEMM, no split
-  size_t off_h, off_u, off_part, off_base, clear_bytes, total;
+  size_t off_h, off_u, off_part, off_next, off_base, clear_bytes, total;
 };
 
 int make_roll_plan(int B, int K, int H, int V, int Ds, int R, bool head, RollPlan* P) {
@@ -719,6 +719,7 @@ int make_roll_plan(int B, int K, int H, int V, int Ds, int R, bool head, RollPla
   p.clear_bytes = off;
   p.off_u = take(static_cast<size_t>(B) * (p.R > 0 ? p.R : 1) * 4);
   p.off_part = take(static_cast<size_t>(p.grid) * dm::kRollMaxB * 16);
+  p.off_next = take(dm::kRollMaxB * 4);  // sampled mode: t_{j+1} of every sequence
   p.off_base = take(static_cast<size_t>(p.M) * V * 4);
   p.total = off;
   return DOMINO_OK;
@@ -731,9 +732,11 @@ size_t domino_rollout_workspace_bytes(int B, int K, int H, int V, int Ds, int R)
   return P.total;
 }
 
-int domino_rollout_greedy(const void* hidden, const int32_t* anchors, const void* w_lm,
-                          const domino_head_weights* head, int B, int K, int H, int V, int32_t* tokens,
-                          float* logp, void* workspace, size_t workspace_bytes, void* stream) {
+namespace {
+// The greedy (uniforms NULL) and the sampled rollout.
+int rollout_entry(const void* hidden, const int32_t* anchors, const float* uniforms, const void* w_lm,
+                  const domino_head_weights* head, int B, int K, int H, int V, int32_t* tokens, float* logp,
+                  void* workspace, size_t workspace_bytes, void* stream) {
   const bool hd = head_active(head);
   if (!hidden || !anchors || !w_lm || !tokens || !logp || !workspace) return DOMINO_ERR_INVALID_ARG;
   if (hd && (!head->emb || !head->w_ih || !head->w_hh || !head->w1)) return DOMINO_ERR_INVALID_ARG;
@@ -796,10 +799,28 @@ int domino_rollout_greedy(const void* hidden, const int32_t* anchors, const void
   rp.tokens = tokens;
   rp.logp = logp;
   rp.status = status;
+  rp.uniforms = uniforms;
+  rp.next_tok = reinterpret_cast<int32_t*>(ws + P.off_next);
   const int ts = timing_open(DOMINO_KERNEL_ROLLOUT, st);
   rc = cuda_rc(dm::launch_rollout(rp, P.grid, st));
   timing_close(ts, st);
   return rc;
+}
+}  // namespace
+
+int domino_rollout_greedy(const void* hidden, const int32_t* anchors, const void* w_lm,
+                          const domino_head_weights* head, int B, int K, int H, int V, int32_t* tokens,
+                          float* logp, void* workspace, size_t workspace_bytes, void* stream) {
+  return rollout_entry(hidden, anchors, nullptr, w_lm, head, B, K, H, V, tokens, logp, workspace, workspace_bytes,
+                       stream);
+}
+
+int domino_rollout_sample(const void* hidden, const int32_t* anchors, const float* uniforms, const void* w_lm,
+                          const domino_head_weights* head, int B, int K, int H, int V, int32_t* tokens,
+                          float* logp, void* workspace, size_t workspace_bytes, void* stream) {
+  if (!uniforms || (reinterpret_cast<uintptr_t>(uniforms) & 3u) != 0) return DOMINO_ERR_INVALID_ARG;
+  return rollout_entry(hidden, anchors, uniforms, w_lm, head, B, K, H, V, tokens, logp, workspace, workspace_bytes,
+                       stream);
 }
 
 int domino_launches_per_step(int B, int K, int H, int V, int Ds, int R, int k, int N) {

@@ -165,6 +165,8 @@ struct RolloutParams {
   int32_t* tokens;              // [B, K] t_1 .. t_K
   float* logp;                  // [B, K]
   int* status;
+  const float* uniforms;        // [B, K] in [0, 1): sampled mode; nullptr: greedy
+  int32_t* next_tok;            // [kRollMaxB] sampled mode: t_{j+1}, written by the CTA holding it
 };
 // dynamic shared memory of one rollout CTA (the resident W2 rows or the W2 ring, u of every
 // sequence and this CTA's rows of base logits + b2): at most kRollMaxSmem, the 227 KB a CTA may

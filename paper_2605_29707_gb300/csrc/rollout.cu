@@ -364,18 +364,125 @@ __device__ __forceinline__ void pass_fma(const float (&wv)[kRowsPerPass][8], con
 // row index row0 (for the staged base logits), vocabulary id vid0 + role.r, nvalid rows valid.
 template <int KB>
 __device__ __forceinline__ void pass_push(const float (&dot)[kRowsPerPass * KB], const PassRole& role, int nvalid,
-                                          int row0, int vid0, const float* s_base, int rows_cta, int B, Lse& mine) {
+                                          int row0, int vid0, float* s_base, int rows_cta, int B, Lse& mine) {
   const float d = ReduceScatter<kRowsPerPass * KB, 16>::run(dot);
-  if (role.rep && role.r < nvalid && role.b < B)
-    lse_push(mine, s_base[role.b * rows_cta + row0 + role.r] + d, vid0 + role.r);
+  if (role.rep && role.r < nvalid && role.b < B) {
+    float* x = s_base + role.b * rows_cta + row0 + role.r;
+    const float logit = *x + d;
+    *x = logit;  // the final logit, for the sampled mode's scan of this CTA's rows
+    lse_push(mine, logit, vid0 + role.r);
+  }
 }
 
 // The end of a step, shared by both kernels: per-CTA partials, grid barrier, every CTA's
 // combine (thread c loads CTA c's partials, then the same block reduction in every CTA, so all
 // reach the same t_{j+1}), the outputs.  Returns false if the barrier gave up.
+// Sampled mode, after the combine (a_all[b]: the merged state of sequence b in every CTA):
+// t_{j+1} = the first id whose cumulative probability in id order exceeds u_{b,j}.  The CTAs'
+// masses w_c = s_c exp(m_c - max) are scanned in CTA order (their slices are consecutive), which
+// names the CTA holding the crossing; that CTA scans its own rows' final logits in id order,
+// writes the token and its log-probability, and one more grid barrier hands the token to all.
+// (If rounding leaves the crossing past its rows, it takes its last row of non-zero mass.)
+template <int KB>
+__device__ bool sample_step(const RolloutParams& p, int j, const float* s_logit, int r_lo, int r_n, int rows_cta,
+                            int* s_tok, unsigned& nbar, volatile int* s_fail, const float* s_max,
+                            const float* s_lz) {
+  __shared__ float s_T[kRollMaxB], s_off[kRollMaxB];
+  __shared__ int s_owner[kRollMaxB], s_pick[kRollMaxB], s_last[kRollMaxB];
+  __shared__ float s_wsum[kRollWarps][kRollMaxB];
+  const int B = p.B, K = p.K, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int grid = static_cast<int>(gridDim.x);  // <= kRollThreads (checked at launch)
+  if (tid < kRollMaxB) { s_owner[tid] = -1; s_off[tid] = 0.f; s_T[tid] = 0.f; }
+  // per-CTA masses (thread c: CTA c) and their inclusive scan in CTA order
+  float incl[KB], w[KB];
+#pragma unroll
+  for (int b = 0; b < KB; ++b) {
+    w[b] = 0.f;
+    if (b < B && tid < grid) {
+      const float4 f = __ldcg(reinterpret_cast<const float4*>(p.partials) + static_cast<size_t>(tid) * kRollMaxB + b);
+      w[b] = f.x == -INFINITY ? 0.f : f.y * __expf(f.x - s_max[b]);
+    }
+    incl[b] = w[b];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float t = __shfl_up_sync(0xffffffffu, incl[b], o);
+      if (lane >= o) incl[b] += t;
+    }
+    if (lane == 31) s_wsum[warp][b] = incl[b];
+  }
+  compute_sync();
+#pragma unroll
+  for (int b = 0; b < KB; ++b) {
+    if (b >= B) continue;
+    float off = 0.f, total = 0.f;
+    for (int ww = 0; ww < kRollWarps; ++ww) {
+      if (ww < warp) off += s_wsum[ww][b];
+    }
+    for (int ww = 0; ww < kRollWarps; ++ww) total += s_wsum[ww][b];
+    const float prev = __shfl_up_sync(0xffffffffu, incl[b], 1);
+    const float excl = (lane == 0 ? 0.f : prev) + off;
+    const float inc = incl[b] + off;
+    float u = p.uniforms[static_cast<size_t>(b) * K + j];
+    u = fminf(fmaxf(u, 0.f), 1.f - 1.2e-7f);  // [0, 1)
+    const float T = u * total;
+    if (tid < grid && w[b] > 0.f && excl <= T && T < inc) {
+      s_owner[b] = tid;
+      s_off[b] = excl;
+      s_T[b] = T;
+    }
+  }
+  compute_sync();
+  for (int b = 0; b < B; ++b) {
+    // no claim (no mass anywhere: non-finite logits) falls to CTA 0 and its first row
+    const int owner = s_owner[b] >= 0 ? s_owner[b] : 0;
+    if (owner != static_cast<int>(blockIdx.x)) continue;  // the same test in every thread
+    const float mx = s_max[b], T = s_T[b];
+    const float* lg = s_logit + b * rows_cta;
+    const int per = (r_n + kRollThreads - 1) / kRollThreads;
+    const int q0 = min(r_n, tid * per), q1 = min(r_n, q0 + per);
+    float loc = 0.f;
+    for (int r = q0; r < q1; ++r) loc += __expf(lg[r] - mx);
+    // exclusive scan of the threads' sums (thread order = row order)
+    float inc = loc;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float t = __shfl_up_sync(0xffffffffu, inc, o);
+      if (lane >= o) inc += t;
+    }
+    if (tid == 0) { s_pick[b] = 0x7fffffff; s_last[b] = -1; }
+    if (lane == 31) s_wsum[warp][b] = inc;
+    compute_sync();
+    float off = s_off[b];
+    for (int ww = 0; ww < warp; ++ww) off += s_wsum[ww][b];
+    float acc = off + inc - loc;
+    int cand = 0x7fffffff, last = -1;
+    for (int r = q0; r < q1; ++r) {
+      const float e = __expf(lg[r] - mx);
+      if (e > 0.f) last = r;
+      acc += e;
+      if (acc > T) { cand = r; break; }
+    }
+    if (cand != 0x7fffffff) atomicMin(&s_pick[b], cand);
+    if (last >= 0) atomicMax(&s_last[b], last);
+    compute_sync();
+    if (tid == 0) {
+      const int r = s_pick[b] != 0x7fffffff ? s_pick[b] : max(0, s_last[b]);
+      const int tok = r_lo + r;
+      p.tokens[static_cast<size_t>(b) * K + j] = tok;
+      p.logp[static_cast<size_t>(b) * K + j] = lg[r] - mx - s_lz[b];
+      p.next_tok[b] = tok;
+    }
+  }
+  if (!grid_barrier(p.barrier, nbar++, p.status, s_fail)) return false;
+  if (tid < B) s_tok[tid] = __ldcg(p.next_tok + tid);
+  compute_sync();
+  return true;
+}
+
 template <int KB>
 __device__ __forceinline__ bool finish_step(const RolloutParams& p, int j, Lse (&st)[KB], Lse (*s_red)[kRollMaxB],
-                                            int* s_tok, unsigned& nbar, volatile int* s_fail) {
+                                            int* s_tok, unsigned& nbar, volatile int* s_fail, const float* s_logit,
+                                            int r_lo, int r_n, int rows_cta) {
   const int B = p.B, K = p.K, tid = threadIdx.x;
   block_reduce(st, s_red, B);
   if (tid < B) {
@@ -399,6 +506,17 @@ __device__ __forceinline__ bool finish_step(const RolloutParams& p, int j, Lse (
     }
   }
   block_reduce(st, s_red, B);
+  if (p.uniforms) {
+    __shared__ float s_gmax[kRollMaxB], s_glz[kRollMaxB];
+    if (tid < B) {
+      Lse a = s_red[0][tid];
+      for (int w = 1; w < kRollWarps; ++w) lse_merge(a, s_red[w][tid]);
+      s_gmax[tid] = a.m;
+      s_glz[tid] = logf(a.s);
+    }
+    compute_sync();
+    return sample_step<KB>(p, j, s_logit, r_lo, r_n, rows_cta, s_tok, nbar, s_fail, s_gmax, s_glz);
+  }
   if (tid < B) {
     Lse a = s_red[0][tid];
     for (int w = 1; w < kRollWarps; ++w) lse_merge(a, s_red[w][tid]);
@@ -449,10 +567,15 @@ __device__ __forceinline__ void group_fma(const uint4 (&raw)[G], int r_in_pass, 
 
 template <int KB>
 __device__ __forceinline__ void wide_push(const float (&dot)[32], int lane, int nvalid, int row0, int vid0,
-                                          const float* s_base, const float* s_b2, int rows_cta, int B, Lse& mine) {
+                                          float* s_base, const float* s_b2, int rows_cta, int B, Lse& mine) {
   const float d = ReduceScatter<32, 16>::run(dot);
   const int r = lane / KB, b = lane % KB;
-  if (r < nvalid && b < B) lse_push(mine, s_base[b * rows_cta + row0 + r] + s_b2[row0 + r] + d, vid0 + r);
+  if (r < nvalid && b < B) {
+    float* x = s_base + b * rows_cta + row0 + r;
+    const float logit = *x + s_b2[row0 + r] + d;
+    *x = logit;  // the final logit, for the sampled mode's scan of this CTA's rows
+    lse_push(mine, logit, vid0 + r);
+  }
 }
 
 // ================================================================ resident kernel (r <= 256)
@@ -629,7 +752,7 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
       Lse st[KB];
 #pragma unroll
       for (int b = 0; b < KB; ++b) st[b] = (b == lane % KB) ? mine : lse_empty();
-      if (!finish_step<KB>(p, j, st, s_red, s_tok, nbar, &s_fail)) break;
+      if (!finish_step<KB>(p, j, st, s_red, s_tok, nbar, &s_fail, s_base, r_lo, r_n, rows_cta)) break;
     }
   }
   // ---- teardown: the asynchronous copies have landed (the fill: bounded), tensor memory is
@@ -798,7 +921,7 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
           if (b < B) lse_push(st[b], s_base[b * rows_cta + r], r_lo + r);
       }
     }
-    if (!finish_step<KB>(p, j, st, s_red, s_tok, nbar, &s_fail)) return;
+    if (!finish_step<KB>(p, j, st, s_red, s_tok, nbar, &s_fail, s_base, r_lo, r_n, rows_cta)) return;
   }
 }
 
@@ -856,6 +979,7 @@ static cudaError_t launch_rollout_kb(const RolloutParams& p, int grid, size_t sm
 
 cudaError_t launch_rollout(const RolloutParams& p, int grid, cudaStream_t stream) {
   if (p.B < 1 || p.B > kRollMaxB || grid < 1) return cudaErrorInvalidValue;
+  if (p.uniforms && (grid > kRollThreads || !p.next_tok)) return cudaErrorInvalidValue;  // one thread per CTA
   const size_t smem = rollout_smem_bytes(p.B, p.V, p.R, p.head, grid);
   if (smem > kRollMaxSmem) return cudaErrorInvalidValue;
   RolloutParams pp = p;

@@ -9,6 +9,8 @@ valid greedy choice there (within 4e-2 of the position's best log-probability) w
 log-probability within 2e-2; and up to the first such near-tie the GPU tokens must equal the
 oracle rollout's exactly.
 """
+import ctypes
+
 import numpy as np
 import pytest
 import torch
@@ -122,3 +124,107 @@ def test_rollout_rejects_bad_anchor_and_sizes():
 @pytest.mark.parametrize("name", ["qwen3-8b", "qwen3-1.7b"])
 def test_rollout_full_size(name):
     _check(inputs.cached_workload(name))
+
+
+# ---------------------------------------------------------------------------- sampled loop
+CDF_TOL = 5e-3  # fp32 logits and sums on the GPU against fp64: how far u may sit past a boundary
+
+
+def _run_gpu_sample(wl, uniforms, head_on=True):
+    c = wl.cfg
+    dev = torch.device("cuda:0")
+    w, head = _device_weights(wl, dev, head_on)
+    hidden = torch.from_numpy(wl.hidden.view(np.int16)).view(torch.bfloat16).to(dev)
+    anchors = torch.from_numpy(np.ascontiguousarray(wl.prefix_ids[:, 0])).to(dev)
+    uni = torch.from_numpy(uniforms).to(dev)
+    nbytes = binding.domino_rollout_workspace_bytes(c.B, c.K, c.H, c.V, c.Ds if head_on else 0, c.R if head_on else 0)
+    ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    tokens = torch.full((c.B, c.K), -7, dtype=torch.int32, device=dev)
+    logp = torch.full((c.B, c.K), 7.0, dtype=torch.float32, device=dev)
+    s = torch.cuda.current_stream(dev)
+    rc = binding.domino_rollout_sample(hidden, anchors, uni, w["w_lm"], head, c.B, c.K, c.H, c.V, tokens, logp, ws,
+                                       nbytes, s)
+    assert rc == 0, binding.domino_status_string(rc)
+    assert binding.domino_check_status(ws, s) == 0
+    return tokens.cpu().numpy(), logp.cpu().numpy()
+
+
+def _check_sample(wl, head_on=True, seed=5):
+    """Teacher-forced: every GPU token's cumulative-probability interval (under the oracle's step
+    fed the GPU's own tokens) holds its uniform within CDF_TOL, with logp within LOGP_TOL; up to
+    the first uniform within CDF_TOL of one of the oracle rollout's boundaries, the tokens equal
+    the oracle rollout's."""
+    c = wl.cfg
+    w = wl.weights if head_on else {"w_lm": wl.weights["w_lm"], "b2": wl.weights.get("b2")}
+    uni = np.random.default_rng(seed).random((c.B, c.K), dtype=np.float32)
+    tokens, logp = _run_gpu_sample(wl, uni, head_on)
+    anchors = np.ascontiguousarray(wl.prefix_ids[:, 0]).astype(np.int32)
+    o_tok, _ = oracle.rollout_sample(w, wl.hidden, anchors, uni)
+    excused = 0
+    for b in range(c.B):
+        prefix = np.concatenate([[anchors[b]], tokens[b, :-1]]).astype(np.int32)[None, :]
+        ref = oracle.draft_step(w, wl.hidden[b:b + 1], prefix, 1, 1, want_logp_full=True)
+        same = True
+        for j in range(c.K):
+            lp = ref["logp_full"][0, j]
+            cdf = np.cumsum(np.exp(lp))
+            t = int(tokens[b, j])
+            assert 0 <= t < c.V
+            lo = cdf[t - 1] if t > 0 else 0.0
+            u = float(uni[b, j])
+            assert lo - CDF_TOL <= u <= cdf[t] + CDF_TOL, (b, j, t, lo, u, cdf[t])
+            assert abs(float(logp[b, j]) - lp[t]) <= LOGP_TOL, (b, j, logp[b, j], lp[t])
+            if same:
+                ot = int(o_tok[b, j])
+                olo = cdf[ot - 1] if ot > 0 else 0.0
+                if min(u - olo, cdf[ot] - u) > CDF_TOL:
+                    assert t == ot, (b, j, t, ot)
+                elif t != ot:
+                    excused += 1
+                    same = False
+    return excused
+
+
+@pytest.mark.parametrize("cfg", [
+    inputs.CONFIGS["tiny"],
+    inputs.custom_config("samp-b3", B=3, K=8, H=512, V=3000, Ds=64, R=64, seed=31, biases=True),
+    inputs.custom_config("samp-b8", B=8, K=5, H=256, V=1000, Ds=32, R=16, seed=32),
+    inputs.custom_config("samp-wide", B=2, K=4, H=256, V=2500, Ds=32, R=512, seed=33, biases=True),
+    inputs.custom_config("samp-tiers", B=8, K=3, H=256, V=167001, Ds=32, R=256, seed=34),
+])
+def test_rollout_sample_matches_oracle(cfg):
+    _check_sample(inputs.make_workload(cfg))
+
+
+def test_rollout_sample_head_off():
+    _check_sample(inputs.make_workload(inputs.custom_config("samp-off", B=2, K=6, H=256, V=2000, seed=35)),
+                  head_on=False)
+
+
+@pytest.mark.parametrize("name", ["qwen3-8b"])
+def test_rollout_sample_full_size(name):
+    _check_sample(inputs.cached_workload(name), seed=7)
+
+
+def test_rollout_sample_uniform_ends_and_bad_pointer():
+    """u = 0 takes the first id of non-zero probability (id 0 here), and a misaligned uniforms
+    pointer is refused before anything is enqueued."""
+    wl = inputs.make_workload(inputs.custom_config("samp-ends", B=2, K=3, H=128, V=700, Ds=16, R=8, seed=36))
+    c = wl.cfg
+    uni = np.zeros((c.B, c.K), np.float32)
+    tokens, _ = _run_gpu_sample(wl, uni)
+    assert (tokens == 0).all()
+    dev = torch.device("cuda:0")
+    w, head = _device_weights(wl, dev)
+    hidden = torch.from_numpy(wl.hidden.view(np.int16)).view(torch.bfloat16).to(dev)
+    anchors = torch.from_numpy(np.ascontiguousarray(wl.prefix_ids[:, 0])).to(dev)
+    raw = torch.zeros(c.B * c.K + 1, dtype=torch.float32, device=dev)
+    nbytes = binding.domino_rollout_workspace_bytes(c.B, c.K, c.H, c.V, c.Ds, c.R)
+    ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    out_t = torch.empty((c.B, c.K), dtype=torch.int32, device=dev)
+    out_l = torch.empty((c.B, c.K), dtype=torch.float32, device=dev)
+    bad = raw.data_ptr() + 2  # not 4-byte aligned
+    f = binding.load().domino_rollout_sample
+    h = ctypes.byref(head)
+    assert f(hidden.data_ptr(), anchors.data_ptr(), bad, w["w_lm"].data_ptr(), h, c.B, c.K, c.H, c.V,
+             out_t.data_ptr(), out_l.data_ptr(), ws.data_ptr(), nbytes, None) == binding.DOMINO_ERR_INVALID_ARG
