@@ -380,6 +380,26 @@ def rollout_timing(st, wl, c, hidden, device, stream, reps=50):
     kern = binding.domino_timing_end()
     status = binding.domino_check_status(ws, stream)
     split = {n: round(v[0] / max(1, v[1]) * 1e3, 2) for n, v in kern.items() if v[1] > 0}
+    # the sampled loop (inverse CDF from uniforms) on the same inputs
+    uni = torch.rand((c.B, c.K), generator=torch.Generator().manual_seed(11)).to(device)
+    stok = torch.empty_like(tok)
+    slp = torch.empty_like(lp)
+
+    def run_s():
+        rc = binding.domino_rollout_sample(hidden, anchors, uni, st.w["w_lm"], st.head, c.B, c.K, c.H, c.V, stok,
+                                           slp, ws, nb, stream)
+        if rc != 0:
+            raise RuntimeError(f"domino_rollout_sample returned {rc}")
+    for _ in range(3):
+        run_s()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(reps):
+        run_s()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    us_s = e0.elapsed_time(e1) / reps * 1e3
+    status_s = binding.domino_check_status(ws, stream)
     # every weight read once (W_lm by the base GEMM; W2, the GRU weights and W1 by the step
     # kernel, which keeps W2 on chip and the rest in L2 across steps) plus the fp32 base logits
     # written and read back once
@@ -389,6 +409,8 @@ def rollout_timing(st, wl, c, hidden, device, stream, reps=50):
     roof_us = unique / (peaks["hbm_gbs"] * 1e9) * 1e6
     return {"us_per_block": round(us, 2), "draft_tokens_per_s": round(c.B * c.K / (us * 1e-6), 1),
             "us_per_kernel": split, "status": status, "unique_bytes_per_block": unique,
+            "sampled": {"us_per_block": round(us_s, 2), "draft_tokens_per_s": round(c.B * c.K / (us_s * 1e-6), 1),
+                        "status": status_s},
             "hbm_roofline_us": round(roof_us, 2), "frac_of_hbm_roofline": round(roof_us / us, 4),
             "note": "B sequences x K greedy draft tokens, each fed back; timing only (parity is in the tests)"}
 
