@@ -105,8 +105,12 @@ DOMINO_API size_t domino_workspace_bytes(int B, int K, int H, int V, int Ds, int
  *   tree_token  int32 [B, N]
  *   tree_depth  int32 [B, N]     1..K
  *   tree_score  fp32  [B, N] or NULL   cumulative log-probability, non-increasing in i
- * workspace: device buffer of at least domino_workspace_bytes(...) bytes, 256-byte aligned;
- * one workspace must not be shared by steps that overlap in time.
+ * workspace: device buffer of at least domino_workspace_bytes(...) bytes, 256-byte aligned,
+ * ZERO-FILLED before its first use (once, e.g. cudaMemsetAsync at allocation); every step
+ * leaves it ready for the next one, whatever the sizes (small batches skip a per-step clear:
+ * the GRU's state words carry a step count the last kernel advances).  Zero it again after a
+ * call that returned DOMINO_ERR_CUDA part-way.  One workspace must not be shared by steps that
+ * overlap in time.
  * Returns DOMINO_OK once everything is enqueued, or a negative code (nothing enqueued). */
 DOMINO_API int domino_draft_step(const void* hidden, const int32_t* prefix_ids, const void* w_lm,
                       const domino_head_weights* head, int B, int K, int H, int V, int k, int N,
@@ -120,7 +124,8 @@ DOMINO_API int domino_draft_step(const void* hidden, const int32_t* prefix_ids, 
  * copy into a pinned staging buffer the library allocates on first use and keeps for the
  * process (calls from several threads take turns on it), from which they are copied to the
  * caller's buffers; the call synchronises the stream before returning.  The workspace must
- * hold domino_workspace_bytes_host(...) bytes.  Returns DOMINO_OK or the first error,
+ * hold domino_workspace_bytes_host(...) bytes and be zero-filled before its first use, as for
+ * domino_draft_step.  Returns DOMINO_OK or the first error,
  * including device-side errors (bad prefix id, timeout). */
 DOMINO_API size_t domino_workspace_bytes_host(int B, int K, int H, int V, int Ds, int R, int k, int N);
 DOMINO_API int domino_draft_step_host(const void* hidden_host, const int32_t* prefix_ids_host,

@@ -210,10 +210,13 @@ int make_plan_sms(int B, int K, int H, int V, int Ds, int R, int k, int N, bool 
   };
   p.ctrl_bytes = align_up(256 + static_cast<size_t>(B) * 4);
   p.off_ctrl = take(p.ctrl_bytes);
-  p.clear_bytes = p.ctrl_bytes;
+  // control words: status at 0, GRU barrier counter at 64, step epoch at 128, merge counters
+  // from 256.  Fused projections need no clear before a step (the GRU resets the status and the
+  // counters, and its state words carry the epoch as a tag); the workspace must only be zero
+  // when first used.
+  p.clear_bytes = p.fused ? 0 : p.ctrl_bytes;
   if (head) {
-    p.off_hx = take(static_cast<size_t>(M) * Ds * 4);  // right after the control words: one clear
-    if (p.fused) p.clear_bytes = p.off_hx + static_cast<size_t>(M) * Ds * 4 - p.off_ctrl;
+    p.off_hx = take(static_cast<size_t>(M) * Ds * 4);
     p.off_E = take(static_cast<size_t>(M) * H * 2);
     p.off_xpart = take(static_cast<size_t>(p.xg.splits) * M * 3 * Ds * 4);
     p.off_upart = take(static_cast<size_t>(p.ug.splits) * M * R * 4);
@@ -338,7 +341,8 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
   int* status = reinterpret_cast<int*>(ws + P.off_ctrl);
   unsigned* barrier = reinterpret_cast<unsigned*>(ws + P.off_ctrl + 64);
   unsigned* seq_done = reinterpret_cast<unsigned*>(ws + P.off_ctrl + 256);
-  if (cudaMemsetAsync(ws + P.off_ctrl, 0, P.clear_bytes, st) != cudaSuccess) return DOMINO_ERR_CUDA;
+  if (P.clear_bytes && cudaMemsetAsync(ws + P.off_ctrl, 0, P.clear_bytes, st) != cudaSuccess) return DOMINO_ERR_CUDA;
+  uint32_t* epoch = reinterpret_cast<uint32_t*>(ws + P.off_ctrl + 128);
 
   __nv_bfloat16* E = P.head ? reinterpret_cast<__nv_bfloat16*>(ws + P.off_E) : nullptr;
   uint32_t* hx = P.head ? reinterpret_cast<uint32_t*>(ws + P.off_hx) : nullptr;
@@ -431,6 +435,9 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
     gr.s_out = P.u_in_gru ? nullptr : S;
     gr.u = P.u_in_gru ? u : nullptr;
     gr.status = status;
+    gr.epoch = epoch;
+    gr.seq_done = seq_done;
+    gr.reset_ctrl = P.fused ? 1 : 0;
     if (P.fused) {
       gr.ids = ids;
       gr.emb = static_cast<const __nv_bfloat16*>(hw->emb);
@@ -496,6 +503,7 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
   tr.tree_parent = tpar; tr.tree_token = ttok; tr.tree_depth = tdep; tr.tree_score = tsc;
   tr.status = status;
   tr.status_out = status_out;
+  tr.epoch = P.head ? epoch : nullptr;
   ts = timing_open(DOMINO_KERNEL_TREE, st);
   rc = cuda_rc(dm::launch_merge_tree(tr, st));
   timing_close(ts, st);

@@ -5,9 +5,9 @@
 // full previous state of a sequence.  One cooperative launch keeps the W_hh rows of a block of
 // hidden units resident in shared memory for all K steps and computes W_hh . h_{t-1} on the
 // tensor cores (mma.sync, bf16 operands, fp32 accumulation).  States cross CTAs through L2 as
-// tagged words (bf16 value in the high half, a non-zero flag in the low half; one row per
-// (sequence, position), cleared by the gather kernel), so a CTA waits for exactly the data it
-// reads: no grid barrier and no release fence.  Every wait is bounded.
+// tagged words (bf16 value in the high half, the step's 16-bit tag in the low half; one row per
+// (sequence, position)), so a CTA waits for exactly the data it reads: no grid barrier and no
+// release fence.  Every wait is bounded.
 #include <math.h>
 
 #include "kernels.h"
@@ -76,23 +76,28 @@ __device__ __forceinline__ uint4 ld_relaxed_v4(const uint32_t* p) {
   return v;
 }
 
-// Reads 4 tagged state words, re-reading until all four carry the "written" flag.  Returns
-// false if that takes longer than kWaitCycles (the caller reports DOMINO_ERR_TIMEOUT).
-__device__ __forceinline__ bool poll_v4(const uint32_t* p, uint4& v) {
+// Four state words all written in this step: their low halves equal the step's tag.
+__device__ __forceinline__ bool all_tagged(const uint4& v, uint32_t tag) {
+  return (((v.x ^ tag) | (v.y ^ tag) | (v.z ^ tag) | (v.w ^ tag)) & 0xFFFFu) == 0u;
+}
+
+// Reads 4 tagged state words, re-reading until all four carry this step's tag.  Returns false
+// if that takes longer than kWaitCycles (the caller reports DOMINO_ERR_TIMEOUT).
+__device__ __forceinline__ bool poll_v4(const uint32_t* p, uint4& v, uint32_t tag) {
   v = ld_relaxed_v4(p);
-  if ((v.x & v.y & v.z & v.w & 1u) != 0u) return true;
+  if (all_tagged(v, tag)) return true;
   const long long t0 = clock64();
   while (true) {
     if (DOMINO_GRU_BACKOFF_NS > 0) __nanosleep(DOMINO_GRU_BACKOFF_NS);  // spare L2 while waiting
     v = ld_relaxed_v4(p);
-    if ((v.x & v.y & v.z & v.w & 1u) != 0u) return true;
+    if (all_tagged(v, tag)) return true;
     if (clock64() - t0 > kWaitCycles) return false;
   }
 }
 
-__device__ __forceinline__ uint32_t tagged(float h) {
+__device__ __forceinline__ uint32_t tagged(float h, uint32_t tag) {
   const uint32_t b = static_cast<uint32_t>(__bfloat16_as_ushort(__float2bfloat16_rn(h)));
-  return (b << 16) | 1u;
+  return (b << 16) | tag;
 }
 
 // two tagged words -> packed bf16x2 (low element first)
@@ -193,9 +198,12 @@ __device__ void fused_projections(const GruParams& p, int j0, int Uc, int b0, in
   const int H = p.H, Ds = p.Ds, K = p.K, R = p.R, M = p.B * p.K;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, t = lane & 3;
-  for (int m = tid; m < M; m += kGruThreads) {
-    const int id = p.ids[m];
-    if (id < 0 || id >= p.V) set_status(p.status, kStatusBadToken);
+  __syncthreads();  // CTA 0: the status reset comes first
+  if (blockIdx.x == 0) {
+    for (int m = tid; m < M; m += kGruThreads) {
+      const int id = p.ids[m];
+      if (id < 0 || id >= p.V) set_status(p.status, kStatusBadToken);
+    }
   }
   const int rows = nbc * K;  // this CTA's positions: m = b0 * K + r
   const int nchunk = (H + 63) / 64;
@@ -304,6 +312,17 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
   float* hprev = reinterpret_cast<float*>(gsmem + L.hprev);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int ldw = L.ldw;
+  // This step's tag for the state words (low half): the workspace's step epoch, advanced by
+  // the merge kernel at the end of every step, so that words a previous step wrote never pass
+  // for this step's; 0 (a cleared word) is never a tag.
+  const uint32_t tag = (*p.epoch % 0xFFFFu) + 1u;
+  // Without a clear before the launch (fused projections) the first CTA resets the step's
+  // status and the merge counters; only it then checks the ids (after the barrier below), so a
+  // reset can never hide an error of this step.
+  if (p.reset_ctrl && blockIdx.x == 0 && tid == 0) {
+    *p.status = 0;
+    for (int b = 0; b < B; ++b) p.seq_done[b] = 0u;
+  }
   // the vocabulary GEMM that follows may start now: its first K segment does not read
   // anything this kernel writes, and it waits for this grid before reading u
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -417,9 +436,9 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
             const int e = e0 + i * 32;
             if (e < total && got) {
               const int bb = e / ncq, cq = q0 + e % ncq;
-              if ((v[i].x & v[i].y & v[i].z & v[i].w & 1u) == 0u) {
+              if (!all_tagged(v[i], tag)) {
                 const size_t m = static_cast<size_t>(b0 + c0 + bb) * K + (t - 1);
-                got = poll_v4(p.hx + m * Ds + cq * 4, v[i]);
+                got = poll_v4(p.hx + m * Ds + cq * 4, v[i], tag);
               }
               *reinterpret_cast<uint2*>(hsm + static_cast<size_t>(bb) * ldw + cq * 4) =
                   make_uint2(pack_hi_halves(v[i].x, v[i].y), pack_hi_halves(v[i].z, v[i].w));
@@ -507,7 +526,7 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
         const float n = tanhf(gx[rr][2] + r * hn);
         const float h = (1.f - z) * n + z * hp;
         hprev[bl * U + jl] = h;
-        p.hx[m * Ds + j] = tagged(h);
+        p.hx[m * Ds + j] = tagged(h, tag);
         if (p.s_out) p.s_out[m * Ds + j] = __float2bfloat16_rn(h);
       }
       __syncthreads();
@@ -548,7 +567,7 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
           if (c >= Ds || !got) continue;
           for (int h = 0; h < 2; ++h) {
             uint4& x = sv[2 * i + h];
-            if ((x.x & x.y & x.z & x.w & 1u) == 0u) got = got && poll_v4(srow + c + 4 * h, x);
+            if (!all_tagged(x, tag)) got = got && poll_v4(srow + c + 4 * h, x, tag);
           }
           const __nv_bfloat162* w2 = reinterpret_cast<const __nv_bfloat162*>(&wv[i]);
           const uint32_t sw[8] = {sv[2 * i].x, sv[2 * i].y, sv[2 * i].z, sv[2 * i].w,

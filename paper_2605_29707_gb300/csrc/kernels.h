@@ -97,7 +97,7 @@ struct GruParams {
   int B, K, H, Ds, R;
   int units, gu, gb, bc;      // grid shape: gu unit blocks x gb sequence groups of bc
   float* xs;                  // [M][3*Ds] input-gate sums (scratch)
-  uint32_t* hx;               // [M][Ds] tagged states (cleared before the launch)
+  uint32_t* hx;               // [M][Ds] tagged states (words of earlier steps carry other tags)
   __nv_bfloat16* s_out;       // [M][Ds] plain bf16 states, or nullptr
   __nv_bfloat16* u;           // [M][R] low-rank code computed in-kernel, or nullptr
   int* status;
@@ -109,6 +109,9 @@ struct GruParams {
   const __nv_bfloat16* w_ih;  // [3*Ds, H]
   const __nv_bfloat16* hidden;  // [M, H]
   int V;
+  const uint32_t* epoch;      // the workspace's step epoch (the state words' tag)
+  unsigned int* seq_done;     // [B] merge counters
+  int reset_ctrl;             // no clear before the launch: CTA 0 resets the status and seq_done
 };
 // Largest number of (rank row, position) pairs of u one warp finalises for which the fused
 // projections apply (their hidden halves wait in shared memory).
@@ -145,6 +148,7 @@ struct TreeParams {
   float* tree_score;      // or nullptr
   const int* status;      // the step's device status word
   int32_t* status_out;    // or nullptr: a copy of it beside the outputs, made once the step is done
+  uint32_t* epoch;        // the workspace's step epoch, advanced once the step's GRU is done
 };
 cudaError_t launch_merge_tree(const TreeParams& p, cudaStream_t stream);
 

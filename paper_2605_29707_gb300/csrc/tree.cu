@@ -265,7 +265,10 @@ __global__ void __launch_bounds__(NT, NT == kMergeThreadsNarrow ? 8 : 1) merge_t
   // launched as a programmatic dependent of the vocabulary GEMM: wait for its partials
   asm volatile("griddepcontrol.wait;" ::: "memory");
   // every earlier kernel of the step has completed: its status is final
-  if (m == 0 && tid == 0 && p.status_out) *p.status_out = *p.status;
+  if (m == 0 && tid == 0) {
+    if (p.status_out) *p.status_out = *p.status;
+    if (p.epoch) *p.epoch += 1u;  // the next step's GRU tags its state words differently
+  }
   const float* base = p.partials + static_cast<size_t>(m) * F * nch;
   const int* ibase = reinterpret_cast<const int*>(base);
 

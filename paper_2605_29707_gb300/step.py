@@ -33,7 +33,8 @@ class DraftStep:
         if self.ws_bytes == 0:
             raise B_.DominoError(B_.DOMINO_ERR_UNSUPPORTED, "domino_workspace_bytes")
         self.ws_host_bytes = B_.domino_workspace_bytes_host(B, K, H, V, self.Ds, self.R, k, N)
-        self.workspace = torch.empty(self.ws_host_bytes, dtype=torch.uint8, device=dev)
+        # zero-filled once: the library expects a zero workspace at its first use
+        self.workspace = torch.zeros(self.ws_host_bytes, dtype=torch.uint8, device=dev)
         M = B * K
         self.topk_ids = torch.empty(M * k, dtype=torch.int32, device=dev)
         self.topk_logp = torch.empty(M * k, dtype=torch.float32, device=dev)
