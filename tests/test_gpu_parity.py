@@ -103,6 +103,27 @@ def test_deterministic_and_host_entry_point_matches():
     np.testing.assert_array_equal(host["tree_score"].numpy().reshape(out1["tree_score"].shape), out1["tree_score"])
 
 
+@pytest.mark.parametrize("B,K", [(1, 6), (4, 16)])
+def test_consecutive_steps_on_one_workspace(B, K):
+    """Steps with different inputs back to back on one workspace each match the oracle: state
+    words a previous step left behind (tagged with its epoch at B <= 2, cleared at larger B)
+    never pass for the current step's."""
+    cfg = inputs.custom_config("consec", B=B, K=K, H=256, V=2000, Ds=64, R=64, k=4, N=8, seed=41, biases=True)
+    wl_a = inputs.make_workload(cfg)
+    # same head and LM head, new hidden states and prefixes
+    wl_b = inputs.make_workload(inputs.custom_config("consec", B=B, K=K, H=256, V=2000, Ds=64, R=64, k=4, N=8,
+                                                     seed=42, biases=True), weights=wl_a.weights)
+    c = wl_a.cfg
+    st = DraftStep(wl_a.weights, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=_dev())
+    for wl in (wl_a, wl_b, wl_a, wl_b):
+        hidden = torch.from_numpy(wl.hidden.view(np.int16)).view(torch.bfloat16).to(_dev())
+        ids = torch.from_numpy(wl.prefix_ids).to(_dev())
+        out = st.run(hidden, ids)
+        ex_topk, ex_tree, _ = _check(wl, out)
+        assert ex_topk <= max(1, c.M * c.k // 50)
+        assert ex_tree <= max(1, c.B * c.N // 10)
+
+
 # the GRU's own id check (3 launches) and the gather kernel's (6 launches)
 @pytest.mark.parametrize("B,K,expect", [(1, 4, 3), (4, 16, 6)])
 def test_bad_token_reported_by_device_status(B, K, expect):
