@@ -19,21 +19,6 @@
 
 namespace dm {
 
-#ifdef DOMINO_GRU_TRACE
-__device__ unsigned long long g_gru_trace[2][64][8];  // [cta 0 / last][step][phase] globaltimer
-__device__ __forceinline__ void gru_trace(int step, int ph) {
-  const int w = blockIdx.x == 0 ? 0 : (blockIdx.x == gridDim.x - 1 ? 1 : -1);
-  if (w >= 0 && threadIdx.x == 0 && step < 64) {
-    unsigned long long t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    g_gru_trace[w][step][ph] = t;
-  }
-}
-#define GRU_TRACE(step, ph) gru_trace(step, ph)
-#else
-#define GRU_TRACE(step, ph)
-#endif
-
 constexpr int kGruThreads = 256;
 constexpr int kGatePairsPerThread = 4;  // (sequence, unit) gate evaluations per thread and chunk
 constexpr int kGruWarps = kGruThreads / 32;
@@ -389,7 +374,6 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
   bool ok = true;
 
   for (int t = 0; t < K && ok; ++t) {
-    GRU_TRACE(t, 0);
     for (int c0 = 0; c0 < nbc; c0 += L.chunk) {
       const int nb = min(L.chunk, nbc - c0);
       const int nt_count = (nb + 7) / 8;
@@ -485,13 +469,11 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
             }
           }
         }
-        GRU_TRACE(t, 4);
         if (__syncthreads_or(!got)) {
           set_status(p.status, kStatusTimeout);
           ok = false;
           break;
         }
-        GRU_TRACE(t, 1);
         // ---- sum the eight k-range partials of every tile
         for (int e = tid; e < tiles * 128; e += kGruThreads) {
           const int tile = e / 128, w = e % 128;
@@ -501,10 +483,8 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
           const int mt = tile / nt_count, nt = tile % nt_count;
           gsm[static_cast<size_t>(mt * 16 + w / 8) * kGsmLd + nt * 8 + (w % 8)] = sum;
         }
-        GRU_TRACE(t, 5);
         __syncthreads();
       }
-      GRU_TRACE(t, 2);
       // ---- gates and the new state (torch.nn.GRU convention); publish the tagged state
 #pragma unroll
       for (int rr = 0; rr < kGatePairsPerThread; ++rr) {
@@ -531,7 +511,6 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
       }
       __syncthreads();
     }
-    GRU_TRACE(t, 3);
   }
   if (!ok || p.u == nullptr) return;
 
@@ -676,9 +655,3 @@ cudaError_t launch_u_finalize(const UFinalParams& p, cudaStream_t stream) {
 }
 
 }  // namespace dm
-
-#ifdef DOMINO_GRU_TRACE
-extern "C" __attribute__((visibility("default"))) int domino_debug_gru_trace(unsigned long long* out) {
-  return cudaMemcpyFromSymbol(out, dm::g_gru_trace, sizeof(dm::g_gru_trace)) == cudaSuccess ? 0 : -3;
-}
-#endif

@@ -60,6 +60,9 @@ SMALL = {
     # the GRU computes its own projections (three launches): H not a multiple of 64 (a short last
     # k chunk), 32 GRU CTAs, four u pairs per warp
     "fused-ragged": dict(B=2, K=7, H=328, V=5000, Ds=256, R=64, k=5, N=12, seed=19, biases=True),
+    # the largest k and N the boundary accepts: 32-entry lists, a 256-node tree (slots past 32
+    # live in shared memory), on a vocabulary with a ragged last chunk
+    "max-k-N": dict(B=2, K=8, H=128, V=3001, Ds=64, R=32, k=32, N=256, seed=20),
 }
 
 
