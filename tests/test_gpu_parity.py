@@ -63,6 +63,10 @@ SMALL = {
     # the largest k and N the boundary accepts: 32-entry lists, a 256-node tree (slots past 32
     # live in shared memory), on a vocabulary with a ragged last chunk
     "max-k-N": dict(B=2, K=8, H=128, V=3001, Ds=64, R=32, k=32, N=256, seed=20),
+    # the largest K (64 positions: the GRU's longest recurrence, the deepest tree rows)
+    "max-K": dict(B=1, K=64, H=64, V=800, Ds=32, R=16, k=3, N=40, seed=21, biases=True),
+    # the longest block the fused-projection GRU takes (M = 32)
+    "fused-K32": dict(B=1, K=32, H=128, V=1500, Ds=256, R=32, k=4, N=30, seed=22),
 }
 
 
