@@ -667,7 +667,7 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
     constexpr int kRows = WidePass<KB>::kRows, kGroup = WidePass<KB>::kGroup;
     const uint64_t pol_ab = l2_policy_evict_normal();
     const uint64_t pol_rest = l2_policy_evict_last();
-      unsigned nbar = 0;
+    unsigned nbar = 0;
     for (int j = 0; j < K; ++j) {
       const float* hprev = p.h + static_cast<size_t>((j + 1) & 1) * B * p.Ds;  // h_{j-1} (zeros at j = 0)
       float* hcur = p.h + static_cast<size_t>(j & 1) * B * p.Ds;
@@ -687,7 +687,7 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
 #pragma unroll
       for (int b = 0; b < KB; ++b)
 #pragma unroll
-        for (int e = 0; e < 8; ++e) ur[b][e] = (b < B && lane * 8 < R) ? s_u[b * R + lane * 8 + e] : 0.f;
+        for (int e = 0; e < 8; ++e) ur[b][e] = (b < B && lane * 8 < R) ? s_u[(b < B && lane * 8 < R) ? b * R + lane * 8 + e : 0] : 0.f;
       Lse mine = lse_empty();
       // rows read through L2 first (the longest latency): one group of rows per warp at a time
       for (int r0 = warp * kGroup; r0 < n_g; r0 += kRollWarps * kGroup) {
@@ -742,7 +742,10 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
 #pragma unroll
             for (int r = 0; r < kGroup; ++r)
               raw[r] = (r0 + g + r < n_s && lane * 8 < R)
-                           ? *reinterpret_cast<const uint4*>(s_w2 + static_cast<size_t>(r0 + g + r) * R + lane * 8)
+                           ? *reinterpret_cast<const uint4*>(
+                                 s_w2 + ((r0 + g + r < n_s && lane * 8 < R) ? static_cast<size_t>(r0 + g + r) * R +
+                                                                                   lane * 8
+                                                                             : 0))
                            : make_uint4(0, 0, 0, 0);
             group_fma<KB, kGroup>(raw, g, ur, dot);
           }
@@ -871,7 +874,7 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
 #pragma unroll
       for (int b = 0; b < KB; ++b)
 #pragma unroll
-        for (int e = 0; e < 8; ++e) ur[b][e] = (b < B && lane * 8 < R) ? s_u[b * R + lane * 8 + e] : 0.f;
+        for (int e = 0; e < 8; ++e) ur[b][e] = (b < B && lane * 8 < R) ? s_u[(b < B && lane * 8 < R) ? b * R + lane * 8 + e : 0] : 0.f;
       Lse mine = lse_empty();
       for (int i = 0; i < nch; ++i) {
         const long long g = static_cast<long long>(j) * nch + i;
