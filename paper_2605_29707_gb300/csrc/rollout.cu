@@ -209,8 +209,11 @@ __device__ __forceinline__ void block_reduce(Lse (&st)[NB], Lse (*red)[kRollMaxB
 
 // Grid barrier number `n` (0, 1, ...) of the compute warps: every CTA arrives once per barrier.
 // Returns false if the wait gave up or the CTA's abort flag is up (status set); the caller
-// then stops.
+// then stops.  Thread 0 alone reads the flag (which the feeding warp may raise at any time) and
+// hands its decision to the compute threads through s_go, so that they all return the same
+// value and leave together.
 __device__ bool grid_barrier(unsigned* ctr, unsigned n, int* status, volatile int* fail) {
+  __shared__ int s_go;
   compute_sync();
   if (threadIdx.x == 0) {
     // release at GPU scope: every write the CTA made before the barrier above is visible to a
@@ -229,9 +232,10 @@ __device__ bool grid_barrier(unsigned* ctr, unsigned n, int* status, volatile in
       }
       __nanosleep(32);
     }
+    s_go = *fail == 0;
   }
   compute_sync();
-  return *fail == 0;
+  return s_go != 0;
 }
 
 // ---- phase A: h_j = GRU(emb[t_j], h_{j-1}) (torch.nn.GRU: gates r|z|n, r multiplies
@@ -460,7 +464,7 @@ __device__ bool sample_step(const RolloutParams& p, int j, const float* s_logit,
       const float e = __expf(lg[r] - mx);
       if (e > 0.f) last = r;
       acc += e;
-      if (acc > T) { cand = r; break; }
+      if (e > 0.f && acc > T) { cand = r; break; }
     }
     if (cand != 0x7fffffff) atomicMin(&s_pick[b], cand);
     if (last >= 0) atomicMax(&s_last[b], last);
@@ -732,8 +736,9 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
         wide_push<KB>(dot, lane, n_t - row0, row0, r_lo + row0, s_base, s_b2, rows_cta, B, mine);
       }
       // rows in shared memory (landed before the first step's phase C)
-      if (j == 0 && n_s > 0) mbar_wait(&s_fill, 0, &s_fail, p.status);
-      if (!s_fail) {
+      bool filled = true;
+      if (j == 0 && n_s > 0) filled = mbar_wait(&s_fill, 0, &s_fail, p.status);
+      if (__all_sync(0xffffffffu, filled && !s_fail)) {  // warp-uniform: the passes shuffle
         for (int r0 = warp * kRows; r0 < n_s; r0 += kRollWarps * kRows) {
           float dot[32] = {};
 #pragma unroll
@@ -879,7 +884,8 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
       for (int i = 0; i < nch; ++i) {
         const long long g = static_cast<long long>(j) * nch + i;
         const int sidx = static_cast<int>(g % kW2Stages);
-        if (!mbar_wait(&s_full[sidx], static_cast<uint32_t>((g / kW2Stages) & 1), &s_fail, p.status)) break;
+        const bool landed = mbar_wait(&s_full[sidx], static_cast<uint32_t>((g / kW2Stages) & 1), &s_fail, p.status);
+        if (!__all_sync(0xffffffffu, landed)) break;  // warp-uniform: the passes shuffle
         const int c = c_lo + i;
         const int rows = min(ch, V - c * ch);
         const __nv_bfloat16* sw = reinterpret_cast<const __nv_bfloat16*>(s_ring + sidx * kW2StageBytes);
