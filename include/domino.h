@@ -39,7 +39,7 @@
 extern "C" {
 #endif
 
-#define DOMINO_ABI_VERSION 1
+#define DOMINO_ABI_VERSION 2
 
 #if defined(__GNUC__)
 #define DOMINO_API __attribute__((visibility("default")))
@@ -84,7 +84,26 @@ typedef struct domino_head_weights {
   const void* b2;
   int Ds;
   int R;
+  /* Optional fp32 [V, 3*Ds] input-projection table, table[t] = W_ih . emb[t] (no bias), made
+   * once per set of weights by domino_build_input_table; NULL = the GRU projects emb[t]
+   * itself.  Read by domino_rollout_greedy / domino_rollout_sample: a step's input-gate sums
+   * are then one row of it. */
+  const float* x_table;
 } domino_head_weights;
+
+/* Bytes of the input-projection table (V * 3 * Ds fp32 values); 0 for invalid sizes. */
+DOMINO_API size_t domino_input_table_bytes(int V, int Ds);
+
+/* table[t][g] = sum_h emb[t][h] * w_ih[g][h] for every token t < V and gate row g < 3*Ds: the
+ * GRU's input projection (section 4.1.2, encoder eq.; b_ih is not included) of every token,
+ * computed once on the tensor cores (fp32 accumulation).  emb bf16 [V, H], w_ih bf16 [3*Ds, H],
+ * table fp32 [V, 3*Ds] (domino_input_table_bytes), all device pointers, 16-byte aligned; H and
+ * Ds multiples of 8.  The table depends on emb and w_ih only: rebuild it when they change.
+ * Synchronises the stream; returns DOMINO_OK, DOMINO_ERR_INVALID_ARG / _UNSUPPORTED (nothing
+ * enqueued), DOMINO_ERR_CUDA or DOMINO_ERR_TIMEOUT (a device-side wait ran out: the table is
+ * not valid). */
+DOMINO_API int domino_build_input_table(const void* emb, const void* w_ih, int V, int H, int Ds, float* table,
+                                        void* stream);
 
 /* Bytes of device workspace domino_draft_step needs for these sizes on the current device
  * (the split of the work depends on the device's SM count).  Returns 0 when the sizes are
@@ -194,8 +213,11 @@ DOMINO_API int domino_verify_tree_greedy(const float* target_logits, const int32
  * Outputs (device): tokens int32 [B, K] = t_1 .. t_K; logp fp32 [B, K].
  * workspace: device memory of domino_rollout_workspace_bytes(...) bytes (16-byte aligned);
  * its first int32 receives the device status (DOMINO_OK, DOMINO_ERR_BAD_TOKEN,
- * DOMINO_ERR_TIMEOUT; domino_check_status reads it).  Two kernels on `stream` (a tensor-core
- * GEMM for W_lm hidden_j of every position, then one cooperative kernel for the K steps).
+ * DOMINO_ERR_TIMEOUT; domino_check_status reads it).  Two kernels on `stream`: a tensor-core
+ * GEMM for W_lm hidden_j of every position, then one cooperative kernel for the K steps (for
+ * r <= 256 it first computes W1[:, :H] hidden_j of every position, which does not depend on the
+ * recurrence).  With head->x_table set, a step's GRU input-gate sums are row t_j of that table
+ * instead of a product with emb[t_j].
  * Returns DOMINO_OK once enqueued, or a negative code with nothing enqueued. */
 DOMINO_API size_t domino_rollout_workspace_bytes(int B, int K, int H, int V, int Ds, int R);
 

@@ -25,7 +25,8 @@ SYMBOLS = ("domino_workspace_bytes", "domino_draft_step", "domino_workspace_byte
            "domino_draft_step_host", "domino_check_status", "domino_status_string",
            "domino_abi_version", "domino_launches_per_step", "domino_timing_begin", "domino_timing_end",
            "domino_draft_step_static_scratch", "domino_verify_tree_greedy", "domino_rollout_workspace_bytes",
-           "domino_rollout_greedy", "domino_rollout_sample")
+           "domino_rollout_greedy", "domino_rollout_sample", "domino_input_table_bytes",
+           "domino_build_input_table")
 
 DOMINO_STATIC_SCRATCH_BYTES = 16 << 20
 
@@ -36,7 +37,7 @@ KERNEL_KINDS = ("gather", "gru_input_proj", "w1_hidden_proj", "gru", "vocab_gemm
 class domino_head_weights(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in
                 ("emb", "w_ih", "w_hh", "b_ih", "b_hh", "w1", "b1", "w2", "b2")] + \
-               [("Ds", ctypes.c_int), ("R", ctypes.c_int)]
+               [("Ds", ctypes.c_int), ("R", ctypes.c_int), ("x_table", ctypes.c_void_p)]
 
 
 class DominoError(RuntimeError):
@@ -92,6 +93,10 @@ def load():
     lib.domino_rollout_sample.argtypes = [P, P, P, P, ctypes.POINTER(domino_head_weights)] + [I] * 4 + [
         P, P, P, ctypes.c_size_t, P]
     lib.domino_rollout_sample.restype = I
+    lib.domino_input_table_bytes.argtypes = [I, I]
+    lib.domino_input_table_bytes.restype = S
+    lib.domino_build_input_table.argtypes = [P, P, I, I, I, P, P]
+    lib.domino_build_input_table.restype = I
     _lib = lib
     return lib
 
@@ -117,9 +122,18 @@ def _stream(s):
 
 
 def make_head(emb=None, w_ih=None, w_hh=None, b_ih=None, b_hh=None, w1=None, b1=None, w2=None, b2=None,
-              Ds=0, R=0) -> domino_head_weights:
+              Ds=0, R=0, x_table=None) -> domino_head_weights:
     return domino_head_weights(_addr(emb), _addr(w_ih), _addr(w_hh), _addr(b_ih), _addr(b_hh), _addr(w1),
-                               _addr(b1), _addr(w2), _addr(b2), int(Ds), int(R))
+                               _addr(b1), _addr(w2), _addr(b2), int(Ds), int(R), _addr(x_table))
+
+
+def domino_input_table_bytes(V, Ds) -> int:
+    return int(load().domino_input_table_bytes(V, Ds))
+
+
+def domino_build_input_table(emb, w_ih, V, H, Ds, table, stream=None) -> int:
+    """table [V, 3 Ds] fp32 = emb . W_ih^T (device); synchronises the stream."""
+    return int(load().domino_build_input_table(_addr(emb), _addr(w_ih), V, H, Ds, _addr(table), _stream(stream)))
 
 
 def domino_workspace_bytes(B, K, H, V, Ds, R, k, N) -> int:

@@ -684,13 +684,65 @@ int domino_verify_tree_greedy(const float* target_logits, const int32_t* tree_pa
   return rc;
 }
 
+// ---------------------------------------------------------------- input-projection table
+namespace {
+__device__ int g_table_status;  // device status of domino_build_input_table's GEMM
+std::mutex g_table_mu;          // one build at a time uses it
+}  // namespace
+
+size_t domino_input_table_bytes(int V, int Ds) {
+  if (V <= 0 || Ds <= 0) return 0;
+  return static_cast<size_t>(V) * 3 * Ds * sizeof(float);
+}
+
+int domino_build_input_table(const void* emb, const void* w_ih, int V, int H, int Ds, float* table, void* stream) {
+  if (!emb || !w_ih || !table || V <= 0 || H <= 0 || Ds <= 0) return DOMINO_ERR_INVALID_ARG;
+  if (H % 8 != 0 || Ds % 8 != 0 || Ds > kMaxDs || V >= kMaxV) return DOMINO_ERR_UNSUPPORTED;
+  if (!aligned16(emb) || !aligned16(w_ih) || !aligned16(table)) return DOMINO_ERR_UNSUPPORTED;
+  int sms = 0, major = 0, minor = 0;
+  int rc = device_sms(&sms, &major, &minor);
+  if (rc != DOMINO_OK) return rc;
+  if (major != 10 || minor != 3) return DOMINO_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_table_mu);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int* status = nullptr;
+  if (cudaGetSymbolAddress(reinterpret_cast<void**>(&status), g_table_status) != cudaSuccess) return DOMINO_ERR_CUDA;
+  if (cudaMemsetAsync(status, 0, sizeof(int), st) != cudaSuccess) return DOMINO_ERR_CUDA;
+  // emb [V, H] . W_ih [3 Ds, H]^T, every token a GEMM row, one split (finished sums)
+  StorePlan g = plan_store(V, 3 * Ds, ceil_div(H, 64), sms);
+  g.splits = 1;
+  g.kb_per_split = g.nkb;
+  g.total_items = g.tok_tiles * g.w_tiles;
+  g.grid = g.total_items < sms ? g.total_items : sms;
+  CUtensorMap maps[4];
+  if (!gemm_maps(&maps[0], &maps[1], g.swap, g.bn, emb, V, H, H, w_ih, 3 * Ds, H)) return DOMINO_ERR_CUDA;
+  maps[2] = maps[0];
+  maps[3] = maps[1];
+  const dm::TcParams b0{};
+  TcParams tp = b0;
+  tp.nkb1 = g.nkb; tp.nkb2 = 0;
+  tp.rows_tok = V; tp.rows_w = 3 * Ds;
+  tp.tok_tiles = g.tok_tiles; tp.w_tiles = g.w_tiles;
+  tp.splits = 1; tp.kb_per_split = g.kb_per_split; tp.total_items = g.total_items;
+  tp.w_evict_first = 0;
+  tp.tmem_cols = pow2_at_least(2 * g.bn, 32);
+  tp.out = table; tp.ld_out = 3 * Ds;
+  tp.status = status;
+  rc = cuda_rc(dm::launch_tc_gemm(dm::kModeStore, g.bn, g.swap, 16, maps, tp, g.grid, st));
+  if (rc) return rc;
+  int h = 0;
+  if (cudaMemcpyAsync(&h, status, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess) return DOMINO_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return DOMINO_ERR_CUDA;
+  return h;
+}
+
 // ---------------------------------------------------------------- greedy rollout
 namespace {
 struct RollPlan {
   int B, K, H, V, Ds, R, M, grid;
   bool head;
   StorePlan g;  // base-logit GEMM, no split
-  size_t off_h, off_u, off_part, off_next, off_base, clear_bytes, total;
+  size_t off_h, off_u, off_part, off_next, off_base, off_uh, clear_bytes, total;
 };
 
 int make_roll_plan(int B, int K, int H, int V, int Ds, int R, bool head, RollPlan* P) {
@@ -729,6 +781,7 @@ int make_roll_plan(int B, int K, int H, int V, int Ds, int R, bool head, RollPla
   p.off_part = take(static_cast<size_t>(p.grid) * dm::kRollMaxB * 16);
   p.off_next = take(dm::kRollMaxB * 4);  // sampled mode: t_{j+1} of every sequence
   p.off_base = take(static_cast<size_t>(p.M) * V * 4);
+  p.off_uh = take(static_cast<size_t>(p.M) * (p.R > 0 ? p.R : 1) * 4);  // hidden . W1[:, :H]^T
   p.total = off;
   return DOMINO_OK;
 }
@@ -795,6 +848,8 @@ int rollout_entry(const void* hidden, const int32_t* anchors, const float* unifo
     rp.w1 = static_cast<const __nv_bfloat16*>(head->w1);
     rp.b1 = static_cast<const __nv_bfloat16*>(head->b1);
     rp.w2 = static_cast<const __nv_bfloat16*>(head->w2);
+    rp.x_table = head->x_table;
+    rp.uh = reinterpret_cast<float*>(ws + P.off_uh);
   }
   rp.b2 = head ? static_cast<const __nv_bfloat16*>(head->b2) : nullptr;
   rp.head = hd ? 1 : 0;

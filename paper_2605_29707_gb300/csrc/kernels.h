@@ -171,6 +171,8 @@ struct RolloutParams {
   int* status;
   const float* uniforms;        // [B, K] in [0, 1): sampled mode; nullptr: greedy
   int32_t* next_tok;            // [kRollMaxB] sampled mode: t_{j+1}, written by the CTA holding it
+  const float* x_table;         // [V, 3 Ds] emb . W_ih^T, or nullptr (phase A projects emb[t] itself)
+  float* uh;                    // [B*K][R] scratch for hidden . W1[:, :H]^T (resident kernel), or nullptr
 };
 // dynamic shared memory of one rollout CTA (the resident W2 rows or the W2 ring, u of every
 // sequence and this CTA's rows of base logits + b2): at most kRollMaxSmem, the 227 KB a CTA may

@@ -239,7 +239,8 @@ __device__ bool grid_barrier(unsigned* ctr, unsigned n, int* status, volatile in
 }
 
 // ---- phase A: h_j = GRU(emb[t_j], h_{j-1}) (torch.nn.GRU: gates r|z|n, r multiplies
-//      W_hn h + b_hn), one warp per hidden unit q, every sequence
+//      W_hn h + b_hn), one warp per hidden unit q, every sequence.  With an input-projection
+//      table the three input-gate sums W_i{r,z,n} emb[t_j] are entries of row t_j of it.
 __device__ __forceinline__ void gru_phase(const RolloutParams& p, const int* s_tok, const float* hprev, float* hcur,
                                           int gw, int nwarps, int lane, uint64_t pol) {
   const int B = p.B, H = p.H, Ds = p.Ds;
@@ -247,18 +248,27 @@ __device__ __forceinline__ void gru_phase(const RolloutParams& p, const int* s_t
     for (int b = 0; b < B; ++b) {
       const __nv_bfloat16* x = p.emb + static_cast<size_t>(s_tok[b]) * H;
       float ar = 0.f, az = 0.f, an = 0.f, hr = 0.f, hz = 0.f, hn = 0.f;
+      if (p.x_table) {
+        if (lane == 0) {  // summed over the warp below with the other lanes' zeros
+          const float* xt = p.x_table + static_cast<size_t>(s_tok[b]) * 3 * Ds;
+          ar = __ldg(xt + q);
+          az = __ldg(xt + Ds + q);
+          an = __ldg(xt + 2 * Ds + q);
+        }
+      } else {
 #pragma unroll 4
-      for (int c = lane * 8; c < H; c += 256) {
-        float xv[8], wr[8], wz[8], wn[8];
-        bf8(x + c, xv);
-        bf8_hint(p.w_ih + static_cast<size_t>(q) * H + c, wr, pol);
-        bf8_hint(p.w_ih + static_cast<size_t>(Ds + q) * H + c, wz, pol);
-        bf8_hint(p.w_ih + static_cast<size_t>(2 * Ds + q) * H + c, wn, pol);
+        for (int c = lane * 8; c < H; c += 256) {
+          float xv[8], wr[8], wz[8], wn[8];
+          bf8(x + c, xv);
+          bf8_hint(p.w_ih + static_cast<size_t>(q) * H + c, wr, pol);
+          bf8_hint(p.w_ih + static_cast<size_t>(Ds + q) * H + c, wz, pol);
+          bf8_hint(p.w_ih + static_cast<size_t>(2 * Ds + q) * H + c, wn, pol);
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          ar += wr[e] * xv[e];
-          az += wz[e] * xv[e];
-          an += wn[e] * xv[e];
+          for (int e = 0; e < 8; ++e) {
+            ar += wr[e] * xv[e];
+            az += wz[e] * xv[e];
+            an += wn[e] * xv[e];
+          }
         }
       }
       const float* hp = hprev + static_cast<size_t>(b) * Ds;
@@ -295,7 +305,46 @@ __device__ __forceinline__ void gru_phase(const RolloutParams& p, const int* s_t
   }
 }
 
-// ---- phase B: u_j = SiLU(W1 [hidden_j ; h_j] + b1), one warp per rank row q, every sequence
+// ---- before the steps (resident kernel): uh[m][q] = W1[q, :H] . hidden_m for every position m
+//      = b K + j and rank row q, the half of u's argument that does not depend on the
+//      recurrence.  Warp w takes row q = w % R and the positions m = w / R, w / R + G, ...
+//      (G = max(1, warps / R)), four at a time, so a W1 row is read once per four positions.
+__device__ void uh_prologue(const RolloutParams& p, int gw, int nwarps, int lane, uint64_t pol) {
+  const int H = p.H, Ds = p.Ds, R = p.R, M = p.B * p.K;
+  const int groups = max(1, nwarps / R);
+  for (int pi = gw; pi < R * groups; pi += nwarps) {
+    const int q = pi % R, mg = pi / R;
+    const __nv_bfloat16* w = p.w1 + static_cast<size_t>(q) * (H + Ds);
+    for (int m0 = mg; m0 < M; m0 += 4 * groups) {
+      float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 2
+      for (int c = lane * 8; c < H; c += 256) {
+        float wv[8];
+        bf8_hint(w + c, wv, pol);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int m = m0 + i * groups;
+          if (m < M) {
+            float xv[8];
+            bf8(p.hidden + static_cast<size_t>(m) * H + c, xv);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) acc[i] += wv[e] * xv[e];
+          }
+        }
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int m = m0 + i * groups;
+        const float a = warp_sum(acc[i]);
+        if (lane == 0 && m < M) p.uh[static_cast<size_t>(m) * R + q] = a;
+      }
+    }
+  }
+}
+
+// ---- phase B: u_j = SiLU(W1 [hidden_j ; h_j] + b1), one warp per rank row q, every sequence.
+//      With uh computed before the steps the warp adds uh[b K + j][q] instead of the 4096-long
+//      hidden half of the dot.
 __device__ __forceinline__ void u_phase(const RolloutParams& p, int j, const float* hcur, int gw, int nwarps,
                                         int lane, uint64_t pol) {
   const int B = p.B, K = p.K, H = p.H, Ds = p.Ds, R = p.R;
@@ -305,13 +354,18 @@ __device__ __forceinline__ void u_phase(const RolloutParams& p, int j, const flo
       const __nv_bfloat16* hid = p.hidden + (static_cast<size_t>(b) * K + j) * H;
       const float* hc = hcur + static_cast<size_t>(b) * Ds;
       float acc = 0.f;
+      if (p.uh) {
+        // written before the steps by other CTAs of this launch (ordered by the grid barriers)
+        if (lane == 0) acc = __ldcg(p.uh + (static_cast<size_t>(b) * K + j) * R + q);
+      } else {
 #pragma unroll 4
-      for (int c = lane * 8; c < H; c += 256) {
-        float wv[8], xv[8];
-        bf8_hint(w + c, wv, pol);
-        bf8(hid + c, xv);
+        for (int c = lane * 8; c < H; c += 256) {
+          float wv[8], xv[8];
+          bf8_hint(w + c, wv, pol);
+          bf8(hid + c, xv);
 #pragma unroll
-        for (int e = 0; e < 8; ++e) acc += wv[e] * xv[e];
+          for (int e = 0; e < 8; ++e) acc += wv[e] * xv[e];
+        }
       }
 #pragma unroll 4
       for (int c = lane * 8; c < Ds; c += 256) {
@@ -641,6 +695,8 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
       }
     }
     fill_issued = true;
+    // ---- u's hidden halves while the bulk copies land (read by phase B after a grid barrier)
+    if (p.uh) uh_prologue(p, gw, nwarps, lane, l2_policy_evict_normal());
     // ---- fill: tensor-memory rows.  Warp w writes lane quarter q = w % 4, rows 64 (w / 4) ..
     //      64 (w / 4) + 63 of the quarter's 128, 4 rows (16 columns) per store.
     const int q = warp & 3, half = warp >> 2;
@@ -993,6 +1049,7 @@ cudaError_t launch_rollout(const RolloutParams& p, int grid, cudaStream_t stream
   if (smem > kRollMaxSmem) return cudaErrorInvalidValue;
   RolloutParams pp = p;
   pp.smem_rows = use_resident(p) ? resident_smem_rows(p.B, p.V, p.R, grid) : 0;
+  if (!use_resident(p)) pp.uh = nullptr;  // only the resident kernel computes it before its steps
   if (p.B <= 1) return launch_rollout_kb<1>(pp, grid, smem, stream);
   if (p.B <= 2) return launch_rollout_kb<2>(pp, grid, smem, stream);
   if (p.B <= 4) return launch_rollout_kb<4>(pp, grid, smem, stream);

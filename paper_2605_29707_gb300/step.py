@@ -17,7 +17,7 @@ def _dev_bf16(a, device):
 
 class DraftStep:
     def __init__(self, weights: dict, B: int, K: int, H: int, V: int, k: int, N: int, Ds: int = 1024,
-                 R: int = 256, device="cuda", head_on: bool = True):
+                 R: int = 256, device="cuda", head_on: bool = True, input_table: bool = False):
         self.B, self.K, self.H, self.V, self.k, self.N = B, K, H, V, k, N
         self.device = torch.device(device)
         self.head_on = head_on and R > 0 and weights.get("w2") is not None
@@ -29,6 +29,17 @@ class DraftStep:
         self.head = B_.make_head(w.get("emb"), w.get("w_ih"), w.get("w_hh"), w.get("b_ih"), w.get("b_hh"),
                                  w.get("w1"), w.get("b1"), w.get("w2") if self.head_on else None, w.get("b2"),
                                  self.Ds, self.R)
+        # optional input-projection table emb . W_ih^T [V, 3 Ds] fp32, built once on the device
+        # (read by the rollout entry points)
+        self.x_table = None
+        if input_table and self.head_on:
+            self.x_table = torch.empty(B_.domino_input_table_bytes(V, self.Ds) // 4, dtype=torch.float32,
+                                       device=dev)
+            rc = B_.domino_build_input_table(w["emb"], w["w_ih"], V, H, self.Ds, self.x_table,
+                                             torch.cuda.current_stream(dev))
+            if rc != B_.DOMINO_OK:
+                raise B_.DominoError(rc, "domino_build_input_table")
+            self.head.x_table = self.x_table.data_ptr()
         self.ws_bytes = B_.domino_workspace_bytes(B, K, H, V, self.Ds, self.R, k, N)
         if self.ws_bytes == 0:
             raise B_.DominoError(B_.DOMINO_ERR_UNSUPPORTED, "domino_workspace_bytes")

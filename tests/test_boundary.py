@@ -33,7 +33,7 @@ def test_library_loads_and_exports_every_declared_symbol():
     lib = _lib()
     for name in declared_entry_points():
         assert hasattr(lib, name), name
-    assert binding.domino_abi_version() == 1
+    assert binding.domino_abi_version() == 2
 
 
 def test_status_strings():
@@ -59,6 +59,22 @@ def test_null_pointers_rejected_before_any_cuda_call():
     rc = binding.domino_draft_step(None, None, None, None, 1, 4, 64, 100, 2, 3, None, None, None, None, None,
                                    None, None, 0)
     assert rc == binding.DOMINO_ERR_INVALID_ARG
+
+
+def test_input_table_size_and_argument_checks():
+    """The input-projection table is V x 3 Ds fp32; NULL pointers and bad sizes are refused
+    before any device query."""
+    _lib()
+    assert binding.domino_input_table_bytes(151936, 1024) == 151936 * 3 * 1024 * 4
+    assert binding.domino_input_table_bytes(0, 1024) == 0
+    assert binding.domino_input_table_bytes(10, 0) == 0
+    bad = binding.DOMINO_ERR_INVALID_ARG
+    assert binding.domino_build_input_table(None, None, 10, 8, 8, None) == bad
+    one = 16  # a non-null stand-in; never dereferenced because validation fails first
+    assert binding.domino_build_input_table(one, one, 0, 8, 8, one) == bad
+    assert binding.domino_build_input_table(one, one, 10, 8, -8, one) == bad
+    assert binding.domino_build_input_table(one, one, 10, 12, 8, one) == binding.DOMINO_ERR_UNSUPPORTED
+    assert binding.domino_build_input_table(one, one, 10, 8, 4096, one) == binding.DOMINO_ERR_UNSUPPORTED
 
 
 def test_launch_count_query():

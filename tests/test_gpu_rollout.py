@@ -10,6 +10,8 @@ log-probability within 2e-2; and up to the first such near-tie the GPU tokens mu
 oracle rollout's exactly.
 """
 import ctypes
+import dataclasses
+import functools
 
 import numpy as np
 import pytest
@@ -24,20 +26,44 @@ LOGP_TOL = 2e-2
 GAP = 4e-2
 
 
-def _device_weights(wl, dev, head_on=True):
+def _full_emb(wl):
+    """The workload with every embedding row drawn.  The generator leaves the rows no prefix id
+    names at zero, but a rollout feeds back tokens of its own choosing, so here every row is
+    live and every step's GRU input is a real embedding."""
+    c = wl.cfg
+    w = dict(wl.weights)
+    w["emb"] = inputs.normal_bf16((c.V, c.H), (c.seed, "emb-all"))
+    return dataclasses.replace(wl, weights=w)
+
+
+@functools.lru_cache(maxsize=2)
+def _full_size(name):
+    return _full_emb(inputs.cached_workload(name))
+
+
+def _device_weights(wl, dev, head_on=True, table=False):
+    """Device weights and the head struct; table=True also builds the input-projection table
+    (kept alive in w["x_table"]) and points the head at it."""
     w = {n: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(dev)
          for n, a in wl.weights.items() if a is not None}
     c = wl.cfg
+    x_table = None
+    if table:
+        x_table = torch.empty(binding.domino_input_table_bytes(c.V, c.Ds) // 4, dtype=torch.float32, device=dev)
+        rc = binding.domino_build_input_table(w["emb"], w["w_ih"], c.V, c.H, c.Ds, x_table,
+                                              torch.cuda.current_stream(dev))
+        assert rc == 0, binding.domino_status_string(rc)
+        w["x_table"] = x_table
     head = binding.make_head(w.get("emb"), w.get("w_ih"), w.get("w_hh"), w.get("b_ih"), w.get("b_hh"), w.get("w1"),
                              w.get("b1"), w.get("w2") if head_on else None, w.get("b2"), c.Ds if head_on else 0,
-                             c.R if head_on else 0)
+                             c.R if head_on else 0, x_table)
     return w, head
 
 
-def _run_gpu(wl, head_on=True):
+def _run_gpu(wl, head_on=True, table=False):
     c = wl.cfg
     dev = torch.device("cuda:0")
-    w, head = _device_weights(wl, dev, head_on)
+    w, head = _device_weights(wl, dev, head_on, table)
     hidden = torch.from_numpy(wl.hidden.view(np.int16)).view(torch.bfloat16).to(dev)
     anchors = torch.from_numpy(np.ascontiguousarray(wl.prefix_ids[:, 0])).to(dev)
     nbytes = binding.domino_rollout_workspace_bytes(c.B, c.K, c.H, c.V, c.Ds if head_on else 0, c.R if head_on else 0)
@@ -53,10 +79,10 @@ def _run_gpu(wl, head_on=True):
     return tokens.cpu().numpy(), logp.cpu().numpy()
 
 
-def _check(wl, head_on=True):
+def _check(wl, head_on=True, table=False):
     c = wl.cfg
     w = wl.weights if head_on else {"w_lm": wl.weights["w_lm"], "b2": wl.weights.get("b2")}
-    tokens, logp = _run_gpu(wl, head_on)
+    tokens, logp = _run_gpu(wl, head_on, table)
     anchors = np.ascontiguousarray(wl.prefix_ids[:, 0]).astype(np.int32)
     o_tok, _ = oracle.rollout_greedy(w, wl.hidden, anchors)
     excused = 0
@@ -94,7 +120,18 @@ def _check(wl, head_on=True):
     inputs.custom_config("roll-tiers-b1", B=1, K=4, H=256, V=160003, Ds=32, R=256, seed=28, biases=True),
 ])
 def test_rollout_matches_oracle(cfg):
-    _check(inputs.make_workload(cfg))
+    _check(_full_emb(inputs.make_workload(cfg)))
+
+
+@pytest.mark.parametrize("cfg", [
+    inputs.CONFIGS["tiny"],
+    inputs.custom_config("roll-b3", B=3, K=8, H=512, V=3000, Ds=64, R=64, seed=21, biases=True),
+    inputs.custom_config("roll-wide", B=2, K=4, H=256, V=2500, Ds=32, R=512, seed=26, biases=True),
+    inputs.custom_config("roll-tiers-b1", B=1, K=4, H=256, V=160003, Ds=32, R=256, seed=28, biases=True),
+])
+def test_rollout_with_input_table_matches_oracle(cfg):
+    """Phase A's input-gate sums read from the table emb . W_ih^T: the same rollout."""
+    _check(_full_emb(inputs.make_workload(cfg)), table=True)
 
 
 def test_rollout_head_off():
@@ -123,17 +160,58 @@ def test_rollout_rejects_bad_anchor_and_sizes():
 
 @pytest.mark.parametrize("name", ["qwen3-8b", "qwen3-1.7b"])
 def test_rollout_full_size(name):
-    _check(inputs.cached_workload(name))
+    _check(_full_size(name))
+
+
+def test_rollout_full_size_with_input_table():
+    _check(_full_size("qwen3-8b"), table=True)
+
+
+# ---------------------------------------------------------------------------- input table
+def _table_case(wl, rows):
+    """GPU table rows against the fp64 product of the same bf16 values, within the fp32
+    summation bound gamma_H = H u / (1 - H u) (u = 2^-24) times sum_h |emb[t, h] W_ih[g, h]|
+    (bf16 x bf16 products are exact in fp32)."""
+    c = wl.cfg
+    dev = torch.device("cuda:0")
+    w, _ = _device_weights(wl, dev, True, table=True)
+    tab = w["x_table"].view(c.V, 3 * c.Ds)
+    got = tab[torch.from_numpy(rows).to(dev).long()].cpu().numpy().astype(np.float64)
+    emb = inputs.bf16_bits_to_f32(wl.weights["emb"][rows]).numpy().astype(np.float64)
+    wih = inputs.bf16_bits_to_f32(wl.weights["w_ih"]).numpy().astype(np.float64)
+    ref = emb @ wih.T
+    mag = np.abs(emb) @ np.abs(wih).T
+    u = 2.0 ** -24
+    gamma = c.H * u / (1 - c.H * u)
+    err = np.abs(got - ref)
+    assert (err <= gamma * mag + 1e-30).all(), float((err - gamma * mag).max())
+
+
+@pytest.mark.parametrize("cfg", [
+    # a ragged last 128-token tile and 3 Ds = 72 gate rows (a ragged 256-row tile)
+    inputs.custom_config("tab-ragged", B=1, K=2, H=256, V=1000, Ds=24, R=8, seed=41),
+    inputs.custom_config("tab-mid", B=1, K=2, H=512, V=3001, Ds=64, R=16, seed=42, biases=True),
+])
+def test_input_table_matches_product(cfg):
+    wl = _full_emb(inputs.make_workload(cfg))
+    _table_case(wl, np.arange(cfg.V, dtype=np.int64))
+
+
+def test_input_table_full_size_sampled_rows():
+    wl = _full_size("qwen3-8b")
+    rows = np.unique(np.concatenate([[0, 1, wl.cfg.V - 1],
+                                     np.random.default_rng(3).integers(0, wl.cfg.V, 61)])).astype(np.int64)
+    _table_case(wl, rows)
 
 
 # ---------------------------------------------------------------------------- sampled loop
 CDF_TOL = 5e-3  # fp32 logits and sums on the GPU against fp64: how far u may sit past a boundary
 
 
-def _run_gpu_sample(wl, uniforms, head_on=True):
+def _run_gpu_sample(wl, uniforms, head_on=True, table=False):
     c = wl.cfg
     dev = torch.device("cuda:0")
-    w, head = _device_weights(wl, dev, head_on)
+    w, head = _device_weights(wl, dev, head_on, table)
     hidden = torch.from_numpy(wl.hidden.view(np.int16)).view(torch.bfloat16).to(dev)
     anchors = torch.from_numpy(np.ascontiguousarray(wl.prefix_ids[:, 0])).to(dev)
     uni = torch.from_numpy(uniforms).to(dev)
@@ -149,7 +227,7 @@ def _run_gpu_sample(wl, uniforms, head_on=True):
     return tokens.cpu().numpy(), logp.cpu().numpy()
 
 
-def _check_sample(wl, head_on=True, seed=5):
+def _check_sample(wl, head_on=True, seed=5, table=False):
     """Teacher-forced: every GPU token's cumulative-probability interval (under the oracle's step
     fed the GPU's own tokens) holds its uniform within CDF_TOL, with logp within LOGP_TOL; up to
     the first uniform within CDF_TOL of one of the oracle rollout's boundaries, the tokens equal
@@ -157,7 +235,7 @@ def _check_sample(wl, head_on=True, seed=5):
     c = wl.cfg
     w = wl.weights if head_on else {"w_lm": wl.weights["w_lm"], "b2": wl.weights.get("b2")}
     uni = np.random.default_rng(seed).random((c.B, c.K), dtype=np.float32)
-    tokens, logp = _run_gpu_sample(wl, uni, head_on)
+    tokens, logp = _run_gpu_sample(wl, uni, head_on, table)
     anchors = np.ascontiguousarray(wl.prefix_ids[:, 0]).astype(np.int32)
     o_tok, _ = oracle.rollout_sample(w, wl.hidden, anchors, uni)
     excused = 0
@@ -193,7 +271,15 @@ def _check_sample(wl, head_on=True, seed=5):
     inputs.custom_config("samp-tiers", B=8, K=3, H=256, V=167001, Ds=32, R=256, seed=34),
 ])
 def test_rollout_sample_matches_oracle(cfg):
-    _check_sample(inputs.make_workload(cfg))
+    _check_sample(_full_emb(inputs.make_workload(cfg)))
+
+
+@pytest.mark.parametrize("cfg", [
+    inputs.custom_config("samp-b3", B=3, K=8, H=512, V=3000, Ds=64, R=64, seed=31, biases=True),
+    inputs.custom_config("samp-tiers", B=8, K=3, H=256, V=167001, Ds=32, R=256, seed=34),
+])
+def test_rollout_sample_with_input_table_matches_oracle(cfg):
+    _check_sample(_full_emb(inputs.make_workload(cfg)), table=True)
 
 
 def test_rollout_sample_head_off():
@@ -203,7 +289,7 @@ def test_rollout_sample_head_off():
 
 @pytest.mark.parametrize("name", ["qwen3-8b"])
 def test_rollout_sample_full_size(name):
-    _check_sample(inputs.cached_workload(name), seed=7)
+    _check_sample(_full_size(name), seed=7)
 
 
 def test_rollout_sample_uniform_ends_and_bad_pointer():
