@@ -569,6 +569,18 @@ def run_ours(args):
                          "note": "head off = W_lm projection + softmax/top-k + tree only (R = 0)"}
         del st_off
 
+    # ---- the same step with the input-projection table emb . W_ih^T (built once, outside the
+    #      timed region): the GRU reads its input-gate sums as table rows instead of projecting
+    #      the embedding rows (no X GEMM at larger B)
+    input_table = None
+    if st.head_on:
+        st_tab = DraftStep(st.w, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=device, input_table=True)
+        us_tab = time_steps(st_tab, hidden, ids, stream, min(args.steps, 1000), args.warmup)
+        input_table = {"us_per_step": round(us_tab, 2), "launches_per_step": st_tab.launches_per_step(),
+                       "table_bytes": st_tab.x_table.numel() * 4,
+                       "note": "the same step reading the GRU's input-gate sums from the table; value is the step without it"}
+        del st_tab
+
     # ---- the step after the draft: greedy verification of this step's trees against synthetic
     #      target logits [B, N+1, V] fp32 (timing only; parity is in the tests)
     verify = verify_timing(st, c, device, stream) if c.B <= 4 else None
@@ -606,7 +618,8 @@ def run_ours(args):
         "e2e": {"value": round(e2e_value, 3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "steps": n_e2e, "api": "domino_draft_step_host (synchronous per step)"},
         "gpu_launches": args.steps * launches, "clocks": clocks,
-        "head_overhead": head_overhead, "tree_verify": verify, "rollout_greedy": rollout,
+        "head_overhead": head_overhead, "input_table_step": input_table, "tree_verify": verify,
+        "rollout_greedy": rollout,
     }
     # ---- last: the same step replayed from a CUDA graph (one captured step, replayed back to
     #      back); a failed capture is reported in the line, after everything else was measured

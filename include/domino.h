@@ -86,8 +86,9 @@ typedef struct domino_head_weights {
   int R;
   /* Optional fp32 [V, 3*Ds] input-projection table, table[t] = W_ih . emb[t] (no bias), made
    * once per set of weights by domino_build_input_table; NULL = the GRU projects emb[t]
-   * itself.  Read by domino_rollout_greedy / domino_rollout_sample: a step's input-gate sums
-   * are then one row of it. */
+   * itself.  When set, every entry point takes the GRU's input-gate sums from it (one row per
+   * token) instead of projecting the embedding rows: the block step then launches no X GEMM
+   * (domino_launches_per_step_table) and the rollout's steps read one row each. */
   const float* x_table;
 } domino_head_weights;
 
@@ -172,6 +173,9 @@ DOMINO_API int domino_abi_version(void);
  * own projections (B <= 2 at K = 16), 6 for other batches of at most 128 positions, 7 above;
  * a negative code for sizes domino_draft_step would reject. */
 DOMINO_API int domino_launches_per_step(int B, int K, int H, int V, int Ds, int R, int k, int N);
+/* The same count for a head that carries an input-projection table (head->x_table): one launch
+ * fewer wherever domino_launches_per_step counts an X GEMM (5 instead of 6, 6 instead of 7). */
+DOMINO_API int domino_launches_per_step_table(int B, int K, int H, int V, int Ds, int R, int k, int N);
 
 /* Greedy verification of draft trees against the target model's logits: the step after the
  * draft.  Section 3.1: the target evaluates the draft in one pass and accepts the longest valid

@@ -26,7 +26,7 @@ SYMBOLS = ("domino_workspace_bytes", "domino_draft_step", "domino_workspace_byte
            "domino_abi_version", "domino_launches_per_step", "domino_timing_begin", "domino_timing_end",
            "domino_draft_step_static_scratch", "domino_verify_tree_greedy", "domino_rollout_workspace_bytes",
            "domino_rollout_greedy", "domino_rollout_sample", "domino_input_table_bytes",
-           "domino_build_input_table")
+           "domino_build_input_table", "domino_launches_per_step_table")
 
 DOMINO_STATIC_SCRATCH_BYTES = 16 << 20
 
@@ -76,6 +76,8 @@ def load():
     lib.domino_abi_version.restype = I
     lib.domino_launches_per_step.argtypes = [I] * 8
     lib.domino_launches_per_step.restype = I
+    lib.domino_launches_per_step_table.argtypes = [I] * 8
+    lib.domino_launches_per_step_table.restype = I
     lib.domino_timing_begin.argtypes = [I]
     lib.domino_timing_begin.restype = I
     lib.domino_timing_end.argtypes = [P, P, I]
@@ -177,6 +179,10 @@ def domino_abi_version() -> int:
 
 def domino_launches_per_step(B, K, H, V, Ds, R, k, N) -> int:
     return int(load().domino_launches_per_step(B, K, H, V, Ds, R, k, N))
+
+
+def domino_launches_per_step_table(B, K, H, V, Ds, R, k, N) -> int:
+    return int(load().domino_launches_per_step_table(B, K, H, V, Ds, R, k, N))
 
 
 def domino_timing_begin(max_launches: int) -> int:

@@ -344,7 +344,9 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
   if (P.clear_bytes && cudaMemsetAsync(ws + P.off_ctrl, 0, P.clear_bytes, st) != cudaSuccess) return DOMINO_ERR_CUDA;
   uint32_t* epoch = reinterpret_cast<uint32_t*>(ws + P.off_ctrl + 128);
 
-  __nv_bfloat16* E = P.head ? reinterpret_cast<__nv_bfloat16*>(ws + P.off_E) : nullptr;
+  // an input-projection table replaces the gathered embeddings and the X GEMM
+  const float* x_table = P.head ? hw->x_table : nullptr;
+  __nv_bfloat16* E = (P.head && !x_table) ? reinterpret_cast<__nv_bfloat16*>(ws + P.off_E) : nullptr;
   uint32_t* hx = P.head ? reinterpret_cast<uint32_t*>(ws + P.off_hx) : nullptr;
   int ts = -1, rc = DOMINO_OK;
   if (!P.fused) {
@@ -361,7 +363,7 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
     float* upart = reinterpret_cast<float*>(ws + P.off_upart);
     u = reinterpret_cast<__nv_bfloat16*>(ws + P.off_u);
     // X partials: E [M, H] . W_ih [3Ds, H]^T
-    if (!P.fused) {
+    if (!P.fused && !x_table) {
       const dm::TcParams base{};
       TcParams tp = base;
       const StorePlan& g = P.xg;
@@ -409,7 +411,8 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
       tp.out = upart; tp.ld_out = R;
       tp.status = status;
       const bool chained = P.chain && !both;
-      tp.pdl_wait = chained ? 2 : 0;  // reads nothing the X GEMM writes; completes after it
+      tp.pdl_wait = chained ? 2 : 0;  // reads nothing the kernel before it (X GEMM or gather)
+                                      // writes; completes after it
       const int slot = timing_open(DOMINO_KERNEL_W1_HIDDEN, st);
       const int r = cuda_rc(chained ? dm::launch_tc_store_chained(g.bn, maps, tp, g.grid, st)
                                     : dm::launch_tc_gemm(dm::kModeStore, g.bn, g.swap, 16, maps, tp, g.grid, st));
@@ -438,6 +441,9 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
     gr.epoch = epoch;
     gr.seq_done = seq_done;
     gr.reset_ctrl = P.fused ? 1 : 0;
+    gr.V = V;
+    gr.x_table = x_table;
+    gr.x_ids = ids;
     if (P.fused) {
       gr.ids = ids;
       gr.emb = static_cast<const __nv_bfloat16*>(hw->emb);
@@ -900,6 +906,13 @@ int domino_launches_per_step(int B, int K, int H, int V, int Ds, int R, int k, i
   // GRU, W1 GEMM, u finalize, vocab GEMM, merge + tree
   if (P.fused) return 3;
   return P.u_in_gru ? 6 : 7;
+}
+
+int domino_launches_per_step_table(int B, int K, int H, int V, int Ds, int R, int k, int N) {
+  const int n = domino_launches_per_step(B, K, H, V, Ds, R, k, N);
+  if (n < 0 || R <= 0) return n;
+  // the table replaces the X GEMM (the fused path has none)
+  return n == 3 ? 3 : n - 1;
 }
 
 }  // extern "C"

@@ -178,6 +178,7 @@ __device__ __forceinline__ void ldg_words8(const __nv_bfloat16* row, int k0, int
 // 16 t .. 16 t + 15 of its A rows (g, g + 8) and B row (g), and MMA step s of the chunk takes
 // words 2 s and 2 s + 1 of those, the same columns in A and B.  The warps split k; their partial
 // tiles meet in `red` (one 16 x 8 tile per warp at a time).
+template <bool kTable>
 __device__ void fused_projections(const GruParams& p, int j0, int Uc, int b0, int nbc, float* red,
                                   float (*s_uh)[kGruMaxUPairs]) {
   const int H = p.H, Ds = p.Ds, K = p.K, R = p.R, M = p.B * p.K;
@@ -201,7 +202,7 @@ __device__ void fused_projections(const GruParams& p, int j0, int Uc, int b0, in
     bvalid[nt] = g < Uc;
     brow[nt] = p.w_ih + static_cast<size_t>(nt * Ds + j0 + (g < Uc ? g : 0)) * H;
   }
-  for (int mt = 0; mt * 16 < rows; ++mt) {
+  for (int mt = 0; !kTable && mt * 16 < rows; ++mt) {  // with a table the steps read its rows
     const int ra = mt * 16 + g, rb = ra + 8;
     const int ida = ra < rows ? p.ids[b0 * K + ra] : 0, idb = rb < rows ? p.ids[b0 * K + rb] : 0;
     const bool va = ra < rows && ida >= 0 && ida < p.V, vb = rb < rows && idb >= 0 && idb < p.V;
@@ -280,6 +281,9 @@ __device__ void fused_projections(const GruParams& p, int j0, int Uc, int b0, in
 
 // At most 128 registers per thread (two CTAs' worth per SM), so that a GRU CTA and a vocabulary
 // GEMM CTA (at most 168 registers x 192 threads) fit in one SM's register file.
+// kTable: the input-gate sums come from the input-projection table (p.x_table) rather than
+// from xs (a separate instantiation, so that the path without a table keeps its registers).
+template <bool kTable>
 __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) {
   extern __shared__ __align__(16) uint8_t gsmem[];
   const int U = p.units, Ds = p.Ds, K = p.K, B = p.B, R = p.R, H = p.H;
@@ -330,7 +334,7 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
   for (int e = tid; e < L.chunk * (ldw / 8); e += kGruThreads) reinterpret_cast<uint4*>(hsm)[e] = make_uint4(0, 0, 0, 0);
   __shared__ float s_uh[kGruWarps][kGruMaxUPairs];  // fused: hidden halves of this warp's u pairs
   if (p.ids != nullptr) {
-    fused_projections(p, j0, Uc, b0, nbc, red, s_uh);
+    fused_projections<kTable>(p, j0, Uc, b0, nbc, red, s_uh);
   } else {
   // Launched as a programmatic dependent of the projection GEMMs: everything below reads
   // what they (and, through their own waits, the gather) wrote -- X partials, u partials and
@@ -338,7 +342,7 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
   asm volatile("griddepcontrol.wait;" ::: "memory");
   // ---- input-gate sums b_ih + E . W_ih^T for this CTA's rows and units, spread over all
   //      threads (made visible to the CTA by the barrier below)
-  const int xs_count = nbc * K * 3 * Uc;
+  const int xs_count = kTable ? 0 : nbc * K * 3 * Uc;  // with a table the steps read its rows
   for (int e0 = tid; e0 < xs_count; e0 += 4 * kGruThreads) {
     float a[4];
     size_t at[4];
@@ -387,10 +391,18 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
           const int bb = e / Uc, jl = e % Uc;
           const int j = j0 + jl;
           const size_t m = static_cast<size_t>(b0 + c0 + bb) * K + t;
-          const float* x = p.xs + m * 3 * Ds;
+          // b_ih + W_i{r,z,n} E_m: summed into xs before the steps, or a row of the table (an id
+          // outside [0, V), reported by the id check, reads row 0)
+          const float* x = p.xs + m * 3 * Ds;  // written by this kernel: plain loads
+          const __nv_bfloat16* xbias = nullptr;
+          if (kTable) {
+            const int id = p.x_ids[m];
+            x = p.x_table + static_cast<size_t>(id >= 0 && id < p.V ? id : 0) * 3 * Ds;
+            xbias = p.b_ih;
+          }
 #pragma unroll
           for (int g = 0; g < 3; ++g) {
-            gx[r][g] = x[g * Ds + j];
+            gx[r][g] = x[g * Ds + j] + bf_or0(xbias, g * Ds + j);
             gb[r][g] = bf_or0(p.b_hh, g * Ds + j);
           }
         }
@@ -598,14 +610,14 @@ GruPlan gru_plan(int B, int Ds, int num_sms) {
   return g;
 }
 
-cudaError_t launch_gru(const GruParams& p, const GruPlan& plan, cudaStream_t stream, bool pdl) {
-  if (plan.smem == 0) return cudaErrorInvalidValue;
+template <bool kTable>
+static cudaError_t launch_gru_t(const GruParams& p, const GruPlan& plan, cudaStream_t stream, bool pdl) {
   static size_t attr_smem = 0;
   if (plan.smem > attr_smem) {
-    cudaError_t e = cudaFuncSetAttribute(gru_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(gru_kernel<kTable>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(plan.smem));
     if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(gru_kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    e = cudaFuncSetAttribute(gru_kernel<kTable>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
     if (e != cudaSuccess) return e;
     attr_smem = plan.smem;
   }
@@ -623,15 +635,20 @@ cudaError_t launch_gru(const GruParams& p, const GruPlan& plan, cudaStream_t str
   // A runtime that refuses the pair gets the cooperative launch alone from then on.
   static bool pdl_refused = false;
   cfg.numAttrs = (pdl && !pdl_refused) ? 2 : 1;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, gru_kernel, p);
+  cudaError_t e = cudaLaunchKernelEx(&cfg, gru_kernel<kTable>, p);
   if (e != cudaSuccess && cfg.numAttrs == 2) {
     (void)cudaGetLastError();
     pdl_refused = true;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, gru_kernel, p);
+    e = cudaLaunchKernelEx(&cfg, gru_kernel<kTable>, p);
   }
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
+}
+
+cudaError_t launch_gru(const GruParams& p, const GruPlan& plan, cudaStream_t stream, bool pdl) {
+  if (plan.smem == 0) return cudaErrorInvalidValue;
+  return p.x_table ? launch_gru_t<true>(p, plan, stream, pdl) : launch_gru_t<false>(p, plan, stream, pdl);
 }
 
 // ---------------------------------------------------------------------------- u finalize

@@ -112,6 +112,11 @@ struct GruParams {
   const uint32_t* epoch;      // the workspace's step epoch (the state words' tag)
   unsigned int* seq_done;     // [B] merge counters
   int reset_ctrl;             // no clear before the launch: CTA 0 resets the status and seq_done
+  // Input-projection table emb . W_ih^T [V, 3*Ds] fp32, or nullptr: when set, each step reads
+  // its input-gate sums as b_ih + row x_ids[m] of it, and xpart / xs / the fused path's own
+  // product are not used.
+  const float* x_table;
+  const int32_t* x_ids;       // [M] the prefix ids (read with x_table)
 };
 // Largest number of (rank row, position) pairs of u one warp finalises for which the fused
 // projections apply (their hidden halves wait in shared memory).

@@ -30,7 +30,7 @@ class DraftStep:
                                  w.get("w1"), w.get("b1"), w.get("w2") if self.head_on else None, w.get("b2"),
                                  self.Ds, self.R)
         # optional input-projection table emb . W_ih^T [V, 3 Ds] fp32, built once on the device
-        # (read by the rollout entry points)
+        # (every entry point then reads the GRU's input-gate sums from it)
         self.x_table = None
         if input_table and self.head_on:
             self.x_table = torch.empty(B_.domino_input_table_bytes(V, self.Ds) // 4, dtype=torch.float32,
@@ -55,7 +55,8 @@ class DraftStep:
         self.tree_score = torch.empty(B * N, dtype=torch.float32, device=dev)
 
     def launches_per_step(self) -> int:
-        return B_.domino_launches_per_step(self.B, self.K, self.H, self.V, self.Ds, self.R, self.k, self.N)
+        f = B_.domino_launches_per_step_table if self.x_table is not None else B_.domino_launches_per_step
+        return f(self.B, self.K, self.H, self.V, self.Ds, self.R, self.k, self.N)
 
     def enqueue(self, hidden: torch.Tensor, prefix_ids: torch.Tensor, stream=None) -> int:
         """Enqueue one step on `stream` (default: torch's current stream); returns the C status."""

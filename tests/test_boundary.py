@@ -87,6 +87,12 @@ def test_launch_count_query():
     assert binding.domino_launches_per_step(32, 16, 4096, 151936, 1024, 256, 8, 16) == 7
     assert binding.domino_launches_per_step(1, 16, 4096, 151936, 0, 0, 8, 16) == 3
     assert binding.domino_launches_per_step(0, 16, 4096, 151936, 1024, 256, 8, 16) < 0
+    # with an input-projection table the X GEMM is not launched
+    assert binding.domino_launches_per_step_table(1, 16, 4096, 151936, 1024, 256, 8, 16) == 3
+    assert binding.domino_launches_per_step_table(4, 16, 4096, 151936, 1024, 256, 8, 16) == 5
+    assert binding.domino_launches_per_step_table(32, 16, 4096, 151936, 1024, 256, 8, 16) == 6
+    assert binding.domino_launches_per_step_table(1, 16, 4096, 151936, 0, 0, 8, 16) == 3
+    assert binding.domino_launches_per_step_table(0, 16, 4096, 151936, 1024, 256, 8, 16) < 0
 
 
 def test_verify_rejects_bad_arguments_before_launch():

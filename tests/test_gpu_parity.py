@@ -22,9 +22,10 @@ def _dev():
     return torch.device("cuda:0")
 
 
-def _run_gpu(wl, head_on=True):
+def _run_gpu(wl, head_on=True, table=False):
     c = wl.cfg
-    st = DraftStep(wl.weights, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=_dev(), head_on=head_on)
+    st = DraftStep(wl.weights, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=_dev(), head_on=head_on,
+                   input_table=table)
     hidden = torch.from_numpy(wl.hidden.view(np.int16)).view(torch.bfloat16).to(_dev())
     ids = torch.from_numpy(wl.prefix_ids).to(_dev())
     out = st.run(hidden, ids)
@@ -79,6 +80,57 @@ def test_small_parity(name):
     # gap-excused differences are allowed but must stay rare on these inputs
     assert ex_topk <= max(1, cfg.M * cfg.k // 50)
     assert ex_tree <= max(1, cfg.B * cfg.N // 10)
+
+
+# the input-projection table in place of the GRU's own E . W_ih^T: the fused path (B <= 2), the
+# chained small-M path, the large-M path, K = 1
+TABLE = ["tiny", "ragged-swap16", "swap64", "normal-2tiles", "normal-ragged", "K1", "fused-ragged", "fused-K32"]
+
+
+@pytest.mark.parametrize("name", TABLE)
+def test_small_parity_with_input_table(name):
+    cfg = inputs.CONFIGS["tiny"] if name == "tiny" else inputs.custom_config(name, **SMALL[name])
+    wl = inputs.make_workload(cfg)
+    _, out, _, _ = _run_gpu(wl, table=True)
+    ex_topk, ex_tree, _ = _check(wl, out)
+    assert ex_topk <= max(1, cfg.M * cfg.k // 50)
+    assert ex_tree <= max(1, cfg.B * cfg.N // 10)
+
+
+@pytest.mark.parametrize("name,table", [("fused-ragged", False), ("fused-ragged", True), ("swap64", False),
+                                        ("swap64", True), ("normal-2tiles", False), ("normal-2tiles", True)])
+def test_launches_per_step_counts_the_kernels(name, table):
+    """The kernels one step launches (the library's per-launch timing hooks) are as many as
+    domino_launches_per_step (_table with an input table) says."""
+    cfg = inputs.custom_config(name, **SMALL[name])
+    wl = inputs.make_workload(cfg)
+    st, _, hidden, ids = _run_gpu(wl, table=table)
+    binding.domino_timing_begin(64)
+    assert st.enqueue(hidden, ids) == 0
+    torch.cuda.synchronize()
+    launched = sum(n for _, n in binding.domino_timing_end().values())
+    assert launched == st.launches_per_step()
+    if table:
+        c = wl.cfg
+        plain = binding.domino_launches_per_step(c.B, c.K, c.H, c.V, c.Ds, c.R, c.k, c.N)
+        assert launched == (3 if plain == 3 else plain - 1)
+
+
+def test_bad_token_reported_with_input_table():
+    """Without the X GEMM an out-of-range id is still reported (the gather's check), and the GRU
+    reads a valid table row for it."""
+    wl = inputs.make_workload(inputs.custom_config("bad-t", B=4, K=16, H=64, V=500, Ds=32, R=16, k=2, N=3, seed=25))
+    c = wl.cfg
+    st = DraftStep(wl.weights, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=_dev(), input_table=True)
+    assert st.launches_per_step() == 5
+    hidden = torch.from_numpy(wl.hidden.view(np.int16)).view(torch.bfloat16).to(_dev())
+    ids = torch.from_numpy(wl.prefix_ids).to(_dev())
+    ids[1, 3] = -2
+    assert st.enqueue(hidden, ids) == 0
+    assert binding.domino_check_status(st.workspace, torch.cuda.current_stream()) == binding.DOMINO_ERR_BAD_TOKEN
+    ids[1, 3] = 7
+    assert st.enqueue(hidden, ids) == 0
+    assert binding.domino_check_status(st.workspace, torch.cuda.current_stream()) == 0
 
 
 def test_correction_off_is_base_distribution():
@@ -172,11 +224,11 @@ FULL = ["qwen3-1.7b", "qwen3-8b", "qwen3-8b-b32", "qwen3-32b-b64"]
 
 
 @pytest.mark.slow
-@pytest.mark.parametrize("name", FULL)
-def test_full_size_parity(name):
+@pytest.mark.parametrize("name,table", [(n, False) for n in FULL] + [("qwen3-8b", True), ("qwen3-8b-b32", True)])
+def test_full_size_parity(name, table):
     wl = inputs.cached_workload(name)
     c = wl.cfg
-    _, out, _, _ = _run_gpu(wl)
+    _, out, _, _ = _run_gpu(wl, table=table)
     seqs = list(range(c.B)) if c.B <= 2 else [0, c.B - 1]
     ex_topk, ex_tree, _ = _check(wl, out, seqs=seqs)
     assert ex_topk <= max(1, len(seqs) * c.K * c.k // 20)
