@@ -232,7 +232,8 @@ DOMINO_API size_t domino_rollout_workspace_bytes(int B, int K, int H, int V, int
  * order, exceeds u (computed in fp32: where u falls within rounding of a boundary either
  * neighbour may be chosen); logp_j = log-softmax(L_j)[t_{j+1}].  Arguments, outputs, workspace
  * (domino_rollout_workspace_bytes) and errors as domino_rollout_greedy; uniforms NULL or not
- * 4-byte aligned: DOMINO_ERR_INVALID_ARG.  One grid barrier per step more than the greedy loop. */
+ * 4-byte aligned: DOMINO_ERR_INVALID_ARG.  The same grid barriers per step as the greedy loop: every
+ * CTA reads the final logits of the CTA whose rows hold the draw and scans them itself. */
 DOMINO_API int domino_rollout_sample(const void* hidden, const int32_t* anchors, const float* uniforms,
                                      const void* w_lm, const domino_head_weights* head, int B, int K, int H,
                                      int V, int32_t* tokens, float* logp, void* workspace,

@@ -748,7 +748,7 @@ struct RollPlan {
   int B, K, H, V, Ds, R, M, grid;
   bool head;
   StorePlan g;  // base-logit GEMM, no split
-  size_t off_h, off_u, off_part, off_next, off_base, off_uh, clear_bytes, total;
+  size_t off_h, off_u, off_part, off_lg, off_base, off_uh, clear_bytes, total;
 };
 
 int make_roll_plan(int B, int K, int H, int V, int Ds, int R, bool head, RollPlan* P) {
@@ -784,8 +784,8 @@ int make_roll_plan(int B, int K, int H, int V, int Ds, int R, bool head, RollPla
   p.off_h = take(static_cast<size_t>(2) * B * (p.Ds > 0 ? p.Ds : 1) * 4);
   p.clear_bytes = off;
   p.off_u = take(static_cast<size_t>(B) * (p.R > 0 ? p.R : 1) * 4);
-  p.off_part = take(static_cast<size_t>(p.grid) * dm::kRollMaxB * 16);
-  p.off_next = take(dm::kRollMaxB * 4);  // sampled mode: t_{j+1} of every sequence
+  p.off_part = take(static_cast<size_t>(2) * p.grid * dm::kRollMaxB * 16);  // two, by step parity
+  p.off_lg = take(static_cast<size_t>(2) * B * V * 4);  // sampled mode: final logits, by step parity
   p.off_base = take(static_cast<size_t>(p.M) * V * 4);
   p.off_uh = take(static_cast<size_t>(p.M) * (p.R > 0 ? p.R : 1) * 4);  // hidden . W1[:, :H]^T
   p.total = off;
@@ -869,7 +869,7 @@ int rollout_entry(const void* hidden, const int32_t* anchors, const float* unifo
   rp.logp = logp;
   rp.status = status;
   rp.uniforms = uniforms;
-  rp.next_tok = reinterpret_cast<int32_t*>(ws + P.off_next);
+  rp.lg = reinterpret_cast<float*>(ws + P.off_lg);
   const int ts = timing_open(DOMINO_KERNEL_ROLLOUT, st);
   rc = cuda_rc(dm::launch_rollout(rp, P.grid, st));
   timing_close(ts, st);

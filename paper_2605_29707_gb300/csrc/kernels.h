@@ -169,13 +169,13 @@ struct RolloutParams {
   const float* base;            // [B*K, V] W_lm hidden (fp32, from the store-mode GEMM)
   float* h;                     // [2][B][Ds] GRU states (cleared: h_{-1} = 0)
   float* u;                     // [B][R]
-  float* partials;              // [grid][kRollMaxB] float4 (max, sum exp, argmax bits, 0)
+  float* partials;              // [2][grid][kRollMaxB] float4 (max, sum exp, argmax bits, 0), by step parity
   unsigned* barrier;            // grid barrier counter (cleared)
   int32_t* tokens;              // [B, K] t_1 .. t_K
   float* logp;                  // [B, K]
   int* status;
   const float* uniforms;        // [B, K] in [0, 1): sampled mode; nullptr: greedy
-  int32_t* next_tok;            // [kRollMaxB] sampled mode: t_{j+1}, written by the CTA holding it
+  float* lg;                    // [2][B][V] sampled mode: every CTA's final logits, by step parity
   const float* x_table;         // [V, 3 Ds] emb . W_ih^T, or nullptr (phase A projects emb[t] itself)
   float* uh;                    // [B*K][R] scratch for hidden . W1[:, :H]^T (resident kernel), or nullptr
 };

@@ -144,6 +144,27 @@ __host__ __device__ inline int rollout_rows_per_cta(int V, int R, int head, int 
   const int nchunk_all = (V + ch - 1) / ch;
   return ((nchunk_all + grid - 1) / grid) * ch;
 }
+// The resident kernel's slices: ceil(V / grid) consecutive rows per CTA.
+__host__ __device__ inline int resident_rows_per_cta(int V, int grid) { return (V + grid - 1) / grid; }
+
+// Rows [lo, lo + n) of CTA c: the resident kernel's equal slices, or the streamed kernel's run
+// of whole W2 chunks (the same split the kernels take for themselves).
+__device__ __forceinline__ void cta_rows(const RolloutParams& p, int c, bool resident, int& lo, int& n) {
+  const int V = p.V, grid = static_cast<int>(gridDim.x);
+  if (resident) {
+    const int rows = resident_rows_per_cta(V, grid);
+    lo = min(V, c * rows);
+    n = min(V, lo + rows) - lo;
+  } else {
+    const int ch = rollout_chunk_rows(p.R, p.head);
+    const int nall = (V + ch - 1) / ch;
+    const int cpc = (nall + grid - 1) / grid;
+    const int c_lo = min(nall, c * cpc);
+    const int nch = min(nall, c_lo + cpc) - c_lo;
+    lo = c_lo * ch;
+    n = max(0, min(V, (c_lo + nch) * ch) - lo);
+  }
+}
 
 // Running (max, sum of exp relative to max, argmax) of a stream of logits.
 struct Lse {
@@ -435,16 +456,17 @@ __device__ __forceinline__ void pass_push(const float (&dot)[kRowsPerPass * KB],
 // The end of a step, shared by both kernels: per-CTA partials, grid barrier, every CTA's
 // combine (thread c loads CTA c's partials, then the same block reduction in every CTA, so all
 // reach the same t_{j+1}), the outputs.  Returns false if the barrier gave up.
-// Sampled mode, after the combine (a_all[b]: the merged state of sequence b in every CTA):
-// t_{j+1} = the first id whose cumulative probability in id order exceeds u_{b,j}.  The CTAs'
-// masses w_c = s_c exp(m_c - max) are scanned in CTA order (their slices are consecutive), which
-// names the CTA holding the crossing; that CTA scans its own rows' final logits in id order,
-// writes the token and its log-probability, and one more grid barrier hands the token to all.
-// (If rounding leaves the crossing past its rows, it takes its last row of non-zero mass.)
+// Sampled mode, after the combine (s_max / s_lz: the merged max and log-sum of every sequence,
+// the same in every CTA): t_{j+1} = the first id whose cumulative probability in id order
+// exceeds u_{b,j}.  The CTAs' masses w_c = s_c exp(m_c - max) are scanned in CTA order (their
+// slices are consecutive), which names the CTA whose rows hold the crossing; every CTA then
+// reads that CTA's final logits (copied to global memory before the partials' barrier) and
+// scans them in id order the same way, so every CTA reaches the same token with no further
+// barrier.  (If rounding leaves the crossing past those rows, the last row of non-zero mass.)
 template <int KB>
-__device__ bool sample_step(const RolloutParams& p, int j, const float* s_logit, int r_lo, int r_n, int rows_cta,
-                            int* s_tok, unsigned& nbar, volatile int* s_fail, const float* s_max,
-                            const float* s_lz) {
+__device__ void sample_step(const RolloutParams& p, int j, const float4* part, const float* lg_all,
+                            float* s_stage, int rows_cta, int* s_tok, const float* s_max, const float* s_lz,
+                            bool resident) {
   __shared__ float s_T[kRollMaxB], s_off[kRollMaxB];
   __shared__ int s_owner[kRollMaxB], s_pick[kRollMaxB], s_last[kRollMaxB];
   __shared__ float s_wsum[kRollWarps][kRollMaxB];
@@ -457,7 +479,7 @@ __device__ bool sample_step(const RolloutParams& p, int j, const float* s_logit,
   for (int b = 0; b < KB; ++b) {
     w[b] = 0.f;
     if (b < B && tid < grid) {
-      const float4 f = __ldcg(reinterpret_cast<const float4*>(p.partials) + static_cast<size_t>(tid) * kRollMaxB + b);
+      const float4 f = __ldcg(part + static_cast<size_t>(tid) * kRollMaxB + b);
       w[b] = f.x == -INFINITY ? 0.f : f.y * __expf(f.x - s_max[b]);
     }
     incl[b] = w[b];
@@ -493,11 +515,15 @@ __device__ bool sample_step(const RolloutParams& p, int j, const float* s_logit,
   for (int b = 0; b < B; ++b) {
     // no claim (no mass anywhere: non-finite logits) falls to CTA 0 and its first row
     const int owner = s_owner[b] >= 0 ? s_owner[b] : 0;
-    if (owner != static_cast<int>(blockIdx.x)) continue;  // the same test in every thread
+    int o_lo, o_n;
+    cta_rows(p, owner, resident, o_lo, o_n);
     const float mx = s_max[b], T = s_T[b];
-    const float* lg = s_logit + b * rows_cta;
-    const int per = (r_n + kRollThreads - 1) / kRollThreads;
-    const int q0 = min(r_n, tid * per), q1 = min(r_n, q0 + per);
+    float* lg = s_stage + b * rows_cta;  // o_n <= rows_cta: the slices differ only at the tail
+    for (int r = tid; r < o_n; r += kRollThreads) lg[r] = __ldcg(lg_all + static_cast<size_t>(b) * p.V + o_lo + r);
+    const int per = (o_n + kRollThreads - 1) / kRollThreads;
+    const int q0 = min(o_n, tid * per), q1 = min(o_n, q0 + per);
+    if (tid == 0) { s_pick[b] = 0x7fffffff; s_last[b] = -1; }
+    compute_sync();
     float loc = 0.f;
     for (int r = q0; r < q1; ++r) loc += __expf(lg[r] - mx);
     // exclusive scan of the threads' sums (thread order = row order)
@@ -507,7 +533,6 @@ __device__ bool sample_step(const RolloutParams& p, int j, const float* s_logit,
       const float t = __shfl_up_sync(0xffffffffu, inc, o);
       if (lane >= o) inc += t;
     }
-    if (tid == 0) { s_pick[b] = 0x7fffffff; s_last[b] = -1; }
     if (lane == 31) s_wsum[warp][b] = inc;
     compute_sync();
     float off = s_off[b];
@@ -525,38 +550,51 @@ __device__ bool sample_step(const RolloutParams& p, int j, const float* s_logit,
     compute_sync();
     if (tid == 0) {
       const int r = s_pick[b] != 0x7fffffff ? s_pick[b] : max(0, s_last[b]);
-      const int tok = r_lo + r;
-      p.tokens[static_cast<size_t>(b) * K + j] = tok;
-      p.logp[static_cast<size_t>(b) * K + j] = lg[r] - mx - s_lz[b];
-      p.next_tok[b] = tok;
+      const int tok = o_lo + r;
+      s_tok[b] = tok;
+      if (blockIdx.x == 0) {
+        p.tokens[static_cast<size_t>(b) * K + j] = tok;
+        p.logp[static_cast<size_t>(b) * K + j] = lg[r] - mx - s_lz[b];
+      }
     }
   }
-  if (!grid_barrier(p.barrier, nbar++, p.status, s_fail)) return false;
-  if (tid < B) s_tok[tid] = __ldcg(p.next_tok + tid);
   compute_sync();
-  return true;
 }
 
+// End of step j: this CTA's (max, sum exp, argmax) per sequence go to the partials, every CTA
+// combines all of them after a grid barrier, and picks t_{j+1} (argmax, or sampled).  The
+// partials and (sampled mode) the final-logit copies alternate between two buffers by step
+// parity: a CTA writes step j + 2's only after every CTA has passed step j + 1's barrier, so
+// after every read of step j's (with the correction branch off no other barrier separates
+// consecutive steps).
 template <int KB>
 __device__ __forceinline__ bool finish_step(const RolloutParams& p, int j, Lse (&st)[KB], Lse (*s_red)[kRollMaxB],
-                                            int* s_tok, unsigned& nbar, volatile int* s_fail, const float* s_logit,
-                                            int r_lo, int r_n, int rows_cta) {
-  const int B = p.B, K = p.K, tid = threadIdx.x;
-  block_reduce(st, s_red, B);
+                                            int* s_tok, unsigned& nbar, volatile int* s_fail, float* s_logit,
+                                            int r_lo, int r_n, int rows_cta, bool resident) {
+  const int B = p.B, K = p.K, V = p.V, tid = threadIdx.x;
+  const int grid = static_cast<int>(gridDim.x);
+  float4* part = reinterpret_cast<float4*>(p.partials) + static_cast<size_t>(j & 1) * grid * kRollMaxB;
+  block_reduce(st, s_red, B);  // ends with a barrier: every row's final logit is in s_logit
   if (tid < B) {
     Lse a = s_red[0][tid];
     for (int w = 1; w < kRollWarps; ++w) lse_merge(a, s_red[w][tid]);
-    float4* out = reinterpret_cast<float4*>(p.partials) + static_cast<size_t>(blockIdx.x) * kRollMaxB + tid;
-    *out = make_float4(a.m, a.s, __int_as_float(a.i), 0.f);
+    part[static_cast<size_t>(blockIdx.x) * kRollMaxB + tid] = make_float4(a.m, a.s, __int_as_float(a.i), 0.f);
+  }
+  float* lg = p.lg ? p.lg + static_cast<size_t>(j & 1) * B * V : nullptr;
+  if (p.uniforms) {  // this CTA's final logits, which the CTA holding the draw's crossing is read from
+    for (int e = tid; e < B * r_n; e += kRollThreads) {
+      const int b = e / r_n, r = e - b * r_n;
+      lg[static_cast<size_t>(b) * V + r_lo + r] = s_logit[b * rows_cta + r];
+    }
   }
   if (!grid_barrier(p.barrier, nbar++, p.status, s_fail)) return false;
 #pragma unroll
   for (int b = 0; b < KB; ++b) st[b] = lse_empty();
-  for (int c = tid; c < static_cast<int>(gridDim.x); c += kRollThreads) {
+  for (int c = tid; c < grid; c += kRollThreads) {
 #pragma unroll
     for (int b = 0; b < KB; ++b) {
       if (b < B) {
-        const float4 f = __ldcg(reinterpret_cast<const float4*>(p.partials) + static_cast<size_t>(c) * kRollMaxB + b);
+        const float4 f = __ldcg(part + static_cast<size_t>(c) * kRollMaxB + b);
         Lse t;
         t.m = f.x; t.s = f.y; t.i = __float_as_int(f.z);
         lse_merge(st[b], t);
@@ -573,7 +611,8 @@ __device__ __forceinline__ bool finish_step(const RolloutParams& p, int j, Lse (
       s_glz[tid] = logf(a.s);
     }
     compute_sync();
-    return sample_step<KB>(p, j, s_logit, r_lo, r_n, rows_cta, s_tok, nbar, s_fail, s_gmax, s_glz);
+    sample_step<KB>(p, j, part, lg, s_logit, rows_cta, s_tok, s_gmax, s_glz, resident);
+    return true;
   }
   if (tid < B) {
     Lse a = s_red[0][tid];
@@ -637,7 +676,6 @@ __device__ __forceinline__ void wide_push(const float (&dot)[32], int lane, int 
 }
 
 // ================================================================ resident kernel (r <= 256)
-__host__ __device__ inline int resident_rows_per_cta(int V, int grid) { return (V + grid - 1) / grid; }
 
 template <int KB>
 __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const RolloutParams p) {
@@ -816,7 +854,7 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
       Lse st[KB];
 #pragma unroll
       for (int b = 0; b < KB; ++b) st[b] = (b == lane % KB) ? mine : lse_empty();
-      if (!finish_step<KB>(p, j, st, s_red, s_tok, nbar, &s_fail, s_base, r_lo, r_n, rows_cta)) break;
+      if (!finish_step<KB>(p, j, st, s_red, s_tok, nbar, &s_fail, s_base, r_lo, r_n, rows_cta, true)) break;
     }
   }
   // ---- teardown: the asynchronous copies have landed (the fill: bounded), tensor memory is
@@ -986,7 +1024,7 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
           if (b < B) lse_push(st[b], s_base[b * rows_cta + r], r_lo + r);
       }
     }
-    if (!finish_step<KB>(p, j, st, s_red, s_tok, nbar, &s_fail, s_base, r_lo, r_n, rows_cta)) return;
+    if (!finish_step<KB>(p, j, st, s_red, s_tok, nbar, &s_fail, s_base, r_lo, r_n, rows_cta, false)) return;
   }
 }
 
@@ -1044,7 +1082,7 @@ static cudaError_t launch_rollout_kb(const RolloutParams& p, int grid, size_t sm
 
 cudaError_t launch_rollout(const RolloutParams& p, int grid, cudaStream_t stream) {
   if (p.B < 1 || p.B > kRollMaxB || grid < 1) return cudaErrorInvalidValue;
-  if (p.uniforms && (grid > kRollThreads || !p.next_tok)) return cudaErrorInvalidValue;  // one thread per CTA
+  if (p.uniforms && (grid > kRollThreads || !p.lg)) return cudaErrorInvalidValue;  // one thread per CTA
   const size_t smem = rollout_smem_bytes(p.B, p.V, p.R, p.head, grid);
   if (smem > kRollMaxSmem) return cudaErrorInvalidValue;
   RolloutParams pp = p;
