@@ -464,7 +464,7 @@ __device__ __forceinline__ void pass_push(const float (&dot)[kRowsPerPass * KB],
 // scans them in id order the same way, so every CTA reaches the same token with no further
 // barrier.  (If rounding leaves the crossing past those rows, the last row of non-zero mass.)
 template <int KB>
-__device__ void sample_step(const RolloutParams& p, int j, const float4* part, const float* lg_all,
+__device__ void sample_step(const RolloutParams& p, int j, const float4 (&mine)[KB], const float* lg_all,
                             float* s_stage, int rows_cta, int* s_tok, const float* s_max, const float* s_lz,
                             bool resident) {
   __shared__ float s_T[kRollMaxB], s_off[kRollMaxB];
@@ -473,13 +473,14 @@ __device__ void sample_step(const RolloutParams& p, int j, const float4* part, c
   const int B = p.B, K = p.K, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int grid = static_cast<int>(gridDim.x);  // <= kRollThreads (checked at launch)
   if (tid < kRollMaxB) { s_owner[tid] = -1; s_off[tid] = 0.f; s_T[tid] = 0.f; }
-  // per-CTA masses (thread c: CTA c) and their inclusive scan in CTA order
+  // per-CTA masses (thread c: CTA c, whose partial the combine loaded into `mine`) and their
+  // inclusive scan in CTA order
   float incl[KB], w[KB];
 #pragma unroll
   for (int b = 0; b < KB; ++b) {
     w[b] = 0.f;
     if (b < B && tid < grid) {
-      const float4 f = __ldcg(part + static_cast<size_t>(tid) * kRollMaxB + b);
+      const float4 f = mine[b];
       w[b] = f.x == -INFINITY ? 0.f : f.y * __expf(f.x - s_max[b]);
     }
     incl[b] = w[b];
@@ -581,20 +582,25 @@ __device__ __forceinline__ bool finish_step(const RolloutParams& p, int j, Lse (
     part[static_cast<size_t>(blockIdx.x) * kRollMaxB + tid] = make_float4(a.m, a.s, __int_as_float(a.i), 0.f);
   }
   float* lg = p.lg ? p.lg + static_cast<size_t>(j & 1) * B * V : nullptr;
-  if (p.uniforms) {  // this CTA's final logits, which the CTA holding the draw's crossing is read from
+  if (p.uniforms && !resident) {  // this CTA's final logits (the resident kernel wrote them in phase C)
     for (int e = tid; e < B * r_n; e += kRollThreads) {
       const int b = e / r_n, r = e - b * r_n;
       lg[static_cast<size_t>(b) * V + r_lo + r] = s_logit[b * rows_cta + r];
     }
   }
   if (!grid_barrier(p.barrier, nbar++, p.status, s_fail)) return false;
+  float4 mine[KB];  // sampled mode: CTA tid's partials (grid <= kRollThreads there)
 #pragma unroll
-  for (int b = 0; b < KB; ++b) st[b] = lse_empty();
+  for (int b = 0; b < KB; ++b) {
+    st[b] = lse_empty();
+    mine[b] = make_float4(-INFINITY, 0.f, 0.f, 0.f);
+  }
   for (int c = tid; c < grid; c += kRollThreads) {
 #pragma unroll
     for (int b = 0; b < KB; ++b) {
       if (b < B) {
         const float4 f = __ldcg(part + static_cast<size_t>(c) * kRollMaxB + b);
+        if (c == tid) mine[b] = f;
         Lse t;
         t.m = f.x; t.s = f.y; t.i = __float_as_int(f.z);
         lse_merge(st[b], t);
@@ -611,7 +617,7 @@ __device__ __forceinline__ bool finish_step(const RolloutParams& p, int j, Lse (
       s_glz[tid] = logf(a.s);
     }
     compute_sync();
-    sample_step<KB>(p, j, part, lg, s_logit, rows_cta, s_tok, s_gmax, s_glz, resident);
+    sample_step<KB>(p, j, mine, lg, s_logit, rows_cta, s_tok, s_gmax, s_glz, resident);
     return true;
   }
   if (tid < B) {
@@ -662,15 +668,19 @@ __device__ __forceinline__ void group_fma(const uint4 (&raw)[G], int r_in_pass, 
   }
 }
 
+// After the reduce-scatter each lane holds one finished dot product: the logit of its row and
+// sequence is pushed into the lane's running (max, sum, argmax).  glg (sampled mode): the
+// step's [B, V] buffer of final logits, which every CTA reads the draw's CTA's rows from;
+// nullptr in greedy mode.
 template <int KB>
 __device__ __forceinline__ void wide_push(const float (&dot)[32], int lane, int nvalid, int row0, int vid0,
-                                          float* s_base, const float* s_b2, int rows_cta, int B, Lse& mine) {
+                                          const float* s_base, const float* s_b2, int rows_cta, int B, Lse& mine,
+                                          float* glg, int V) {
   const float d = ReduceScatter<32, 16>::run(dot);
   const int r = lane / KB, b = lane % KB;
   if (r < nvalid && b < B) {
-    float* x = s_base + b * rows_cta + row0 + r;
-    const float logit = *x + s_b2[row0 + r] + d;
-    *x = logit;  // the final logit, for the sampled mode's scan of this CTA's rows
+    const float logit = s_base[b * rows_cta + row0 + r] + s_b2[row0 + r] + d;
+    if (glg) glg[static_cast<size_t>(b) * V + vid0 + r] = logit;
     lse_push(mine, logit, vid0 + r);
   }
 }
@@ -787,6 +797,7 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
 #pragma unroll
         for (int e = 0; e < 8; ++e) ur[b][e] = (b < B && lane * 8 < R) ? s_u[(b < B && lane * 8 < R) ? b * R + lane * 8 + e : 0] : 0.f;
       Lse mine = lse_empty();
+      float* glg = p.uniforms ? p.lg + static_cast<size_t>(j & 1) * B * V : nullptr;  // sampled: final logits
       // rows read through L2 first (the longest latency): one group of rows per warp at a time
       for (int r0 = warp * kGroup; r0 < n_g; r0 += kRollWarps * kGroup) {
         uint4 raw[kGroup];
@@ -798,7 +809,7 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
         float dot[32] = {};
         group_fma<KB, kGroup>(raw, 0, ur, dot);
         wide_push<KB>(dot, lane, min(kGroup, n_g - r0), n_t + n_s + r0, r_lo + n_t + n_s + r0, s_base, s_b2,
-                      rows_cta, B, mine);
+                      rows_cta, B, mine, glg, V);
       }
       // rows in tensor memory: this warp's 64 rows of its lane quarter, 8 rows (32 columns) a load
       for (int rho0 = 64 * half; rho0 < 64 * half + 64; rho0 += kRows) {
@@ -827,7 +838,7 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
           }
           group_fma<KB, kGroup>(raw, g, ur, dot);
         }
-        wide_push<KB>(dot, lane, n_t - row0, row0, r_lo + row0, s_base, s_b2, rows_cta, B, mine);
+        wide_push<KB>(dot, lane, n_t - row0, row0, r_lo + row0, s_base, s_b2, rows_cta, B, mine, glg, V);
       }
       // rows in shared memory (landed before the first step's phase C)
       bool filled = true;
@@ -848,7 +859,8 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
                            : make_uint4(0, 0, 0, 0);
             group_fma<KB, kGroup>(raw, g, ur, dot);
           }
-          wide_push<KB>(dot, lane, n_s - r0, n_t + r0, r_lo + n_t + r0, s_base, s_b2, rows_cta, B, mine);
+          wide_push<KB>(dot, lane, n_s - r0, n_t + r0, r_lo + n_t + r0, s_base, s_b2, rows_cta, B, mine, glg,
+                        V);
         }
       }
       Lse st[KB];
