@@ -56,6 +56,22 @@ def dist_env():
     return rank, world, local
 
 
+def max_over_ranks(x: float, world: int, device) -> float:
+    """The slowest rank's value (replicas: the job ends when its slowest rank does)."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(world: int, blocks_per_rank_step: int, steps: int, seconds: float) -> float:
+    """Whole-job draft blocks/s: every rank ran `steps` steps of `blocks_per_rank_step` blocks."""
+    return world * blocks_per_rank_step * steps / seconds
+
+
 def load_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -519,12 +535,9 @@ def run_ours(args):
     kern = binding.domino_timing_end()
     if bad:
         raise RuntimeError("a step of the per-kernel region returned an error")
-    if world > 1:
-        t = torch.tensor([ms], dtype=torch.float64, device=device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, world, device)
     ms_step = ms / args.steps
-    value = world * c.B * args.steps / (ms / 1e3)
+    value = job_throughput(world, c.B, args.steps, ms / 1e3)
 
     # ---- e2e through the host-buffer entry point (pinned inputs and outputs)
     M = c.M
@@ -546,11 +559,8 @@ def run_ours(args):
         if rc != 0:
             raise binding.DominoError(rc, "host-buffer step")
     t_e2e = time.perf_counter() - t0
-    if world > 1:
-        t = torch.tensor([t_e2e], dtype=torch.float64, device=device)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        t_e2e = float(t.item())
-    e2e_value = world * c.B * n_e2e / t_e2e
+    t_e2e = max_over_ranks(t_e2e, world, device)
+    e2e_value = job_throughput(world, c.B, n_e2e, t_e2e)
     h2d = M * c.H * 2 + M * 4
     # the host entry point reads its outputs (top-k ids and log-probs, the four tree arrays) and a
     # copy of the status in one copy of the workspace region that holds them (256-byte aligned)
