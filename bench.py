@@ -436,6 +436,37 @@ def rollout_timing(st, wl, c, hidden, device, stream, reps=50):
             "note": "B sequences x K draft tokens, each fed back; timing only (parity is in the tests)"}
 
 
+def torch_unfused_timing(st, c, hidden, stream, reps=50):
+    """Context only, not the library: the vocabulary GEMM of the step done the unfused way in
+    PyTorch -- cuBLAS bf16 matmuls of hidden with W_lm and of u with W2 writing full logits to
+    HBM, then log_softmax and topk -- on the same weights and hidden states (u is a zero tensor
+    of the right shape: the GRU and W1 are left out, so this times S5 + S6 only)."""
+    import torch
+    h = hidden.view(c.M, c.H)
+    w_lm, w2 = st.w["w_lm"], (st.w.get("w2") if st.head_on else None)
+    u = torch.zeros(c.M, c.R, dtype=torch.bfloat16, device=h.device) if w2 is not None else None
+
+    def run():
+        z = torch.matmul(h, w_lm.t())
+        if w2 is not None:
+            z = z + torch.matmul(u, w2.t())
+        return torch.topk(torch.log_softmax(z.float(), dim=-1), c.k, dim=-1)
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            run()
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            run()
+        e1.record(stream)
+        torch.cuda.synchronize()
+    return {"us": round(e0.elapsed_time(e1) / reps * 1e3, 2),
+            "note": "context only: torch matmul (cuBLAS) for W_lm and W2 with full logits in HBM, then "
+                    "log_softmax + topk (S5 + S6 of the step, the GRU and W1 left out); not part of the library"}
+
+
 def graph_replay(st, hidden, ids, device, n, blocks_per_step):
     """Capture one step in a CUDA graph and time n replays; on a capture failure, say why."""
     import torch
@@ -596,6 +627,8 @@ def run_ours(args):
     verify = verify_timing(st, c, device, stream) if c.B <= 4 else None
     # ---- the sequential draft loop (the paper's inference loop) on the same weights
     rollout = rollout_timing(st, wl, c, hidden, device, stream)
+    # ---- context: the vocabulary GEMM + log_softmax + topk the unfused way in PyTorch
+    unfused = torch_unfused_timing(st, c, hidden, stream)
 
     # ---- roofline of the dominant kernel, measured in the timed region
     peaks = load_peaks()
@@ -628,7 +661,8 @@ def run_ours(args):
         "e2e": {"value": round(e2e_value, 3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "steps": n_e2e, "api": "domino_draft_step_host (synchronous per step)"},
         "gpu_launches": args.steps * launches, "clocks": clocks,
-        "head_overhead": head_overhead, "input_table_step": input_table, "tree_verify": verify,
+        "head_overhead": head_overhead, "input_table_step": input_table, "torch_unfused": unfused,
+        "tree_verify": verify,
         "rollout_greedy": rollout,
     }
     # ---- last: the same step replayed from a CUDA graph (one captured step, replayed back to
