@@ -116,19 +116,20 @@ def test_launches_per_step_counts_the_kernels(name, table):
         assert launched == (3 if plain == 3 else plain - 1)
 
 
-def test_bad_token_reported_with_input_table():
-    """Without the X GEMM an out-of-range id is still reported (the gather's check), and the GRU
-    reads a valid table row for it."""
-    wl = inputs.make_workload(inputs.custom_config("bad-t", B=4, K=16, H=64, V=500, Ds=32, R=16, k=2, N=3, seed=25))
+@pytest.mark.parametrize("B,K,launches", [(1, 4, 3), (4, 16, 5)])
+def test_bad_token_reported_with_input_table(B, K, launches):
+    """With the table an out-of-range id is still reported (the GRU's own check at B <= 2, the
+    gather's otherwise), and the GRU reads a valid table row for it."""
+    wl = inputs.make_workload(inputs.custom_config("bad-t", B=B, K=K, H=64, V=500, Ds=32, R=16, k=2, N=3, seed=25))
     c = wl.cfg
     st = DraftStep(wl.weights, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=_dev(), input_table=True)
-    assert st.launches_per_step() == 5
+    assert st.launches_per_step() == launches
     hidden = torch.from_numpy(wl.hidden.view(np.int16)).view(torch.bfloat16).to(_dev())
     ids = torch.from_numpy(wl.prefix_ids).to(_dev())
-    ids[1, 3] = -2
+    ids[B - 1, K - 1] = -2
     assert st.enqueue(hidden, ids) == 0
     assert binding.domino_check_status(st.workspace, torch.cuda.current_stream()) == binding.DOMINO_ERR_BAD_TOKEN
-    ids[1, 3] = 7
+    ids[B - 1, K - 1] = 7
     assert st.enqueue(hidden, ids) == 0
     assert binding.domino_check_status(st.workspace, torch.cuda.current_stream()) == 0
 
@@ -162,8 +163,8 @@ def test_deterministic_and_host_entry_point_matches():
     np.testing.assert_array_equal(host["tree_score"].numpy().reshape(out1["tree_score"].shape), out1["tree_score"])
 
 
-@pytest.mark.parametrize("B,K", [(1, 6), (4, 16)])
-def test_consecutive_steps_on_one_workspace(B, K):
+@pytest.mark.parametrize("B,K,table", [(1, 6, False), (4, 16, False), (1, 6, True), (4, 16, True)])
+def test_consecutive_steps_on_one_workspace(B, K, table):
     """Steps with different inputs back to back on one workspace each match the oracle: state
     words a previous step left behind (tagged with its epoch at B <= 2, cleared at larger B)
     never pass for the current step's."""
@@ -173,7 +174,7 @@ def test_consecutive_steps_on_one_workspace(B, K):
     wl_b = inputs.make_workload(inputs.custom_config("consec", B=B, K=K, H=256, V=2000, Ds=64, R=64, k=4, N=8,
                                                      seed=42, biases=True), weights=wl_a.weights)
     c = wl_a.cfg
-    st = DraftStep(wl_a.weights, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=_dev())
+    st = DraftStep(wl_a.weights, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=_dev(), input_table=table)
     for wl in (wl_a, wl_b, wl_a, wl_b):
         hidden = torch.from_numpy(wl.hidden.view(np.int16)).view(torch.bfloat16).to(_dev())
         ids = torch.from_numpy(wl.prefix_ids).to(_dev())

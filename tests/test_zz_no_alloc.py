@@ -19,11 +19,11 @@ pytestmark = pytest.mark.gpu
 LOGP_TOL = 2e-2  # the tolerance the parity tests use for log-probabilities
 
 
-def _compare(cfg):
+def _compare(cfg, table=False):
     dev = torch.device("cuda:0")
     wl = inputs.make_workload(cfg)
     c = wl.cfg
-    st = DraftStep(wl.weights, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=dev)
+    st = DraftStep(wl.weights, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=dev, input_table=table)
     hidden = torch.from_numpy(wl.hidden.view(np.int16)).view(torch.bfloat16).to(dev)
     ids = torch.from_numpy(wl.prefix_ids).to(dev)
     ref = st.run(hidden, ids)  # existing entry point, caller-allocated workspace
@@ -55,11 +55,11 @@ def _compare(cfg):
                                    atol=LOGP_TOL * c.K, rtol=0)
 
 
-@pytest.mark.parametrize("name", ["tiny", "B2"])
-def test_static_scratch_matches_workspace_entry_point(name):
+@pytest.mark.parametrize("name,table", [("tiny", False), ("B2", False), ("B2", True)])
+def test_static_scratch_matches_workspace_entry_point(name, table):
     cfg = inputs.CONFIGS["tiny"] if name == "tiny" else inputs.custom_config(
         name, B=2, K=8, H=256, V=3000, Ds=64, R=64, k=6, N=12, seed=31, biases=True)
-    _compare(cfg)
+    _compare(cfg, table)
 
 
 def test_static_scratch_rejects_sizes_beyond_the_array():
