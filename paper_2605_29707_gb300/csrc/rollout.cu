@@ -1,4 +1,4 @@
-// rollout.cu -- the greedy sequential draft loop (section 4.1.2 and Fig. 3: at inference each
+// rollout.cu -- the sequential draft loop, greedy or sampled (section 4.1.2 and Fig. 3: at inference each
 // draft token is chosen from the final logits L_j = L_base_j + W2 u_j + b2 and becomes the
 // causal encoder's next input).  The base logits W_lm hidden_j of every position come first from
 // the tensor-core GEMM (store mode, fp32); a persistent cooperative kernel then runs the K
@@ -8,7 +8,12 @@
 //   C  L_j = base_j + W2 u_j + b2 over the CTA's slice of the vocabulary, with a running max,
 //      sum of exp and argmax (equal values: the lowest id) per sequence, reduced per CTA;
 // after the third barrier every CTA combines the per-CTA partials itself (the same result
-// everywhere), so t_{j+1} needs no fourth barrier.  Every wait is bounded.
+// everywhere), so t_{j+1} needs no fourth barrier.  The sampled loop (t_{j+1} by inverse CDF
+// from the caller's uniform) keeps the same barriers: every CTA reads the final logits of the
+// CTA whose rows hold the draw and scans them itself.  With an input-projection table
+// (emb . W_ih^T) phase A reads one row of it instead of projecting emb[t_j]; the resident
+// kernel computes u's hidden half W1[:, :H] hidden_j for all positions before the steps.
+// Every wait is bounded.
 //
 // W2 (V x r bf16, 78 MB at the Qwen3 vocabulary) is the operand phase C reads every step.  With
 // r <= 256 the resident kernel keeps each CTA's slice of it on chip for the whole block: 512
