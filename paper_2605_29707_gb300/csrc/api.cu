@@ -1,15 +1,19 @@
 // api.cu -- host side of the C ABI declared in include/domino.h: argument checks, the launch
 // plan for the current device, workspace layout, TMA tensor maps and the launch sequence.
 //
-// Launch sequence of one step (all on the caller's stream):
-//   memset   clear the status word and the GRU grid-barrier counter
-//   gather   E_j = emb[prefix_ids] (section 4.1.2) and the prefix-id range check
-//   tc store Xp = E . W_ih^T            (tcgen05, split-K fp32 partials)
-//   tc store Up = hidden . W1[:, :H]^T  (tcgen05, split-K fp32 partials)
-//   gru      S_j = GRU(E_0..E_j); u = SiLU(Up + S . W1[:, H:]^T + b1)   (cooperative)
+// Launch sequence of one step (all on the caller's stream).  Small batches (B <= 2 at K = 16):
+//   gru      prologue: prefix-id check, E . W_ih^T from the embedding rows by id (or rows of the
+//            input-projection table) and hidden . W1[:, :H]^T; then S_j = GRU(E_0..E_j) and
+//            u = SiLU(. + S . W1[:, H:]^T + b1)  (cooperative; its first CTA resets the status)
 //   tc soft  logits = [hidden | u] . [W_lm | W2]^T + b2, online max / sum-exp / top-k
+//            (a programmatic dependent of the GRU: the W_lm segment streams beside it)
 //   tree     merge the partials -> lse, top-k log-probs; best-first draft tree
-// With the correction branch off only memset, gather (id check), tc soft and tree run.
+// Other batches: memset (the control words: status, merge counters), gather (id check, state
+// words cleared; E = emb[ids] unless a table is given), tc store Xp = E . W_ih^T (not with a
+// table), tc store Up = hidden .
+// W1[:, :H]^T, gru, tc soft, tree; large M moves the W1 GEMM (both halves) and a SiLU kernel
+// after the GRU.  With the correction branch off only memset, gather (id check), tc soft and
+// tree run.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
@@ -742,7 +746,7 @@ int domino_build_input_table(const void* emb, const void* w_ih, int V, int H, in
   return h;
 }
 
-// ---------------------------------------------------------------- greedy rollout
+// ---------------------------------------------------------------- sequential rollout (greedy, sampled)
 namespace {
 struct RollPlan {
   int B, K, H, V, Ds, R, M, grid;
