@@ -10,9 +10,8 @@
 //   tree     merge the partials -> lse, top-k log-probs; best-first draft tree
 // Other batches: memset (the control words: status, merge counters), gather (id check, state
 // words cleared; E = emb[ids] unless a table is given), tc store Xp = E . W_ih^T (not with a
-// table), tc store Up = hidden .
-// W1[:, :H]^T, gru, tc soft, tree; large M moves the W1 GEMM (both halves) and a SiLU kernel
-// after the GRU.  With the correction branch off only memset, gather (id check), tc soft and
+// table), tc store Up = hidden . W1[:, :H]^T, gru, tc soft, tree; large M moves the W1 GEMM
+// (both halves) and a SiLU kernel after the GRU.  With the correction branch off only memset, gather (id check), tc soft and
 // tree run.
 #include <cuda.h>
 #include <cudaTypedefs.h>
