@@ -75,6 +75,9 @@ def test_input_table_size_and_argument_checks():
     assert binding.domino_build_input_table(one, one, 10, 8, -8, one) == bad
     assert binding.domino_build_input_table(one, one, 10, 12, 8, one) == binding.DOMINO_ERR_UNSUPPORTED
     assert binding.domino_build_input_table(one, one, 10, 8, 4096, one) == binding.DOMINO_ERR_UNSUPPORTED
+    # pointers must be 16-byte aligned (TMA); refused before any device query
+    assert binding.domino_build_input_table(one + 2, one, 10, 8, 8, one) == binding.DOMINO_ERR_UNSUPPORTED
+    assert binding.domino_build_input_table(one, one, 10, 8, 8, one + 4) == binding.DOMINO_ERR_UNSUPPORTED
 
 
 def test_launch_count_query():
