@@ -88,7 +88,8 @@ typedef struct domino_head_weights {
    * once per set of weights by domino_build_input_table; NULL = the GRU projects emb[t]
    * itself.  When set, every entry point takes the GRU's input-gate sums from it (one row per
    * token) instead of projecting the embedding rows: the block step then launches no X GEMM
-   * (domino_launches_per_step_table) and the rollout's steps read one row each. */
+   * (domino_launches_per_step_table) and the rollout's steps read one row each.  16-byte
+   * aligned, like every tensor (refused as the other pointers are). */
   const float* x_table;
 } domino_head_weights;
 

@@ -527,7 +527,7 @@ int check_pointers(const void* hidden, const int32_t* ids, const void* w_lm, con
   if (head && (!hw->emb || !hw->w_ih || !hw->w_hh || !hw->w1 || !hw->w2)) return DOMINO_ERR_INVALID_ARG;
   if (!aligned16(hidden) || !aligned16(w_lm)) return DOMINO_ERR_UNSUPPORTED;
   if (head && (!aligned16(hw->emb) || !aligned16(hw->w_ih) || !aligned16(hw->w_hh) || !aligned16(hw->w1) ||
-               !aligned16(hw->w2)))
+               !aligned16(hw->w2) || !aligned16(hw->x_table)))
     return DOMINO_ERR_UNSUPPORTED;
   return DOMINO_OK;
 }
@@ -812,7 +812,7 @@ int rollout_entry(const void* hidden, const int32_t* anchors, const float* unifo
   if (hd && (!head->emb || !head->w_ih || !head->w_hh || !head->w1)) return DOMINO_ERR_INVALID_ARG;
   if (!aligned16(hidden) || !aligned16(w_lm)) return DOMINO_ERR_INVALID_ARG;
   if (hd && (!aligned16(head->w2) || !aligned16(head->w1) || !aligned16(head->w_ih) || !aligned16(head->w_hh) ||
-             !aligned16(head->emb)))
+             !aligned16(head->emb) || !aligned16(head->x_table)))  // x_table: NULL passes
     return DOMINO_ERR_INVALID_ARG;
   RollPlan P;
   int rc = make_roll_plan(B, K, H, V, hd ? head->Ds : 0, hd ? head->R : 0, hd, &P);

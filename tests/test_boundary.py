@@ -80,6 +80,14 @@ def test_input_table_size_and_argument_checks():
     assert binding.domino_build_input_table(one, one, 10, 8, 8, one + 4) == binding.DOMINO_ERR_UNSUPPORTED
 
 
+def test_rollout_refuses_a_misaligned_input_table_before_any_device_call():
+    _lib()
+    one = 16  # non-null, 16-byte aligned stand-ins; never dereferenced
+    head = binding.make_head(one, one, one, None, None, one, None, one, None, 16, 8, x_table=one + 4)
+    rc = binding.domino_rollout_greedy(one, one, one, head, 1, 2, 64, 100, one, one, one, 1 << 20, None)
+    assert rc == binding.DOMINO_ERR_INVALID_ARG
+
+
 def test_launch_count_query():
     _lib()
     # B = 1: the GRU (with its own projections), the vocab GEMM, merge + tree
