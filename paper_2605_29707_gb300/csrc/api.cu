@@ -19,12 +19,37 @@
 #include <stdint.h>
 #include <string.h>
 
+#include <atomic>
 #include <cmath>
+#include <map>
 #include <mutex>
+#include <utility>
 #include <vector>
 
 #include "domino.h"
 #include "kernels.h"
+
+// ---------------------------------------------------------------- kernel attributes
+namespace dm {
+cudaError_t ensure_smem_attr(const void* func, size_t smem, bool carveout) {
+  static std::mutex mu;
+  static std::map<std::pair<int, const void*>, size_t> done;  // (device, kernel) -> limit set
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  size_t& have = done[std::make_pair(dev, func)];
+  if (have >= smem) return cudaSuccess;
+  e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  if (carveout) {
+    e = cudaFuncSetAttribute(func, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    if (e != cudaSuccess) return e;
+  }
+  have = smem;
+  return cudaSuccess;
+}
+}  // namespace dm
 
 namespace {
 
@@ -295,6 +320,7 @@ bool gemm_maps(CUtensorMap* a, CUtensorMap* b, bool swap, int bn, const void* X,
 
 int cuda_rc(cudaError_t e) { return e == cudaSuccess ? DOMINO_OK : DOMINO_ERR_CUDA; }
 
+
 // ---------------------------------------------------------------- host staging
 // Pinned host buffer the host entry point copies a step's outputs into (one copy), grown on
 // demand and kept for the process; callers hold g_stage_mu while they use it.
@@ -316,7 +342,7 @@ uint8_t* stage_buffer(size_t bytes) {
 
 // ---------------------------------------------------------------- per-kernel timing
 struct Timing {
-  bool on = false;
+  std::atomic<bool> on{false};  // read by every launch, on any thread; set by begin / end
   int used = 0;
   std::vector<cudaEvent_t> start, stop;
   std::vector<int> kind;

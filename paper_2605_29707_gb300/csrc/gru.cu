@@ -10,6 +10,8 @@
 // release fence.  Every wait is bounded.
 #include <math.h>
 
+#include <atomic>
+
 #include "kernels.h"
 #include "ptx.cuh"
 
@@ -612,14 +614,9 @@ GruPlan gru_plan(int B, int Ds, int num_sms) {
 
 template <bool kTable>
 static cudaError_t launch_gru_t(const GruParams& p, const GruPlan& plan, cudaStream_t stream, bool pdl) {
-  static size_t attr_smem = 0;
-  if (plan.smem > attr_smem) {
-    cudaError_t e = cudaFuncSetAttribute(gru_kernel<kTable>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(plan.smem));
+  {
+    const cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(gru_kernel<kTable>), plan.smem, true);
     if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(gru_kernel<kTable>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
-    if (e != cudaSuccess) return e;
-    attr_smem = plan.smem;
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(plan.gu * plan.gb);
@@ -633,7 +630,7 @@ static cudaError_t launch_gru_t(const GruParams& p, const GruPlan& plan, cudaStr
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   // A runtime that refuses the pair gets the cooperative launch alone from then on.
-  static bool pdl_refused = false;
+  static std::atomic<bool> pdl_refused{false};
   cfg.numAttrs = (pdl && !pdl_refused) ? 2 : 1;
   cudaError_t e = cudaLaunchKernelEx(&cfg, gru_kernel<kTable>, p);
   if (e != cudaSuccess && cfg.numAttrs == 2) {

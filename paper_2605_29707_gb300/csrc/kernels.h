@@ -10,6 +10,11 @@ namespace dm {
 
 enum TcMode { kModeSoftmax = 0, kModeStore = 1 };
 
+// Raises a kernel's dynamic shared-memory limit to at least `smem` bytes on the current device
+// (with `carveout`, also asks for the largest shared-memory carveout), once per device, kernel
+// and size; safe to call from several host threads (api.cu).
+cudaError_t ensure_smem_attr(const void* func, size_t smem, bool carveout);
+
 // Most deferred tiles one CTA of the vocabulary GEMM can hold (each has its own completion
 // barrier in shared memory).
 constexpr int kMaxDefer = 32;

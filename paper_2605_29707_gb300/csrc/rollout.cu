@@ -1072,12 +1072,11 @@ size_t rollout_smem_bytes(int B, int V, int R, bool head, int grid) {
 }
 
 template <typename Kern>
-static cudaError_t launch_coop(Kern kern, size_t& attr_smem, const RolloutParams& p, int grid, int threads,
-                               size_t smem, cudaStream_t stream) {
-  if (smem > 48 * 1024 && smem > attr_smem) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+static cudaError_t launch_coop(Kern kern, const RolloutParams& p, int grid, int threads, size_t smem,
+                               cudaStream_t stream) {
+  if (smem > 48 * 1024) {
+    const cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(kern), smem, false);
     if (e != cudaSuccess) return e;
-    attr_smem = smem;
   }
   RolloutParams pp = p;
   void* args[] = {&pp};
@@ -1089,12 +1088,8 @@ static cudaError_t launch_coop(Kern kern, size_t& attr_smem, const RolloutParams
 
 template <int KB>
 static cudaError_t launch_rollout_kb(const RolloutParams& p, int grid, size_t smem, cudaStream_t stream) {
-  if (use_resident(p)) {
-    static size_t attr = 0;
-    return launch_coop(rollout_resident_kernel<KB>, attr, p, grid, kRollThreads, smem, stream);
-  }
-  static size_t attr = 0;
-  return launch_coop(rollout_kernel<KB>, attr, p, grid, kRollThreadsAll, smem, stream);
+  if (use_resident(p)) return launch_coop(rollout_resident_kernel<KB>, p, grid, kRollThreads, smem, stream);
+  return launch_coop(rollout_kernel<KB>, p, grid, kRollThreadsAll, smem, stream);
 }
 
 cudaError_t launch_rollout(const RolloutParams& p, int grid, cudaStream_t stream) {

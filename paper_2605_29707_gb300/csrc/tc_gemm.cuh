@@ -590,13 +590,9 @@ cudaError_t launch_tc_instance(const CUtensorMap* maps, const TcParams& p, int g
                                bool pdl = false) {
   using C = TcCfg<BN, SWAP, MODE, KMAX, ST>;
   auto kern = tc_gemm_kernel<BN, SWAP, MODE, KMAX, ST>;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+  {
+    const cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(kern), C::kSmemBytes, true);
     if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
