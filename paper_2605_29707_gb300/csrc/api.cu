@@ -162,7 +162,7 @@ int check_sizes(int B, int K, int H, int V, int Ds, int R, int k, int N, bool he
 // The plan for a GPU with `sms` SMs (sizes already checked).
 int make_plan_sms(int B, int K, int H, int V, int Ds, int R, int k, int N, bool head, int sms, Plan* P) {
   Plan& p = *P;
-  memset(&p, 0, sizeof p);
+  p = Plan{};  // every member zero (the nested plans' defaults are zero too)
   p.B = B; p.K = K; p.H = H; p.V = V; p.k = k; p.N = N;
   p.head = head;
   p.Ds = head ? Ds : 0;
@@ -368,7 +368,6 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
              uint8_t* ws, cudaStream_t st, int32_t* status_out = nullptr) {
   const int M = P.M, H = P.H, V = P.V, Ds = P.Ds, R = P.R;
   int* status = reinterpret_cast<int*>(ws + P.off_ctrl);
-  unsigned* barrier = reinterpret_cast<unsigned*>(ws + P.off_ctrl + 64);
   unsigned* seq_done = reinterpret_cast<unsigned*>(ws + P.off_ctrl + 256);
   if (P.clear_bytes && cudaMemsetAsync(ws + P.off_ctrl, 0, P.clear_bytes, st) != cudaSuccess) return DOMINO_ERR_CUDA;
   uint32_t* epoch = reinterpret_cast<uint32_t*>(ws + P.off_ctrl + 128);
