@@ -223,6 +223,48 @@ def test_tree_invariants(ties):
     assert len({(par[i], tok[i]) for i in range(N)}) == N
 
 
+def _tree_by_frontier_scan(ids, lp, N):
+    """The best-first tree by its definition, slowly: before every pop the frontier is rebuilt
+    from scratch (every depth-1 candidate and every child of a selected node that is not selected
+    yet), and the pop is the greatest (score, lower token, lower parent index)."""
+    K, k = lp.shape
+    nodes = []  # (parent, token, depth, score, list index)
+    taken = set()  # (parent, list index)
+    for _ in range(N):
+        best = None
+        for parent in [-1] + list(range(len(nodes))):
+            d = 1 if parent < 0 else nodes[parent][2] + 1
+            if d > K:
+                continue
+            base = 0.0 if parent < 0 else nodes[parent][3]
+            for q in range(k):
+                if (parent, q) in taken:
+                    continue
+                key = (base + lp[d - 1, q], -int(ids[d - 1, q]), -parent)
+                if best is None or key > best[0]:
+                    best = (key, parent, q, d)
+        (score, _, _), parent, q, d = best
+        taken.add((parent, q))
+        nodes.append((parent, int(ids[d - 1, q]), d, score, q))
+    return (np.array([n[0] for n in nodes]), np.array([n[1] for n in nodes]), np.array([n[2] for n in nodes]),
+            np.array([n[3] for n in nodes]))
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_tree_with_ties_matches_a_frontier_scan(seed):
+    """Tie-heavy lists (log-probs on a 1/4 grid, so equal scores are common at every depth):
+    the oracle's tree equals the definition computed by rescanning the whole frontier."""
+    rng = np.random.default_rng(100 + seed)
+    K, k = [(3, 3), (4, 2), (2, 4), (5, 3), (3, 4), (6, 2)][seed]
+    ids, lp = _random_lists(rng, K, k, ties=True)
+    total = sum(k ** d for d in range(1, K + 1))
+    for N in sorted({1, 2, 3, min(total, 12), min(total, 31), total}):
+        par, tok, dep, sc = oracle.tree(ids, lp, N)
+        rpar, rtok, rdep, rsc = _tree_by_frontier_scan(ids, lp, N)
+        assert par.tolist() == rpar.tolist() and tok.tolist() == rtok.tolist() and dep.tolist() == rdep.tolist()
+        np.testing.assert_array_equal(sc, rsc)
+
+
 def test_tree_special_cases():
     rng = np.random.default_rng(11)
     K, k = 6, 4
