@@ -19,9 +19,11 @@ def test_same_seed_same_bytes():
     np.testing.assert_array_equal(a.prefix_ids, b.prefix_ids)
 
 
-def test_chunks_are_seeded_by_key_and_index_not_by_thread_count():
-    """A tensor of two 2^24-element chunks: chunk 0 equals a one-chunk draw with the same key and
-    chunk 1 the first values of the generator keyed (key, 1), with one thread or many."""
+def test_chunks_are_seeded_by_key_and_index_not_by_thread_count(monkeypatch):
+    """A tensor of two chunks (the chunk size shrunk from 2^24 to 4096 for the test): chunk 0
+    equals a one-chunk draw with the same key and chunk 1 the first values of the generator keyed
+    (key, 1), with one thread or many."""
+    monkeypatch.setattr(inputs, "_CHUNK", 4096)
     key = (7, "chunk-test")
     n_tail = 1000
     old = torch.get_num_threads()
