@@ -34,3 +34,26 @@ def test_head_weights_layout_matches_the_header():
     assert c["sizeof"] == ctypes.sizeof(binding.domino_head_weights)
     for f in FIELDS:
         assert c[f] == getattr(binding.domino_head_weights, f).offset, f
+
+
+def _prototypes():
+    """{entry point: number of parameters} from the header's DOMINO_API declarations."""
+    import re
+    with open(os.path.join(ROOT, "include", "domino.h")) as f:
+        text = re.sub(r"/\*.*?\*/", " ", f.read(), flags=re.S)  # drop comments
+    out = {}
+    for m in re.finditer(r"DOMINO_API\s+[\w\s\*]+?\b(domino_\w+)\s*\(([^)]*)\)\s*;", text):
+        params = m.group(2).strip()
+        out[m.group(1)] = 0 if params in ("", "void") else params.count(",") + 1
+    return out
+
+
+def test_binding_argument_counts_match_the_prototypes():
+    """Every entry point the binding declares takes as many arguments as its C prototype."""
+    protos = _prototypes()
+    assert sorted(protos) == sorted(binding.SYMBOLS)
+    lib = binding.load()
+    for name, n in protos.items():
+        argtypes = getattr(lib, name).argtypes
+        assert argtypes is not None, name
+        assert len(argtypes) == n, (name, len(argtypes), n)
