@@ -3,7 +3,7 @@
  *
  * TEST INFRASTRUCTURE ONLY.  This library exists to check the CUDA path; it is
  * called from the tests, from the package smoke check and from the CPU-baseline
- * leg of the benchmark, never from the product path.  It shares no code, header,
+ * leg and the reference arm of the benchmark, never from the product path.  It shares no code, header,
  * table or helper with the CUDA library (include/domino.h) and includes nothing
  * from it.
  *
