@@ -128,10 +128,13 @@ DOMINO_API size_t domino_workspace_bytes(int B, int K, int H, int V, int Ds, int
  *   tree_score  fp32  [B, N] or NULL   cumulative log-probability, non-increasing in i
  * workspace: device buffer of at least domino_workspace_bytes(...) bytes, 256-byte aligned,
  * ZERO-FILLED before its first use (once, e.g. cudaMemsetAsync at allocation); every step
- * leaves it ready for the next one, whatever the sizes (small batches skip a per-step clear:
- * the GRU's state words carry a step count the last kernel advances).  Zero it again after a
- * call that returned DOMINO_ERR_CUDA part-way.  One workspace must not be shared by steps that
- * overlap in time.
+ * leaves it ready for the next one, whatever the sizes or the kind of the step before.  Small
+ * batches skip a per-step clear: the GRU's state words carry a step count the last kernel
+ * advances, and are trusted only over the byte range the control words record as holding state
+ * words; when a step of another shape or kind used the workspace last, the GRU first zeroes its
+ * own state words behind a grid barrier.  A call that fails part-way with DOMINO_ERR_CUDA zeroes
+ * the control words itself; if the CUDA context is broken, zero the whole workspace before
+ * reusing it.  One workspace must not be shared by steps that overlap in time.
  * Returns DOMINO_OK once everything is enqueued, or a negative code (nothing enqueued). */
 DOMINO_API int domino_draft_step(const void* hidden, const int32_t* prefix_ids, const void* w_lm,
                       const domino_head_weights* head, int B, int K, int H, int V, int k, int N,
@@ -162,6 +165,26 @@ DOMINO_API int domino_draft_step_host(const void* hidden_host, const int32_t* pr
  * read itself fails).  Each domino_draft_step clears the word when it starts. */
 DOMINO_API int domino_check_status(const void* workspace, void* stream);
 
+/* Failure-detection test hook; the paper has no counterpart.  It lets a test check that a
+ * step whose inter-CTA wait can never be satisfied reports DOMINO_ERR_TIMEOUT instead of
+ * hanging, without faulting anything.  It arms, on the current device, one withheld event in
+ * the next GRU launch that has a CTA numbered gru_cta; the launch's other CTAs wait for that
+ * event, their bounded waits run out (about one second of SM clock cycles each), and the step
+ * records DOMINO_ERR_TIMEOUT in its device status word (domino_check_status):
+ *   DOMINO_HOLD_STATE          CTA gru_cta does not publish its hidden states of position
+ *                              `step` (0 <= step < 64; a step >= K withholds nothing);
+ *   DOMINO_HOLD_CLEAR_BARRIER  CTA gru_cta does not arrive at the barrier of the state clear
+ *                              that a small-batch step (B <= 2 at K = 16) runs when the workspace
+ *                              last held another kind or shape of step (or is fresh); `step` is
+ *                              ignored, and a step that needs no clear withholds nothing;
+ *   DOMINO_HOLD_OFF            disarms the hook.
+ * The held CTA disarms the hook when its launch ends, so it affects one step.  Every kernel of
+ * the held step still completes (its outputs are undefined) and the workspace stays usable: the
+ * next step runs normally.  Synchronous (a copy to a device symbol); not for use while steps
+ * run on other threads.  Returns DOMINO_OK, DOMINO_ERR_INVALID_ARG or DOMINO_ERR_CUDA. */
+enum domino_hold { DOMINO_HOLD_OFF = 0, DOMINO_HOLD_STATE = 1, DOMINO_HOLD_CLEAR_BARRIER = 2 };
+DOMINO_API int domino_debug_hold(int what, int gru_cta, int step);
+
 /* Static, human-readable name of a status code. */
 DOMINO_API const char* domino_status_string(int status);
 
@@ -179,8 +202,8 @@ DOMINO_API int domino_launches_per_step(int B, int K, int H, int V, int Ds, int 
 DOMINO_API int domino_launches_per_step_table(int B, int K, int H, int V, int Ds, int R, int k, int N);
 
 /* Greedy verification of draft trees against the target model's logits: the step after the
- * draft.  Section 3.1: the target evaluates the draft in one pass and accepts the longest valid
- * prefix; tau counts the accepted tokens plus the bonus token the target produces.  At
+ * draft.  Section 3.1: one target pass checks the whole draft, the draft tokens are kept up to the
+ * first one the target rejects, and tau counts them plus the one extra token the target adds.  At
  * temperature 0 a draft token is valid when it equals the target's most likely next token.
  * For each sequence b, from the anchor: a = argmax of the current node's row (equal values: the
  * lowest id); if a child of the current node carries token a (several: the lowest node index),
@@ -258,9 +281,10 @@ DOMINO_API int domino_rollout_greedy(const void* hidden, const int32_t* anchors,
  *     DOMINO_STATIC_SCRATCH_BYTES; e.g. the B = 32 serving batch) return DOMINO_ERR_UNSUPPORTED
  *     before anything is enqueued.
  *   - Every call on a device shares the one array and it keeps the last call's contents; each
- *     call clears the words that must start at zero (status and counters) itself.  Calls whose
- *     work overlaps on the GPU (other streams, other host threads) race on the array: serialise
- *     them.
+ *     call clears the words that must start at zero (status and counters) itself, and a small
+ *     batch whose state words overlap what a call of another shape or kind left there zeroes
+ *     them first, as for a caller's workspace.  Calls whose work overlaps on the GPU (other
+ *     streams, other host threads) race on the array: serialise them.
  *   - No allocation of any kind is made (no cudaMalloc / cudaFree, no library allocator).
  * device_status: optional device int32; after the step it receives the device status word
  * (DOMINO_OK, DOMINO_ERR_BAD_TOKEN or DOMINO_ERR_TIMEOUT) by an asynchronous copy on `stream`.

@@ -26,9 +26,14 @@ SYMBOLS = ("domino_workspace_bytes", "domino_draft_step", "domino_workspace_byte
            "domino_abi_version", "domino_launches_per_step", "domino_timing_begin", "domino_timing_end",
            "domino_draft_step_static_scratch", "domino_verify_tree_greedy", "domino_rollout_workspace_bytes",
            "domino_rollout_greedy", "domino_rollout_sample", "domino_input_table_bytes",
-           "domino_build_input_table", "domino_launches_per_step_table")
+           "domino_build_input_table", "domino_launches_per_step_table", "domino_debug_hold")
 
 DOMINO_STATIC_SCRATCH_BYTES = 16 << 20
+
+# domino_debug_hold: what a GRU CTA withholds (a failure-detection test hook)
+DOMINO_HOLD_OFF = 0
+DOMINO_HOLD_STATE = 1
+DOMINO_HOLD_CLEAR_BARRIER = 2
 
 KERNEL_KINDS = ("gather", "gru_input_proj", "w1_hidden_proj", "gru", "vocab_gemm_softmax_topk", "merge_tree",
                 "rollout_base_gemm", "rollout_steps", "tree_verify")
@@ -99,6 +104,8 @@ def load():
     lib.domino_input_table_bytes.restype = S
     lib.domino_build_input_table.argtypes = [P, P, I, I, I, P, P]
     lib.domino_build_input_table.restype = I
+    lib.domino_debug_hold.argtypes = [I, I, I]
+    lib.domino_debug_hold.restype = I
     _lib = lib
     return lib
 
@@ -240,3 +247,10 @@ def domino_rollout_sample(hidden, anchors, uniforms, w_lm, head, B, K, H, V, tok
     return int(load().domino_rollout_sample(_addr(hidden), _addr(anchors), _addr(uniforms), _addr(w_lm), h, B, K, H,
                                             V, _addr(tokens), _addr(logp), _addr(workspace), int(workspace_bytes),
                                             _stream(stream)))
+
+
+def domino_debug_hold(what, gru_cta=-1, step=-1) -> int:
+    """Test hook: the next GRU launch's CTA ``gru_cta`` withholds its states of position ``step``
+    (DOMINO_HOLD_STATE) or its clear-barrier arrival (DOMINO_HOLD_CLEAR_BARRIER); DOMINO_HOLD_OFF
+    disarms.  The step then reports DOMINO_ERR_TIMEOUT through its device status."""
+    return int(load().domino_debug_hold(int(what), int(gru_cta), int(step)))

@@ -238,10 +238,12 @@ int make_plan_sms(int B, int K, int H, int V, int Ds, int R, int k, int N, bool 
   };
   p.ctrl_bytes = align_up(256 + static_cast<size_t>(B) * 4);
   p.off_ctrl = take(p.ctrl_bytes);
-  // control words: status at 0, GRU barrier counter at 64, step epoch at 128, merge counters
-  // from 256.  Fused projections need no clear before a step (the GRU resets the status and the
-  // counters, and its state words carry the epoch as a tag); the workspace must only be zero
-  // when first used.
+  // control words: status at 0, the GRU's clear barrier at 64, step epoch at 128, the hx range
+  // record at 160, merge counters from 256.  Fused projections need no clear before a step (the
+  // GRU resets the status and the counters; its state words carry the epoch as a tag, trusted
+  // where the range record covers them, and cleared by the GRU itself where it does not); the
+  // workspace must only be zero when first used.  Every other plan clears all control words,
+  // the range record with them.
   p.clear_bytes = p.fused ? 0 : p.ctrl_bytes;
   if (head) {
     p.off_hx = take(static_cast<size_t>(M) * Ds * 4);
@@ -363,9 +365,10 @@ void timing_close(int slot, cudaStream_t st) {
   if (slot >= 0) cudaEventRecord(g_timing.stop[slot], st);
 }
 
-int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* w_lm, const domino_head_weights* hw,
-             int32_t* topk_ids, float* topk_logp, int32_t* tpar, int32_t* ttok, int32_t* tdep, float* tsc,
-             uint8_t* ws, cudaStream_t st, int32_t* status_out = nullptr) {
+int run_step_launches(const Plan& P, const void* hidden, const int32_t* ids, const void* w_lm,
+                      const domino_head_weights* hw, int32_t* topk_ids, float* topk_logp, int32_t* tpar,
+                      int32_t* ttok, int32_t* tdep, float* tsc, uint8_t* ws, cudaStream_t st,
+                      int32_t* status_out) {
   const int M = P.M, H = P.H, V = P.V, Ds = P.Ds, R = P.R;
   int* status = reinterpret_cast<int*>(ws + P.off_ctrl);
   unsigned* seq_done = reinterpret_cast<unsigned*>(ws + P.off_ctrl + 256);
@@ -469,6 +472,11 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
     gr.epoch = epoch;
     gr.seq_done = seq_done;
     gr.reset_ctrl = P.fused ? 1 : 0;
+    if (P.fused) {
+      gr.layout = reinterpret_cast<unsigned long long*>(ws + P.off_ctrl + 160);
+      gr.layout_range = dm::hx_range(P.off_hx, P.off_hx + static_cast<size_t>(M) * Ds * 4);
+      gr.clear_bar = reinterpret_cast<unsigned long long*>(ws + P.off_ctrl + 64);
+    }
     gr.V = V;
     gr.x_table = x_table;
     gr.x_ids = ids;
@@ -541,6 +549,21 @@ int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* 
   ts = timing_open(DOMINO_KERNEL_TREE, st);
   rc = cuda_rc(dm::launch_merge_tree(tr, st));
   timing_close(ts, st);
+  return rc;
+}
+
+// One step.  A launch that fails part-way leaves the step's later kernels (among them the one
+// that advances the step epoch) unlaunched; the control words are then zeroed, as in a fresh
+// workspace, so the next step neither trusts this one's state words nor counts from its barrier.
+int run_step(const Plan& P, const void* hidden, const int32_t* ids, const void* w_lm, const domino_head_weights* hw,
+             int32_t* topk_ids, float* topk_logp, int32_t* tpar, int32_t* ttok, int32_t* tdep, float* tsc,
+             uint8_t* ws, cudaStream_t st, int32_t* status_out = nullptr) {
+  const int rc = run_step_launches(P, hidden, ids, w_lm, hw, topk_ids, topk_logp, tpar, ttok, tdep, tsc, ws, st,
+                                   status_out);
+  if (rc != DOMINO_OK) {
+    (void)cudaGetLastError();
+    (void)cudaMemsetAsync(ws + P.off_ctrl, 0, P.ctrl_bytes, st);
+  }
   return rc;
 }
 
@@ -665,6 +688,14 @@ const char* domino_status_string(int status) {
 }
 
 int domino_abi_version(void) { return DOMINO_ABI_VERSION; }
+
+int domino_debug_hold(int what, int gru_cta, int step) {
+  if (what == DOMINO_HOLD_OFF) return cuda_rc(dm::arm_gru_hold(dm::kHoldOff, -1, -1));
+  if (what != DOMINO_HOLD_STATE && what != DOMINO_HOLD_CLEAR_BARRIER) return DOMINO_ERR_INVALID_ARG;
+  if (gru_cta < 0 || (what == DOMINO_HOLD_STATE && (step < 0 || step >= kMaxK))) return DOMINO_ERR_INVALID_ARG;
+  const int kind = what == DOMINO_HOLD_STATE ? dm::kHoldPublish : dm::kHoldClearBarrier;
+  return cuda_rc(dm::arm_gru_hold(kind, gru_cta, what == DOMINO_HOLD_STATE ? step : -1));
+}
 
 int domino_timing_begin(int max_launches) {
   if (max_launches <= 0) return DOMINO_ERR_INVALID_ARG;

@@ -82,6 +82,66 @@ __device__ __forceinline__ bool poll_v4(const uint32_t* p, uint4& v, uint32_t ta
   }
 }
 
+__device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Does the recorded range `have` (lo | hi << 32; 0 = none) contain the range `want`?
+__device__ __forceinline__ bool range_contains(unsigned long long have, unsigned long long want) {
+  const uint32_t hl = static_cast<uint32_t>(have), hh = static_cast<uint32_t>(have >> 32);
+  const uint32_t wl = static_cast<uint32_t>(want), wh = static_cast<uint32_t>(want >> 32);
+  return have != 0ull && hl <= wl && wh <= hh;
+}
+
+// Test hook state (domino_debug_hold): what to withhold, from which CTA, at which position.
+__device__ int3 g_gru_hold = {kHoldOff, -1, -1};
+
+cudaError_t arm_gru_hold(int what, int cta, int step) {
+  const int3 v = make_int3(what, cta, step);
+  return cudaMemcpyToSymbol(g_gru_hold, &v, sizeof(v));
+}
+
+// Grid barrier of a cooperative launch that needs no reset: the word holds the generation in its
+// high half and the arrivals of that generation in its low half; the first arrival of a new
+// generation restarts the count.  Every generation is used by one launch only (the step epoch),
+// so a word another launch left behind never counts.  Called by every thread of the CTA; false
+// when the wait ran past kWaitCycles (or the hook withheld this CTA's arrival and its peers').
+__device__ bool grid_barrier_gen(unsigned long long* bar, uint32_t gen, uint32_t count, bool skip_arrival) {
+  __syncthreads();
+  int ok = 1;
+  if (threadIdx.x == 0) {
+    __threadfence();  // this CTA's writes before its arrival
+    if (!skip_arrival) {
+      unsigned long long old = ld_relaxed_u64(bar), assumed;
+      int tries = 0;
+      do {
+        assumed = old;
+        const unsigned long long next = static_cast<uint32_t>(assumed >> 32) == gen
+                                            ? assumed + 1ull
+                                            : (static_cast<unsigned long long>(gen) << 32) | 1ull;
+        old = atomicCAS(bar, assumed, next);
+      } while (old != assumed && ++tries < (1 << 20));
+      if (old != assumed) ok = 0;
+    }
+    const unsigned long long want = (static_cast<unsigned long long>(gen) << 32) | count;
+    const long long t0 = clock64();
+    while (ok && ld_acquire_u64(bar) != want) {
+      __nanosleep(64);
+      if (clock64() - t0 > kWaitCycles) ok = 0;
+    }
+    __threadfence();
+  }
+  return __syncthreads_and(ok) != 0;
+}
+
 __device__ __forceinline__ uint32_t tagged(float h, uint32_t tag) {
   const uint32_t b = static_cast<uint32_t>(__bfloat16_as_ushort(__float2bfloat16_rn(h)));
   return (b << 16) | tag;
@@ -317,6 +377,34 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
   // the vocabulary GEMM that follows may start now: its first K segment does not read
   // anything this kernel writes, and it waits for this grid before reading u
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  const int3 hold = g_gru_hold;
+  const bool held = hold.x != kHoldOff && hold.y == static_cast<int>(blockIdx.x);
+
+  // ---- no clear before the launch: a stale word passes for this step's only if its low half
+  //      equals the tag, which words of earlier steps never do (the epoch advances every step) but
+  //      other data may.  So the tags are trusted only where the workspace held nothing but state
+  //      words at the end of the last step: the range recorded in the control words (written by
+  //      the last step of this kind, zeroed by any other step).  When it does not cover this
+  //      launch's hx, every CTA zeroes the words it will itself write and the grid meets at a
+  //      barrier before any CTA reads a state.
+  if (p.layout != nullptr) {
+    const unsigned long long have = ld_relaxed_u64(p.layout);
+    if (!range_contains(have, p.layout_range)) {
+      const int Ucl = Uc;
+      for (int e = tid; e < nbc * K * Ucl; e += kGruThreads) {
+        const size_t m = static_cast<size_t>(b0) * K + e / Ucl;
+        p.hx[m * Ds + j0 + e % Ucl] = 0u;
+      }
+      const bool skip = held && hold.x == kHoldClearBarrier;
+      if (!grid_barrier_gen(p.clear_bar, *p.epoch + 1u, gridDim.x, skip)) {
+        if (tid == 0) set_status(p.status, kStatusTimeout);
+        if (held && tid == 0) g_gru_hold = make_int3(kHoldOff, -1, -1);
+        return;
+      }
+    }
+    // every CTA has read the record (before the barrier, or it already covered this range)
+    if (blockIdx.x == 0 && tid == 0 && have != p.layout_range) *p.layout = p.layout_range;
+  }
 
   // ---- W_hh rows of this CTA's units (asynchronous); zero rows past 3U and the state tile
   const int rowlen8 = Ds / 8;
@@ -520,12 +608,14 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
         const float n = tanhf(gx[rr][2] + r * hn);
         const float h = (1.f - z) * n + z * hp;
         hprev[bl * U + jl] = h;
+        if (held && hold.x == kHoldPublish && hold.z == t) continue;  // test hook: withheld
         p.hx[m * Ds + j] = tagged(h, tag);
         if (p.s_out) p.s_out[m * Ds + j] = __float2bfloat16_rn(h);
       }
       __syncthreads();
     }
   }
+  if (held && tid == 0) g_gru_hold = make_int3(kHoldOff, -1, -1);  // the hook holds one launch
   if (!ok || p.u == nullptr) return;
 
   // ---- u[m, q] = SiLU(b1[q] + hidden_m . W1[q, :H] + S_m . W1[q, H:]) (small batches): the

@@ -108,7 +108,7 @@ struct GruParams {
   int* status;
   // Fused projections (small batches, u computed in-kernel): with ids set, the kernel computes
   // its own input-gate sums E . W_ih^T (E = emb rows of ids, checked against V) and the hidden
-  // half of u, and xpart / upart are unused; hx must arrive cleared.
+  // half of u, and xpart / upart are unused; hx is not cleared before the launch (see layout).
   const int32_t* ids;         // [M] or nullptr
   const __nv_bfloat16* emb;   // [V, H]
   const __nv_bfloat16* w_ih;  // [3*Ds, H]
@@ -122,7 +122,24 @@ struct GruParams {
   // product are not used.
   const float* x_table;
   const int32_t* x_ids;       // [M] the prefix ids (read with x_table)
+  // No clear before the launch (fused projections): the control word recording which byte range
+  // of the workspace held nothing but state words at the end of the last step (lo | hi << 32, 0 =
+  // none; every other kind of step zeroes it), this launch's hx range packed the same way, and
+  // the grid barrier word (generation << 32 | arrivals) of the clear that runs when the recorded
+  // range does not contain this launch's.  layout == nullptr: hx arrives cleared.
+  unsigned long long* layout;
+  unsigned long long layout_range;
+  unsigned long long* clear_bar;
 };
+// Packs a workspace byte range [lo, hi) the way GruParams::layout holds it.
+inline unsigned long long hx_range(size_t lo, size_t hi) {
+  return static_cast<unsigned long long>(lo) | (static_cast<unsigned long long>(hi) << 32);
+}
+// Failure-detection test hook (domino_debug_hold): while armed, GRU CTA `cta` withholds one
+// thing its peers wait for -- kHoldPublish: its states of position `step`; kHoldClearBarrier: its
+// arrival at the clear barrier -- so their bounded waits run out.  The held CTA disarms it.
+constexpr int kHoldOff = 0, kHoldPublish = 1, kHoldClearBarrier = 2;
+cudaError_t arm_gru_hold(int what, int cta, int step);
 // Largest number of (rank row, position) pairs of u one warp finalises for which the fused
 // projections apply (their hidden halves wait in shared memory).
 constexpr int kGruMaxUPairs = 8;

@@ -127,3 +127,21 @@ def test_rollout_rejects_bad_sizes_before_any_device_work():
     assert f(1, 4, 256, 100, 60, 64) == 0       # d_s not a multiple of 8
     assert binding.domino_rollout_greedy(None, None, None, None, 1, 4, 256, 100, None, None, None, 0) == \
         binding.DOMINO_ERR_INVALID_ARG
+
+
+def test_debug_hold_argument_checks_and_header_constants():
+    """The failure-detection hook refuses unknown kinds and negative CTAs / positions before any
+    device call, and its constants match the header's."""
+    _lib()
+    with open(os.path.join(ROOT, "include", "domino.h")) as f:
+        text = f.read()
+    for name in ("DOMINO_HOLD_OFF", "DOMINO_HOLD_STATE", "DOMINO_HOLD_CLEAR_BARRIER"):
+        m = re.search(name + r"\s*=\s*(\d+)", text)
+        assert m and int(m.group(1)) == getattr(binding, name), name
+    bad = binding.DOMINO_ERR_INVALID_ARG
+    assert binding.domino_debug_hold(7, 0, 0) == bad
+    assert binding.domino_debug_hold(-1, 0, 0) == bad
+    assert binding.domino_debug_hold(binding.DOMINO_HOLD_STATE, -1, 0) == bad
+    assert binding.domino_debug_hold(binding.DOMINO_HOLD_STATE, 0, -1) == bad
+    assert binding.domino_debug_hold(binding.DOMINO_HOLD_STATE, 0, 64) == bad
+    assert binding.domino_debug_hold(binding.DOMINO_HOLD_CLEAR_BARRIER, -3) == bad
