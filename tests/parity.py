@@ -10,7 +10,7 @@ Rules (floating point: bf16 inputs, fp32 accumulation on the GPU, fp64 in the or
     the GPU's own top-k lists) of the anchor or of an earlier pick, and its oracle cumulative
     score must be within GAP of the best such candidate; where the best candidate leads by more
     than GAP the pick is that candidate.  GPU scores match the oracle's cumulative score of the
-    same path within LOGP_TOL per level.
+    same path within LOGP_TOL (the same bound as a single log-prob, at every depth).
 Differences that these rules excuse are counted and returned.
 """
 from __future__ import annotations
@@ -77,7 +77,8 @@ def check_tree(par, tok, dep, score, gpu_topk_ids, logp_full, K, N, logp_tol=LOG
         if len(ranked) > 1 and ranked[0][0] - ranked[1][0] > gap:
             assert (ranked[0][1], ranked[0][2]) == (p, t), f"node {i}: clear best not picked"
         if score is not None:
-            assert abs(float(score[i]) - mine) <= logp_tol * d, f"node {i}: score {score[i]:.5f} vs {mine:.5f}"
+            assert abs(float(score[i]) - mine) <= logp_tol, (
+                f"node {i} (depth {d}): score {score[i]:.5f} vs oracle path score {mine:.5f}")
         oscore.append(mine)
         picked.add((p, t))
         expanded.append((i, d, mine))

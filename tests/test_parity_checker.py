@@ -85,8 +85,14 @@ def test_tree_mistakes_fail():
     p[1] = 1
     with pytest.raises(AssertionError):
         check_tree(p, tok, dep, sc, ids, lp, K, N)
-    # a cumulative score off by more than the tolerance
+    # a cumulative score off by more than the tolerance, at the deepest node: the bound does not
+    # grow with depth
     s = sc.copy()
-    s[3] += 3 * LOGP_TOL * dep[3]
+    deep = int(np.argmax(dep))
+    assert dep[deep] >= 2
+    s[deep] += 1.5 * LOGP_TOL
     with pytest.raises(AssertionError):
         check_tree(par, tok, dep, s, ids, lp, K, N)
+    s = sc.copy()
+    s[deep] += 0.5 * LOGP_TOL
+    check_tree(par, tok, dep, s, ids, lp, K, N)
