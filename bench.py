@@ -16,8 +16,13 @@ e2e     the same metric through domino_draft_step_host: per step, hidden + prefi
         copied from pinned host memory and the top-k lists and tree are copied back.
 roofline  the dominant kernel (vocabulary GEMM + softmax/top-k): algorithmic bytes (or
         FLOPs) per launch / its mean CUDA-event duration in the timed region.
-Multi-GPU: one process per GPU (torchrun); each rank runs its own independent draft step
-(sequences are independent problems), no collective on the data path: weak scaling.
+configs the other Qwen3-shaped workloads (1.7B B=1, 8B B=32, 32B B=64) timed the same way in
+        the same run: us per step, blocks/s, the vocabulary kernel's roofline (HBM-bound at
+        B=1, tensor-bound against the sustained bf16 peak at B=32/64), the step roofline and
+        the per-kernel breakdown.
+One GPU only: the library is a single-GPU library (its vocabulary GEMM shares weight tiles
+between the CTAs of a cluster by TMA multicast, which only 1-GPU runs may use), so a launch
+with WORLD_SIZE > 1 or --gpus > 1 prints a line saying so and runs nothing.
 """
 from __future__ import annotations
 
@@ -56,20 +61,16 @@ def dist_env():
     return rank, world, local
 
 
-def max_over_ranks(x: float, world: int, device) -> float:
-    """The slowest rank's value (replicas: the job ends when its slowest rank does)."""
-    if world <= 1:
-        return x
-    import torch
-    import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device=device)
-    dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    return float(t.item())
+EXTRA_CONFIGS = ("qwen3-1.7b", "qwen3-8b-b32", "qwen3-32b-b64")
+SINGLE_GPU = ("one GPU only: the library's vocabulary GEMM shares weight tiles within a CTA cluster by TMA "
+              "multicast, which only 1-GPU runs may use; run bench.py without torchrun and --gpus 1")
 
 
-def job_throughput(world: int, blocks_per_rank_step: int, steps: int, seconds: float) -> float:
-    """Whole-job draft blocks/s: every rank ran `steps` steps of `blocks_per_rank_step` blocks."""
-    return world * blocks_per_rank_step * steps / seconds
+def single_gpu_refusal(world: int, gpus: int):
+    """The line a multi-GPU launch prints instead of running (None for a 1-GPU launch)."""
+    if world <= 1 and gpus <= 1:
+        return None
+    return {"metric": METRIC, "unit": UNIT, "n_gpus": max(world, gpus), "unavailable": SINGLE_GPU}
 
 
 def load_peaks():
@@ -241,7 +242,7 @@ def cpu_baseline(wl, budget_s=12.0):
 def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
-        return 0
+        return 0  # under torchrun the oracle runs on rank 0 alone
     import numpy as np
     import oracle
     from paper_2605_29707_gb300 import inputs
@@ -288,7 +289,7 @@ def run_reference(args):
     line = {"impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(sec_step * 1e3, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": config_dict(c, world),
+            "config": config_dict(c),
             "cpu_baseline": {"value": round(value, 4), "unit": UNIT, "cores": cores, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": round(value, 4), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -296,11 +297,11 @@ def run_reference(args):
     return 0
 
 
-def config_dict(c, world):
+def config_dict(c):
     return {"workload": f"{c.name}: B={c.B} K={c.K} H={c.H} V={c.V} d_s={c.Ds} r={c.R} k={c.k} N={c.N}",
             "B": c.B, "K": c.K, "H": c.H, "V": c.V, "d_s": c.Ds, "r": c.R, "k": c.k, "N": c.N,
-            "parallelism": f"replicas x{world} (independent sequences per GPU)",
-            "l2": "no flush: weights (W_lm alone 1.2 GB at H=4096) exceed the 129 MB L2"}
+            "parallelism": "one GPU",
+            "l2": f"no flush: the weights ({c.V * c.H * 2 / 1e9:.2f} GB of W_lm alone) exceed the 129 MB L2"}
 
 
 # ---------------------------------------------------------------------------- our arm
@@ -496,16 +497,89 @@ def graph_replay(st, hidden, ids, device, n, blocks_per_step):
         return {"error": str(e).splitlines()[0][:200]}
 
 
+def per_kernel(st, hidden, ids, stream, n, launches):
+    """Per-kernel device time of n steps, each kernel bracketed by an event pair (the library's
+    timing hooks): {kind: (total ms, launches)}.  Events between launches serialise the
+    GRU / vocabulary-GEMM overlap, so step times come from time_steps, not from this."""
+    import torch
+    from paper_2605_29707_gb300 import binding
+    torch.cuda.synchronize()
+    binding.domino_timing_begin(n * launches)
+    bad = False
+    for _ in range(n):
+        bad |= st.enqueue(hidden, ids, stream) != 0
+    torch.cuda.synchronize()
+    kern = binding.domino_timing_end()
+    if bad:
+        raise RuntimeError("a step of the per-kernel region returned an error")
+    return kern
+
+
+def vocab_roofline(c, kern, num_sms, peaks, has_b2, n):
+    """Roofline entry of the vocabulary kernel from its mean event-timed launch."""
+    vw = vocab_work(c, num_sms, has_b2=has_b2)
+    vk_ms, vk_n = kern["vocab_gemm_softmax_topk"]
+    vk_mean = vk_ms / max(1, vk_n)
+    roof = roofline_entry(vw["bytes"], vw["flops"], vk_mean, peaks, sustained=True)
+    traffic, traffic_note = traffic_for(c.name)
+    roof.update({"kernel": "vocab_gemm_softmax_topk", "traffic": traffic,
+                 "algorithmic_bytes_per_launch": vw["bytes"], "algorithmic_flops_per_launch": vw["flops"],
+                 "mean_launch_us": round(vk_mean * 1e3, 2), "launches": vk_n, "traffic_note": traffic_note,
+                 "timing": f"CUDA events around each launch, {n} steps right after the timed region",
+                 "share_of_step": round(vk_ms / max(1e-9, sum(v[0] for v in kern.values())), 4)})
+    return roof
+
+
+def step_roofline(c, peaks, us):
+    sw = step_work(c)
+    t = max(sw["bytes"] / (peaks["hbm_gbs"] * 1e9), sw["flops"] / (peaks["bf16_tflops_sustained"] * 1e12))
+    return {"us": round(t * 1e6, 2), "frac": round(t / (us * 1e-6), 4), "bytes": sw["bytes"], "flops": sw["flops"],
+            "note": "max(every weight once / HBM peak, FLOPs / sustained bf16 peak)"}
+
+
+def measure_config(name, device, stream, steps, warmup, num_sms, peaks):
+    """One more workload in the same run: µs per step (CUDA events around `steps` back-to-back
+    steps, clocks sampled meanwhile), the per-kernel breakdown, the vocabulary kernel's roofline,
+    the step roofline and the step with the correction branch off."""
+    import torch
+    from paper_2605_29707_gb300 import binding, inputs
+    from paper_2605_29707_gb300.step import DraftStep
+    wl = inputs.make_workload(name)
+    c = wl.cfg
+    st = DraftStep(wl.weights, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=device)
+    hidden = dev_bf16(wl.hidden, device)
+    ids = torch.from_numpy(wl.prefix_ids).to(device)
+    sampler = ClockSampler(device.index or 0)
+    sampler.start()
+    us = time_steps(st, hidden, ids, stream, steps, warmup)
+    clocks = sampler.stop()
+    rc = binding.domino_check_status(st.workspace, stream)
+    if rc != 0:
+        raise binding.DominoError(rc, f"{name}: device status")
+    n = min(steps, 200)
+    kern = per_kernel(st, hidden, ids, stream, n, st.launches_per_step())
+    st_off = DraftStep(st.w, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=device, head_on=False)
+    us_off = time_steps(st_off, hidden, ids, stream, steps, warmup)
+    del st_off
+    out = {"config": config_dict(c), "us_per_step": round(us, 2), "value": round(c.B * 1e6 / us, 3), "unit": UNIT,
+           "steps": steps, "warmup": max(3, warmup), "gpu_launches": steps * st.launches_per_step(),
+           "roofline": vocab_roofline(c, kern, num_sms, peaks, wl.weights.get("b2") is not None, n),
+           "step_roofline": step_roofline(c, peaks, us),
+           "kernel_breakdown": {k: {"us_per_step": round(v[0] / n * 1e3, 2), "launches": v[1]}
+                                for k, v in kern.items() if v[1] > 0},
+           "head_overhead": {"us_head_off": round(us_off, 2), "overhead_us": round(us - us_off, 2),
+                             "overhead_pct": round(100.0 * (us / us_off - 1.0), 2)},
+           "clocks": clocks}
+    del st, hidden, ids, wl
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_ours(args):
     import numpy as np
     import torch
-    import torch.distributed as dist
 
-    rank, world, local = dist_env()
-    if world > 1:
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo", init_method="env://")
-    device = torch.device("cuda", local if world > 1 else 0)
+    device = torch.device("cuda", 0)
     torch.cuda.set_device(device)
 
     from paper_2605_29707_gb300 import binding, inputs
@@ -520,10 +594,6 @@ def run_ours(args):
     launches = st.launches_per_step()
     num_sms = torch.cuda.get_device_properties(device).multi_processor_count
 
-    def barrier():
-        if world > 1:
-            dist.barrier()
-
     for _ in range(args.warmup):
         rc = st.enqueue(hidden, ids, stream)
         if rc != 0:
@@ -533,9 +603,8 @@ def run_ours(args):
         raise binding.DominoError(rc, "warm-up device status")
 
     # ---- timed region: exactly K steps, CUDA events on the launching stream
-    sampler = ClockSampler(local)
+    sampler = ClockSampler(0)
     sampler.start()
-    barrier()
     torch.cuda.synchronize(device)
     ev0 = torch.cuda.Event(enable_timing=True)
     ev1 = torch.cuda.Event(enable_timing=True)
@@ -545,7 +614,6 @@ def run_ours(args):
         bad |= st.enqueue(hidden, ids, stream) != 0
     ev1.record(stream)
     torch.cuda.synchronize(device)
-    barrier()
     clocks = sampler.stop()
     if bad:
         raise RuntimeError("a timed step returned an error")
@@ -555,20 +623,11 @@ def run_ours(args):
     ms = ev0.elapsed_time(ev1)
 
     # ---- second timed region: the same steps with an event pair around every kernel (the
-    #      per-kernel breakdown and the roofline).  Events between launches serialise the
-    #      GRU / vocabulary-GEMM overlap, so the step value comes from the region above.
+    #      per-kernel breakdown and the roofline)
     k_steps = min(args.steps, 1000)
-    torch.cuda.synchronize(device)
-    binding.domino_timing_begin(k_steps * launches)
-    for _ in range(k_steps):
-        bad |= st.enqueue(hidden, ids, stream) != 0
-    torch.cuda.synchronize(device)
-    kern = binding.domino_timing_end()
-    if bad:
-        raise RuntimeError("a step of the per-kernel region returned an error")
-    ms = max_over_ranks(ms, world, device)
+    kern = per_kernel(st, hidden, ids, stream, k_steps, launches)
     ms_step = ms / args.steps
-    value = job_throughput(world, c.B, args.steps, ms / 1e3)
+    value = c.B * args.steps / (ms / 1e3)
 
     # ---- e2e through the host-buffer entry point (pinned inputs and outputs)
     M = c.M
@@ -583,15 +642,13 @@ def run_ours(args):
     n_e2e = max(3, min(args.steps, 1000))
     for _ in range(3):
         st.run_host(h_hidden, h_ids, host, stream)
-    barrier()
     t0 = time.perf_counter()
     for _ in range(n_e2e):
         rc = st.run_host(h_hidden, h_ids, host, stream)
         if rc != 0:
             raise binding.DominoError(rc, "host-buffer step")
     t_e2e = time.perf_counter() - t0
-    t_e2e = max_over_ranks(t_e2e, world, device)
-    e2e_value = job_throughput(world, c.B, n_e2e, t_e2e)
+    e2e_value = c.B * n_e2e / t_e2e
     h2d = M * c.H * 2 + M * 4
     # the host entry point reads its outputs (top-k ids and log-probs, the four tree arrays) and a
     # copy of the status in one copy of the workspace region that holds them (256-byte aligned)
@@ -633,30 +690,17 @@ def run_ours(args):
     # ---- roofline of the dominant kernel, measured in the timed region
     peaks = load_peaks()
     dominant = max(kern, key=lambda n: kern[n][0])
-    vw = vocab_work(c, num_sms, has_b2=wl.weights.get("b2") is not None)
-    vk_ms, vk_n = kern["vocab_gemm_softmax_topk"]
-    vk_mean = vk_ms / max(1, vk_n)
-    roof = roofline_entry(vw["bytes"], vw["flops"], vk_mean, peaks, sustained=True)
-    traffic, traffic_note = traffic_for(c.name)
-    roof.update({"kernel": "vocab_gemm_softmax_topk", "traffic": traffic,
-                 "algorithmic_bytes_per_launch": vw["bytes"], "algorithmic_flops_per_launch": vw["flops"],
-                 "mean_launch_us": round(vk_mean * 1e3, 2), "launches": vk_n, "traffic_note": traffic_note,
-                 "timing": f"CUDA events around each launch, {k_steps} steps right after the timed region",
-                 "share_of_step": round(vk_ms / max(1e-9, sum(v[0] for v in kern.values())), 4)})
-    sw = step_work(c)
-    step_roof = max(sw["bytes"] / (peaks["hbm_gbs"] * 1e9), sw["flops"] / (peaks["bf16_tflops_sustained"] * 1e12))
+    roof = vocab_roofline(c, kern, num_sms, peaks, wl.weights.get("b2") is not None, k_steps)
     breakdown = {n: {"us_per_step": round(v[0] / k_steps * 1e3, 2), "launches": v[1]} for n, v in kern.items()
                  if v[1] > 0}
 
     line = {
-        "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms_step, 5), "us_per_step": round(ms_step * 1e3, 2),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic (seeded, Qwen3-shaped, random-init weights)", "config": config_dict(c, world),
+        "data": "synthetic (seeded, Qwen3-shaped, random-init weights)", "config": config_dict(c),
         "roofline": roof,
-        "step_roofline": {"us": round(step_roof * 1e6, 2), "frac": round(step_roof / (ms_step * 1e-3), 4),
-                          "bytes": sw["bytes"], "flops": sw["flops"],
-                          "note": "max(every weight once / HBM peak, FLOPs / sustained bf16 peak)"},
+        "step_roofline": step_roofline(c, peaks, ms_step * 1e3),
         "kernel_breakdown": breakdown, "dominant_kernel": dominant,
         "e2e": {"value": round(e2e_value, 3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "steps": n_e2e, "api": "domino_draft_step_host (synchronous per step)"},
@@ -665,15 +709,22 @@ def run_ours(args):
         "tree_verify": verify,
         "rollout_greedy": rollout,
     }
-    # ---- last: the same step replayed from a CUDA graph (one captured step, replayed back to
-    #      back); a failed capture is reported in the line, after everything else was measured
-    line["graph_replay"] = graph_replay(st, hidden, ids, device, min(args.steps, 1000), c.B * world)
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    # ---- last for this workload: the same step replayed from a CUDA graph (one captured step,
+    #      replayed back to back); a failed capture is reported in the line
+    line["graph_replay"] = graph_replay(st, hidden, ids, device, min(args.steps, 1000), c.B)
+    del st, hidden, ids
+    torch.cuda.empty_cache()
+    # ---- the other Qwen3-shaped workloads: 1.7B at B = 1 (HBM-bound), the 8B and 32B serving
+    #      batches (tensor-bound), each timed the same way
+    if args.extra_configs:
+        line["configs"] = {}
+        for name in args.extra_configs.split(","):
+            if name and name != c.name:
+                steps = max(20, min(args.steps, 2000 // max(1, inputs.CONFIGS[name].B)))
+                line["configs"][name] = measure_config(name, device, stream, steps, args.warmup, num_sms, peaks)
+    if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, args.cpu_seconds)
-    if rank == 0:
-        print(json.dumps(line), flush=True)
-    if world > 1:
-        dist.destroy_process_group()
+    print(json.dumps(line), flush=True)
     return 0
 
 
@@ -686,11 +737,19 @@ def main():
     ap.add_argument("--config", default=DEFAULT_CONFIG)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--extra-configs", default=",".join(EXTRA_CONFIGS),
+                    help="other workloads timed in the same run (comma-separated; empty for none)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
     if args.impl == "reference":
         return run_reference(args)
+    rank, world, _ = dist_env()
+    refusal = single_gpu_refusal(world, args.gpus)
+    if refusal is not None:
+        if rank == 0:
+            print(json.dumps(refusal), flush=True)
+        return 0
     return run_ours(args)
 
 

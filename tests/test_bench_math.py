@@ -45,3 +45,29 @@ def test_roofline_takes_the_slower_of_memory_and_tensor_time():
     # 3 PFLOP in 2 s against the sustained 1500 TFLOP/s: tensor-bound, frac 1.0
     r = bench.roofline_entry(1e6, 3e15, 2000.0, peaks, sustained=True)
     assert r["bound"] == "tensor" and r["frac"] == pytest.approx(1.0) and r["unit"] == "TFLOP/s"
+
+
+def test_multi_gpu_launch_is_refused_without_running():
+    """The library is single-GPU (its vocabulary GEMM multicasts weight tiles within a cluster,
+    which only 1-GPU runs may use): a torchrun launch or --gpus > 1 prints one 'unavailable' line
+    from rank 0, the other ranks print nothing, and nothing runs."""
+    import json
+    import os
+    import subprocess
+    import sys
+
+    assert bench.single_gpu_refusal(1, 1) is None
+    line = bench.single_gpu_refusal(2, 1)
+    assert line["unavailable"] and line["n_gpus"] == 2
+    assert bench.single_gpu_refusal(1, 4)["n_gpus"] == 4
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    for rank, expect in (("0", True), ("1", False)):
+        env = dict(os.environ, WORLD_SIZE="2", RANK=rank, LOCAL_RANK=rank)
+        r = subprocess.run([sys.executable, os.path.join(root, "bench.py"), "--gpus", "2", "--steps", "3"],
+                           env=env, capture_output=True, text=True, timeout=120)
+        assert r.returncode == 0, r.stderr
+        out = [ln for ln in r.stdout.splitlines() if ln.strip()]
+        if expect:
+            assert len(out) == 1 and json.loads(out[0])["unavailable"] == bench.SINGLE_GPU
+        else:
+            assert out == []
