@@ -55,7 +55,8 @@ int oracle_max_threads(void) {
 #endif
 }
 
-/* O1: E[i] = emb[ids[i]] (section 4.1.2, "E_j denotes the token embedding"). */
+/* O1: E[i] = emb[ids[i]]: the GRU input at a position is the embedding row of the token there
+   (section 4.1.2, causal encoder equation). */
 int oracle_embed(const uint16_t* emb, int V, int H, const int32_t* ids, int n, double* E) {
   if (!emb || !ids || !E || V <= 0 || H <= 0 || n < 0) return ORACLE_ERR_ARG;
   for (int i = 0; i < n; ++i) {
@@ -176,7 +177,7 @@ static int ranks_before(double va, int ia, double vb, int ib) {
   return va > vb || (va == vb && ia < ib);
 }
 
-/* O6: k passes of "take the best remaining entry" under (value desc, id asc). */
+/* O6: k passes, each taking the best entry not yet taken under (value desc, id asc). */
 int oracle_topk(const double* logp, int n, int V, int k, int32_t* ids, double* vals) {
   if (!logp || !ids || !vals || n < 0 || V <= 0 || k <= 0 || k > V) return ORACLE_ERR_ARG;
   unsigned char* taken = (unsigned char*)malloc((size_t)V);
@@ -319,7 +320,8 @@ int oracle_draft_step(const uint16_t* hidden, const int32_t* prefix_ids, const u
   return rc;
 }
 
-/* O8: greedy verification of one tree (section 3.1, "accepts the longest valid prefix"). */
+/* O8: greedy verification of one tree (section 3.1): the target checks the whole draft at once and
+   keeps the draft tokens up to the first one it would not have produced itself. */
 int oracle_verify_greedy(const float* target, int N, int V, const int32_t* parent, const int32_t* token,
                          int32_t* row_argmax, int32_t* nodes, int32_t* n_acc, int32_t* bonus) {
   if (!target || !row_argmax || !nodes || !n_acc || !bonus || N < 0 || V <= 0) return ORACLE_ERR_ARG;

@@ -95,9 +95,9 @@ int oracle_draft_step(const uint16_t* hidden, const int32_t* prefix_ids, const u
                       int32_t* tree_parent, int32_t* tree_token, int32_t* tree_depth,
                       double* tree_score, int nthreads);
 
-/* O8, the step after the draft (section 3.1: the target model evaluates the draft in one pass
- * and "accepts the longest valid prefix"; tau counts the accepted tokens plus the bonus token
- * the target produces).  Greedy verification of one draft tree at temperature 0, where a draft
+/* O8, the step after the draft (section 3.1: one target pass checks the whole draft, the draft
+ * tokens are kept up to the first one the target rejects, and tau counts the kept tokens plus
+ * the one extra token the target itself contributes).  Greedy verification of one draft tree at temperature 0, where a draft
  * token is valid when it equals the target's most likely next token:
  *   parent/token [N]: the tree (parent -1 = the anchor, otherwise an earlier node), as from
  *     oracle_tree; target [N+1, V] fp32: the target's next-token logits after the anchor
@@ -126,8 +126,8 @@ int oracle_rollout_greedy(const uint16_t* hidden, const int32_t* anchors, const 
                           int H, int V, int Ds, int R, const int32_t* seqs, int nseq, int32_t* tokens,
                           double* logp, int nthreads);
 
-/* O10, the same loop with each token sampled from the final distribution (section 4.1.2: "each
- * draft token is sampled from the final logits"): with u_j = uniforms[b * K + j] in [0, 1)
+/* O10, the same loop with each token sampled from the final distribution (section 4.1.2 and
+ * Fig. 3: every draft token is drawn from the refined logits l_i + c_i): with u_j = uniforms[b * K + j] in [0, 1)
  * (the caller's random draws), t_{j+1} = the first id v whose cumulative probability
  * sum_{v' <= v} softmax(L_j)[v'] (in id order) exceeds u_j; a u_j at or past the rounded total
  * takes the last id of non-zero probability.  logp_j = log-softmax(L_j)[t_{j+1}].  Returns

@@ -1,6 +1,6 @@
 // verify.cu -- greedy verification of a draft tree against the target's logits (the step after
-// the draft, section 3.1: the target evaluates the draft in one pass and accepts the longest
-// valid prefix; tau counts the accepted tokens plus the bonus token the target produces).
+// the draft, section 3.1: one target pass checks the whole draft, draft tokens are kept up to the
+// first one the target rejects, and tau counts them plus the target's own extra token).
 //
 // Row argmax: a cluster of kSplit CTAs per row of target logits (the target's next-token logits
 // after the anchor, row 0, and after each tree node i, row i + 1); each CTA finds the greatest

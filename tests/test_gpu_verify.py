@@ -1,8 +1,8 @@
 """Greedy tree verification on the GPU (domino_verify_tree_greedy) against the oracle.
 
-Section 3.1: the target model evaluates the draft in one pass and accepts the longest valid
-prefix; at temperature 0 a draft token is valid when it equals the target's most likely next
-token.  The argmax decisions are taken on the same fp32 logits on both sides, so every output
+Section 3.1: one target pass checks the whole draft and the draft tokens are kept up to the
+first one the target rejects; at temperature 0 a draft token is kept when it equals the target's
+most likely next token.  The argmax decisions are taken on the same fp32 logits on both sides, so every output
 (row argmaxes, accepted nodes, their count, the bonus token) must match exactly.
 """
 import numpy as np
