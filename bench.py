@@ -575,6 +575,32 @@ def measure_config(name, device, stream, steps, warmup, num_sms, peaks):
     return out
 
 
+def run_step_only(args):
+    """Only the draft step of one workload (W warm-up + K timed steps, then one greedy tree
+    verification when B <= 4): a short, fixed launch sequence for profiler captures.  Prints one
+    JSON line with the step time; not a benchmark line."""
+    import torch
+    from paper_2605_29707_gb300 import binding, inputs
+    from paper_2605_29707_gb300.step import DraftStep
+    device = torch.device("cuda", 0)
+    torch.cuda.set_device(device)
+    wl = inputs.make_workload(args.config)
+    c = wl.cfg
+    st = DraftStep(wl.weights, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=device)
+    hidden = dev_bf16(wl.hidden, device)
+    ids = torch.from_numpy(wl.prefix_ids).to(device)
+    stream = torch.cuda.current_stream(device)
+    us = time_steps(st, hidden, ids, stream, args.steps, args.warmup)
+    rc = binding.domino_check_status(st.workspace, stream)
+    if rc != 0:
+        raise binding.DominoError(rc, "device status")
+    verify = verify_timing(st, c, device, stream, reps=3) if c.B <= 4 else None
+    print(json.dumps({"step_only": c.name, "us_per_step": round(us, 2), "launches_per_step": st.launches_per_step(),
+                      "steps": args.steps, "warmup": max(3, args.warmup),
+                      "verify_us": verify["us"] if verify else None}), flush=True)
+    return 0
+
+
 def run_ours(args):
     import numpy as np
     import torch
@@ -739,6 +765,9 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--extra-configs", default=",".join(EXTRA_CONFIGS),
                     help="other workloads timed in the same run (comma-separated; empty for none)")
+    ap.add_argument("--step-only", action="store_true",
+                    help="run only the step of --config (warm-up, steps, one verification at B <= 4): "
+                         "a short launch sequence for profiler captures; prints no benchmark line")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -750,7 +779,7 @@ def main():
         if rank == 0:
             print(json.dumps(refusal), flush=True)
         return 0
-    return run_ours(args)
+    return run_step_only(args) if args.step_only else run_ours(args)
 
 
 if __name__ == "__main__":
