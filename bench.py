@@ -595,9 +595,12 @@ def run_step_only(args):
     if rc != 0:
         raise binding.DominoError(rc, "device status")
     verify = verify_timing(st, c, device, stream, reps=3) if c.B <= 4 else None
+    kern = per_kernel(st, hidden, ids, stream, args.steps, st.launches_per_step())
     print(json.dumps({"step_only": c.name, "us_per_step": round(us, 2), "launches_per_step": st.launches_per_step(),
                       "steps": args.steps, "warmup": max(3, args.warmup),
-                      "verify_us": verify["us"] if verify else None}), flush=True)
+                      "verify_us": verify["us"] if verify else None,
+                      "us_per_kernel": {k: round(v[0] / max(1, v[1]) * 1e3, 2) for k, v in kern.items() if v[1]}}),
+          flush=True)
     return 0
 
 
