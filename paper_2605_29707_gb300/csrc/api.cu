@@ -488,7 +488,8 @@ int run_step_launches(const Plan& P, const void* hidden, const int32_t* ids, con
       gr.V = V;
     }
     ts = timing_open(DOMINO_KERNEL_GRU, st);
-    rc = cuda_rc(dm::launch_gru(gr, P.gru, st, P.chain && !P.fused));
+    // no vocabulary CTA shares the GRU's SMs unless the two overlap
+    rc = cuda_rc(dm::launch_gru(gr, P.gru, st, P.chain && !P.fused, !P.overlap));
     timing_close(ts, st);
     if (rc) return rc;
     if (!P.u_in_gru) {

@@ -345,8 +345,14 @@ __device__ void fused_projections(const GruParams& p, int j0, int Uc, int b0, in
 // GEMM CTA (at most 168 registers x 192 threads) fit in one SM's register file.
 // kTable: the input-gate sums come from the input-projection table (p.x_table) rather than
 // from xs (a separate instantiation, so that the path without a table keeps its registers).
-template <bool kTable>
-__global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) {
+// kWide: a launch that shares no SM with the vocabulary GEMM (large batches): the register
+// budget of one CTA per SM, so that a lane issues all 16 of its state loads of a step at once
+// (one L2 round trip instead of two at 16 sequences per CTA), and the steps read the input-gate
+// sums as split-K partial sums of the X GEMM directly (prefetched before each step's wait)
+// instead of a prologue pass that first sums them into xs.
+template <bool kTable, bool kWide>
+__global__ void __launch_bounds__(kGruThreads, kWide ? 1 : 2) gru_kernel(const GruParams p) {
+  constexpr int kPollBatch = kWide ? 16 : 8;  // state loads a lane issues before checking tags
   extern __shared__ __align__(16) uint8_t gsmem[];
   const int U = p.units, Ds = p.Ds, K = p.K, B = p.B, R = p.R, H = p.H;
   const int M = B * K;
@@ -432,7 +438,8 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
   asm volatile("griddepcontrol.wait;" ::: "memory");
   // ---- input-gate sums b_ih + E . W_ih^T for this CTA's rows and units, spread over all
   //      threads (made visible to the CTA by the barrier below)
-  const int xs_count = kTable ? 0 : nbc * K * 3 * Uc;  // with a table the steps read its rows
+  // with a table the steps read its rows; wide launches read the partial sums at each step
+  const int xs_count = (kTable || kWide) ? 0 : nbc * K * 3 * Uc;
   for (int e0 = tid; e0 < xs_count; e0 += 4 * kGruThreads) {
     float a[4];
     size_t at[4];
@@ -485,14 +492,23 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
           // outside [0, V), reported by the id check, reads row 0)
           const float* x = p.xs + m * 3 * Ds;  // written by this kernel: plain loads
           const __nv_bfloat16* xbias = nullptr;
+          int nsplit = 1;
+          size_t split_stride = 0;
           if (kTable) {
             const int id = p.x_ids[m];
             x = p.x_table + static_cast<size_t>(id >= 0 && id < p.V ? id : 0) * 3 * Ds;
             xbias = p.b_ih;
+          } else if (kWide) {  // the X GEMM's split-K partial sums, summed here
+            x = p.xpart + m * 3 * Ds;
+            xbias = p.b_ih;
+            nsplit = p.xsplits;
+            split_stride = static_cast<size_t>(M) * 3 * Ds;
           }
 #pragma unroll
           for (int g = 0; g < 3; ++g) {
-            gx[r][g] = x[g * Ds + j] + bf_or0(xbias, g * Ds + j);
+            float xv = x[g * Ds + j];
+            for (int s = 1; s < nsplit; ++s) xv += x[s * split_stride + g * Ds + j];
+            gx[r][g] = xv + bf_or0(xbias, g * Ds + j);
             gb[r][g] = bf_or0(p.b_hh, g * Ds + j);
           }
         }
@@ -507,10 +523,10 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
         const int ncq = max(0, q1 - q0);
         const int total = nb * ncq;
         bool got = true;
-        for (int e0 = lane; e0 < total && got; e0 += 8 * 32) {
-          uint4 v[8];
+        for (int e0 = lane; e0 < total && got; e0 += kPollBatch * 32) {
+          uint4 v[kPollBatch];
 #pragma unroll
-          for (int i = 0; i < 8; ++i) {  // issue every load first, then check the flags
+          for (int i = 0; i < kPollBatch; ++i) {  // issue every load first, then check the flags
             const int e = e0 + i * 32;
             if (e < total) {
               const size_t m = static_cast<size_t>(b0 + c0 + e / ncq) * K + (t - 1);
@@ -518,7 +534,7 @@ __global__ void __launch_bounds__(kGruThreads, 2) gru_kernel(const GruParams p) 
             }
           }
 #pragma unroll
-          for (int i = 0; i < 8; ++i) {
+          for (int i = 0; i < kPollBatch; ++i) {
             const int e = e0 + i * 32;
             if (e < total && got) {
               const int bb = e / ncq, cq = q0 + e % ncq;
@@ -702,10 +718,11 @@ GruPlan gru_plan(int B, int Ds, int num_sms) {
   return g;
 }
 
-template <bool kTable>
+template <bool kTable, bool kWide>
 static cudaError_t launch_gru_t(const GruParams& p, const GruPlan& plan, cudaStream_t stream, bool pdl) {
   {
-    const cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(gru_kernel<kTable>), plan.smem, true);
+    const cudaError_t e =
+        ensure_smem_attr(reinterpret_cast<const void*>(gru_kernel<kTable, kWide>), plan.smem, true);
     if (e != cudaSuccess) return e;
   }
   cudaLaunchConfig_t cfg = {};
@@ -722,20 +739,23 @@ static cudaError_t launch_gru_t(const GruParams& p, const GruPlan& plan, cudaStr
   // A runtime that refuses the pair gets the cooperative launch alone from then on.
   static std::atomic<bool> pdl_refused{false};
   cfg.numAttrs = (pdl && !pdl_refused) ? 2 : 1;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, gru_kernel<kTable>, p);
+  cudaError_t e = cudaLaunchKernelEx(&cfg, gru_kernel<kTable, kWide>, p);
   if (e != cudaSuccess && cfg.numAttrs == 2) {
     (void)cudaGetLastError();
     pdl_refused = true;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, gru_kernel<kTable>, p);
+    e = cudaLaunchKernelEx(&cfg, gru_kernel<kTable, kWide>, p);
   }
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
-cudaError_t launch_gru(const GruParams& p, const GruPlan& plan, cudaStream_t stream, bool pdl) {
+cudaError_t launch_gru(const GruParams& p, const GruPlan& plan, cudaStream_t stream, bool pdl, bool wide) {
   if (plan.smem == 0) return cudaErrorInvalidValue;
-  return p.x_table ? launch_gru_t<true>(p, plan, stream, pdl) : launch_gru_t<false>(p, plan, stream, pdl);
+  if (wide && p.ids != nullptr) return cudaErrorInvalidValue;  // fused projections share SMs
+  if (wide)
+    return p.x_table ? launch_gru_t<true, true>(p, plan, stream, pdl) : launch_gru_t<false, true>(p, plan, stream, pdl);
+  return p.x_table ? launch_gru_t<true, false>(p, plan, stream, pdl) : launch_gru_t<false, false>(p, plan, stream, pdl);
 }
 
 // ---------------------------------------------------------------------------- u finalize

@@ -149,8 +149,9 @@ struct GruPlan {
 };
 GruPlan gru_plan(int B, int Ds, int num_sms);
 // Cooperative launch; with pdl, also as a programmatic dependent of the preceding kernel (the
-// kernel waits for that grid before it reads the projections).
-cudaError_t launch_gru(const GruParams& p, const GruPlan& plan, cudaStream_t stream, bool pdl);
+// kernel waits for that grid before it reads the projections).  wide: the launch shares no SM
+// with the vocabulary GEMM (not with fused projections): one CTA's worth of registers per SM.
+cudaError_t launch_gru(const GruParams& p, const GruPlan& plan, cudaStream_t stream, bool pdl, bool wide);
 
 // u = bf16(SiLU(b1 + sum over splits of part)) for the large-batch path.
 struct UFinalParams {
