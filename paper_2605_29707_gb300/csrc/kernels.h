@@ -67,6 +67,10 @@ cudaError_t launch_tc_softmax_k8(int bn, bool swap, const CUtensorMap* maps, con
 cudaError_t launch_tc_softmax_deferred_k8(int bn, const CUtensorMap* maps, const TcParams& p, int grid,
                                           cudaStream_t stream);
 int tc_softmax_deferred_smem_k8(int bn);
+// Tokens on M in CTA pairs (mcast = 2, bn 256): the 2-SM MMA variant (tc_pair.cuh); the maps are
+// the same as for the multicast kernel (weight boxes 128 rows high).
+cudaError_t launch_tc_vocab_pair(int kmax, const CUtensorMap* maps, const TcParams& p, int grid, cudaStream_t stream);
+cudaError_t launch_tc_vocab_pair_k8(const CUtensorMap* maps, const TcParams& p, int grid, cudaStream_t stream);
 // Small-M (swap, bn 16..128) store-mode GEMM with four pipeline stages, launched as a
 // programmatic dependent of the preceding kernel (p.pdl_wait says where it waits for it).
 cudaError_t launch_tc_store_chained(int bn, const CUtensorMap* maps, const TcParams& p, int grid,

@@ -1,11 +1,20 @@
 // tc_softmax.cu -- instantiations of the fused vocabulary GEMM + online softmax / top-k
 // epilogue (section 4.1.1 base logits and the section 4.1.2 W2 term in one accumulator).
-#include "tc_gemm.cuh"
+#include "tc_pair.cuh"
 
 namespace dm {
 
+cudaError_t launch_tc_vocab_pair(int kmax, const CUtensorMap* maps, const TcParams& p, int grid, cudaStream_t s) {
+  if (kmax == 8) return launch_tc_vocab_pair_k8(maps, p, grid, s);
+  if (kmax == 16) return launch_tc_vocab_pair_instance<16>(maps, p, grid, s);
+  if (kmax == 32) return launch_tc_vocab_pair_instance<32>(maps, p, grid, s);
+  return cudaErrorInvalidValue;
+}
+
 cudaError_t launch_tc_softmax(int bn, bool swap, int kmax, const CUtensorMap* maps, const TcParams& p,
                               int grid, cudaStream_t s) {
+  // tokens on M in CTA pairs: the 2-SM MMA kernel (tc_pair.cuh)
+  if (!swap && bn == 256 && p.mcast == 2) return launch_tc_vocab_pair(kmax, maps, p, grid, s);
   if (kmax == 8) return launch_tc_softmax_k8(bn, swap, maps, p, grid, s);
 #define DM_SM(BN, SW, KM)                                                              \
   if (bn == BN && swap == SW && kmax == KM)                                            \

@@ -1,8 +1,12 @@
 // tc_softmax_k8.cu -- the fused vocabulary GEMM + online softmax / top-k with 8-entry lists
 // (draft branching k <= 8), compiled apart from the 16 / 32-entry variants.
-#include "tc_gemm.cuh"
+#include "tc_pair.cuh"
 
 namespace dm {
+
+cudaError_t launch_tc_vocab_pair_k8(const CUtensorMap* maps, const TcParams& p, int grid, cudaStream_t s) {
+  return launch_tc_vocab_pair_instance<8>(maps, p, grid, s);
+}
 
 cudaError_t launch_tc_softmax_k8(int bn, bool swap, const CUtensorMap* maps, const TcParams& p, int grid,
                                  cudaStream_t s) {

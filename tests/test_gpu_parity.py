@@ -72,6 +72,10 @@ SMALL = {
     "max-K": dict(B=1, K=64, H=64, V=800, Ds=32, R=16, k=3, N=40, seed=21, biases=True),
     # the longest block the fused-projection GRU takes (M = 32)
     "fused-K32": dict(B=1, K=32, H=128, V=1500, Ds=256, R=32, k=4, N=30, seed=22),
+    # tokens on M in CTA pairs (the 2-SM MMA kernel): 32-entry lists (k = 20), and a second token
+    # tile of 22 rows (M = 150) with a ragged vocabulary and biases
+    "pair-k20": dict(B=10, K=16, H=192, V=3001, Ds=64, R=64, k=20, N=24, seed=26, biases=True),
+    "pair-ragged": dict(B=10, K=15, H=136, V=2333, Ds=72, R=40, k=6, N=10, seed=27, biases=True),
 }
 
 
