@@ -45,7 +45,8 @@ METRIC = "µs per draft step & draft blocks/s (1 GB300); LM-head HBM GB/s / roof
 UNIT = "draft blocks/s"
 DEFAULT_CONFIG = "qwen3-8b"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-VOCAB_SOURCES = ["paper_2605_29707_gb300/csrc/tc_gemm.cuh", "paper_2605_29707_gb300/csrc/tc_softmax.cu",
+VOCAB_SOURCES = ["paper_2605_29707_gb300/csrc/tc_gemm.cuh", "paper_2605_29707_gb300/csrc/tc_pair.cuh",
+                 "paper_2605_29707_gb300/csrc/tc_softmax.cu", "paper_2605_29707_gb300/csrc/tc_softmax_k8.cu",
                  "paper_2605_29707_gb300/csrc/ptx.cuh", "paper_2605_29707_gb300/csrc/topk.cuh"]
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "vocab_gemm_traffic.json")
 
