@@ -22,7 +22,7 @@
 namespace dm {
 
 constexpr int kGruThreads = 256;
-constexpr int kGatePairsPerThread = 4;  // (sequence, unit) gate evaluations per thread and chunk
+constexpr int kGatePairsPerThread = 2;  // (sequence, unit) gate evaluations per thread and chunk
 constexpr int kGruWarps = kGruThreads / 32;
 constexpr int kChunkSeqs = 32;  // sequences staged per MMA pass (4 n-tiles of 8)
 constexpr int kGsmLd = kChunkSeqs + 1;  // padded row stride of the W_hh . h tile (bank spread)
@@ -473,43 +473,59 @@ __global__ void __launch_bounds__(kGruThreads, kWide ? 1 : 2) gru_kernel(const G
 
   const int nk = (Ds + 15) / 16;  // a k tail of 8 reads the zero padding columns
   bool ok = true;
+  // The biases of this thread's gate pairs do not change from step to step (pair e of a chunk is
+  // unit e % Uc).  b_ih is already in xs except when the steps read a table row or X partials.
+  float bih[kGatePairsPerThread][3], bhh[kGatePairsPerThread][3];
+#pragma unroll
+  for (int r = 0; r < kGatePairsPerThread; ++r) {
+    const int j = j0 + (Uc > 0 ? (tid + r * kGruThreads) % Uc : 0);
+#pragma unroll
+    for (int g = 0; g < 3; ++g) {
+      bih[r][g] = (kTable || kWide) ? bf_or0(p.b_ih, g * Ds + j) : 0.f;
+      bhh[r][g] = bf_or0(p.b_hh, g * Ds + j);
+    }
+  }
 
   for (int t = 0; t < K && ok; ++t) {
     for (int c0 = 0; c0 < nbc; c0 += L.chunk) {
       const int nb = min(L.chunk, nbc - c0);
       const int nt_count = (nb + 7) / 8;
       const int tiles = L.mt * nt_count;
-      // gate inputs of this step (input-gate sums, b_hh) into registers before the wait
-      float gx[kGatePairsPerThread][3], gb[kGatePairsPerThread][3];
+      // gate inputs of this step: issued as loads now and summed only at the gates, after the
+      // wait for h_{t-1}, so that no instruction stalls on them before the wait
+      constexpr int kXr = kWide ? 3 : 1;  // X partial sums held per gate (more are summed at once)
+      float gx[kGatePairsPerThread][3][kXr];
 #pragma unroll
       for (int r = 0; r < kGatePairsPerThread; ++r) {
         const int e = tid + r * kGruThreads;
+#pragma unroll
+        for (int g = 0; g < 3; ++g)
+#pragma unroll
+          for (int s = 0; s < kXr; ++s) gx[r][g][s] = 0.f;
         if (e < nb * Uc) {
           const int bb = e / Uc, jl = e % Uc;
           const int j = j0 + jl;
           const size_t m = static_cast<size_t>(b0 + c0 + bb) * K + t;
           // b_ih + W_i{r,z,n} E_m: summed into xs before the steps, or a row of the table (an id
-          // outside [0, V), reported by the id check, reads row 0)
+          // outside [0, V), reported by the id check, reads row 0), or the X GEMM's split-K partial
+          // sums (wide launches)
           const float* x = p.xs + m * 3 * Ds;  // written by this kernel: plain loads
-          const __nv_bfloat16* xbias = nullptr;
           int nsplit = 1;
           size_t split_stride = 0;
           if (kTable) {
             const int id = p.x_ids[m];
             x = p.x_table + static_cast<size_t>(id >= 0 && id < p.V ? id : 0) * 3 * Ds;
-            xbias = p.b_ih;
-          } else if (kWide) {  // the X GEMM's split-K partial sums, summed here
+          } else if (kWide) {
             x = p.xpart + m * 3 * Ds;
-            xbias = p.b_ih;
             nsplit = p.xsplits;
             split_stride = static_cast<size_t>(M) * 3 * Ds;
           }
 #pragma unroll
           for (int g = 0; g < 3; ++g) {
-            float xv = x[g * Ds + j];
-            for (int s = 1; s < nsplit; ++s) xv += x[s * split_stride + g * Ds + j];
-            gx[r][g] = xv + bf_or0(xbias, g * Ds + j);
-            gb[r][g] = bf_or0(p.b_hh, g * Ds + j);
+#pragma unroll
+            for (int s = 0; s < kXr; ++s)
+              if (s < nsplit) gx[r][g][s] = x[s * split_stride + g * Ds + j];
+            for (int s = kXr; s < nsplit; ++s) gx[r][g][0] += x[s * split_stride + g * Ds + j];  // rare
           }
         }
       }
@@ -612,16 +628,24 @@ __global__ void __launch_bounds__(kGruThreads, kWide ? 1 : 2) gru_kernel(const G
         const int j = j0 + jl;
         const int bl = c0 + bb;  // sequence index within this CTA
         const size_t m = static_cast<size_t>(b0 + bl) * K + t;
-        float hr = gb[rr][0], hz = gb[rr][1], hn = gb[rr][2];
+        float hr = bhh[rr][0], hz = bhh[rr][1], hn = bhh[rr][2];
         if (t > 0) {
           hr += gsm[static_cast<size_t>(jl) * kGsmLd + bb];
           hz += gsm[static_cast<size_t>(U + jl) * kGsmLd + bb];
           hn += gsm[static_cast<size_t>(2 * U + jl) * kGsmLd + bb];
         }
+        float xin[3];
+#pragma unroll
+        for (int g = 0; g < 3; ++g) {
+          float s = gx[rr][g][0];
+#pragma unroll
+          for (int q = 1; q < kXr; ++q) s += gx[rr][g][q];
+          xin[g] = s + bih[rr][g];
+        }
         const float hp = hprev[bl * U + jl];
-        const float r = sigmoidf_(gx[rr][0] + hr);
-        const float z = sigmoidf_(gx[rr][1] + hz);
-        const float n = tanhf(gx[rr][2] + r * hn);
+        const float r = sigmoidf_(xin[0] + hr);
+        const float z = sigmoidf_(xin[1] + hz);
+        const float n = tanhf(xin[2] + r * hn);
         const float h = (1.f - z) * n + z * hp;
         hprev[bl * U + jl] = h;
         if (held && hold.x == kHoldPublish && hold.z == t) continue;  // test hook: withheld
