@@ -808,7 +808,7 @@ struct RollPlan {
   int B, K, H, V, Ds, R, M, grid;
   bool head;
   StorePlan g;  // base-logit GEMM, no split
-  size_t off_h, off_u, off_part, off_lg, off_base, off_uh, clear_bytes, total;
+  size_t off_h, off_u, off_part, off_lg, off_base, off_uh, off_gh, clear_bytes, total;
 };
 
 int make_roll_plan(int B, int K, int H, int V, int Ds, int R, bool head, RollPlan* P) {
@@ -848,6 +848,7 @@ int make_roll_plan(int B, int K, int H, int V, int Ds, int R, bool head, RollPla
   p.off_lg = take(static_cast<size_t>(2) * B * V * 4);  // sampled mode: final logits, by step parity
   p.off_base = take(static_cast<size_t>(p.M) * V * 4);
   p.off_uh = take(static_cast<size_t>(p.M) * (p.R > 0 ? p.R : 1) * 4);  // hidden . W1[:, :H]^T
+  p.off_gh = take(static_cast<size_t>(2) * B * 3 * (p.Ds > 0 ? p.Ds : 1) * 4);  // W_hh h_j, by step parity
   p.total = off;
   return DOMINO_OK;
 }
@@ -916,6 +917,7 @@ int rollout_entry(const void* hidden, const int32_t* anchors, const float* unifo
     rp.w2 = static_cast<const __nv_bfloat16*>(head->w2);
     rp.x_table = head->x_table;
     rp.uh = reinterpret_cast<float*>(ws + P.off_uh);
+    rp.gh = reinterpret_cast<float*>(ws + P.off_gh);
   }
   rp.b2 = head ? static_cast<const __nv_bfloat16*>(head->b2) : nullptr;
   rp.head = hd ? 1 : 0;

@@ -331,6 +331,129 @@ __device__ __forceinline__ void gru_phase(const RolloutParams& p, const int* s_t
   }
 }
 
+// Four consecutive bf16 values (8-byte aligned) as floats.
+__device__ __forceinline__ void bf4(const __nv_bfloat16* p, float (&f)[4]) {
+  const uint2 v = *reinterpret_cast<const uint2*>(p);
+  const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&v.x));
+  const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&v.y));
+  f[0] = a.x; f[1] = a.y; f[2] = b.x; f[3] = b.y;
+}
+
+// ---- phase A with the input-projection table, two barriers per step (resident kernel): every
+//      CTA computes h_j of every unit and sequence itself, so that no grid barrier follows.  The
+//      input-gate sums are row t_j of the table, the recurrent sums W_hh h_{j-1} were computed in
+//      the previous step's phase B (gh; none at j = 0), and h_{j-1} is the CTA's own copy in
+//      shared memory, updated in place (unit q of h_j needs unit q of h_{j-1} only); four consecutive
+//      units per thread, every load of them issued before any arithmetic.
+__device__ __forceinline__ void gates_all(const RolloutParams& p, int j, const int* s_tok, float* s_h) {
+  const int B = p.B, Ds = p.Ds, D4 = Ds / 4;
+  const float* gh = p.gh + static_cast<size_t>((j + 1) & 1) * B * 3 * Ds;  // W_hh h_{j-1}
+  for (int e = threadIdx.x; e < B * D4; e += kRollThreads) {
+    const int b = e / D4, q = (e - b * D4) * 4;
+    const float* xt = p.x_table + static_cast<size_t>(s_tok[b]) * 3 * Ds;
+    float4 x[3], hh[3];
+    float bi[3][4], bh[3][4];
+#pragma unroll
+    for (int g = 0; g < 3; ++g) {
+      x[g] = __ldg(reinterpret_cast<const float4*>(xt + g * Ds + q));
+      // written by other CTAs in this launch: read through L2
+      hh[g] = j > 0 ? __ldcg(reinterpret_cast<const float4*>(gh + static_cast<size_t>(b) * 3 * Ds + g * Ds + q))
+                    : make_float4(0.f, 0.f, 0.f, 0.f);
+      if (p.b_ih) bf4(p.b_ih + g * Ds + q, bi[g]); else bi[g][0] = bi[g][1] = bi[g][2] = bi[g][3] = 0.f;
+      if (p.b_hh) bf4(p.b_hh + g * Ds + q, bh[g]); else bh[g][0] = bh[g][1] = bh[g][2] = bh[g][3] = 0.f;
+    }
+    float* hrow = s_h + static_cast<size_t>(b) * Ds + q;
+    const float4 hp = j > 0 ? *reinterpret_cast<const float4*>(hrow) : make_float4(0.f, 0.f, 0.f, 0.f);
+    const float xa[3][4] = {{x[0].x, x[0].y, x[0].z, x[0].w}, {x[1].x, x[1].y, x[1].z, x[1].w},
+                            {x[2].x, x[2].y, x[2].z, x[2].w}};
+    const float ha[3][4] = {{hh[0].x, hh[0].y, hh[0].z, hh[0].w}, {hh[1].x, hh[1].y, hh[1].z, hh[1].w},
+                            {hh[2].x, hh[2].y, hh[2].z, hh[2].w}};
+    const float hpa[4] = {hp.x, hp.y, hp.z, hp.w};
+    float out[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float r = 1.f / (1.f + expf(-(xa[0][i] + bi[0][i] + ha[0][i] + bh[0][i])));
+      const float z = 1.f / (1.f + expf(-(xa[1][i] + bi[1][i] + ha[1][i] + bh[1][i])));
+      const float n = tanhf(xa[2][i] + bi[2][i] + r * (ha[2][i] + bh[2][i]));
+      out[i] = (1.f - z) * n + z * hpa[i];
+    }
+    *reinterpret_cast<float4*>(hrow) = make_float4(out[0], out[1], out[2], out[3]);
+  }
+}
+
+// ---- phase B of the two-barrier step: one warp per row of [W1[:, H:]; W_hh] (R + 3 Ds rows;
+//      the W_hh rows only when a next step follows), each multiplied with h_j of every sequence
+//      from the CTA's shared memory: u_j = SiLU(uh + W1[q, H:] h_j + b1), and gh_j = W_hh h_j for
+//      the next step's gates.  A warp takes its rows two at a time, with every weight load of both
+//      issued before the arithmetic (Ds <= 2048: at most 8 chunks of 8 columns per lane and row).
+template <int KB>
+__device__ __forceinline__ void ub_phase(const RolloutParams& p, int j, const float* s_h, int gw, int nwarps,
+                                         int lane, uint64_t pol) {
+  const int B = p.B, K = p.K, H = p.H, Ds = p.Ds, R = p.R;
+  const int rows = R + (j + 1 < K ? 3 * Ds : 0);
+  float* gh = p.gh + static_cast<size_t>(j & 1) * B * 3 * Ds;
+  constexpr int kCh = 8;
+  for (int row0 = gw; row0 < rows; row0 += 2 * nwarps) {
+    uint4 wraw[2][kCh];
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const int row = row0 + k * nwarps;
+      const __nv_bfloat16* w = row >= rows ? nullptr
+                               : row < R   ? p.w1 + static_cast<size_t>(row) * (H + Ds) + H
+                                           : p.w_hh + static_cast<size_t>(row - R) * Ds;
+#pragma unroll
+      for (int i = 0; i < kCh; ++i) {
+        const int c = lane * 8 + 256 * i;
+        wraw[k][i] = (w != nullptr && c < Ds) ? ld16_hint(w + c, pol) : make_uint4(0, 0, 0, 0);
+      }
+    }
+    float acc[2][KB];
+#pragma unroll
+    for (int k = 0; k < 2; ++k)
+#pragma unroll
+      for (int b = 0; b < KB; ++b) acc[k][b] = 0.f;
+#pragma unroll
+    for (int i = 0; i < kCh; ++i) {
+      const int c = lane * 8 + 256 * i;
+      if (c >= Ds) break;
+      float wv[2][8];
+      unpack8(wraw[0][i], wv[0]);
+      unpack8(wraw[1][i], wv[1]);
+#pragma unroll
+      for (int b = 0; b < KB; ++b) {
+        if (b < B) {
+          const float4 h0 = *reinterpret_cast<const float4*>(s_h + static_cast<size_t>(b) * Ds + c);
+          const float4 h1 = *reinterpret_cast<const float4*>(s_h + static_cast<size_t>(b) * Ds + c + 4);
+#pragma unroll
+          for (int k = 0; k < 2; ++k)
+            acc[k][b] += wv[k][0] * h0.x + wv[k][1] * h0.y + wv[k][2] * h0.z + wv[k][3] * h0.w +
+                         wv[k][4] * h1.x + wv[k][5] * h1.y + wv[k][6] * h1.z + wv[k][7] * h1.w;
+        }
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const int row = row0 + k * nwarps;
+#pragma unroll
+      for (int b = 0; b < KB; ++b) {
+        if (b < B) {
+          const float a = warp_sum(acc[k][b]);
+          if (lane == 0 && row < rows) {
+            if (row < R) {
+              // uh: written before the steps by other CTAs of this launch (ordered by the barriers)
+              const float x = a + __ldcg(p.uh + (static_cast<size_t>(b) * K + j) * R + row) +
+                              (p.b1 ? bf2f(p.b1[row]) : 0.f);
+              p.u[static_cast<size_t>(b) * R + row] = x / (1.f + expf(-x));
+            } else {
+              gh[static_cast<size_t>(b) * 3 * Ds + row - R] = a;
+            }
+          }
+        }
+      }
+    }
+  }
+}
+
 // ---- before the steps (resident kernel): uh[m][q] = W1[q, :H] . hidden_m for every position m
 //      = b K + j and rank row q, the half of u's argument that does not depend on the
 //      recurrence.  Warp w takes row q = w % R and the positions m = w / R, w / R + G, ...
@@ -711,6 +834,8 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
   float* s_u = reinterpret_cast<float*>(s_dyn + static_cast<size_t>(p.smem_rows) * R * 2);  // [B][R]
   float* s_base = s_u + B * R;                                                          // [B][rows_cta]
   float* s_b2 = s_base + B * rows_cta;                                                  // [rows_cta]
+  // [B][Ds] h_j of every sequence (two-barrier steps only), 16-byte aligned for vector reads
+  float* s_h = reinterpret_cast<float*>((reinterpret_cast<uintptr_t>(s_b2 + rows_cta) + 15) & ~static_cast<uintptr_t>(15));
   __shared__ __align__(8) uint64_t s_fill;  // the shared-memory rows landed
   __shared__ uint32_t s_tmem;
   __shared__ int s_tok[kRollMaxB];
@@ -789,10 +914,17 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
         const int b = e / r_n, r = e - b * r_n;
         cp_async4(s_base + b * rows_cta + r, p.base + (static_cast<size_t>(b) * K + j) * V + r_lo + r);
       }
-      gru_phase(p, s_tok, hprev, hcur, gw, nwarps, lane, pol_ab);
-      if (!grid_barrier(p.barrier, nbar++, p.status, &s_fail)) break;
-      u_phase(p, j, hcur, gw, nwarps, lane, pol_ab);
-      if (!grid_barrier(p.barrier, nbar++, p.status, &s_fail)) break;
+      if (p.fast_gates) {
+        gates_all(p, j, s_tok, s_h);
+        compute_sync();  // h_j of every sequence in this CTA's shared memory
+        ub_phase<KB>(p, j, s_h, gw, nwarps, lane, pol_ab);
+        if (!grid_barrier(p.barrier, nbar++, p.status, &s_fail)) break;
+      } else {
+        gru_phase(p, s_tok, hprev, hcur, gw, nwarps, lane, pol_ab);
+        if (!grid_barrier(p.barrier, nbar++, p.status, &s_fail)) break;
+        u_phase(p, j, hcur, gw, nwarps, lane, pol_ab);
+        if (!grid_barrier(p.barrier, nbar++, p.status, &s_fail)) break;
+      }
       for (int e = tid; e < B * R; e += kRollThreads) s_u[e] = __ldcg(p.u + e);
       cp_async_wait_all();
       compute_sync();
@@ -1048,10 +1180,12 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
 // ================================================================ launch
 static bool use_resident(const RolloutParams& p) { return p.head && p.R <= kResidentMaxR; }
 
-// Resident kernel: shared-memory W2 rows that fit beside u and the staged base logits.
-static int resident_smem_rows(int B, int V, int R, int grid) {
+// Resident kernel: shared-memory W2 rows that fit beside u, the staged base logits and `extra`
+// bytes (h_j of every sequence for two-barrier steps); -1 when those alone do not fit.
+static int resident_smem_rows(int B, int V, int R, int grid, long long extra = 0) {
   const int rows_cta = resident_rows_per_cta(V, grid);
-  const long long fixed = static_cast<long long>(B) * R * 4 + static_cast<long long>(B + 1) * rows_cta * 4;
+  const long long fixed =
+      static_cast<long long>(B) * R * 4 + static_cast<long long>(B + 1) * rows_cta * 4 + extra;
   const long long avail = static_cast<long long>(kRollMaxSmem) - fixed;
   if (avail < 0) return -1;
   const long long fit = (avail / (2LL * R)) & ~3LL;
@@ -1086,6 +1220,16 @@ static cudaError_t launch_coop(Kern kern, const RolloutParams& p, int grid, int 
   return cudaGetLastError();
 }
 
+// Two grid barriers per step (phase A done by every CTA for all units, gates_all / ub_phase):
+// the resident kernel with a table, when h_j of every sequence fits in shared memory beside u and
+// the base logits (the shared-memory W2 rows give way to it).
+static bool use_fast_gates(const RolloutParams& p, int grid) {
+  // gates_all reads the biases four at a time (8-byte loads)
+  const bool bias_ok = (reinterpret_cast<uintptr_t>(p.b_ih) & 7u) == 0 && (reinterpret_cast<uintptr_t>(p.b_hh) & 7u) == 0;
+  return use_resident(p) && p.x_table && p.uh && p.gh && p.Ds <= 2048 && bias_ok &&
+         resident_smem_rows(p.B, p.V, p.R, grid, static_cast<long long>(p.B) * p.Ds * 4 + 16) >= 0;
+}
+
 template <int KB>
 static cudaError_t launch_rollout_kb(const RolloutParams& p, int grid, size_t smem, cudaStream_t stream) {
   if (use_resident(p)) return launch_coop(rollout_resident_kernel<KB>, p, grid, kRollThreads, smem, stream);
@@ -1095,10 +1239,18 @@ static cudaError_t launch_rollout_kb(const RolloutParams& p, int grid, size_t sm
 cudaError_t launch_rollout(const RolloutParams& p, int grid, cudaStream_t stream) {
   if (p.B < 1 || p.B > kRollMaxB || grid < 1) return cudaErrorInvalidValue;
   if (p.uniforms && (grid > kRollThreads || !p.lg)) return cudaErrorInvalidValue;  // one thread per CTA
-  const size_t smem = rollout_smem_bytes(p.B, p.V, p.R, p.head, grid);
+  size_t smem = rollout_smem_bytes(p.B, p.V, p.R, p.head, grid);
   if (smem > kRollMaxSmem) return cudaErrorInvalidValue;
   RolloutParams pp = p;
   pp.smem_rows = use_resident(p) ? resident_smem_rows(p.B, p.V, p.R, grid) : 0;
+  pp.fast_gates = use_fast_gates(p, grid) ? 1 : 0;
+  if (pp.fast_gates) {
+    const long long hbytes = static_cast<long long>(p.B) * p.Ds * 4 + 16;  // + alignment of s_h
+    pp.smem_rows = resident_smem_rows(p.B, p.V, p.R, grid, hbytes);
+    smem = static_cast<size_t>(pp.smem_rows) * p.R * 2 + static_cast<size_t>(p.B) * p.R * 4 +
+           static_cast<size_t>(p.B + 1) * resident_rows_per_cta(p.V, grid) * 4 + static_cast<size_t>(hbytes);
+    if (smem > kRollMaxSmem) return cudaErrorInvalidValue;
+  }
   if (!use_resident(p)) pp.uh = nullptr;  // only the resident kernel computes it before its steps
   if (p.B <= 1) return launch_rollout_kb<1>(pp, grid, smem, stream);
   if (p.B <= 2) return launch_rollout_kb<2>(pp, grid, smem, stream);
