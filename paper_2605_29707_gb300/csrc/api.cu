@@ -927,6 +927,7 @@ int rollout_entry(const void* hidden, const int32_t* anchors, const float* unifo
   rp.u = reinterpret_cast<float*>(ws + P.off_u);
   rp.partials = reinterpret_cast<float*>(ws + P.off_part);
   rp.barrier = reinterpret_cast<unsigned*>(ws + 64);
+  rp.ucount = reinterpret_cast<unsigned*>(ws + 128);  // cleared with the status and the barrier
   rp.tokens = tokens;
   rp.logp = logp;
   rp.status = status;

@@ -206,8 +206,9 @@ struct RolloutParams {
   const float* x_table;         // [V, 3 Ds] emb . W_ih^T, or nullptr (phase A projects emb[t] itself)
   float* uh;                    // [B*K][R] scratch for hidden . W1[:, :H]^T (resident kernel), or nullptr
   float* gh;                    // [2][B][3 Ds] W_hh h_j of the next step's gates, by step parity
-  int fast_gates;               // set by launch_rollout: two grid barriers per step (resident kernel,
+  int fast_gates;               // set by launch_rollout: one grid barrier per step (resident kernel,
                                 // table, h_j of every sequence in each CTA's shared memory)
+  unsigned* ucount;             // rows of u finished so far in this launch (cleared), fast_gates only
 };
 // dynamic shared memory of one rollout CTA (the resident W2 rows or the W2 ring, u of every
 // sequence and this CTA's rows of base logits + b2): at most kRollMaxSmem, the 227 KB a CTA may

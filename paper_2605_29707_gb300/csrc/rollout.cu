@@ -264,6 +264,29 @@ __device__ bool grid_barrier(unsigned* ctr, unsigned n, int* status, volatile in
   return s_go != 0;
 }
 
+// Waits until *ctr >= target (acquire at GPU scope): the rows of u phase C needs are written.  The
+// same bounded wait and CTA-wide decision as grid_barrier, without an arrival.
+__device__ bool wait_count(const unsigned* ctr, unsigned target, int* status, volatile int* fail) {
+  __shared__ int s_go;
+  if (threadIdx.x == 0) {
+    const long long t0 = clock64();
+    while (true) {
+      unsigned v;
+      asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+      if (v >= target) break;
+      if (clock64() - t0 > kWaitCycles) {
+        set_status(status, kStatusTimeout);
+        *fail = 1;
+        break;
+      }
+      __nanosleep(32);
+    }
+    s_go = *fail == 0;
+  }
+  compute_sync();
+  return s_go != 0;
+}
+
 // ---- phase A: h_j = GRU(emb[t_j], h_{j-1}) (torch.nn.GRU: gates r|z|n, r multiplies
 //      W_hn h + b_hn), one warp per hidden unit q, every sequence.  With an input-projection
 //      table the three input-gate sums W_i{r,z,n} emb[t_j] are entries of row t_j of it.
@@ -381,11 +404,13 @@ __device__ __forceinline__ void gates_all(const RolloutParams& p, int j, const i
   }
 }
 
-// ---- phase B of the two-barrier step: one warp per row of [W1[:, H:]; W_hh] (R + 3 Ds rows;
+// ---- phase B of the one-barrier step: one warp per row of [W1[:, H:]; W_hh] (R + 3 Ds rows;
 //      the W_hh rows only when a next step follows), each multiplied with h_j of every sequence
 //      from the CTA's shared memory: u_j = SiLU(uh + W1[q, H:] h_j + b1), and gh_j = W_hh h_j for
-//      the next step's gates.  A warp takes its rows two at a time, with every weight load of both
-//      issued before the arithmetic (Ds <= 2048: at most 8 chunks of 8 columns per lane and row).
+//      the next step's gates.  A finished row of u is counted in p.ucount (release), which phase C
+//      waits for instead of a grid barrier; the gh rows are next needed after the step's partials
+//      barrier.  A warp takes its rows two at a time, with every weight load of both issued
+//      before the arithmetic (Ds <= 2048: at most 8 chunks of 8 columns per lane and row).
 template <int KB>
 __device__ __forceinline__ void ub_phase(const RolloutParams& p, int j, const float* s_h, int gw, int nwarps,
                                          int lane, uint64_t pol) {
@@ -450,6 +475,8 @@ __device__ __forceinline__ void ub_phase(const RolloutParams& p, int j, const fl
           }
         }
       }
+      if (lane == 0 && row < R)  // this row of u_j is written for every sequence
+        asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(p.ucount) : "memory");
     }
   }
 }
@@ -918,7 +945,8 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
         gates_all(p, j, s_tok, s_h);
         compute_sync();  // h_j of every sequence in this CTA's shared memory
         ub_phase<KB>(p, j, s_h, gw, nwarps, lane, pol_ab);
-        if (!grid_barrier(p.barrier, nbar++, p.status, &s_fail)) break;
+        // phase C needs u_j only: every one of its R rows counted, not a grid barrier
+        if (!wait_count(p.ucount, static_cast<unsigned>(R) * (j + 1), p.status, &s_fail)) break;
       } else {
         gru_phase(p, s_tok, hprev, hcur, gw, nwarps, lane, pol_ab);
         if (!grid_barrier(p.barrier, nbar++, p.status, &s_fail)) break;
@@ -1226,7 +1254,7 @@ static cudaError_t launch_coop(Kern kern, const RolloutParams& p, int grid, int 
 static bool use_fast_gates(const RolloutParams& p, int grid) {
   // gates_all reads the biases four at a time (8-byte loads)
   const bool bias_ok = (reinterpret_cast<uintptr_t>(p.b_ih) & 7u) == 0 && (reinterpret_cast<uintptr_t>(p.b_hh) & 7u) == 0;
-  return use_resident(p) && p.x_table && p.uh && p.gh && p.Ds <= 2048 && bias_ok &&
+  return use_resident(p) && p.x_table && p.uh && p.gh && p.ucount && p.Ds <= 2048 && bias_ok &&
          resident_smem_rows(p.B, p.V, p.R, grid, static_cast<long long>(p.B) * p.Ds * 4 + 16) >= 0;
 }
 
