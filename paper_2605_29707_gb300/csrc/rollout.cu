@@ -409,19 +409,20 @@ __device__ __forceinline__ void gates_all(const RolloutParams& p, int j, const i
 //      from the CTA's shared memory: u_j = SiLU(uh + W1[q, H:] h_j + b1), and gh_j = W_hh h_j for
 //      the next step's gates.  A finished row of u is counted in p.ucount (release), which phase C
 //      waits for instead of a grid barrier; the gh rows are next needed after the step's partials
-//      barrier.  A warp takes its rows two at a time, with every weight load of both issued
-//      before the arithmetic (Ds <= 2048: at most 8 chunks of 8 columns per lane and row).
+//      barrier.  A warp takes its rows three at a time (R + 3 Ds rows over the grid's warps: one
+//      round for d_s = 1024 and r = 256 on 152 SMs), with every weight load of the three issued
+//      before the arithmetic (Ds <= 1024: at most 4 chunks of 8 columns per lane and row).
 template <int KB>
 __device__ __forceinline__ void ub_phase(const RolloutParams& p, int j, const float* s_h, int gw, int nwarps,
                                          int lane, uint64_t pol) {
   const int B = p.B, K = p.K, H = p.H, Ds = p.Ds, R = p.R;
   const int rows = R + (j + 1 < K ? 3 * Ds : 0);
   float* gh = p.gh + static_cast<size_t>(j & 1) * B * 3 * Ds;
-  constexpr int kCh = 8;
-  for (int row0 = gw; row0 < rows; row0 += 2 * nwarps) {
-    uint4 wraw[2][kCh];
+  constexpr int kCh = 4, kRowsAt = 3;
+  for (int row0 = gw; row0 < rows; row0 += kRowsAt * nwarps) {
+    uint4 wraw[kRowsAt][kCh];
 #pragma unroll
-    for (int k = 0; k < 2; ++k) {
+    for (int k = 0; k < kRowsAt; ++k) {
       const int row = row0 + k * nwarps;
       const __nv_bfloat16* w = row >= rows ? nullptr
                                : row < R   ? p.w1 + static_cast<size_t>(row) * (H + Ds) + H
@@ -432,32 +433,32 @@ __device__ __forceinline__ void ub_phase(const RolloutParams& p, int j, const fl
         wraw[k][i] = (w != nullptr && c < Ds) ? ld16_hint(w + c, pol) : make_uint4(0, 0, 0, 0);
       }
     }
-    float acc[2][KB];
+    float acc[kRowsAt][KB];
 #pragma unroll
-    for (int k = 0; k < 2; ++k)
+    for (int k = 0; k < kRowsAt; ++k)
 #pragma unroll
       for (int b = 0; b < KB; ++b) acc[k][b] = 0.f;
 #pragma unroll
     for (int i = 0; i < kCh; ++i) {
       const int c = lane * 8 + 256 * i;
       if (c >= Ds) break;
-      float wv[2][8];
-      unpack8(wraw[0][i], wv[0]);
-      unpack8(wraw[1][i], wv[1]);
+      float wv[kRowsAt][8];
+#pragma unroll
+      for (int k = 0; k < kRowsAt; ++k) unpack8(wraw[k][i], wv[k]);
 #pragma unroll
       for (int b = 0; b < KB; ++b) {
         if (b < B) {
           const float4 h0 = *reinterpret_cast<const float4*>(s_h + static_cast<size_t>(b) * Ds + c);
           const float4 h1 = *reinterpret_cast<const float4*>(s_h + static_cast<size_t>(b) * Ds + c + 4);
 #pragma unroll
-          for (int k = 0; k < 2; ++k)
+          for (int k = 0; k < kRowsAt; ++k)
             acc[k][b] += wv[k][0] * h0.x + wv[k][1] * h0.y + wv[k][2] * h0.z + wv[k][3] * h0.w +
                          wv[k][4] * h1.x + wv[k][5] * h1.y + wv[k][6] * h1.z + wv[k][7] * h1.w;
         }
       }
     }
 #pragma unroll
-    for (int k = 0; k < 2; ++k) {
+    for (int k = 0; k < kRowsAt; ++k) {
       const int row = row0 + k * nwarps;
 #pragma unroll
       for (int b = 0; b < KB; ++b) {
@@ -1254,7 +1255,7 @@ static cudaError_t launch_coop(Kern kern, const RolloutParams& p, int grid, int 
 static bool use_fast_gates(const RolloutParams& p, int grid) {
   // gates_all reads the biases four at a time (8-byte loads)
   const bool bias_ok = (reinterpret_cast<uintptr_t>(p.b_ih) & 7u) == 0 && (reinterpret_cast<uintptr_t>(p.b_hh) & 7u) == 0;
-  return use_resident(p) && p.x_table && p.uh && p.gh && p.ucount && p.Ds <= 2048 && bias_ok &&
+  return use_resident(p) && p.x_table && p.uh && p.gh && p.ucount && p.Ds <= 1024 && bias_ok &&
          resident_smem_rows(p.B, p.V, p.R, grid, static_cast<long long>(p.B) * p.Ds * 4 + 16) >= 0;
 }
 
