@@ -55,6 +55,9 @@ def _load():
         _lib.oracle_tree.argtypes = [P, P, I, I, I, P, P, P, P]
         _lib.oracle_draft_step.argtypes = [P] * 12 + [I] * 8 + [P, I] + [P] * 8 + [I]
         _lib.oracle_verify_greedy.argtypes = [P, I, I, P, P, P, P, P, P]
+        _lib.oracle_tree_walk.argtypes = [I, P, P, P, P, P, P]
+        _lib.oracle_row_sample.argtypes = [P, I, ctypes.c_double, ctypes.c_double, P]
+        _lib.oracle_verify_sample.argtypes = [P, I, I, ctypes.c_double, P, P, P, P, P, P, P]
         _lib.oracle_rollout_greedy.argtypes = [P] * 12 + [I] * 6 + [P, I, P, P, I]
         _lib.oracle_rollout_sample.argtypes = [P] * 13 + [I] * 6 + [P, I, P, P, I]
         _lib.oracle_max_threads.restype = I
@@ -186,6 +189,46 @@ def verify_greedy(target, parent, token):
     _check(_load().oracle_verify_greedy(_p(target), N, V, _p(parent), _p(token), _p(ra), _p(nodes), _p(n),
                                         _p(bonus)), "oracle_verify_greedy")
     return ra, nodes[: int(n[0])].copy(), int(bonus[0])
+
+
+def tree_walk(parent, token, row_choice):
+    """The verification walk of one tree for given per-row target choices [N+1].
+    Returns (accepted nodes [n_acc], bonus token)."""
+    parent = _i32(parent); token = _i32(token); row_choice = _i32(row_choice)
+    N = parent.shape[0]
+    if row_choice.shape[0] != N + 1:
+        raise OracleError(-1, "oracle_tree_walk: row_choice must have N + 1 entries")
+    nodes = np.empty(max(N, 1), np.int32)
+    n = np.zeros(1, np.int32); bonus = np.zeros(1, np.int32)
+    _check(_load().oracle_tree_walk(N, _p(parent), _p(token), _p(row_choice), _p(nodes), _p(n), _p(bonus)),
+           "oracle_tree_walk")
+    return nodes[: int(n[0])].copy(), int(bonus[0])
+
+
+def row_sample(row, T, u):
+    """One draw from softmax(row / T) with uniform u in [0, 1) (first id whose cumulative
+    probability in id order exceeds u)."""
+    row = np.ascontiguousarray(row, np.float32)
+    out = np.zeros(1, np.int32)
+    _check(_load().oracle_row_sample(_p(row), row.shape[0], float(T), float(u), _p(out)), "oracle_row_sample")
+    return int(out[0])
+
+
+def verify_sample(target, parent, token, T, uniforms):
+    """Tree verification of one sequence at temperature T > 0: target fp32 [N+1, V],
+    parent/token [N], uniforms fp32 [N+1].  Returns (row_sample [N+1], accepted nodes, bonus)."""
+    target = np.ascontiguousarray(target, np.float32)
+    parent = _i32(parent); token = _i32(token)
+    uniforms = np.ascontiguousarray(uniforms, np.float32)
+    N = parent.shape[0]
+    V = target.shape[1]
+    if target.shape[0] != N + 1 or uniforms.shape[0] != N + 1:
+        raise OracleError(-1, "oracle_verify_sample: target and uniforms must have N + 1 rows")
+    rs = np.empty(N + 1, np.int32); nodes = np.empty(max(N, 1), np.int32)
+    n = np.zeros(1, np.int32); bonus = np.zeros(1, np.int32)
+    _check(_load().oracle_verify_sample(_p(target), N, V, float(T), _p(uniforms), _p(parent), _p(token), _p(rs),
+                                        _p(nodes), _p(n), _p(bonus)), "oracle_verify_sample")
+    return rs, nodes[: int(n[0])].copy(), int(bonus[0])
 
 
 def rollout_greedy(w, hidden, anchors, seqs=None, nthreads=0):

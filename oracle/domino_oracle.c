@@ -14,7 +14,8 @@
  *                  L_i = L_base_i + dL_i                          -> oracle_logits (sum)
  *   Fig. 3 caption: tokens are drawn from the final logits        -> oracle_log_softmax
  *   Fig. 1 caption: the "Tree" construction cost                  -> oracle_topk, oracle_tree
- *   section 3.1, verification of the draft (the step after it)     -> oracle_verify_greedy
+ *   section 3.1, verification of the draft (the step after it)     -> oracle_verify_greedy,
+ *                                                                       oracle_verify_sample
  *   section 4.1.2 / Fig. 3, tokens chosen and fed back one by one   -> oracle_rollout_greedy,
  *                                                                       oracle_rollout_sample
  * Readings of points the paper leaves open (GRU gate convention, which ids feed which
@@ -335,10 +336,23 @@ int oracle_verify_greedy(const float* target, int N, int V, const int32_t* paren
       if (row[v] > row[best]) best = v; /* strict: an equal value keeps the lower id */
     row_argmax[r] = best;
   }
+  return oracle_tree_walk(N, parent, token, row_argmax, nodes, n_acc, bonus);
+}
+
+/* The walk shared by both verification rules: from the anchor, the target's choice a for the
+   current node's row is kept when a child of that node carries it (the first such child in node
+   order), and the walk continues from that child; the first choice that no child carries ends
+   the walk and is the token the target adds itself (section 3.1). */
+int oracle_tree_walk(int N, const int32_t* parent, const int32_t* token, const int32_t* row_choice,
+                     int32_t* nodes, int32_t* n_acc, int32_t* bonus) {
+  if (!row_choice || !nodes || !n_acc || !bonus || N < 0) return ORACLE_ERR_ARG;
+  if (N > 0 && (!parent || !token)) return ORACLE_ERR_ARG;
+  for (int i = 0; i < N; ++i)
+    if (parent[i] < -1 || parent[i] >= i) return ORACLE_ERR_ARG;
   for (int i = 0; i < N; ++i) nodes[i] = -1;
   int cur = -1, n = 0;
   for (;;) {
-    const int a = row_argmax[cur + 1];
+    const int a = row_choice[cur + 1];
     int next = -1;
     for (int c = 0; c < N; ++c)
       if (parent[c] == cur && token[c] == a) { next = c; break; }
@@ -351,6 +365,52 @@ int oracle_verify_greedy(const float* target, int N, int V, const int32_t* paren
   }
   *n_acc = n;
   return 0;
+}
+
+/* O11: one draw from the target's distribution at temperature T for one row of logits:
+   p(v) = exp(l_v / T) / sum_v' exp(l_v' / T), computed as exp((l_v - max) / T) over its sum;
+   the draw is the first id whose cumulative probability, summed in id order, exceeds u.  A u at
+   or past the total (rounding) takes the last id of non-zero mass; a row with no finite value
+   takes id 0. */
+int oracle_row_sample(const float* row, int V, double T, double u, int32_t* id) {
+  if (!row || !id || V <= 0 || !(T > 0.0) || !isfinite(T) || !(u >= 0.0 && u < 1.0)) return ORACLE_ERR_ARG;
+  double m = -INFINITY;
+  for (int v = 0; v < V; ++v)
+    if ((double)row[v] > m) m = (double)row[v];
+  if (!isfinite(m)) {
+    *id = 0;
+    return 0;
+  }
+  double Z = 0.0;
+  for (int v = 0; v < V; ++v) Z += exp(((double)row[v] - m) / T);
+  const double theta = u * Z;
+  double c = 0.0;
+  int last = 0;
+  for (int v = 0; v < V; ++v) {
+    const double w = exp(((double)row[v] - m) / T);
+    if (w > 0.0) last = v;
+    c += w;
+    if (c > theta) {
+      *id = v;
+      return 0;
+    }
+  }
+  *id = last;
+  return 0;
+}
+
+/* O12: verification of one tree at temperature T > 0 (section 3.1's rule for sampled decoding,
+   applied to a tree whose children are fixed proposals; the reading is in oracle_verify_sample's
+   declaration): every row's draw (O11) with its own uniform, then the walk above. */
+int oracle_verify_sample(const float* target, int N, int V, double T, const float* uniforms,
+                         const int32_t* parent, const int32_t* token, int32_t* row_sample, int32_t* nodes,
+                         int32_t* n_acc, int32_t* bonus) {
+  if (!target || !uniforms || !row_sample || N < 0 || V <= 0) return ORACLE_ERR_ARG;
+  for (int r = 0; r <= N; ++r) {
+    const int rc = oracle_row_sample(target + (long)r * V, V, T, (double)uniforms[r], row_sample + r);
+    if (rc) return rc;
+  }
+  return oracle_tree_walk(N, parent, token, row_sample, nodes, n_acc, bonus);
 }
 
 /* O9: the greedy sequential draft loop.  Each position is computed from scratch out of the

@@ -111,6 +111,29 @@ int oracle_draft_step(const uint16_t* hidden, const int32_t* prefix_ids, const u
 int oracle_verify_greedy(const float* target, int N, int V, const int32_t* parent, const int32_t* token,
                          int32_t* row_argmax, int32_t* nodes, int32_t* n_acc, int32_t* bonus);
 
+/* The walk of oracle_verify_greedy for any per-row choice: row_choice [N+1] = the target's token
+ * after the anchor (row 0) and after each node i (row i+1); same outputs and tree checks. */
+int oracle_tree_walk(int N, const int32_t* parent, const int32_t* token, const int32_t* row_choice,
+                     int32_t* nodes, int32_t* n_acc, int32_t* bonus);
+
+/* O11: one draw from softmax(row / T) (temperature T > 0) with the caller's uniform u in [0, 1):
+ * the first id whose cumulative probability in id order exceeds u; at or past the total
+ * (rounding) the last id of non-zero mass; a row without a finite value gives id 0. */
+int oracle_row_sample(const float* row, int V, double T, double u, int32_t* id);
+
+/* O12, verification at temperature T > 0 (section 3.1: the target keeps draft tokens by the
+ * speculative sampling rule, so that what it emits is distributed as its own samples).  Reading:
+ * the tree's children are fixed proposals (chosen best-first, not drawn), a point mass per
+ * child.  Against a point mass at x the rule accepts x with probability p(x) and otherwise draws
+ * from p with x removed, renormalised; applied child after child (recursive rejection) that is
+ * the same as drawing one token y from p and moving to the child that carries y, or emitting y
+ * when no child does.  So, per tree: row_sample[r] = oracle_row_sample(row r, T, uniforms[r]),
+ * then oracle_tree_walk on those draws; uniforms [N+1] in [0, 1).  Lossless: the emitted tokens
+ * follow the target's own distribution whatever the tree. */
+int oracle_verify_sample(const float* target, int N, int V, double T, const float* uniforms,
+                         const int32_t* parent, const int32_t* token, int32_t* row_sample, int32_t* nodes,
+                         int32_t* n_acc, int32_t* bonus);
+
 /* O9, the sequential draft loop at inference (section 4.1.2 and Fig. 3: each draft token is
  * chosen from the final logits and is the causal encoder's next input), greedy: per sequence,
  * t_0 = anchors[b]; for j = 0..K-1: S_j = the GRU state after E_0..E_j with E_i = emb[t_i];

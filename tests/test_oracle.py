@@ -487,6 +487,106 @@ def test_verify_special_cases():
         oracle.verify_greedy(np.zeros((2, 4), np.float32), np.array([-1, 0], np.int32), np.array([0, 1], np.int32))
 
 
+# ---------------------------------------------------------------------------- O11/O12 verification at T > 0
+def _fixture_logits(rows):
+    return np.array([[float(x) if x == "-inf" else _ev(x) for x in r] for r in rows], np.float32)
+
+
+@pytest.mark.parametrize("case", [0, 1, 2])
+def test_verify_sample_hand_case_a(case):
+    """Hand-worked verification at T = 1, 0.5, 2 (section 3.1): draws by the id-order inverse CDF,
+    a zero-mass id skipped at u = 0, accepted and rejected children."""
+    g = _golden("verify_sample_case_a.json")
+    c = g["cases"][case]
+    rs, nodes, bonus = oracle.verify_sample(_fixture_logits(g["target"]), g["parent"], g["token"], c["T"],
+                                            np.array(g["uniforms"], np.float32))
+    assert rs.tolist() == c["expect_row_sample"]
+    assert nodes.tolist() == c["expect_nodes"]
+    assert bonus == c["expect_bonus"]
+    assert len(nodes) + 1 == c["expect_tau"]
+
+
+@pytest.mark.parametrize("T", [0.6, 1.0, 1.7])
+def test_row_sample_is_the_inverse_cdf_of_the_tempered_softmax(T):
+    """Stratified uniforms (i + 1/2) / M: each id is drawn for M p(id) +- 1 of them, p from scipy's
+    softmax of logits / T, and the draw never decreases as u grows (cumulative in id order)."""
+    from scipy.special import softmax
+    rng = np.random.default_rng(11)
+    V, M = 37, 20000
+    row = (rng.standard_normal(V) * 2.0).astype(np.float32)
+    row[5] = -np.inf
+    p = softmax(row.astype(np.float64) / T)
+    draws = np.array([oracle.row_sample(row, T, (i + 0.5) / M) for i in range(M)])
+    assert np.all(np.diff(draws) >= 0)
+    counts = np.bincount(draws, minlength=V)
+    assert counts[5] == 0
+    assert np.all(np.abs(counts - M * p) <= 1.0 + 1e-9)
+
+
+def test_verify_sample_first_emitted_token_follows_the_target():
+    """Lossless: whatever the tree, the first token the verification emits (the accepted child's or
+    the bonus) is distributed as the target's own draw after the anchor; stratified over row 0's
+    uniform, the other rows' uniforms fixed."""
+    from scipy.special import softmax
+    from paper_2605_29707_gb300 import inputs
+    c = inputs.make_verify_case(1, 8, 6, 21, p_plant=1.0)
+    T, M = 1.3, 6000
+    tgt, par, tok = c.target[0], c.parent[0], c.token[0]
+    p0 = softmax(tgt[0].astype(np.float64) / T)
+    rest = inputs.uniform01(9, (21, "verify-sample-rest")).astype(np.float32)
+    first = []
+    for i in range(M):
+        u = rest.copy()
+        u[0] = (i + 0.5) / M
+        rs, nodes, bonus = oracle.verify_sample(tgt, par, tok, T, u)
+        first.append(int(tok[nodes[0]]) if len(nodes) else bonus)
+        assert (int(tok[nodes[0]]) if len(nodes) else bonus) == rs[0]
+    counts = np.bincount(first, minlength=6)
+    assert np.all(np.abs(counts - M * p0) <= 1.0 + 1e-9)
+
+
+@pytest.mark.parametrize("seed,N,V,chain", [(1, 12, 300, False), (3, 16, 1000, True), (5, 30, 64, False)])
+def test_verify_sample_at_low_temperature_is_greedy(seed, N, V, chain):
+    """With every row's maximum at least 1 above the rest and T = 0.01, the tempered softmax puts all
+    but e^-100 of its mass on the argmax: every draw is the argmax and the walk is the greedy one."""
+    from paper_2605_29707_gb300 import inputs
+    c = inputs.make_verify_case(2, N, V, seed, p_plant=0.8, chain=chain)
+    for b in range(2):
+        t = c.target[b].copy()
+        for r in range(N + 1):
+            a = int(np.argmax(t[r]))
+            t[r, a] = np.float32(np.max(np.delete(t[r], a)) + 1.0)
+        u = inputs.uniform01(N + 1, (seed, "verify-sample-u", b)).astype(np.float32) * np.float32(0.999)
+        rs, nodes, bonus = oracle.verify_sample(t, c.parent[b], c.token[b], 0.01, u)
+        ra, gnodes, gbonus = oracle.verify_greedy(t, c.parent[b], c.token[b])
+        assert rs.tolist() == ra.tolist()
+        assert nodes.tolist() == gnodes.tolist() and bonus == gbonus
+
+
+def test_verify_sample_special_cases():
+    below_one = float(np.nextafter(np.float32(1.0), np.float32(0.0)))
+    # u = 0: the first id of non-zero mass; u just below 1: the last one
+    row = np.array([-np.inf, 0.0, 0.0, -np.inf], np.float32)
+    assert oracle.row_sample(row, 1.0, 0.0) == 1
+    assert oracle.row_sample(row, 1.0, below_one) == 2
+    # a row with no finite value: id 0
+    assert oracle.row_sample(np.full(4, -np.inf, np.float32), 1.0, 0.5) == 0
+    # no nodes: the draw after the anchor is the bonus, tau = 1
+    rs, nodes, bonus = oracle.verify_sample(np.array([[0.0, 0.0, 0.0, 0.0]], np.float32), np.zeros(0, np.int32),
+                                            np.zeros(0, np.int32), 1.0, np.array([0.6], np.float32))
+    assert rs.tolist() == [2] and len(nodes) == 0 and bonus == 2
+    # bad temperature, bad uniforms, bad tree
+    for T in (0.0, -1.0, float("inf"), float("nan")):
+        with pytest.raises(oracle.OracleError):
+            oracle.row_sample(row, T, 0.5)
+    for u in (1.0, -0.1, float("nan")):
+        with pytest.raises(oracle.OracleError):
+            oracle.row_sample(row, 1.0, u)
+    with pytest.raises(oracle.OracleError):
+        oracle.verify_sample(np.zeros((3, 4), np.float32), np.array([-1, 1], np.int32), np.array([0, 1], np.int32),
+                             1.0, np.zeros(3, np.float32))
+
+
 # ---------------------------------------------------------------------------- O9 greedy rollout
 def test_rollout_hand_case_c():
     """Hand-worked greedy rollout (section 4.1.2 / Fig. 3) from hand case C's numbers."""
