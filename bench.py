@@ -355,9 +355,33 @@ def verify_timing(st, c, device, stream, reps=200):
     torch.cuda.synchronize()
     us = e0.elapsed_time(e1) / reps * 1e3
     nbytes = c.B * (c.N + 1) * c.V * 4
+    greedy_tau = round(float(cnt.float().mean().item()) + 1.0, 3)
+
+    # the same trees at temperature 1 (domino_verify_tree_sample): planted tokens raised by 9 so
+    # that they carry about two thirds of a row's mass, one seeded uniform per row
+    T = 1.0
+    case_s = inputs.make_verify_case(c.B, c.N, c.V, 98, p_plant=0.8, trees=trees, margin=9.0)
+    t_s = torch.from_numpy(case_s.target).to(device)
+    uu = torch.from_numpy(inputs.uniform01(c.B * (c.N + 1), (98, "verify-sample-u")).astype("float32")).to(device)
+
+    def run_s():
+        rc = binding.domino_verify_tree_sample(t_s, par, tok, uu, T, c.B, c.N, c.V, ra, nodes, cnt, bon, stream)
+        if rc != 0:
+            raise RuntimeError(f"domino_verify_tree_sample returned {rc}")
+    for _ in range(3):
+        run_s()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(reps):
+        run_s()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    us_s = e0.elapsed_time(e1) / reps * 1e3
     return {"us": round(us, 2), "logits_bytes": nbytes, "GB_per_s": round(nbytes / (us * 1e-6) / 1e9, 1),
-            "tau_mean": round(float(cnt.float().mean().item()) + 1.0, 3),
-            "note": "synthetic target logits (planted argmaxes); tau is a mechanics check, not a quality number"}
+            "tau_mean": greedy_tau,
+            "sampled": {"temperature": T, "us": round(us_s, 2), "GB_per_s": round(nbytes / (us_s * 1e-6) / 1e9, 1),
+                        "tau_mean": round(float(cnt.float().mean().item()) + 1.0, 3)},
+            "note": "synthetic target logits (planted tokens); tau is a mechanics check, not a quality number"}
 
 
 def rollout_timing(st, wl, c, hidden, device, stream, reps=50):
@@ -709,8 +733,8 @@ def run_ours(args):
                        "note": "the same step reading the GRU's input-gate sums from the table; value is the step without it"}
         del st_tab
 
-    # ---- the step after the draft: greedy verification of this step's trees against synthetic
-    #      target logits [B, N+1, V] fp32 (timing only; parity is in the tests)
+    # ---- the step after the draft: verification of this step's trees against synthetic target
+    #      logits [B, N+1, V] fp32, greedy and at temperature 1 (timing only; parity is in the tests)
     verify = verify_timing(st, c, device, stream) if c.B <= 4 else None
     # ---- the sequential draft loop (the paper's inference loop) on the same weights
     rollout = rollout_timing(st, wl, c, hidden, device, stream)

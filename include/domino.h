@@ -221,6 +221,36 @@ DOMINO_API int domino_verify_tree_greedy(const float* target_logits, const int32
                                          int32_t* accepted_nodes, int32_t* accepted_count,
                                          int32_t* bonus_token, void* stream);
 
+/* Verification of draft trees at temperature T > 0 (section 3.1: the target keeps draft tokens by
+ * the speculative sampling rule, which leaves what it emits distributed as its own samples).
+ * The tree's children are fixed proposals (chosen best-first, not drawn): against a proposal x
+ * that is certain, the rule keeps x with probability p(x) and otherwise draws from p without x,
+ * renormalised; tried child after child, that is one draw y from the target's p at the node,
+ * kept when a child carries y.  So, for each sequence b, from the anchor: y = the draw of the
+ * current node's row; if a child of the current node carries y (several: the lowest node index),
+ * accept it and continue from it; otherwise stop, and y is the bonus token.
+ *   The draw of row r: p = softmax(target_logits[r] / T); y = the first id v whose cumulative
+ *   probability sum_{v' <= v} p(v'), in id order, exceeds u = uniforms[r] (values outside [0, 1)
+ *   are clamped to it), computed in fp32: where u falls within rounding of a boundary either
+ *   neighbour may be drawn, and past the computed total the last id of non-zero probability is.
+ *   Ids of zero probability (logit -inf) are never drawn; a row with no finite logit gives id 0.
+ *   target_logits: device fp32 [B, N + 1, V] as for domino_verify_tree_greedy; finite or -inf
+ *     (NaN is not ordered).  V <= 8 * 53248 (a row is staged in shared memory once).
+ *   uniforms: device fp32 [B, N + 1], the caller's random draws, one per row (only the rows the
+ *     walk visits matter).
+ *   temperature: T > 0 with 1 / T finite in fp32.
+ *   tree_parent / tree_token: as for domino_verify_tree_greedy.
+ * Outputs (device int32): row_sample [B, N + 1] = every row's draw; accepted_nodes [B, N],
+ *   accepted_count [B] (tau = accepted_count + 1) and bonus_token [B] as for
+ *   domino_verify_tree_greedy.
+ * Two kernels on `stream`; no workspace.  Returns DOMINO_OK once enqueued, DOMINO_ERR_UNSUPPORTED
+ * for a larger V, or another negative code (bad sizes, pointers or temperature) with nothing
+ * enqueued. */
+DOMINO_API int domino_verify_tree_sample(const float* target_logits, const int32_t* tree_parent,
+                                         const int32_t* tree_token, const float* uniforms, float temperature,
+                                         int B, int N, int V, int32_t* row_sample, int32_t* accepted_nodes,
+                                         int32_t* accepted_count, int32_t* bonus_token, void* stream);
+
 /* The greedy sequential draft loop, the paper's inference loop (section 4.1.2 and Fig. 3: each
  * draft token is chosen from the final logits and becomes the causal encoder's next input), as
  * a variant of domino_draft_step for callers that do not have the prefix:
@@ -317,7 +347,8 @@ enum domino_kernel_kind {
   DOMINO_KERNEL_TREE = 5,         /* merge to log-probs and top-k; best-first tree */
   DOMINO_KERNEL_ROLLOUT_BASE = 6, /* domino_rollout_greedy: W_lm hidden_j of every position */
   DOMINO_KERNEL_ROLLOUT = 7,      /* domino_rollout_greedy: the K sequential steps */
-  DOMINO_KERNEL_VERIFY = 8,       /* domino_verify_tree_greedy: row argmax and tree walk */
+  DOMINO_KERNEL_VERIFY = 8,       /* domino_verify_tree_greedy / _sample: row argmax or draw, and
+                                     tree walk */
   DOMINO_KERNEL_KINDS = 9
 };
 DOMINO_API int domino_timing_begin(int max_launches);

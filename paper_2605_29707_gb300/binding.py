@@ -26,7 +26,8 @@ SYMBOLS = ("domino_workspace_bytes", "domino_draft_step", "domino_workspace_byte
            "domino_abi_version", "domino_launches_per_step", "domino_timing_begin", "domino_timing_end",
            "domino_draft_step_static_scratch", "domino_verify_tree_greedy", "domino_rollout_workspace_bytes",
            "domino_rollout_greedy", "domino_rollout_sample", "domino_input_table_bytes",
-           "domino_build_input_table", "domino_launches_per_step_table", "domino_debug_hold")
+           "domino_build_input_table", "domino_launches_per_step_table", "domino_debug_hold",
+           "domino_verify_tree_sample")
 
 DOMINO_STATIC_SCRATCH_BYTES = 16 << 20
 
@@ -92,6 +93,8 @@ def load():
     lib.domino_draft_step_static_scratch.restype = I
     lib.domino_verify_tree_greedy.argtypes = [P, P, P, I, I, I, P, P, P, P, P]
     lib.domino_verify_tree_greedy.restype = I
+    lib.domino_verify_tree_sample.argtypes = [P, P, P, P, ctypes.c_float, I, I, I, P, P, P, P, P]
+    lib.domino_verify_tree_sample.restype = I
     lib.domino_rollout_workspace_bytes.argtypes = [I] * 6
     lib.domino_rollout_workspace_bytes.restype = ctypes.c_size_t
     lib.domino_rollout_greedy.argtypes = [P, P, P, ctypes.POINTER(domino_head_weights)] + [I] * 4 + [P, P, P,
@@ -225,6 +228,16 @@ def domino_verify_tree_greedy(target_logits, tree_parent, tree_token, B, N, V, r
     return int(load().domino_verify_tree_greedy(_addr(target_logits), _addr(tree_parent), _addr(tree_token), B, N, V,
                                                 _addr(row_argmax), _addr(accepted_nodes), _addr(accepted_count),
                                                 _addr(bonus_token), _stream(stream)))
+
+
+def domino_verify_tree_sample(target_logits, tree_parent, tree_token, uniforms, temperature, B, N, V, row_sample,
+                              accepted_nodes, accepted_count, bonus_token, stream=None) -> int:
+    """Verification at temperature T > 0 of B draft trees against the target's fp32 logits
+    [B, N+1, V] with one uniform per row [B, N+1] (device)."""
+    return int(load().domino_verify_tree_sample(_addr(target_logits), _addr(tree_parent), _addr(tree_token),
+                                                _addr(uniforms), float(temperature), B, N, V, _addr(row_sample),
+                                                _addr(accepted_nodes), _addr(accepted_count), _addr(bonus_token),
+                                                _stream(stream)))
 
 
 def domino_rollout_workspace_bytes(B, K, H, V, Ds, R) -> int:

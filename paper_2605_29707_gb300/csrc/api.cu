@@ -750,6 +750,24 @@ int domino_verify_tree_greedy(const float* target_logits, const int32_t* tree_pa
   return rc;
 }
 
+int domino_verify_tree_sample(const float* target_logits, const int32_t* tree_parent, const int32_t* tree_token,
+                              const float* uniforms, float temperature, int B, int N, int V, int32_t* row_sample,
+                              int32_t* accepted_nodes, int32_t* accepted_count, int32_t* bonus_token, void* stream) {
+  if (B < 1 || N < 0 || V < 1 || N > (1 << 20)) return DOMINO_ERR_INVALID_ARG;
+  if (static_cast<long long>(B) * (N + 1) > 0x7fffffffLL) return DOMINO_ERR_INVALID_ARG;
+  if (!target_logits || !uniforms || !row_sample || !accepted_count || !bonus_token) return DOMINO_ERR_INVALID_ARG;
+  if (N > 0 && (!tree_parent || !tree_token || !accepted_nodes)) return DOMINO_ERR_INVALID_ARG;
+  const float inv_t = 1.0f / temperature;
+  if (!(temperature > 0.f) || !std::isfinite(temperature) || !std::isfinite(inv_t)) return DOMINO_ERR_INVALID_ARG;
+  if (((V + 7) / 8 + 3) / 4 * 4 > dm::kMaxSampleSlice) return DOMINO_ERR_UNSUPPORTED;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int ts = timing_open(DOMINO_KERNEL_VERIFY, st);
+  const int rc = cuda_rc(dm::launch_verify_sample(target_logits, tree_parent, tree_token, uniforms, B, N, V, inv_t,
+                                                  row_sample, accepted_nodes, accepted_count, bonus_token, st));
+  timing_close(ts, st);
+  return rc;
+}
+
 // ---------------------------------------------------------------- input-projection table
 namespace {
 __device__ int g_table_status;  // device status of domino_build_input_table's GEMM

@@ -221,5 +221,11 @@ cudaError_t launch_rollout(const RolloutParams& p, int grid, cudaStream_t stream
 cudaError_t launch_verify_greedy(const float* logits, const int32_t* parent, const int32_t* token, int B, int N,
                                  int V, int32_t* row_argmax, int32_t* nodes, int32_t* count, int32_t* bonus,
                                  cudaStream_t stream);
+// Row draws from softmax(logits / T) (inv_t = 1 / T) with one uniform per row, then the same walk;
+// a row slice of at most kMaxSampleSlice floats is staged in shared memory (V <= 8 of them).
+constexpr int kMaxSampleSlice = 53248;
+cudaError_t launch_verify_sample(const float* logits, const int32_t* parent, const int32_t* token,
+                                 const float* uniforms, int B, int N, int V, float inv_t, int32_t* row_sample,
+                                 int32_t* nodes, int32_t* count, int32_t* bonus, cudaStream_t stream);
 
 }  // namespace dm

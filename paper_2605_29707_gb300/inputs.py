@@ -299,11 +299,12 @@ def random_tree(N: int, V: int, key: tuple, chain: bool = False):
 
 
 def make_verify_case(B: int, N: int, V: int, seed: int, p_plant: float = 0.7, chain: bool = False,
-                     trees=None) -> VerifyCase:
+                     trees=None, margin: float = 1.0) -> VerifyCase:
     """Target logits ~ N(0, 1) fp32; with probability p_plant the row after a node (or after the
-    anchor) gets one of that node's children's tokens raised to the row maximum + 1, so that
-    accepted paths of every length occur.  `trees` ([B] pairs of parent/token) replaces the
-    random trees, e.g. with trees a draft step produced."""
+    anchor) gets one of that node's children's tokens raised to the row maximum + margin, so that
+    accepted paths of every length occur (greedy: any margin > 0; sampled at T = 1 over 151936
+    ids, margin 9 gives the planted token about two thirds of the mass).  `trees` ([B] pairs of
+    parent/token) replaces the random trees, e.g. with trees a draft step produced."""
     parent = np.empty((B, N), np.int32)
     token = np.empty((B, N), np.int32)
     target = np.empty((B, N + 1, V), np.float32)
@@ -318,6 +319,6 @@ def make_verify_case(B: int, N: int, V: int, seed: int, p_plant: float = 0.7, ch
             kids = [c for c in range(N) if parent[b, c] == r - 1]
             if kids and u[2 * r] < p_plant:
                 c = kids[min(len(kids) - 1, int(u[2 * r + 1] * len(kids)))]
-                t[r, token[b, c]] = t[r].max() + 1.0
+                t[r, token[b, c]] = t[r].max() + margin
         target[b] = t
     return VerifyCase(parent, token, target)

@@ -119,6 +119,23 @@ def test_verify_rejects_bad_arguments_before_launch():
     assert f(one, one, one, 1, 4, 10, one, None, one, one) == bad       # no accepted_nodes
 
 
+def test_verify_sample_rejects_bad_arguments_before_launch():
+    """Argument errors of domino_verify_tree_sample (sizes, pointers, temperature, a vocabulary past
+    the shared-memory staging limit) come back before anything is enqueued."""
+    f = binding.domino_verify_tree_sample
+    bad, unsup = binding.DOMINO_ERR_INVALID_ARG, binding.DOMINO_ERR_UNSUPPORTED
+    one = 1  # a non-null stand-in; never dereferenced because validation fails first
+    assert f(one, one, one, one, 1.0, 0, 4, 10, one, one, one, one) == bad       # B < 1
+    assert f(one, one, one, one, 1.0, 1, -1, 10, one, one, one, one) == bad      # N < 0
+    assert f(one, one, one, one, 1.0, 1, 4, 0, one, one, one, one) == bad        # V < 1
+    assert f(one, one, one, None, 1.0, 1, 4, 10, one, one, one, one) == bad      # no uniforms
+    assert f(one, None, one, one, 1.0, 1, 4, 10, one, one, one, one) == bad      # N > 0 without a tree
+    assert f(one, one, one, one, 1.0, 1, 4, 10, None, one, one, one) == bad      # no row_sample
+    for T in (0.0, -1.0, float("inf"), float("nan"), 1e-40):                     # 1 / 1e-40 overflows
+        assert f(one, one, one, one, T, 1, 4, 10, one, one, one, one) == bad
+    assert f(one, one, one, one, 1.0, 1, 4, 8 * 53248 + 1, one, one, one, one) == unsup
+
+
 def test_rollout_rejects_bad_sizes_before_any_device_work():
     f = binding.domino_rollout_workspace_bytes
     assert f(0, 4, 256, 100, 64, 64) == 0       # B < 1
