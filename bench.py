@@ -586,6 +586,15 @@ def measure_config(name, device, stream, steps, warmup, num_sms, peaks):
     st_off = DraftStep(st.w, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=device, head_on=False)
     us_off = time_steps(st_off, hidden, ids, stream, steps, warmup)
     del st_off
+    # the same step with the input-projection table (built once per set of weights, outside the
+    # timed region): the GRU reads a table row per position instead of the E . W_ih^T GEMM
+    st_tab = DraftStep(st.w, c.B, c.K, c.H, c.V, c.k, c.N, Ds=c.Ds, R=c.R, device=device, input_table=True)
+    us_tab = time_steps(st_tab, hidden, ids, stream, steps, warmup)
+    input_table = {"us_per_step": round(us_tab, 2), "value": round(c.B * 1e6 / us_tab, 3),
+                   "launches_per_step": st_tab.launches_per_step(),
+                   "step_roofline_frac": step_roofline(c, peaks, us_tab)["frac"],
+                   "note": "the same step reading the GRU's input-gate sums from the table; us_per_step is without it"}
+    del st_tab
     out = {"config": config_dict(c), "us_per_step": round(us, 2), "value": round(c.B * 1e6 / us, 3), "unit": UNIT,
            "steps": steps, "warmup": max(3, warmup), "gpu_launches": steps * st.launches_per_step(),
            "roofline": vocab_roofline(c, kern, num_sms, peaks, wl.weights.get("b2") is not None, n),
@@ -594,6 +603,7 @@ def measure_config(name, device, stream, steps, warmup, num_sms, peaks):
                                 for k, v in kern.items() if v[1] > 0},
            "head_overhead": {"us_head_off": round(us_off, 2), "overhead_us": round(us - us_off, 2),
                              "overhead_pct": round(100.0 * (us / us_off - 1.0), 2)},
+           "input_table_step": input_table,
            "clocks": clocks}
     del st, hidden, ids, wl
     torch.cuda.empty_cache()
