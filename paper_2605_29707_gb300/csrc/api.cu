@@ -858,11 +858,14 @@ int make_roll_plan(int B, int K, int H, int V, int Ds, int R, bool head, RollPla
     off = align_up(off + bytes);
     return o;
   };
-  take(256);  // status (offset 0, as for domino_check_status) and the grid barrier counter
+  // status (offset 0, as for domino_check_status), the grid barrier counter (64), the u-row
+  // counter (128), the greedy argmax keys (256)
+  take(512);
   p.off_h = take(static_cast<size_t>(2) * B * (p.Ds > 0 ? p.Ds : 1) * 4);
   p.clear_bytes = off;
   p.off_u = take(static_cast<size_t>(B) * (p.R > 0 ? p.R : 1) * 4);
-  p.off_part = take(static_cast<size_t>(2) * p.grid * dm::kRollMaxB * 16);  // two, by step parity
+  // greedy: every step's (the log-probabilities are merged at the end); sampled: two, by step parity
+  p.off_part = take(static_cast<size_t>(K > 2 ? K : 2) * p.grid * dm::kRollMaxB * 16);
   p.off_lg = take(static_cast<size_t>(2) * B * V * 4);  // sampled mode: final logits, by step parity
   p.off_base = take(static_cast<size_t>(p.M) * V * 4);
   p.off_uh = take(static_cast<size_t>(p.M) * (p.R > 0 ? p.R : 1) * 4);  // hidden . W1[:, :H]^T
@@ -946,13 +949,19 @@ int rollout_entry(const void* hidden, const int32_t* anchors, const float* unifo
   rp.partials = reinterpret_cast<float*>(ws + P.off_part);
   rp.barrier = reinterpret_cast<unsigned*>(ws + 64);
   rp.ucount = reinterpret_cast<unsigned*>(ws + 128);  // cleared with the status and the barrier
+  // greedy: the argmax keys of the sequences (cleared with them), ids below 2^22
+  rp.best = (!uniforms && V <= static_cast<int>(dm::kGreedyIdMask)) ? reinterpret_cast<unsigned long long*>(ws + 256)
+                                                                   : nullptr;
   rp.tokens = tokens;
   rp.logp = logp;
   rp.status = status;
   rp.uniforms = uniforms;
   rp.lg = reinterpret_cast<float*>(ws + P.off_lg);
+  // W2 as 64 x 128 swizzled tiles, for phase C on the tensor cores (r a multiple of 64 up to 256)
+  CUtensorMap tm_w2;
+  const bool have_tm = hd && P.R % 64 == 0 && P.R <= 256 && make_map(&tm_w2, head->w2, P.R, V, P.R, 128);
   const int ts = timing_open(DOMINO_KERNEL_ROLLOUT, st);
-  rc = cuda_rc(dm::launch_rollout(rp, P.grid, st));
+  rc = cuda_rc(dm::launch_rollout(rp, P.grid, st, have_tm ? &tm_w2 : nullptr));
   timing_close(ts, st);
   return rc;
 }

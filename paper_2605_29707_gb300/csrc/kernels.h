@@ -186,6 +186,7 @@ cudaError_t launch_merge_tree(const TreeParams& p, cudaStream_t stream);
 
 // ---------------------------------------------------------------- greedy rollout (rollout.cu)
 constexpr int kRollMaxB = 8;  // sequences per rollout launch
+constexpr unsigned kGreedyIdMask = 0x3FFFFFu;  // greedy rollout keys: token ids below 2^22
 struct RolloutParams {
   const __nv_bfloat16* hidden;  // [B, K, H]
   const int32_t* anchors;       // [B]
@@ -196,7 +197,11 @@ struct RolloutParams {
   const float* base;            // [B*K, V] W_lm hidden (fp32, from the store-mode GEMM)
   float* h;                     // [2][B][Ds] GRU states (cleared: h_{-1} = 0)
   float* u;                     // [B][R]
-  float* partials;              // [2][grid][kRollMaxB] float4 (max, sum exp, argmax bits, 0), by step parity
+  float* partials;              // float4 (max, sum exp, argmax bits, 0) per CTA and sequence:
+                                // greedy [K][grid][kRollMaxB]; sampled [2][grid][kRollMaxB], by step parity
+  unsigned long long* best;     // greedy: [2][kRollMaxB] keys of each sequence's argmax by step parity
+                                // (cleared), or nullptr
+                                // (sampled mode, or V >= 2^22: every CTA combines the partials instead)
   unsigned* barrier;            // grid barrier counter (cleared)
   int32_t* tokens;              // [B, K] t_1 .. t_K
   float* logp;                  // [B, K]
@@ -209,13 +214,18 @@ struct RolloutParams {
   int fast_gates;               // set by launch_rollout: one grid barrier per step (resident kernel,
                                 // table, h_j of every sequence in each CTA's shared memory)
   unsigned* ucount;             // rows of u finished so far in this launch (cleared), fast_gates only
+  int mma_tb, mma_sb;           // set by launch_rollout: phase C on the tensor cores over mma_tb
+                                // 128-row W2 blocks in tensor memory and mma_sb in shared memory
+                                // (both 0: phase C on the CUDA cores)
 };
 // dynamic shared memory of one rollout CTA (the resident W2 rows or the W2 ring, u of every
 // sequence and this CTA's rows of base logits + b2): at most kRollMaxSmem, the 227 KB a CTA may
 // hold less 2 KB for the kernels' static shared memory
 constexpr size_t kRollMaxSmem = 225 * 1024;
 size_t rollout_smem_bytes(int B, int V, int R, bool head, int grid);
-cudaError_t launch_rollout(const RolloutParams& p, int grid, cudaStream_t stream);
+// tm_w2: tensor map of W2 [V, r] bf16 (boxes of 64 x 128, 128-byte swizzle), or nullptr; without it
+// phase C stays on the CUDA cores.
+cudaError_t launch_rollout(const RolloutParams& p, int grid, cudaStream_t stream, const CUtensorMap* tm_w2);
 
 // ---------------------------------------------------------------- tree verification (verify.cu)
 cudaError_t launch_verify_greedy(const float* logits, const int32_t* parent, const int32_t* token, int B, int N,

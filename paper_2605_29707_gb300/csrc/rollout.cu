@@ -21,6 +21,9 @@
 // tcgen05.ld), as many rows as fit in shared memory, and the few rows left read through L2.
 // Wider r uses the streamed kernel, which feeds W2 through a shared-memory ring every step.
 #include <math.h>
+#include <string.h>
+
+#include <algorithm>
 
 #include "kernels.h"
 #include "ptx.cuh"
@@ -718,24 +721,36 @@ __device__ void sample_step(const RolloutParams& p, int j, const float4 (&mine)[
   compute_sync();
 }
 
-// End of step j: this CTA's (max, sum exp, argmax) per sequence go to the partials, every CTA
-// combines all of them after a grid barrier, and picks t_{j+1} (argmax, or sampled).  The
-// partials and (sampled mode) the final-logit copies alternate between two buffers by step
-// parity: a CTA writes step j + 2's only after every CTA has passed step j + 1's barrier, so
-// after every read of step j's (with the correction branch off no other barrier separates
-// consecutive steps).
+// Greedy key of a CTA's best row at step j: the step (so that no earlier step's key competes),
+// the logit in order-preserving form, then the id inverted, so that the largest key over the CTAs
+// is the step's maximum with ties to the lowest id (ids below 2^22).
+__device__ __forceinline__ unsigned long long greedy_key(int j, float m, int id) {
+  return (static_cast<unsigned long long>(j + 1) << 54) | (static_cast<unsigned long long>(f32_ord(m)) << 22) |
+         static_cast<unsigned long long>(kGreedyIdMask - static_cast<unsigned>(id));
+}
+
+// End of step j: this CTA's (max, sum exp, argmax) per sequence go to the partials and every CTA
+// picks t_{j+1} after a grid barrier.  Greedy (p.best set): each CTA also folds its argmax into
+// the sequence's key with one atomicMax before the barrier, and after it every CTA reads that key
+// (the log-probabilities come at the end of the launch from every step's partials, kept for
+// all K steps: greedy_logp); the keys alternate between two slots by step parity.  Sampled: every CTA combines all partials, and the partials and the
+// final-logit copies alternate between two buffers by step parity: a CTA writes step j + 2's
+// only after every CTA has passed step j + 1's barrier, so after every read of step j's (with
+// the correction branch off no other barrier separates consecutive steps).
 template <int KB>
 __device__ __forceinline__ bool finish_step(const RolloutParams& p, int j, Lse (&st)[KB], Lse (*s_red)[kRollMaxB],
                                             int* s_tok, unsigned& nbar, volatile int* s_fail, float* s_logit,
                                             int r_lo, int r_n, int rows_cta, bool resident) {
   const int B = p.B, K = p.K, V = p.V, tid = threadIdx.x;
   const int grid = static_cast<int>(gridDim.x);
-  float4* part = reinterpret_cast<float4*>(p.partials) + static_cast<size_t>(j & 1) * grid * kRollMaxB;
+  const bool greedy = p.best != nullptr;
+  float4* part = reinterpret_cast<float4*>(p.partials) + static_cast<size_t>(greedy ? j : (j & 1)) * grid * kRollMaxB;
   block_reduce(st, s_red, B);  // ends with a barrier: every row's final logit is in s_logit
   if (tid < B) {
     Lse a = s_red[0][tid];
     for (int w = 1; w < kRollWarps; ++w) lse_merge(a, s_red[w][tid]);
     part[static_cast<size_t>(blockIdx.x) * kRollMaxB + tid] = make_float4(a.m, a.s, __int_as_float(a.i), 0.f);
+    if (greedy && a.i != 0x7fffffff) atomicMax(p.best + (j & 1) * kRollMaxB + tid, greedy_key(j, a.m, a.i));
   }
   float* lg = p.lg ? p.lg + static_cast<size_t>(j & 1) * B * V : nullptr;
   if (p.uniforms && !resident) {  // this CTA's final logits (the resident kernel wrote them in phase C)
@@ -745,6 +760,21 @@ __device__ __forceinline__ bool finish_step(const RolloutParams& p, int j, Lse (
     }
   }
   if (!grid_barrier(p.barrier, nbar++, p.status, s_fail)) return false;
+  if (greedy) {
+    if (tid < B) {
+      // every CTA's atomicMax came before its arrival at the barrier; the keys alternate between
+      // two slots by step parity (a CTA updates step j + 2's only after every CTA has passed
+      // step j + 1's barrier, hence after this read)
+      const unsigned long long key = __ldcg(p.best + (j & 1) * kRollMaxB + tid);
+      const int tok = static_cast<int>(key >> 54) == j + 1
+                          ? static_cast<int>(kGreedyIdMask - static_cast<unsigned>(key & kGreedyIdMask))
+                          : 0;  // no row with a finite logit anywhere
+      s_tok[tid] = tok;
+      if (blockIdx.x == 0) p.tokens[static_cast<size_t>(tid) * K + j] = tok;
+    }
+    compute_sync();
+    return true;
+  }
   float4 mine[KB];  // sampled mode: CTA tid's partials (grid <= kRollThreads there)
 #pragma unroll
   for (int b = 0; b < KB; ++b) {
@@ -788,6 +818,40 @@ __device__ __forceinline__ bool finish_step(const RolloutParams& p, int j, Lse (
   }
   compute_sync();
   return true;
+}
+
+// Greedy mode, after the last step: the log-probability of each step's token.  The token is the
+// step's argmax, so its log-softmax is -log of the sum of exp(L - max) over the vocabulary, the
+// merge of every CTA's partials of that step (CTA c takes steps c, c + grid, ...).  Called by
+// the compute threads of every CTA once every step has passed its barrier.
+template <int KB>
+__device__ void greedy_logp(const RolloutParams& p, Lse (*s_red)[kRollMaxB]) {
+  const int B = p.B, K = p.K, tid = threadIdx.x;
+  const int grid = static_cast<int>(gridDim.x);
+  for (int j = blockIdx.x; j < K; j += grid) {
+    const float4* part = reinterpret_cast<const float4*>(p.partials) + static_cast<size_t>(j) * grid * kRollMaxB;
+    Lse st[KB];
+#pragma unroll
+    for (int b = 0; b < KB; ++b) st[b] = lse_empty();
+    for (int c = tid; c < grid; c += kRollThreads) {
+#pragma unroll
+      for (int b = 0; b < KB; ++b) {
+        if (b < B) {
+          const float4 f = __ldcg(part + static_cast<size_t>(c) * kRollMaxB + b);
+          Lse t;
+          t.m = f.x; t.s = f.y; t.i = __float_as_int(f.z);
+          lse_merge(st[b], t);
+        }
+      }
+    }
+    block_reduce(st, s_red, B);
+    if (tid < B) {
+      Lse a = s_red[0][tid];
+      for (int w = 1; w < kRollWarps; ++w) lse_merge(a, s_red[w][tid]);
+      p.logp[static_cast<size_t>(tid) * K + j] = -logf(a.s);
+    }
+    compute_sync();  // s_red is read before the next step's reduction overwrites it
+  }
 }
 
 // Base logits + b2 of step j for this CTA's rows [r_lo, r_lo + r_n), staged in shared memory.
@@ -843,8 +907,34 @@ __device__ __forceinline__ void wide_push(const float (&dot)[32], int lane, int 
 
 // ================================================================ resident kernel (r <= 256)
 
-template <int KB>
-__global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const RolloutParams p) {
+// Phase C on the tensor cores (kMma).  A CTA's W2 rows form 128-row blocks: the first mma_tb in
+// tensor memory as the MMA's A operand (row in lane, K along the columns), the next mma_sb in
+// shared memory as 128-byte swizzled K-major tiles (loaded once by TMA); rows past those blocks
+// are read through L2 on the CUDA cores as in the other layout.  u_j is the B operand with
+// N = 16 rows: row 2b holds bf16(u_j[b]) and row 2b + 1 the bf16 of what that rounding left out,
+// so that D[:, 2b] + D[:, 2b + 1] is W2 u_j to about 2^-16 relative (fp32 accumulation, the
+// precision the CUDA-core layout keeps u in).  Each block's MMAs go into its own 16 columns of D,
+// issued by one thread of its own warp; the epilogue adds the staged base logit and b2 of each row.
+// Tensor memory (512 columns): A block i at columns [i r/2, (i+1) r/2), D of block i at
+// mma_tb r/2 + 16 i.  Shared memory from a 1024-byte boundary: the A blocks (r/64 tiles of
+// 128 rows x 64 columns each), the B operand (r/64 tiles of 16 rows x 64 columns), then u, the
+// base logits, b2 and h as in the other layout.
+constexpr int kMmaBopTileBytes = 16 * 128;   // B operand: 16 rows x 64 bf16 columns
+constexpr int kMmaTileBytes = 128 * 128;     // A block: 128 rows x 64 bf16 columns
+constexpr int kMmaMaxL2Rows = 384;           // at most this many rows a CTA reads through L2
+
+// Byte offset of element (n, k) of the B operand in its 128-byte swizzled K-major tiles: tile
+// k / 64, 8-row groups 1024 bytes apart, 16-byte chunk c of row r stored at chunk c ^ (r % 8).
+__device__ __forceinline__ uint32_t bop_offset(int n, int k) {
+  const int kin = k & 63, r = n & 7;
+  return static_cast<uint32_t>((k >> 6) * kMmaBopTileBytes + (n >> 3) * 1024 + r * 128 + (((kin >> 3) ^ r) << 4) +
+                               (kin & 7) * 2);
+}
+
+template <int KB, bool kMma>
+__global__ void __launch_bounds__(kRollThreads, 1)
+    rollout_resident_kernel(const RolloutParams p, const __grid_constant__ CUtensorMap tm_w2) {
+  static_assert(!kMma || KB <= 2, "the B operand holds two rows per sequence in its 16");
   const int B = p.B, K = p.K, V = p.V, R = p.R;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int nwarps = gridDim.x * kRollWarps;
@@ -854,17 +944,24 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
   const int rows_cta = resident_rows_per_cta(V, gridDim.x);
   const int r_lo = min(V, static_cast<int>(blockIdx.x) * rows_cta);
   const int r_n = min(V, r_lo + rows_cta) - r_lo;
-  const int n_t = min(r_n, kTmemRows);
-  const int n_s = min(r_n - n_t, p.smem_rows);
+  const int n_blk = kMma ? p.mma_tb + p.mma_sb : 0;
+  const int n_t = kMma ? min(r_n, 128 * p.mma_tb) : min(r_n, kTmemRows);
+  const int n_s = kMma ? max(0, min(r_n, 128 * n_blk) - n_t) : min(r_n - n_t, p.smem_rows);
   const int n_g = r_n - n_t - n_s;
   extern __shared__ __align__(128) uint8_t s_dyn[];
-  __nv_bfloat16* s_w2 = reinterpret_cast<__nv_bfloat16*>(s_dyn);                      // [smem_rows][R]
-  float* s_u = reinterpret_cast<float*>(s_dyn + static_cast<size_t>(p.smem_rows) * R * 2);  // [B][R]
+  uint8_t* s_al = kMma ? reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(s_dyn) + 1023) &
+                                                    ~static_cast<uintptr_t>(1023))
+                       : s_dyn;
+  uint8_t* s_bop = s_al + static_cast<size_t>(kMma ? p.mma_sb : 0) * (R / 64) * kMmaTileBytes;  // kMma
+  __nv_bfloat16* s_w2 = reinterpret_cast<__nv_bfloat16*>(s_dyn);  // [smem_rows][R] (!kMma)
+  float* s_u = kMma ? reinterpret_cast<float*>(s_bop + (R / 64) * kMmaBopTileBytes)
+                    : reinterpret_cast<float*>(s_dyn + static_cast<size_t>(p.smem_rows) * R * 2);  // [B][R]
   float* s_base = s_u + B * R;                                                          // [B][rows_cta]
   float* s_b2 = s_base + B * rows_cta;                                                  // [rows_cta]
   // [B][Ds] h_j of every sequence (two-barrier steps only), 16-byte aligned for vector reads
   float* s_h = reinterpret_cast<float*>((reinterpret_cast<uintptr_t>(s_b2 + rows_cta) + 15) & ~static_cast<uintptr_t>(15));
   __shared__ __align__(8) uint64_t s_fill;  // the shared-memory rows landed
+  __shared__ __align__(8) uint64_t s_mma;   // kMma: this step's MMAs completed
   __shared__ uint32_t s_tmem;
   __shared__ int s_tok[kRollMaxB];
   __shared__ Lse s_red[kRollWarps][kRollMaxB];
@@ -872,6 +969,7 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
   if (tid == 0) {
     s_fail = 0;
     mbar_init(&s_fill, 1);
+    mbar_init(&s_mma, kMma ? max(1, min(n_blk, kRollWarps)) : 1);  // one commit per issuing thread
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -883,6 +981,10 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
   __syncthreads();
   tc_fence_after();
   const uint32_t tbase = s_tmem;
+  const int dcol0 = kMma ? p.mma_tb * (R / 2) : 0;  // first D column
+  // shared-memory rows were requested (the TMA tiles of the last CTAs may lie past V: zero fill)
+  const bool fill_any = kMma ? p.mma_sb > 0 : n_s > 0;
+  int mma_steps = 0;  // thread 0: steps whose MMAs were issued (their completion is awaited)
   bool tokens_ok = true;
   for (int b = 0; b < B; ++b)
     if (s_tok[b] < 0 || s_tok[b] >= V) tokens_ok = false;  // the same ids in every CTA
@@ -890,44 +992,84 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
   if (!tokens_ok) {
     if (tid == 0) set_status(p.status, kStatusBadToken);
   } else {
-    // ---- fill: shared-memory rows by bulk copies (one barrier, pieces of at most 64 KB)
+    // ---- fill: shared-memory rows by bulk copies (one barrier, pieces of at most 64 KB), or
+    //      with the MMA layout the A blocks' swizzled tiles by TMA
     if (tid == 0) {
-      const uint32_t bytes = static_cast<uint32_t>(n_s) * R * 2;
-      mbar_arrive_expect_tx(&s_fill, bytes);
-      const uint8_t* src = reinterpret_cast<const uint8_t*>(p.w2 + static_cast<size_t>(r_lo + n_t) * R);
-      for (uint32_t off = 0; off < bytes; off += 64 * 1024) {
-        const uint32_t n = min(bytes - off, 64u * 1024u);
-        bulk_load(reinterpret_cast<uint8_t*>(s_w2) + off, src + off, n, &s_fill, l2_policy_evict_first());
+      if constexpr (kMma) {
+        const int tiles = R / 64;
+        mbar_arrive_expect_tx(&s_fill, static_cast<uint32_t>(p.mma_sb * tiles * kMmaTileBytes));
+        const uint64_t pol = l2_policy_evict_first();
+        for (int sb = 0; sb < p.mma_sb; ++sb)
+          for (int a = 0; a < tiles; ++a)
+            tma_load_2d(s_al + static_cast<size_t>(sb * tiles + a) * kMmaTileBytes, &tm_w2, &s_fill, 64 * a,
+                        r_lo + 128 * (p.mma_tb + sb), pol);
+      } else {
+        const uint32_t bytes = static_cast<uint32_t>(n_s) * R * 2;
+        mbar_arrive_expect_tx(&s_fill, bytes);
+        const uint8_t* src = reinterpret_cast<const uint8_t*>(p.w2 + static_cast<size_t>(r_lo + n_t) * R);
+        for (uint32_t off = 0; off < bytes; off += 64 * 1024) {
+          const uint32_t n = min(bytes - off, 64u * 1024u);
+          bulk_load(reinterpret_cast<uint8_t*>(s_w2) + off, src + off, n, &s_fill, l2_policy_evict_first());
+        }
       }
     }
     fill_issued = true;
     // ---- u's hidden halves while the bulk copies land (read by phase B after a grid barrier)
     if (p.uh) uh_prologue(p, gw, nwarps, lane, l2_policy_evict_normal());
-    // ---- fill: tensor-memory rows.  Warp w writes lane quarter q = w % 4, rows 64 (w / 4) ..
-    //      64 (w / 4) + 63 of the quarter's 128, 4 rows (16 columns) per store.
     const int q = warp & 3, half = warp >> 2;
     const uint32_t tq = tbase + (static_cast<uint32_t>(32 * q) << 16);
     const uint64_t pol_once = l2_policy_evict_first();
-#pragma unroll 1
-    for (int g0 = 0; g0 < 64; g0 += 32) {
-      uint4 v[32];  // 8 groups of 4 rows in flight
+    if constexpr (kMma) {
+      // ---- fill: the tensor-memory A blocks.  Thread l of warp w writes lane 32 (w % 4) + l, the
+      //      row 128 i + 32 (w % 4) + l of block i in its natural order (two elements a column);
+      //      warps w and w + 4 take the two halves of the block's r / 2 columns.  Rows past the
+      //      CTA's slice are zero.
+      const int cols = R / 2, hc = R / 4;  // hc, the columns of a half: a multiple of 16
+      for (int i = 0; i < p.mma_tb; ++i) {
+        const int row = 128 * i + 32 * q + lane;
+        const bool valid = row < r_n;
+        const __nv_bfloat16* src = p.w2 + static_cast<size_t>(r_lo + (valid ? row : 0)) * R + 2 * half * hc;
+        for (int c0 = 0; c0 < hc; c0 += 16) {
+          uint32_t r[16];
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const int row = 128 * q + 64 * half + g0 + i;  // CTA-local
-        v[i] = (row < n_t && lane * 8 < R)
-                   ? ld16_hint(p.w2 + static_cast<size_t>(r_lo + row) * R + lane * 8, pol_once)
-                   : make_uint4(0, 0, 0, 0);
+          for (int v = 0; v < 4; ++v) {
+            const uint4 x = valid ? ld16_hint(src + 2 * c0 + 8 * v, pol_once) : make_uint4(0, 0, 0, 0);
+            r[4 * v] = x.x;
+            r[4 * v + 1] = x.y;
+            r[4 * v + 2] = x.z;
+            r[4 * v + 3] = x.w;
+          }
+          tc_st_x16(tq + static_cast<uint32_t>(i * cols + half * hc + c0), r);
+        }
       }
+      // the B operand's rows 2B .. 15 stay zero
+      for (int e = tid; e < (R / 64) * kMmaBopTileBytes / 16; e += kRollThreads)
+        reinterpret_cast<uint4*>(s_bop)[e] = make_uint4(0, 0, 0, 0);
+    } else {
+      // ---- fill: tensor-memory rows.  Warp w writes lane quarter q = w % 4, rows 64 (w / 4) ..
+      //      64 (w / 4) + 63 of the quarter's 128, 4 rows (16 columns) per store.
+#pragma unroll 1
+      for (int g0 = 0; g0 < 64; g0 += 32) {
+        uint4 v[32];  // 8 groups of 4 rows in flight
 #pragma unroll
-      for (int gi = 0; gi < 8; ++gi) {
-        const uint32_t r[16] = {v[4 * gi].x,     v[4 * gi].y,     v[4 * gi].z,     v[4 * gi].w,
-                                v[4 * gi + 1].x, v[4 * gi + 1].y, v[4 * gi + 1].z, v[4 * gi + 1].w,
-                                v[4 * gi + 2].x, v[4 * gi + 2].y, v[4 * gi + 2].z, v[4 * gi + 2].w,
-                                v[4 * gi + 3].x, v[4 * gi + 3].y, v[4 * gi + 3].z, v[4 * gi + 3].w};
-        tc_st_x16(tq + static_cast<uint32_t>(4 * (64 * half + g0 + 4 * gi)), r);
+        for (int i = 0; i < 32; ++i) {
+          const int row = 128 * q + 64 * half + g0 + i;  // CTA-local
+          v[i] = (row < n_t && lane * 8 < R)
+                     ? ld16_hint(p.w2 + static_cast<size_t>(r_lo + row) * R + lane * 8, pol_once)
+                     : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int gi = 0; gi < 8; ++gi) {
+          const uint32_t r[16] = {v[4 * gi].x,     v[4 * gi].y,     v[4 * gi].z,     v[4 * gi].w,
+                                  v[4 * gi + 1].x, v[4 * gi + 1].y, v[4 * gi + 1].z, v[4 * gi + 1].w,
+                                  v[4 * gi + 2].x, v[4 * gi + 2].y, v[4 * gi + 2].z, v[4 * gi + 2].w,
+                                  v[4 * gi + 3].x, v[4 * gi + 3].y, v[4 * gi + 3].z, v[4 * gi + 3].w};
+          tc_st_x16(tq + static_cast<uint32_t>(4 * (64 * half + g0 + 4 * gi)), r);
+        }
       }
     }
-    tc_wait_st();  // a warp reads back only what it wrote itself
+    tc_wait_st();  // (!kMma) a warp reads back only what it wrote itself; (kMma) the MMA reads
+                   // the A blocks after the step's first barrier
     for (int r = tid; r < r_n; r += kRollThreads) s_b2[r] = p.b2 ? bf2f(p.b2[r_lo + r]) : 0.f;
 
     constexpr int kRows = WidePass<KB>::kRows, kGroup = WidePass<KB>::kGroup;
@@ -954,9 +1096,62 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
         u_phase(p, j, hcur, gw, nwarps, lane, pol_ab);
         if (!grid_barrier(p.barrier, nbar++, p.status, &s_fail)) break;
       }
-      for (int e = tid; e < B * R; e += kRollThreads) s_u[e] = __ldcg(p.u + e);
+      for (int e = tid; e < B * R; e += kRollThreads) {
+        const float v = __ldcg(p.u + e);
+        s_u[e] = v;
+        if constexpr (kMma) {  // u_j as the B operand: rows 2b (bf16 of u) and 2b + 1 (the rest)
+          const int b = e / R, k = e - b * R;
+          const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+          const __nv_bfloat16 lo = __float2bfloat16_rn(v - __bfloat162float(hi));
+          *reinterpret_cast<__nv_bfloat16*>(s_bop + bop_offset(2 * b, k)) = hi;
+          *reinterpret_cast<__nv_bfloat16*>(s_bop + bop_offset(2 * b + 1, k)) = lo;
+        }
+      }
+      if constexpr (kMma) {
+        fence_proxy_async_smem();  // the B operand, for the tensor core
+        tc_fence_before();
+      }
       cp_async_wait_all();
       compute_sync();
+      if constexpr (kMma) {
+        // ---- lane 0 of warp 7 - (i % 8) issues block i's MMAs, and each issuing thread commits
+        //      once (a thread issues a K step in about 150 cycles, so the blocks go out in
+        //      parallel); the epilogue below waits for every commit
+        if (lane == 0 && kRollWarps - 1 - warp < n_blk) {
+          bool ok = true;
+          if (j == 0 && fill_any) ok = mbar_wait(&s_fill, 0, &s_fail, p.status);
+          if (ok) {
+            tc_fence_after();
+            constexpr uint32_t kIdesc = idesc_bf16_f32(128, 16);
+            const uint64_t bd0 = smem_desc_sw128(smem_u32(s_bop));
+            const uint32_t ab_a = smem_u32(s_al);
+            const int ksteps = R / 16;
+            for (int i = kRollWarps - 1 - warp; i < n_blk; i += kRollWarps) {
+              const uint32_t d = tbase + static_cast<uint32_t>(dcol0 + 16 * i);
+              if (i < p.mma_tb) {
+                const uint32_t a0 = tbase + static_cast<uint32_t>(i * (R / 2));
+#pragma unroll 4
+                for (int kk = 0; kk < ksteps; ++kk)
+                  tc_mma_bf16_ta(d, a0 + static_cast<uint32_t>(8 * kk),
+                                 bd0 + static_cast<uint64_t>((kk >> 2) * (kMmaBopTileBytes >> 4) + 2 * (kk & 3)), kIdesc,
+                                 kk > 0 ? 1u : 0u);
+              } else {
+                const uint64_t ad0 =
+                    smem_desc_sw128(ab_a + static_cast<uint32_t>((i - p.mma_tb) * (R / 64) * kMmaTileBytes));
+#pragma unroll 4
+                for (int kk = 0; kk < ksteps; ++kk)
+                  tc_mma_bf16(d, ad0 + static_cast<uint64_t>((kk >> 2) * (kMmaTileBytes >> 4) + 2 * (kk & 3)),
+                              bd0 + static_cast<uint64_t>((kk >> 2) * (kMmaBopTileBytes >> 4) + 2 * (kk & 3)), kIdesc,
+                              kk > 0 ? 1u : 0u);
+              }
+            }
+            tc_commit(&s_mma);
+          } else {
+            mbar_arrive(&s_mma);  // nothing issued: the epilogue's wait ends (the step fails)
+          }
+        }
+        if (tid == 0) ++mma_steps;
+      }
       float ur[KB][8];  // u at this lane's 8 columns (zero past r)
 #pragma unroll
       for (int b = 0; b < KB; ++b)
@@ -977,70 +1172,107 @@ __global__ void __launch_bounds__(kRollThreads, 1) rollout_resident_kernel(const
         wide_push<KB>(dot, lane, min(kGroup, n_g - r0), n_t + n_s + r0, r_lo + n_t + n_s + r0, s_base, s_b2,
                       rows_cta, B, mine, glg, V);
       }
-      // rows in tensor memory: this warp's 64 rows of its lane quarter, 8 rows (32 columns) a load
-      for (int rho0 = 64 * half; rho0 < 64 * half + 64; rho0 += kRows) {
-        const int row0 = 128 * q + rho0;
-        if (row0 >= n_t) break;
-        float dot[32] = {};
+      Lse st[KB];
 #pragma unroll
-        for (int g = 0; g < kRows; g += kGroup) {
-          uint4 raw[kGroup];
-          if (kGroup == 8) {
-            float t[32];
-            tc_ld_x32(tq + static_cast<uint32_t>(4 * (rho0 + g)), t);
+      for (int b = 0; b < KB; ++b) st[b] = lse_empty();
+      if constexpr (kMma) {
+        // ---- epilogue: warp w reads lane quarter w % 4 of every other D block (warps w and
+        //      w + 4 alternate), one row per thread, in increasing row order
+        const bool done = mbar_wait(&s_mma, static_cast<uint32_t>(j & 1), &s_fail, p.status);
+        if (__all_sync(0xffffffffu, done)) {  // warp-uniform: the loads are .sync.aligned
+          tc_fence_after();
+          for (int i = half; i < n_blk; i += 2) {
+            float d[4];
+            tc_ld_x4(tq + static_cast<uint32_t>(dcol0 + 16 * i), d);
             tc_wait_ld();
+            const int row = 128 * i + 32 * q + lane;
+            if (row < r_n) {
 #pragma unroll
-            for (int r = 0; r < kGroup; ++r)
-              raw[r] = make_uint4(__float_as_uint(t[4 * r]), __float_as_uint(t[4 * r + 1]),
-                                  __float_as_uint(t[4 * r + 2]), __float_as_uint(t[4 * r + 3]));
-          } else {
-            float t[16];
-            tc_ld_x16(tq + static_cast<uint32_t>(4 * (rho0 + g)), t);
-            tc_wait_ld();
-#pragma unroll
-            for (int r = 0; r < kGroup; ++r)
-              raw[r] = make_uint4(__float_as_uint(t[4 * r]), __float_as_uint(t[4 * r + 1]),
-                                  __float_as_uint(t[4 * r + 2]), __float_as_uint(t[4 * r + 3]));
+              for (int b = 0; b < KB; ++b) {
+                if (b < B) {
+                  const float logit = s_base[b * rows_cta + row] + s_b2[row] + (d[2 * b] + d[2 * b + 1]);
+                  if (glg) glg[static_cast<size_t>(b) * V + r_lo + row] = logit;
+                  lse_push(st[b], logit, r_lo + row);
+                }
+              }
+            }
           }
-          group_fma<KB, kGroup>(raw, g, ur, dot);
         }
-        wide_push<KB>(dot, lane, n_t - row0, row0, r_lo + row0, s_base, s_b2, rows_cta, B, mine, glg, V);
-      }
-      // rows in shared memory (landed before the first step's phase C)
-      bool filled = true;
-      if (j == 0 && n_s > 0) filled = mbar_wait(&s_fill, 0, &s_fail, p.status);
-      if (__all_sync(0xffffffffu, filled && !s_fail)) {  // warp-uniform: the passes shuffle
-        for (int r0 = warp * kRows; r0 < n_s; r0 += kRollWarps * kRows) {
+        tc_fence_before();  // every read of D before the next step's MMAs overwrite it
+      } else {
+        // rows in tensor memory: this warp's 64 rows of its lane quarter, 8 rows (32 columns) a load
+        for (int rho0 = 64 * half; rho0 < 64 * half + 64; rho0 += kRows) {
+          const int row0 = 128 * q + rho0;
+          if (row0 >= n_t) break;
           float dot[32] = {};
 #pragma unroll
           for (int g = 0; g < kRows; g += kGroup) {
             uint4 raw[kGroup];
+            if (kGroup == 8) {
+              float t[32];
+              tc_ld_x32(tq + static_cast<uint32_t>(4 * (rho0 + g)), t);
+              tc_wait_ld();
 #pragma unroll
-            for (int r = 0; r < kGroup; ++r)
-              raw[r] = (r0 + g + r < n_s && lane * 8 < R)
-                           ? *reinterpret_cast<const uint4*>(
-                                 s_w2 + ((r0 + g + r < n_s && lane * 8 < R) ? static_cast<size_t>(r0 + g + r) * R +
-                                                                                   lane * 8
-                                                                             : 0))
-                           : make_uint4(0, 0, 0, 0);
+              for (int r = 0; r < kGroup; ++r)
+                raw[r] = make_uint4(__float_as_uint(t[4 * r]), __float_as_uint(t[4 * r + 1]),
+                                    __float_as_uint(t[4 * r + 2]), __float_as_uint(t[4 * r + 3]));
+            } else {
+              float t[16];
+              tc_ld_x16(tq + static_cast<uint32_t>(4 * (rho0 + g)), t);
+              tc_wait_ld();
+#pragma unroll
+              for (int r = 0; r < kGroup; ++r)
+                raw[r] = make_uint4(__float_as_uint(t[4 * r]), __float_as_uint(t[4 * r + 1]),
+                                    __float_as_uint(t[4 * r + 2]), __float_as_uint(t[4 * r + 3]));
+            }
             group_fma<KB, kGroup>(raw, g, ur, dot);
           }
-          wide_push<KB>(dot, lane, n_s - r0, n_t + r0, r_lo + n_t + r0, s_base, s_b2, rows_cta, B, mine, glg,
-                        V);
+          wide_push<KB>(dot, lane, n_t - row0, row0, r_lo + row0, s_base, s_b2, rows_cta, B, mine, glg, V);
+        }
+        // rows in shared memory (landed before the first step's phase C)
+        bool filled = true;
+        if (j == 0 && n_s > 0) filled = mbar_wait(&s_fill, 0, &s_fail, p.status);
+        if (__all_sync(0xffffffffu, filled && !s_fail)) {  // warp-uniform: the passes shuffle
+          for (int r0 = warp * kRows; r0 < n_s; r0 += kRollWarps * kRows) {
+            float dot[32] = {};
+#pragma unroll
+            for (int g = 0; g < kRows; g += kGroup) {
+              uint4 raw[kGroup];
+#pragma unroll
+              for (int r = 0; r < kGroup; ++r)
+                raw[r] = (r0 + g + r < n_s && lane * 8 < R)
+                             ? *reinterpret_cast<const uint4*>(
+                                   s_w2 + ((r0 + g + r < n_s && lane * 8 < R) ? static_cast<size_t>(r0 + g + r) * R +
+                                                                                     lane * 8
+                                                                               : 0))
+                             : make_uint4(0, 0, 0, 0);
+              group_fma<KB, kGroup>(raw, g, ur, dot);
+            }
+            wide_push<KB>(dot, lane, n_s - r0, n_t + r0, r_lo + n_t + r0, s_base, s_b2, rows_cta, B, mine, glg,
+                          V);
+          }
         }
       }
-      Lse st[KB];
+      // the L2 rows (and, in the CUDA-core layout, every row) of this lane's sequence
+      // lane % KB; ties go to the lower id
 #pragma unroll
-      for (int b = 0; b < KB; ++b) st[b] = (b == lane % KB) ? mine : lse_empty();
+      for (int b = 0; b < KB; ++b)
+        if (b == lane % KB) lse_merge(st[b], mine);
       if (!finish_step<KB>(p, j, st, s_red, s_tok, nbar, &s_fail, s_base, r_lo, r_n, rows_cta, true)) break;
+      if (j + 1 == K && p.best) greedy_logp<KB>(p, s_red);
     }
   }
-  // ---- teardown: the asynchronous copies have landed (the fill: bounded), tensor memory is
-  //      released
+  // ---- teardown: the asynchronous copies have landed (the fill: bounded), the MMAs are done
+  //      (bounded), tensor memory is released
   cp_async_wait_all();
-  if (tid == 0 && fill_issued && n_s > 0) {
+  if (tid == 0 && fill_issued && fill_any) {
     const long long t0 = clock64();
     while (!mbar_try_wait(&s_fill, 0))
+      if (clock64() - t0 > kWaitCycles) break;
+  }
+  if (kMma && tid == 0 && mma_steps > 0) {
+    const long long t0 = clock64();
+    while (!mbar_try_wait(&s_mma, static_cast<uint32_t>((mma_steps - 1) & 1)))
       if (clock64() - t0 > kWaitCycles) break;
   }
   tc_fence_before();
@@ -1204,6 +1436,7 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
     }
     if (!finish_step<KB>(p, j, st, s_red, s_tok, nbar, &s_fail, s_base, r_lo, r_n, rows_cta, false)) return;
   }
+  if (p.best) greedy_logp<KB>(p, s_red);
 }
 
 // ================================================================ launch
@@ -1234,15 +1467,15 @@ size_t rollout_smem_bytes(int B, int V, int R, bool head, int grid) {
          static_cast<size_t>(B) * rollout_rows_per_cta(V, R, head, grid) * sizeof(float);
 }
 
-template <typename Kern>
+template <typename Kern, typename... Extra>
 static cudaError_t launch_coop(Kern kern, const RolloutParams& p, int grid, int threads, size_t smem,
-                               cudaStream_t stream) {
+                               cudaStream_t stream, Extra... extra) {
   if (smem > 48 * 1024) {
     const cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(kern), smem, false);
     if (e != cudaSuccess) return e;
   }
   RolloutParams pp = p;
-  void* args[] = {&pp};
+  void* args[] = {&pp, &extra...};
   cudaError_t e = cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(kern), dim3(grid), dim3(threads), args,
                                               smem, stream);
   if (e != cudaSuccess) return e;
@@ -1259,13 +1492,51 @@ static bool use_fast_gates(const RolloutParams& p, int grid) {
          resident_smem_rows(p.B, p.V, p.R, grid, static_cast<long long>(p.B) * p.Ds * 4 + 16) >= 0;
 }
 
+// Phase C on the tensor cores (two-barrier steps, at most two sequences, r a multiple of 64 up to
+// 256): the 128-row blocks of a CTA's rows, tb in tensor memory and sb in shared memory, that
+// cover the most rows (tensor memory first: an A block there costs r/2 columns and its D 16 more;
+// one in shared memory costs 128 r bf16 beside the fixed buffers).  False when the layout does
+// not apply or would leave more than kMmaMaxL2Rows rows of a CTA to read through L2 every step.
+static bool mma_blocks(const RolloutParams& p, int grid, int* tb, int* sb, size_t* smem) {
+  *tb = *sb = 0;
+  if (!use_fast_gates(p, grid) || p.B > 2 || p.R % 64 != 0 || p.R > 256) return false;
+  const int rows_cta = resident_rows_per_cta(p.V, grid);
+  const int need = (rows_cta + 127) / 128;
+  const long long fixed = 1024 + static_cast<long long>(p.R / 64) * kMmaBopTileBytes +
+                          static_cast<long long>(p.B) * p.R * 4 + static_cast<long long>(p.B + 1) * rows_cta * 4 +
+                          static_cast<long long>(p.B) * p.Ds * 4 + 16;
+  const long long blk = static_cast<long long>(p.R / 64) * kMmaTileBytes;
+  if (fixed > static_cast<long long>(kRollMaxSmem)) return false;
+  const int s_max = static_cast<int>((static_cast<long long>(kRollMaxSmem) - fixed) / blk);
+  int bt = 0, bs = 0;
+  for (int t = 0; t <= need; ++t) {
+    const int room = kTmemCols - t * (p.R / 2);  // columns left for the D blocks
+    if (room < 16 * t) break;
+    const int s = std::min(std::min(s_max, need - t), room / 16 - t);
+    if (s < 0) continue;
+    if (t + s > bt + bs || (t + s == bt + bs && t > bt)) { bt = t; bs = s; }
+  }
+  if (bt + bs == 0 || rows_cta - 128 * (bt + bs) > kMmaMaxL2Rows) return false;
+  *tb = bt;
+  *sb = bs;
+  *smem = static_cast<size_t>(fixed + bs * blk);
+  return true;
+}
+
 template <int KB>
-static cudaError_t launch_rollout_kb(const RolloutParams& p, int grid, size_t smem, cudaStream_t stream) {
-  if (use_resident(p)) return launch_coop(rollout_resident_kernel<KB>, p, grid, kRollThreads, smem, stream);
+static cudaError_t launch_rollout_kb(const RolloutParams& p, int grid, size_t smem, cudaStream_t stream,
+                                     const CUtensorMap& tm) {
+  if (use_resident(p)) {
+    if constexpr (KB <= 2) {
+      if (p.mma_tb + p.mma_sb > 0)
+        return launch_coop(rollout_resident_kernel<KB, true>, p, grid, kRollThreads, smem, stream, tm);
+    }
+    return launch_coop(rollout_resident_kernel<KB, false>, p, grid, kRollThreads, smem, stream, tm);
+  }
   return launch_coop(rollout_kernel<KB>, p, grid, kRollThreadsAll, smem, stream);
 }
 
-cudaError_t launch_rollout(const RolloutParams& p, int grid, cudaStream_t stream) {
+cudaError_t launch_rollout(const RolloutParams& p, int grid, cudaStream_t stream, const CUtensorMap* tm_w2) {
   if (p.B < 1 || p.B > kRollMaxB || grid < 1) return cudaErrorInvalidValue;
   if (p.uniforms && (grid > kRollThreads || !p.lg)) return cudaErrorInvalidValue;  // one thread per CTA
   size_t smem = rollout_smem_bytes(p.B, p.V, p.R, p.head, grid);
@@ -1273,18 +1544,30 @@ cudaError_t launch_rollout(const RolloutParams& p, int grid, cudaStream_t stream
   RolloutParams pp = p;
   pp.smem_rows = use_resident(p) ? resident_smem_rows(p.B, p.V, p.R, grid) : 0;
   pp.fast_gates = use_fast_gates(p, grid) ? 1 : 0;
+  pp.mma_tb = pp.mma_sb = 0;
   if (pp.fast_gates) {
     const long long hbytes = static_cast<long long>(p.B) * p.Ds * 4 + 16;  // + alignment of s_h
     pp.smem_rows = resident_smem_rows(p.B, p.V, p.R, grid, hbytes);
     smem = static_cast<size_t>(pp.smem_rows) * p.R * 2 + static_cast<size_t>(p.B) * p.R * 4 +
            static_cast<size_t>(p.B + 1) * resident_rows_per_cta(p.V, grid) * 4 + static_cast<size_t>(hbytes);
+    int tb = 0, sb = 0;
+    size_t mma_smem = 0;
+    if (tm_w2 != nullptr && mma_blocks(pp, grid, &tb, &sb, &mma_smem)) {
+      pp.mma_tb = tb;
+      pp.mma_sb = sb;
+      pp.smem_rows = 0;
+      smem = mma_smem;
+    }
     if (smem > kRollMaxSmem) return cudaErrorInvalidValue;
   }
   if (!use_resident(p)) pp.uh = nullptr;  // only the resident kernel computes it before its steps
-  if (p.B <= 1) return launch_rollout_kb<1>(pp, grid, smem, stream);
-  if (p.B <= 2) return launch_rollout_kb<2>(pp, grid, smem, stream);
-  if (p.B <= 4) return launch_rollout_kb<4>(pp, grid, smem, stream);
-  return launch_rollout_kb<8>(pp, grid, smem, stream);
+  CUtensorMap tm;
+  if (tm_w2 != nullptr) tm = *tm_w2;
+  else memset(&tm, 0, sizeof(tm));  // never read: phase C stays on the CUDA cores
+  if (p.B <= 1) return launch_rollout_kb<1>(pp, grid, smem, stream, tm);
+  if (p.B <= 2) return launch_rollout_kb<2>(pp, grid, smem, stream, tm);
+  if (p.B <= 4) return launch_rollout_kb<4>(pp, grid, smem, stream, tm);
+  return launch_rollout_kb<8>(pp, grid, smem, stream, tm);
 }
 
 }  // namespace dm

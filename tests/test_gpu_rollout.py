@@ -134,6 +134,22 @@ def test_rollout_with_input_table_matches_oracle(cfg):
     _check(_full_emb(inputs.make_workload(cfg)), table=True)
 
 
+# Phase C on the tensor cores (the table's two-barrier step, B <= 2, r a multiple of 64 up to 256):
+# W2 blocks of 128 rows in tensor memory only (small vocabularies), in tensor and shared memory
+# (r = 128 and 256), and with the rows past those blocks read through L2 (V past 152 x 768).
+MMA_CASES = [
+    inputs.custom_config("mma-r64", B=1, K=6, H=256, V=5000, Ds=64, R=64, seed=51, biases=True),
+    inputs.custom_config("mma-r128-b2", B=2, K=4, H=256, V=160003, Ds=64, R=128, seed=52),
+    inputs.custom_config("mma-r256-b2", B=2, K=4, H=256, V=160003, Ds=32, R=256, seed=53, biases=True),
+    inputs.custom_config("mma-r192-b1", B=1, K=3, H=128, V=120007, Ds=32, R=192, seed=54),
+]
+
+
+@pytest.mark.parametrize("cfg", MMA_CASES)
+def test_rollout_tensor_core_phase_c_matches_oracle(cfg):
+    _check(_full_emb(inputs.make_workload(cfg)), table=True)
+
+
 def test_rollout_head_off():
     _check(inputs.make_workload(inputs.custom_config("roll-off", B=2, K=6, H=256, V=2000, seed=24)), head_on=False)
 
@@ -282,6 +298,11 @@ def test_rollout_sample_with_input_table_matches_oracle(cfg):
     _check_sample(_full_emb(inputs.make_workload(cfg)), table=True)
 
 
+@pytest.mark.parametrize("cfg", [MMA_CASES[0], MMA_CASES[1], MMA_CASES[2]])
+def test_rollout_sample_tensor_core_phase_c_matches_oracle(cfg):
+    _check_sample(_full_emb(inputs.make_workload(cfg)), seed=9, table=True)
+
+
 def test_rollout_sample_head_off():
     _check_sample(inputs.make_workload(inputs.custom_config("samp-off", B=2, K=6, H=256, V=2000, seed=35)),
                   head_on=False)
@@ -290,6 +311,10 @@ def test_rollout_sample_head_off():
 @pytest.mark.parametrize("name", ["qwen3-8b"])
 def test_rollout_sample_full_size(name):
     _check_sample(_full_size(name), seed=7)
+
+
+def test_rollout_sample_full_size_with_input_table():
+    _check_sample(_full_size("qwen3-8b"), seed=8, table=True)
 
 
 def test_rollout_sample_uniform_ends_and_bad_pointer():
