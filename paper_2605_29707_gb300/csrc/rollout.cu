@@ -412,76 +412,90 @@ __device__ __forceinline__ void gates_all(const RolloutParams& p, int j, const i
 //      from the CTA's shared memory: u_j = SiLU(uh + W1[q, H:] h_j + b1), and gh_j = W_hh h_j for
 //      the next step's gates.  A finished row of u is counted in p.ucount (release), which phase C
 //      waits for instead of a grid barrier; the gh rows are next needed after the step's partials
-//      barrier.  A warp takes its rows three at a time (R + 3 Ds rows over the grid's warps: one
-//      round for d_s = 1024 and r = 256 on 152 SMs), with every weight load of the three issued
-//      before the arithmetic (Ds <= 1024: at most 4 chunks of 8 columns per lane and row).
-template <int KB>
-__device__ __forceinline__ void ub_phase(const RolloutParams& p, int j, const float* s_h, int gw, int nwarps,
-                                         int lane, uint64_t pol) {
+//      barrier.  When the grid has more warps than u has rows, warp q < R computes row q of u
+//      alone (phase C waits for those) and the other warps take the W_hh rows four at a time;
+//      otherwise every warp takes its rows three at a time.  Every weight load of a warp's rows is
+//      issued before the arithmetic (Ds <= 1024: at most 4 chunks of 8 columns per lane and row).
+template <int KB, int NR>
+__device__ __forceinline__ void ub_rows(const RolloutParams& p, int j, const float* s_h, int row0, int stride,
+                                        int rows, int lane, uint64_t pol) {
   const int B = p.B, K = p.K, H = p.H, Ds = p.Ds, R = p.R;
-  const int rows = R + (j + 1 < K ? 3 * Ds : 0);
   float* gh = p.gh + static_cast<size_t>(j & 1) * B * 3 * Ds;
-  constexpr int kCh = 4, kRowsAt = 3;
-  for (int row0 = gw; row0 < rows; row0 += kRowsAt * nwarps) {
-    uint4 wraw[kRowsAt][kCh];
+  constexpr int kCh = 4;
+  uint4 wraw[NR][kCh];
 #pragma unroll
-    for (int k = 0; k < kRowsAt; ++k) {
-      const int row = row0 + k * nwarps;
-      const __nv_bfloat16* w = row >= rows ? nullptr
-                               : row < R   ? p.w1 + static_cast<size_t>(row) * (H + Ds) + H
-                                           : p.w_hh + static_cast<size_t>(row - R) * Ds;
-#pragma unroll
-      for (int i = 0; i < kCh; ++i) {
-        const int c = lane * 8 + 256 * i;
-        wraw[k][i] = (w != nullptr && c < Ds) ? ld16_hint(w + c, pol) : make_uint4(0, 0, 0, 0);
-      }
-    }
-    float acc[kRowsAt][KB];
-#pragma unroll
-    for (int k = 0; k < kRowsAt; ++k)
-#pragma unroll
-      for (int b = 0; b < KB; ++b) acc[k][b] = 0.f;
+  for (int k = 0; k < NR; ++k) {
+    const int row = row0 + k * stride;
+    const __nv_bfloat16* w = row >= rows ? nullptr
+                             : row < R   ? p.w1 + static_cast<size_t>(row) * (H + Ds) + H
+                                         : p.w_hh + static_cast<size_t>(row - R) * Ds;
 #pragma unroll
     for (int i = 0; i < kCh; ++i) {
       const int c = lane * 8 + 256 * i;
-      if (c >= Ds) break;
-      float wv[kRowsAt][8];
+      wraw[k][i] = (w != nullptr && c < Ds) ? ld16_hint(w + c, pol) : make_uint4(0, 0, 0, 0);
+    }
+  }
+  float acc[NR][KB];
 #pragma unroll
-      for (int k = 0; k < kRowsAt; ++k) unpack8(wraw[k][i], wv[k]);
+  for (int k = 0; k < NR; ++k)
 #pragma unroll
-      for (int b = 0; b < KB; ++b) {
-        if (b < B) {
-          const float4 h0 = *reinterpret_cast<const float4*>(s_h + static_cast<size_t>(b) * Ds + c);
-          const float4 h1 = *reinterpret_cast<const float4*>(s_h + static_cast<size_t>(b) * Ds + c + 4);
+    for (int b = 0; b < KB; ++b) acc[k][b] = 0.f;
 #pragma unroll
-          for (int k = 0; k < kRowsAt; ++k)
-            acc[k][b] += wv[k][0] * h0.x + wv[k][1] * h0.y + wv[k][2] * h0.z + wv[k][3] * h0.w +
-                         wv[k][4] * h1.x + wv[k][5] * h1.y + wv[k][6] * h1.z + wv[k][7] * h1.w;
-        }
+  for (int i = 0; i < kCh; ++i) {
+    const int c = lane * 8 + 256 * i;
+    if (c >= Ds) break;
+    float wv[NR][8];
+#pragma unroll
+    for (int k = 0; k < NR; ++k) unpack8(wraw[k][i], wv[k]);
+#pragma unroll
+    for (int b = 0; b < KB; ++b) {
+      if (b < B) {
+        const float4 h0 = *reinterpret_cast<const float4*>(s_h + static_cast<size_t>(b) * Ds + c);
+        const float4 h1 = *reinterpret_cast<const float4*>(s_h + static_cast<size_t>(b) * Ds + c + 4);
+#pragma unroll
+        for (int k = 0; k < NR; ++k)
+          acc[k][b] += wv[k][0] * h0.x + wv[k][1] * h0.y + wv[k][2] * h0.z + wv[k][3] * h0.w +
+                       wv[k][4] * h1.x + wv[k][5] * h1.y + wv[k][6] * h1.z + wv[k][7] * h1.w;
       }
     }
+  }
 #pragma unroll
-    for (int k = 0; k < kRowsAt; ++k) {
-      const int row = row0 + k * nwarps;
+  for (int k = 0; k < NR; ++k) {
+    const int row = row0 + k * stride;
 #pragma unroll
-      for (int b = 0; b < KB; ++b) {
-        if (b < B) {
-          const float a = warp_sum(acc[k][b]);
-          if (lane == 0 && row < rows) {
-            if (row < R) {
-              // uh: written before the steps by other CTAs of this launch (ordered by the barriers)
-              const float x = a + __ldcg(p.uh + (static_cast<size_t>(b) * K + j) * R + row) +
-                              (p.b1 ? bf2f(p.b1[row]) : 0.f);
-              p.u[static_cast<size_t>(b) * R + row] = x / (1.f + expf(-x));
-            } else {
-              gh[static_cast<size_t>(b) * 3 * Ds + row - R] = a;
-            }
+    for (int b = 0; b < KB; ++b) {
+      if (b < B) {
+        const float a = warp_sum(acc[k][b]);
+        if (lane == 0 && row < rows) {
+          if (row < R) {
+            const float x = a + __ldcg(p.uh + (static_cast<size_t>(b) * K + j) * R + row) +
+                            (p.b1 ? bf2f(p.b1[row]) : 0.f);
+            p.u[static_cast<size_t>(b) * R + row] = x / (1.f + expf(-x));
+          } else {
+            gh[static_cast<size_t>(b) * 3 * Ds + row - R] = a;
           }
         }
       }
-      if (lane == 0 && row < R)  // this row of u_j is written for every sequence
-        asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(p.ucount) : "memory");
     }
+    if (lane == 0 && row < R)  // this row of u_j is written for every sequence
+      asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(p.ucount) : "memory");
+  }
+}
+
+template <int KB>
+__device__ __forceinline__ void ub_phase(const RolloutParams& p, int j, const float* s_h, int gw, int nwarps,
+                                         int lane, uint64_t pol) {
+  const int R = p.R;
+  const int rows = R + (j + 1 < p.K ? 3 * p.Ds : 0);
+  if (nwarps > R) {
+    if (gw < R) {
+      ub_rows<KB, 1>(p, j, s_h, gw, 0, R, lane, pol);
+    } else {
+      const int n = nwarps - R;
+      for (int row0 = gw; row0 < rows; row0 += 4 * n) ub_rows<KB, 4>(p, j, s_h, row0, n, rows, lane, pol);
+    }
+  } else {
+    for (int row0 = gw; row0 < rows; row0 += 3 * nwarps) ub_rows<KB, 3>(p, j, s_h, row0, nwarps, rows, lane, pol);
   }
 }
 
