@@ -864,8 +864,9 @@ int make_roll_plan(int B, int K, int H, int V, int Ds, int R, bool head, RollPla
   p.off_h = take(static_cast<size_t>(2) * B * (p.Ds > 0 ? p.Ds : 1) * 4);
   p.clear_bytes = off;
   p.off_u = take(static_cast<size_t>(B) * (p.R > 0 ? p.R : 1) * 4);
-  // greedy: every step's (the log-probabilities are merged at the end); sampled: two, by step parity
-  p.off_part = take(static_cast<size_t>(K > 2 ? K : 2) * p.grid * dm::kRollMaxB * 16);
+  // greedy: every step's, per warp (the log-probabilities are merged at the end); sampled: two,
+  // by step parity, per CTA
+  p.off_part = take(static_cast<size_t>(K > 2 ? K : 2) * p.grid * dm::kRollComputeWarps * dm::kRollMaxB * 16);
   p.off_lg = take(static_cast<size_t>(2) * B * V * 4);  // sampled mode: final logits, by step parity
   p.off_base = take(static_cast<size_t>(p.M) * V * 4);
   p.off_uh = take(static_cast<size_t>(p.M) * (p.R > 0 ? p.R : 1) * 4);  // hidden . W1[:, :H]^T

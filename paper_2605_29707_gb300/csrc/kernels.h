@@ -187,6 +187,7 @@ cudaError_t launch_merge_tree(const TreeParams& p, cudaStream_t stream);
 // ---------------------------------------------------------------- greedy rollout (rollout.cu)
 constexpr int kRollMaxB = 8;  // sequences per rollout launch
 constexpr unsigned kGreedyIdMask = 0x3FFFFFu;  // greedy rollout keys: token ids below 2^22
+constexpr int kRollComputeWarps = 8;             // compute warps of a rollout CTA
 struct RolloutParams {
   const __nv_bfloat16* hidden;  // [B, K, H]
   const int32_t* anchors;       // [B]
@@ -197,8 +198,9 @@ struct RolloutParams {
   const float* base;            // [B*K, V] W_lm hidden (fp32, from the store-mode GEMM)
   float* h;                     // [2][B][Ds] GRU states (cleared: h_{-1} = 0)
   float* u;                     // [B][R]
-  float* partials;              // float4 (max, sum exp, argmax bits, 0) per CTA and sequence:
-                                // greedy [K][grid][kRollMaxB]; sampled [2][grid][kRollMaxB], by step parity
+  float* partials;              // float4 (max, sum exp, argmax bits, 0) per sequence: greedy with keys
+                                // [K][grid][kRollComputeWarps][kRollMaxB] (per warp); otherwise
+                                // [2][grid][kRollMaxB] (per CTA), by step parity
   unsigned long long* best;     // greedy: [2][kRollMaxB] keys of each sequence's argmax by step parity
                                 // (cleared), or nullptr
                                 // (sampled mode, or V >= 2^22: every CTA combines the partials instead)

@@ -32,6 +32,7 @@ namespace dm {
 
 constexpr int kRollThreads = 256;                   // the compute warps
 constexpr int kRollWarps = kRollThreads / 32;
+static_assert(kRollWarps == kRollComputeWarps, "the greedy partials are sized per compute warp");
 constexpr int kRollThreadsAll = kRollThreads + 32;  // streamed kernel: + one warp feeding the W2 ring
 constexpr int kW2Stages = 6;                        // shared-memory ring of W2 chunks
 constexpr int kW2StageBytes = 16 * 1024;            // one chunk: kW2StageBytes / (2 r) rows of W2
@@ -765,19 +766,101 @@ __device__ void sample_step(const RolloutParams& p, int j, const float4 (&mine)[
   compute_sync();
 }
 
-// Greedy key of a CTA's best row at step j: the step (so that no earlier step's key competes),
-// the logit in order-preserving form, then the id inverted, so that the largest key over the CTAs
-// is the step's maximum with ties to the lowest id (ids below 2^22).
-__device__ __forceinline__ unsigned long long greedy_key(int j, float m, int id) {
-  return (static_cast<unsigned long long>(j + 1) << 54) | (static_cast<unsigned long long>(f32_ord(m)) << 22) |
-         static_cast<unsigned long long>(kGreedyIdMask - static_cast<unsigned>(id));
+// Greedy end of step j (p.best set): the CTA's best row of each sequence as one key -- the step
+// (so that no earlier step's key competes), the logit in order-preserving form, then the id
+// inverted, so that the largest key over the CTAs is the step's maximum with ties to the lowest
+// id (ids below 2^22) -- from two integer warp reductions per warp; thread 0 folds the warps'
+// keys into the sequence's slot with one red.max and arrives at the grid barrier.  While the
+// other CTAs arrive, each warp reduces its (max, sum of exp) of every sequence and writes it to
+// the step's partials (the log-probabilities are merged from them once, after the last step:
+// greedy_logp); then every CTA reads the slot.  The slots alternate by step parity: a CTA
+// updates step j + 2's only after every CTA has passed step j + 1's barrier, so after every read
+// of step j's.  Returns false if the barrier gave up.
+template <int KB>
+__device__ bool finish_greedy(const RolloutParams& p, int j, Lse (&st)[KB], int* s_tok, unsigned& nbar,
+                              volatile int* s_fail) {
+  __shared__ unsigned long long s_key[kRollWarps][kRollMaxB];
+  __shared__ int s_go;
+  const int B = p.B, K = p.K, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int grid = static_cast<int>(gridDim.x);
+  unsigned long long* slot = p.best + (j & 1) * kRollMaxB;
+#pragma unroll
+  for (int b = 0; b < KB; ++b) {
+    if (b < B) {
+      const bool has = st[b].i != 0x7fffffff;
+      const uint32_t hi = has ? f32_ord(st[b].m) : 0u;
+      const uint32_t lo = has ? kGreedyIdMask - static_cast<unsigned>(st[b].i) : 0u;
+      const uint32_t mhi = __reduce_max_sync(0xffffffffu, hi);
+      const uint32_t mlo = __reduce_max_sync(0xffffffffu, hi == mhi ? lo : 0u);
+      // mhi == 0: no lane has a row (an order-preserving logit is never 0)
+      if (lane == 0)
+        s_key[warp][b] = mhi != 0u ? (static_cast<unsigned long long>(j + 1) << 54) |
+                                         (static_cast<unsigned long long>(mhi) << 22) | mlo
+                                   : 0ull;
+    }
+  }
+  compute_sync();
+  if (tid == 0) {
+    for (int b = 0; b < B; ++b) {
+      unsigned long long k = 0ull;
+      for (int w = 0; w < kRollWarps; ++w) k = s_key[w][b] > k ? s_key[w][b] : k;
+      if (k != 0ull) asm volatile("red.relaxed.gpu.global.max.u64 [%0], %1;" ::"l"(slot + b), "l"(k) : "memory");
+    }
+    // release at GPU scope: this CTA's keys (and its earlier writes) before its arrival
+    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(p.barrier) : "memory");
+  }
+  // the warps' (max, sum of exp) for the log-probabilities, while the other CTAs arrive
+  float4* part = reinterpret_cast<float4*>(p.partials) +
+                 (static_cast<size_t>(j) * grid + blockIdx.x) * kRollWarps * kRollMaxB;
+#pragma unroll
+  for (int b = 0; b < KB; ++b) {
+    if (b < B) {
+      Lse a = st[b];
+#pragma unroll
+      for (int o = 16; o; o >>= 1) {
+        Lse t;
+        t.m = __shfl_xor_sync(0xffffffffu, a.m, o);
+        t.s = __shfl_xor_sync(0xffffffffu, a.s, o);
+        t.i = __shfl_xor_sync(0xffffffffu, a.i, o);
+        lse_merge(a, t);
+      }
+      if (lane == 0) part[warp * kRollMaxB + b] = make_float4(a.m, a.s, __int_as_float(a.i), 0.f);
+    }
+  }
+  if (tid == 0) {
+    const unsigned target = (nbar + 1) * static_cast<unsigned>(grid);
+    const long long t0 = clock64();
+    while (true) {
+      unsigned v;
+      asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p.barrier) : "memory");
+      if (v >= target) break;
+      if (clock64() - t0 > kWaitCycles) {
+        set_status(p.status, kStatusTimeout);
+        *s_fail = 1;
+        break;
+      }
+      __nanosleep(32);
+    }
+    s_go = *s_fail == 0;
+  }
+  ++nbar;
+  compute_sync();
+  if (!s_go) return false;
+  if (tid < B) {
+    const unsigned long long key = __ldcg(slot + tid);
+    const int tok = static_cast<int>(key >> 54) == j + 1
+                        ? static_cast<int>(kGreedyIdMask - static_cast<unsigned>(key & kGreedyIdMask))
+                        : 0;  // no row with a finite logit anywhere
+    s_tok[tid] = tok;
+    if (blockIdx.x == 0) p.tokens[static_cast<size_t>(tid) * K + j] = tok;
+  }
+  compute_sync();
+  return true;
 }
 
-// End of step j: this CTA's (max, sum exp, argmax) per sequence go to the partials and every CTA
-// picks t_{j+1} after a grid barrier.  Greedy (p.best set): each CTA also folds its argmax into
-// the sequence's key with one atomicMax before the barrier, and after it every CTA reads that key
-// (the log-probabilities come at the end of the launch from every step's partials, kept for
-// all K steps: greedy_logp); the keys alternate between two slots by step parity.  Sampled: every CTA combines all partials, and the partials and the
+// End of step j: greedy with keys (p.best set), finish_greedy.  Otherwise this CTA's (max,
+// sum exp, argmax) per sequence go to the partials, and after a grid barrier every CTA combines
+// all of them and picks t_{j+1} (argmax, or sampled).  The partials and (sampled mode) the
 // final-logit copies alternate between two buffers by step parity: a CTA writes step j + 2's
 // only after every CTA has passed step j + 1's barrier, so after every read of step j's (with
 // the correction branch off no other barrier separates consecutive steps).
@@ -787,14 +870,13 @@ __device__ __forceinline__ bool finish_step(const RolloutParams& p, int j, Lse (
                                             int r_lo, int r_n, int rows_cta, bool resident) {
   const int B = p.B, K = p.K, V = p.V, tid = threadIdx.x;
   const int grid = static_cast<int>(gridDim.x);
-  const bool greedy = p.best != nullptr;
-  float4* part = reinterpret_cast<float4*>(p.partials) + static_cast<size_t>(greedy ? j : (j & 1)) * grid * kRollMaxB;
+  if (p.best != nullptr) return finish_greedy<KB>(p, j, st, s_tok, nbar, s_fail);
+  float4* part = reinterpret_cast<float4*>(p.partials) + static_cast<size_t>(j & 1) * grid * kRollMaxB;
   block_reduce(st, s_red, B);  // ends with a barrier: every row's final logit is in s_logit
   if (tid < B) {
     Lse a = s_red[0][tid];
     for (int w = 1; w < kRollWarps; ++w) lse_merge(a, s_red[w][tid]);
     part[static_cast<size_t>(blockIdx.x) * kRollMaxB + tid] = make_float4(a.m, a.s, __int_as_float(a.i), 0.f);
-    if (greedy && a.i != 0x7fffffff) atomicMax(p.best + (j & 1) * kRollMaxB + tid, greedy_key(j, a.m, a.i));
   }
   float* lg = p.lg ? p.lg + static_cast<size_t>(j & 1) * B * V : nullptr;
   if (p.uniforms && !resident) {  // this CTA's final logits (the resident kernel wrote them in phase C)
@@ -804,21 +886,6 @@ __device__ __forceinline__ bool finish_step(const RolloutParams& p, int j, Lse (
     }
   }
   if (!grid_barrier(p.barrier, nbar++, p.status, s_fail)) return false;
-  if (greedy) {
-    if (tid < B) {
-      // every CTA's atomicMax came before its arrival at the barrier; the keys alternate between
-      // two slots by step parity (a CTA updates step j + 2's only after every CTA has passed
-      // step j + 1's barrier, hence after this read)
-      const unsigned long long key = __ldcg(p.best + (j & 1) * kRollMaxB + tid);
-      const int tok = static_cast<int>(key >> 54) == j + 1
-                          ? static_cast<int>(kGreedyIdMask - static_cast<unsigned>(key & kGreedyIdMask))
-                          : 0;  // no row with a finite logit anywhere
-      s_tok[tid] = tok;
-      if (blockIdx.x == 0) p.tokens[static_cast<size_t>(tid) * K + j] = tok;
-    }
-    compute_sync();
-    return true;
-  }
   float4 mine[KB];  // sampled mode: CTA tid's partials (grid <= kRollThreads there)
 #pragma unroll
   for (int b = 0; b < KB; ++b) {
@@ -866,18 +933,21 @@ __device__ __forceinline__ bool finish_step(const RolloutParams& p, int j, Lse (
 
 // Greedy mode, after the last step: the log-probability of each step's token.  The token is the
 // step's argmax, so its log-softmax is -log of the sum of exp(L - max) over the vocabulary, the
-// merge of every CTA's partials of that step (CTA c takes steps c, c + grid, ...).  Called by
-// the compute threads of every CTA once every step has passed its barrier.
+// merge of every warp's partials of that step (CTA c takes steps c, c + grid, ...).  Called by
+// the compute threads of every CTA after the last step; a grid barrier first orders the last
+// step's partials, which the warps write after their arrival at that step's barrier.
 template <int KB>
-__device__ void greedy_logp(const RolloutParams& p, Lse (*s_red)[kRollMaxB]) {
+__device__ void greedy_logp(const RolloutParams& p, Lse (*s_red)[kRollMaxB], unsigned& nbar, volatile int* s_fail) {
   const int B = p.B, K = p.K, tid = threadIdx.x;
   const int grid = static_cast<int>(gridDim.x);
+  if (!grid_barrier(p.barrier, nbar++, p.status, s_fail)) return;
+  const int nw = grid * kRollWarps;
   for (int j = blockIdx.x; j < K; j += grid) {
-    const float4* part = reinterpret_cast<const float4*>(p.partials) + static_cast<size_t>(j) * grid * kRollMaxB;
+    const float4* part = reinterpret_cast<const float4*>(p.partials) + static_cast<size_t>(j) * nw * kRollMaxB;
     Lse st[KB];
 #pragma unroll
     for (int b = 0; b < KB; ++b) st[b] = lse_empty();
-    for (int c = tid; c < grid; c += kRollThreads) {
+    for (int c = tid; c < nw; c += kRollThreads) {
 #pragma unroll
       for (int b = 0; b < KB; ++b) {
         if (b < B) {
@@ -1303,7 +1373,7 @@ __global__ void __launch_bounds__(kRollThreads, 1)
       for (int b = 0; b < KB; ++b)
         if (b == lane % KB) lse_merge(st[b], mine);
       if (!finish_step<KB>(p, j, st, s_red, s_tok, nbar, &s_fail, s_base, r_lo, r_n, rows_cta, true)) break;
-      if (j + 1 == K && p.best) greedy_logp<KB>(p, s_red);
+      if (j + 1 == K && p.best) greedy_logp<KB>(p, s_red, nbar, &s_fail);
     }
   }
   // ---- teardown: the asynchronous copies have landed (the fill: bounded), the MMAs are done
@@ -1480,7 +1550,7 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
     }
     if (!finish_step<KB>(p, j, st, s_red, s_tok, nbar, &s_fail, s_base, r_lo, r_n, rows_cta, false)) return;
   }
-  if (p.best) greedy_logp<KB>(p, s_red);
+  if (p.best) greedy_logp<KB>(p, s_red, nbar, &s_fail);
 }
 
 // ================================================================ launch
