@@ -859,7 +859,7 @@ int make_roll_plan(int B, int K, int H, int V, int Ds, int R, bool head, RollPla
     return o;
   };
   // status (offset 0, as for domino_check_status), the grid barrier counter (64), the u-row
-  // counter (128), the greedy argmax keys (256)
+  // counter (128), the count of warps done with uh (192), the greedy argmax keys (256)
   take(512);
   p.off_h = take(static_cast<size_t>(2) * B * (p.Ds > 0 ? p.Ds : 1) * 4);
   p.clear_bytes = off;
@@ -950,6 +950,7 @@ int rollout_entry(const void* hidden, const int32_t* anchors, const float* unifo
   rp.partials = reinterpret_cast<float*>(ws + P.off_part);
   rp.barrier = reinterpret_cast<unsigned*>(ws + 64);
   rp.ucount = reinterpret_cast<unsigned*>(ws + 128);  // cleared with the status and the barrier
+  rp.uhcount = reinterpret_cast<unsigned*>(ws + 192);
   // greedy: the argmax keys of the sequences (cleared with them), ids below 2^22
   rp.best = (!uniforms && V <= static_cast<int>(dm::kGreedyIdMask)) ? reinterpret_cast<unsigned long long*>(ws + 256)
                                                                    : nullptr;

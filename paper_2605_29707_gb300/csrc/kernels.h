@@ -216,6 +216,7 @@ struct RolloutParams {
   int fast_gates;               // set by launch_rollout: one grid barrier per step (resident kernel,
                                 // table, h_j of every sequence in each CTA's shared memory)
   unsigned* ucount;             // rows of u finished so far in this launch (cleared), fast_gates only
+  unsigned* uhcount;            // warps done with uh before the steps (cleared), fast_gates only
   int mma_tb, mma_sb;           // set by launch_rollout: phase C on the tensor cores over mma_tb
                                 // 128-row W2 blocks in tensor memory and mma_sb in shared memory
                                 // (both 0: phase C on the CUDA cores)

@@ -490,6 +490,22 @@ __device__ __forceinline__ void ub_rows(const RolloutParams& p, int j, const flo
       }
     }
   }
+  // step 0: uh comes from every warp's uh_prologue (other CTAs included); lane 0, which reads
+  // it, first waits for all of them (bounded; a timeout leaves the status set)
+  if (j == 0 && lane == 0 && row0 < R) {
+    const unsigned target = gridDim.x * static_cast<unsigned>(kRollWarps);
+    const long long t0 = clock64();
+    while (true) {
+      unsigned v;
+      asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p.uhcount) : "memory");
+      if (v >= target) break;
+      if (clock64() - t0 > kWaitCycles) {
+        set_status(p.status, kStatusTimeout);
+        break;
+      }
+      __nanosleep(32);
+    }
+  }
 #pragma unroll
   for (int k = 0; k < NR; ++k) {
     const int row = row0 + k * stride;
@@ -534,6 +550,8 @@ __device__ __forceinline__ void ub_phase(const RolloutParams& p, int j, const fl
 //      = b K + j and rank row q, the half of u's argument that does not depend on the
 //      recurrence.  Warp w takes row q = w % R and the positions m = w / R, w / R + G, ...
 //      (G = max(1, warps / R)), four at a time, so a W1 row is read once per four positions.
+//      Each warp then counts itself in p.uhcount (release): the two-barrier step reads uh before
+//      any grid barrier, so its first phase B acquires that count instead.
 __device__ void uh_prologue(const RolloutParams& p, int gw, int nwarps, int lane, uint64_t pol) {
   const int H = p.H, Ds = p.Ds, R = p.R, M = p.B * p.K;
   const int groups = max(1, nwarps / R);
@@ -565,6 +583,8 @@ __device__ void uh_prologue(const RolloutParams& p, int gw, int nwarps, int lane
       }
     }
   }
+  // every warp, with rows or without: the two-barrier step's first phase B waits for all of them
+  if (lane == 0 && p.uhcount) asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(p.uhcount) : "memory");
 }
 
 // ---- phase B: u_j = SiLU(W1 [hidden_j ; h_j] + b1), one warp per rank row q, every sequence.
@@ -1602,7 +1622,7 @@ static cudaError_t launch_coop(Kern kern, const RolloutParams& p, int grid, int 
 static bool use_fast_gates(const RolloutParams& p, int grid) {
   // gates_all reads the biases four at a time (8-byte loads)
   const bool bias_ok = (reinterpret_cast<uintptr_t>(p.b_ih) & 7u) == 0 && (reinterpret_cast<uintptr_t>(p.b_hh) & 7u) == 0;
-  return use_resident(p) && p.x_table && p.uh && p.gh && p.ucount && p.Ds <= 1024 && bias_ok &&
+  return use_resident(p) && p.x_table && p.uh && p.gh && p.ucount && p.uhcount && p.Ds <= 1024 && bias_ok &&
          resident_smem_rows(p.B, p.V, p.R, grid, static_cast<long long>(p.B) * p.Ds * 4 + 16) >= 0;
 }
 
