@@ -149,7 +149,12 @@ DOMINO_API int domino_draft_step(const void* hidden, const int32_t* prefix_ids, 
  * process (calls from several threads take turns on it), from which they are copied to the
  * caller's buffers; the call synchronises the stream before returning.  The workspace must
  * hold domino_workspace_bytes_host(...) bytes and be zero-filled before its first use, as for
- * domino_draft_step.  Returns DOMINO_OK or the first error,
+ * domino_draft_step.  From the second call with the same arguments (pointers and sizes) on, the
+ * library replays a CUDA graph of the whole call that it captured on a stream of its own
+ * (launched on `stream`), so that the step's launches need not reach the GPU one by one after
+ * the previous call returned; the inputs are read afresh on every call.  Calls it cannot
+ * capture (pageable inputs, for instance) run directly.  The graphs hold no device memory of
+ * their own; at most 16 are kept.  Returns DOMINO_OK or the first error,
  * including device-side errors (bad prefix id, timeout). */
 DOMINO_API size_t domino_workspace_bytes_host(int B, int K, int H, int V, int Ds, int R, int k, int N);
 DOMINO_API int domino_draft_step_host(const void* hidden_host, const int32_t* prefix_ids_host,

@@ -330,8 +330,11 @@ std::mutex g_stage_mu;
 uint8_t* g_stage = nullptr;
 size_t g_stage_bytes = 0;
 
+void drop_host_graphs();
+
 uint8_t* stage_buffer(size_t bytes) {
   if (bytes <= g_stage_bytes) return g_stage;
+  drop_host_graphs();  // their output copies target the buffer that is about to move
   if (g_stage) cudaFreeHost(g_stage);
   g_stage = nullptr;
   g_stage_bytes = 0;
@@ -340,6 +343,58 @@ uint8_t* stage_buffer(size_t bytes) {
   g_stage = static_cast<uint8_t*>(p);
   g_stage_bytes = bytes;
   return g_stage;
+}
+
+// ---------------------------------------------------------------- host entry point: graphs
+// domino_draft_step_host returns only once its step is done, so a call's launches reach the GPU
+// one by one after the previous call came back.  The second call with the same arguments
+// captures the whole call (the input copies, the step's kernels, the output copy into the
+// staging buffer) into a CUDA graph on a stream of this library; it and every later call with
+// those arguments launch that graph on the caller's stream.  The first call runs directly, so
+// that every kernel attribute is set outside a capture.  Guarded by g_stage_mu (every host
+// entry call holds it); at most kMaxHostGraphs graphs are kept (all are dropped when full, and
+// when the staging buffer moves).
+struct HostKey {
+  const void* hidden;
+  const void* ids;
+  const void* w_lm;
+  domino_head_weights head;
+  int hd, B, K, H, V, k, N, dev;
+  void* ws;
+  size_t ws_bytes;
+  const uint8_t* stage;
+};
+
+struct HostKeyLess {
+  bool operator()(const HostKey& a, const HostKey& b) const { return memcmp(&a, &b, sizeof(HostKey)) < 0; }
+};
+
+struct HostGraph {
+  int calls = 0;
+  bool failed = false;  // capture or instantiation failed once: this key runs directly
+  cudaGraphExec_t exec = nullptr;
+};
+
+constexpr size_t kMaxHostGraphs = 16;
+std::map<HostKey, HostGraph, HostKeyLess> g_host_graphs;
+std::map<int, cudaStream_t> g_capture_streams;  // per device
+
+void drop_host_graphs() {
+  for (auto& kv : g_host_graphs)
+    if (kv.second.exec) cudaGraphExecDestroy(kv.second.exec);
+  g_host_graphs.clear();
+}
+
+cudaStream_t capture_stream(int dev) {
+  auto it = g_capture_streams.find(dev);
+  if (it != g_capture_streams.end()) return it->second;
+  cudaStream_t cs = nullptr;
+  if (cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return nullptr;
+  }
+  g_capture_streams[dev] = cs;
+  return cs;
 }
 
 // ---------------------------------------------------------------- per-kernel timing
@@ -637,8 +692,6 @@ int domino_draft_step_host(const void* hidden_host, const int32_t* prefix_ids_ho
   int32_t* d_ids = reinterpret_cast<int32_t*>(ws + P.off_ids);
   rc = check_pointers(d_hid, d_ids, w_lm, head, hd);
   if (rc) return rc;
-  if (cudaMemcpyAsync(d_hid, hidden_host, M * H * 2, cudaMemcpyHostToDevice, st) != cudaSuccess) return DOMINO_ERR_CUDA;
-  if (cudaMemcpyAsync(d_ids, prefix_ids_host, M * 4, cudaMemcpyHostToDevice, st) != cudaSuccess) return DOMINO_ERR_CUDA;
   int32_t* d_tid = reinterpret_cast<int32_t*>(ws + P.off_tid);
   float* d_tlp = reinterpret_cast<float*>(ws + P.off_tlp);
   int32_t* d_par = reinterpret_cast<int32_t*>(ws + P.off_tpar);
@@ -646,14 +699,63 @@ int domino_draft_step_host(const void* hidden_host, const int32_t* prefix_ids_ho
   int32_t* d_dep = reinterpret_cast<int32_t*>(ws + P.off_tdep);
   float* d_sc = reinterpret_cast<float*>(ws + P.off_tsc);
   int32_t* d_ostat = reinterpret_cast<int32_t*>(ws + P.off_ostat);
-  rc = run_step(P, d_hid, d_ids, w_lm, head, d_tid, d_tlp, d_par, d_tok, d_dep, d_sc, ws, st, d_ostat);
-  if (rc) return rc;
   // every output and the status in one copy, through a pinned staging buffer of this library
   const size_t lo = P.off_tid, bytes = P.off_ostat + 4 - lo;
   std::lock_guard<std::mutex> lock(g_stage_mu);
   uint8_t* h = stage_buffer(bytes);
   if (!h) return DOMINO_ERR_CUDA;
-  if (cudaMemcpyAsync(h, ws + lo, bytes, cudaMemcpyDeviceToHost, st) != cudaSuccess) return DOMINO_ERR_CUDA;
+  // the whole call on stream s: input copies, the step, the output copy
+  auto enqueue = [&](cudaStream_t s) -> int {
+    if (cudaMemcpyAsync(d_hid, hidden_host, M * H * 2, cudaMemcpyHostToDevice, s) != cudaSuccess) return DOMINO_ERR_CUDA;
+    if (cudaMemcpyAsync(d_ids, prefix_ids_host, M * 4, cudaMemcpyHostToDevice, s) != cudaSuccess) return DOMINO_ERR_CUDA;
+    const int r = run_step(P, d_hid, d_ids, w_lm, head, d_tid, d_tlp, d_par, d_tok, d_dep, d_sc, ws, s, d_ostat);
+    if (r) return r;
+    return cuda_rc(cudaMemcpyAsync(h, ws + lo, bytes, cudaMemcpyDeviceToHost, s));
+  };
+  cudaGraphExec_t exec = nullptr;
+  int dev = 0;
+  if (!g_timing.on && cudaGetDevice(&dev) == cudaSuccess) {
+    HostKey key;
+    memset(&key, 0, sizeof(key));  // padding included: keys compare as bytes
+    key.hidden = hidden_host;
+    key.ids = prefix_ids_host;
+    key.w_lm = w_lm;
+    if (hd) key.head = *head;
+    key.hd = hd ? 1 : 0;
+    key.B = B; key.K = K; key.H = H; key.V = V; key.k = k; key.N = N; key.dev = dev;
+    key.ws = workspace;
+    key.ws_bytes = workspace_bytes;
+    key.stage = h;
+    if (g_host_graphs.size() >= kMaxHostGraphs && g_host_graphs.find(key) == g_host_graphs.end()) drop_host_graphs();
+    HostGraph& g = g_host_graphs[key];
+    if (!g.exec && !g.failed && g.calls >= 1) {
+      // capture on this library's stream (the caller's may be the legacy default stream, which
+      // cannot be captured); a capture that fails leaves this key on the direct path
+      cudaStream_t cs = capture_stream(dev);
+      cudaGraph_t graph = nullptr;
+      g.failed = true;
+      if (cs && cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal) == cudaSuccess) {
+        const int r = enqueue(cs);
+        const cudaError_t e = cudaStreamEndCapture(cs, &graph);
+        if (r == DOMINO_OK && e == cudaSuccess && graph &&
+            cudaGraphInstantiate(&g.exec, graph, 0) == cudaSuccess)
+          g.failed = false;
+        if (graph) cudaGraphDestroy(graph);
+      }
+      if (g.failed) {  // nothing captured ran: the workspace is as the last call left it
+        g.exec = nullptr;
+        (void)cudaGetLastError();
+      }
+    }
+    ++g.calls;
+    exec = g.exec;
+  }
+  if (exec) {
+    if (cudaGraphLaunch(exec, st) != cudaSuccess) return DOMINO_ERR_CUDA;
+  } else {
+    rc = enqueue(st);
+    if (rc) return rc;
+  }
   if (cudaStreamSynchronize(st) != cudaSuccess) return DOMINO_ERR_CUDA;
   const size_t BN = static_cast<size_t>(P.B) * N;
   memcpy(topk_ids_host, h + (P.off_tid - lo), M * k * 4);
