@@ -453,6 +453,32 @@ __device__ __forceinline__ void ub_rows(const RolloutParams& p, int j, const flo
   const int B = p.B, K = p.K, H = p.H, Ds = p.Ds, R = p.R;
   float* gh = p.gh + static_cast<size_t>(j & 1) * B * 3 * Ds;
   constexpr int kCh = 4;
+  // step 0: uh comes from every warp's uh_prologue (other CTAs included); lane 0 first waits
+  // for all of them (bounded; a timeout leaves the status set), and the warp's loads of uh follow
+  if (j == 0 && lane == 0 && row0 < R) {
+    const unsigned target = gridDim.x * static_cast<unsigned>(kRollWarps);
+    const long long t0 = clock64();
+    while (true) {
+      unsigned v;
+      asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p.uhcount) : "memory");
+      if (v >= target) break;
+      if (clock64() - t0 > kWaitCycles) {
+        set_status(p.status, kStatusTimeout);
+        break;
+      }
+      __nanosleep(32);
+    }
+  }
+  __syncwarp();  // lane 0's acquire orders the other lanes' loads of uh below
+  // lane b < B: uh + b1 of sequence b for each u row, loaded with the weights
+  float uhb[NR];
+#pragma unroll
+  for (int k = 0; k < NR; ++k) {
+    const int row = row0 + k * stride;
+    uhb[k] = (row < R && row < rows && lane < B)
+                 ? __ldcg(p.uh + (static_cast<size_t>(lane) * K + j) * R + row) + (p.b1 ? bf2f(p.b1[row]) : 0.f)
+                 : 0.f;
+  }
   uint4 wraw[NR][kCh];
 #pragma unroll
   for (int k = 0; k < NR; ++k) {
@@ -490,22 +516,6 @@ __device__ __forceinline__ void ub_rows(const RolloutParams& p, int j, const flo
       }
     }
   }
-  // step 0: uh comes from every warp's uh_prologue (other CTAs included); lane 0, which reads
-  // it, first waits for all of them (bounded; a timeout leaves the status set)
-  if (j == 0 && lane == 0 && row0 < R) {
-    const unsigned target = gridDim.x * static_cast<unsigned>(kRollWarps);
-    const long long t0 = clock64();
-    while (true) {
-      unsigned v;
-      asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p.uhcount) : "memory");
-      if (v >= target) break;
-      if (clock64() - t0 > kWaitCycles) {
-        set_status(p.status, kStatusTimeout);
-        break;
-      }
-      __nanosleep(32);
-    }
-  }
 #pragma unroll
   for (int k = 0; k < NR; ++k) {
     const int row = row0 + k * stride;
@@ -513,10 +523,10 @@ __device__ __forceinline__ void ub_rows(const RolloutParams& p, int j, const flo
     for (int b = 0; b < KB; ++b) {
       if (b < B) {
         const float a = warp_sum(acc[k][b]);
+        const float ub = __shfl_sync(0xffffffffu, uhb[k], b);
         if (lane == 0 && row < rows) {
           if (row < R) {
-            const float x = a + __ldcg(p.uh + (static_cast<size_t>(b) * K + j) * R + row) +
-                            (p.b1 ? bf2f(p.b1[row]) : 0.f);
+            const float x = a + ub;
             p.u[static_cast<size_t>(b) * R + row] = x / (1.f + expf(-x));
           } else {
             gh[static_cast<size_t>(b) * 3 * Ds + row - R] = a;
@@ -796,9 +806,11 @@ __device__ void sample_step(const RolloutParams& p, int j, const float4 (&mine)[
 // greedy_logp); then every CTA reads the slot.  The slots alternate by step parity: a CTA
 // updates step j + 2's only after every CTA has passed step j + 1's barrier, so after every read
 // of step j's.  Returns false if the barrier gave up.
+// s_base_next (the resident kernel): the next step's base logits are copied into it (cp.async)
+// while the barrier completes.
 template <int KB>
 __device__ bool finish_greedy(const RolloutParams& p, int j, Lse (&st)[KB], int* s_tok, unsigned& nbar,
-                              volatile int* s_fail) {
+                              volatile int* s_fail, float* s_base_next, int r_lo, int r_n, int rows_cta) {
   __shared__ unsigned long long s_key[kRollWarps][kRollMaxB];
   __shared__ int s_go;
   const int B = p.B, K = p.K, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -828,6 +840,12 @@ __device__ bool finish_greedy(const RolloutParams& p, int j, Lse (&st)[KB], int*
     }
     // release at GPU scope: this CTA's keys (and its earlier writes) before its arrival
     asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(p.barrier) : "memory");
+  }
+  if (s_base_next != nullptr && j + 1 < K) {  // phase C has read this step's
+    for (int e = tid; e < B * r_n; e += kRollThreads) {
+      const int b = e / r_n, r = e - b * r_n;
+      cp_async4(s_base_next + b * rows_cta + r, p.base + (static_cast<size_t>(b) * K + j + 1) * p.V + r_lo + r);
+    }
   }
   // the warps' (max, sum of exp) for the log-probabilities, while the other CTAs arrive
   float4* part = reinterpret_cast<float4*>(p.partials) +
@@ -862,20 +880,20 @@ __device__ bool finish_greedy(const RolloutParams& p, int j, Lse (&st)[KB], int*
       __nanosleep(32);
     }
     s_go = *s_fail == 0;
+    if (s_go) {  // every CTA's red.max came before its arrival
+      for (int b = 0; b < B; ++b) {
+        const unsigned long long key = __ldcg(slot + b);
+        const int tok = static_cast<int>(key >> 54) == j + 1
+                            ? static_cast<int>(kGreedyIdMask - static_cast<unsigned>(key & kGreedyIdMask))
+                            : 0;  // no row with a finite logit anywhere
+        s_tok[b] = tok;
+        if (blockIdx.x == 0) p.tokens[static_cast<size_t>(b) * K + j] = tok;
+      }
+    }
   }
   ++nbar;
   compute_sync();
-  if (!s_go) return false;
-  if (tid < B) {
-    const unsigned long long key = __ldcg(slot + tid);
-    const int tok = static_cast<int>(key >> 54) == j + 1
-                        ? static_cast<int>(kGreedyIdMask - static_cast<unsigned>(key & kGreedyIdMask))
-                        : 0;  // no row with a finite logit anywhere
-    s_tok[tid] = tok;
-    if (blockIdx.x == 0) p.tokens[static_cast<size_t>(tid) * K + j] = tok;
-  }
-  compute_sync();
-  return true;
+  return s_go != 0;
 }
 
 // End of step j: greedy with keys (p.best set), finish_greedy.  Otherwise this CTA's (max,
@@ -890,7 +908,9 @@ __device__ __forceinline__ bool finish_step(const RolloutParams& p, int j, Lse (
                                             int r_lo, int r_n, int rows_cta, bool resident) {
   const int B = p.B, K = p.K, V = p.V, tid = threadIdx.x;
   const int grid = static_cast<int>(gridDim.x);
-  if (p.best != nullptr) return finish_greedy<KB>(p, j, st, s_tok, nbar, s_fail);
+  if (p.best != nullptr)
+    return finish_greedy<KB>(p, j, st, s_tok, nbar, s_fail, (resident && p.fast_gates) ? s_logit : nullptr, r_lo,
+                             r_n, rows_cta);
   float4* part = reinterpret_cast<float4*>(p.partials) + static_cast<size_t>(j & 1) * grid * kRollMaxB;
   block_reduce(st, s_red, B);  // ends with a barrier: every row's final logit is in s_logit
   if (tid < B) {
@@ -1214,9 +1234,12 @@ __global__ void __launch_bounds__(kRollThreads, 1)
       const float* hprev = p.h + static_cast<size_t>((j + 1) & 1) * B * p.Ds;  // h_{j-1} (zeros at j = 0)
       float* hcur = p.h + static_cast<size_t>(j & 1) * B * p.Ds;
       // this step's base logits for the CTA's rows: asynchronous copies that land during A and B
-      for (int e = tid; e < B * r_n; e += kRollThreads) {
-        const int b = e / r_n, r = e - b * r_n;
-        cp_async4(s_base + b * rows_cta + r, p.base + (static_cast<size_t>(b) * K + j) * V + r_lo + r);
+      // (greedy two-barrier step: issued by the previous step's finish, from step 1 on)
+      if (j == 0 || p.best == nullptr || !p.fast_gates) {
+        for (int e = tid; e < B * r_n; e += kRollThreads) {
+          const int b = e / r_n, r = e - b * r_n;
+          cp_async4(s_base + b * rows_cta + r, p.base + (static_cast<size_t>(b) * K + j) * V + r_lo + r);
+        }
       }
       if (p.fast_gates) {
         gates_all(p, j, s_tok, s_h);
