@@ -447,16 +447,17 @@ __device__ __forceinline__ void gates_all(const RolloutParams& p, int j, const i
 //      alone (phase C waits for those) and the other warps take the W_hh rows four at a time;
 //      otherwise every warp takes its rows three at a time.  Every weight load of a warp's rows is
 //      issued before the arithmetic (Ds <= 1024: at most 4 chunks of 8 columns per lane and row).
+// count_u: each finished row of u is counted in p.ucount here (otherwise the caller counts them).
 template <int KB, int NR>
 __device__ __forceinline__ void ub_rows(const RolloutParams& p, int j, const float* s_h, int row0, int stride,
-                                        int rows, int lane, uint64_t pol) {
+                                        int rows, int lane, uint64_t pol, bool count_u = true) {
   const int B = p.B, K = p.K, H = p.H, Ds = p.Ds, R = p.R;
   float* gh = p.gh + static_cast<size_t>(j & 1) * B * 3 * Ds;
   constexpr int kCh = 4;
-  // step 0: uh comes from every warp's uh_prologue (other CTAs included); lane 0 first waits
-  // for all of them (bounded; a timeout leaves the status set), and the warp's loads of uh follow
+  // step 0: uh comes from every CTA's uh_prologue; lane 0 first waits for all of them (bounded;
+  // a timeout leaves the status set), and the warp's loads of uh follow
   if (j == 0 && lane == 0 && row0 < R) {
-    const unsigned target = gridDim.x * static_cast<unsigned>(kRollWarps);
+    const unsigned target = gridDim.x;
     const long long t0 = clock64();
     while (true) {
       unsigned v;
@@ -534,7 +535,7 @@ __device__ __forceinline__ void ub_rows(const RolloutParams& p, int j, const flo
         }
       }
     }
-    if (lane == 0 && row < R)  // this row of u_j is written for every sequence
+    if (count_u && lane == 0 && row < R)  // this row of u_j is written for every sequence
       asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(p.ucount) : "memory");
   }
 }
@@ -546,7 +547,14 @@ __device__ __forceinline__ void ub_phase(const RolloutParams& p, int j, const fl
   const int rows = R + (j + 1 < p.K ? 3 * p.Ds : 0);
   if (nwarps > R) {
     if (gw < R) {
-      ub_rows<KB, 1>(p, j, s_h, gw, 0, R, lane, pol);
+      // the CTA's warps with a row of u (warps 0 .. nu - 1) meet at a named barrier and one
+      // thread counts their nu rows (one atomic per CTA rather than per row)
+      const int warp = gw - static_cast<int>(blockIdx.x) * kRollWarps;
+      const int nu = min(kRollWarps, R - static_cast<int>(blockIdx.x) * kRollWarps);
+      ub_rows<KB, 1>(p, j, s_h, gw, 0, R, lane, pol, false);
+      asm volatile("bar.sync 2, %0;" ::"r"(nu * 32) : "memory");
+      if (warp == 0 && lane == 0)
+        asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p.ucount), "r"(static_cast<unsigned>(nu)) : "memory");
     } else {
       const int n = nwarps - R;
       for (int row0 = gw; row0 < rows; row0 += 4 * n) ub_rows<KB, 4>(p, j, s_h, row0, n, rows, lane, pol);
@@ -560,8 +568,8 @@ __device__ __forceinline__ void ub_phase(const RolloutParams& p, int j, const fl
 //      = b K + j and rank row q, the half of u's argument that does not depend on the
 //      recurrence.  Warp w takes row q = w % R and the positions m = w / R, w / R + G, ...
 //      (G = max(1, warps / R)), four at a time, so a W1 row is read once per four positions.
-//      Each warp then counts itself in p.uhcount (release): the two-barrier step reads uh before
-//      any grid barrier, so its first phase B acquires that count instead.
+//      The caller then counts its CTA in p.uhcount (release): the two-barrier step reads uh
+//      before any grid barrier, so its first phase B acquires that count instead.
 __device__ void uh_prologue(const RolloutParams& p, int gw, int nwarps, int lane, uint64_t pol) {
   const int H = p.H, Ds = p.Ds, R = p.R, M = p.B * p.K;
   const int groups = max(1, nwarps / R);
@@ -593,8 +601,6 @@ __device__ void uh_prologue(const RolloutParams& p, int gw, int nwarps, int lane
       }
     }
   }
-  // every warp, with rows or without: the two-barrier step's first phase B waits for all of them
-  if (lane == 0 && p.uhcount) asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(p.uhcount) : "memory");
 }
 
 // ---- phase B: u_j = SiLU(W1 [hidden_j ; h_j] + b1), one warp per rank row q, every sequence.
@@ -801,9 +807,10 @@ __device__ void sample_step(const RolloutParams& p, int j, const float4 (&mine)[
 // inverted, so that the largest key over the CTAs is the step's maximum with ties to the lowest
 // id (ids below 2^22) -- from two integer warp reductions per warp; thread 0 folds the warps'
 // keys into the sequence's slot with one red.max and arrives at the grid barrier.  While the
-// other CTAs arrive, each warp reduces its (max, sum of exp) of every sequence and writes it to
-// the step's partials (the log-probabilities are merged from them once, after the last step:
-// greedy_logp); then every CTA reads the slot.  The slots alternate by step parity: a CTA
+// other CTAs arrive (before the arrival at the last step, which no later barrier follows), each
+// warp reduces its (max, sum of exp) of every sequence and writes it to the step's partials (the
+// log-probabilities are merged from them once, after the last step: greedy_logp); then thread 0
+// reads the slot.  The slots alternate by step parity: a CTA
 // updates step j + 2's only after every CTA has passed step j + 1's barrier, so after every read
 // of step j's.  Returns false if the barrier gave up.
 // s_base_next (the resident kernel): the next step's base logits are copied into it (cp.async)
@@ -816,6 +823,30 @@ __device__ bool finish_greedy(const RolloutParams& p, int j, Lse (&st)[KB], int*
   const int B = p.B, K = p.K, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int grid = static_cast<int>(gridDim.x);
   unsigned long long* slot = p.best + (j & 1) * kRollMaxB;
+  // each warp's (max, sum of exp) of every sequence, for the log-probabilities
+  float4* part = reinterpret_cast<float4*>(p.partials) +
+                 (static_cast<size_t>(j) * grid + blockIdx.x) * kRollWarps * kRollMaxB;
+  auto write_partials = [&]() {
+#pragma unroll
+    for (int b = 0; b < KB; ++b) {
+      if (b < B) {
+        Lse a = st[b];
+#pragma unroll
+        for (int o = 16; o; o >>= 1) {
+          Lse t;
+          t.m = __shfl_xor_sync(0xffffffffu, a.m, o);
+          t.s = __shfl_xor_sync(0xffffffffu, a.s, o);
+          t.i = __shfl_xor_sync(0xffffffffu, a.i, o);
+          lse_merge(a, t);
+        }
+        if (lane == 0) part[warp * kRollMaxB + b] = make_float4(a.m, a.s, __int_as_float(a.i), 0.f);
+      }
+    }
+  };
+  // the last step's before the arrival (no barrier follows it), the others' while the barrier
+  // completes
+  const bool last = j + 1 == K;
+  if (last) write_partials();
 #pragma unroll
   for (int b = 0; b < KB; ++b) {
     if (b < B) {
@@ -847,24 +878,7 @@ __device__ bool finish_greedy(const RolloutParams& p, int j, Lse (&st)[KB], int*
       cp_async4(s_base_next + b * rows_cta + r, p.base + (static_cast<size_t>(b) * K + j + 1) * p.V + r_lo + r);
     }
   }
-  // the warps' (max, sum of exp) for the log-probabilities, while the other CTAs arrive
-  float4* part = reinterpret_cast<float4*>(p.partials) +
-                 (static_cast<size_t>(j) * grid + blockIdx.x) * kRollWarps * kRollMaxB;
-#pragma unroll
-  for (int b = 0; b < KB; ++b) {
-    if (b < B) {
-      Lse a = st[b];
-#pragma unroll
-      for (int o = 16; o; o >>= 1) {
-        Lse t;
-        t.m = __shfl_xor_sync(0xffffffffu, a.m, o);
-        t.s = __shfl_xor_sync(0xffffffffu, a.s, o);
-        t.i = __shfl_xor_sync(0xffffffffu, a.i, o);
-        lse_merge(a, t);
-      }
-      if (lane == 0) part[warp * kRollMaxB + b] = make_float4(a.m, a.s, __int_as_float(a.i), 0.f);
-    }
-  }
+  if (!last) write_partials();
   if (tid == 0) {
     const unsigned target = (nbar + 1) * static_cast<unsigned>(grid);
     const long long t0 = clock64();
@@ -974,13 +988,12 @@ __device__ __forceinline__ bool finish_step(const RolloutParams& p, int j, Lse (
 // Greedy mode, after the last step: the log-probability of each step's token.  The token is the
 // step's argmax, so its log-softmax is -log of the sum of exp(L - max) over the vocabulary, the
 // merge of every warp's partials of that step (CTA c takes steps c, c + grid, ...).  Called by
-// the compute threads of every CTA after the last step; a grid barrier first orders the last
-// step's partials, which the warps write after their arrival at that step's barrier.
+// the compute threads of every CTA after the last step's barrier: every step's partials were
+// written before some later arrival at a grid barrier (the last step's before its own).
 template <int KB>
-__device__ void greedy_logp(const RolloutParams& p, Lse (*s_red)[kRollMaxB], unsigned& nbar, volatile int* s_fail) {
+__device__ void greedy_logp(const RolloutParams& p, Lse (*s_red)[kRollMaxB]) {
   const int B = p.B, K = p.K, tid = threadIdx.x;
   const int grid = static_cast<int>(gridDim.x);
-  if (!grid_barrier(p.barrier, nbar++, p.status, s_fail)) return;
   const int nw = grid * kRollWarps;
   for (int j = blockIdx.x; j < K; j += grid) {
     const float4* part = reinterpret_cast<const float4*>(p.partials) + static_cast<size_t>(j) * nw * kRollMaxB;
@@ -1169,7 +1182,11 @@ __global__ void __launch_bounds__(kRollThreads, 1)
     }
     fill_issued = true;
     // ---- u's hidden halves while the bulk copies land (read by phase B after a grid barrier)
-    if (p.uh) uh_prologue(p, gw, nwarps, lane, l2_policy_evict_normal());
+    if (p.uh) {
+      uh_prologue(p, gw, nwarps, lane, l2_policy_evict_normal());
+      compute_sync();  // one count per CTA: every warp's share of uh is written
+      if (tid == 0 && p.uhcount) asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(p.uhcount) : "memory");
+    }
     const int q = warp & 3, half = warp >> 2;
     const uint32_t tq = tbase + (static_cast<uint32_t>(32 * q) << 16);
     const uint64_t pol_once = l2_policy_evict_first();
@@ -1416,7 +1433,7 @@ __global__ void __launch_bounds__(kRollThreads, 1)
       for (int b = 0; b < KB; ++b)
         if (b == lane % KB) lse_merge(st[b], mine);
       if (!finish_step<KB>(p, j, st, s_red, s_tok, nbar, &s_fail, s_base, r_lo, r_n, rows_cta, true)) break;
-      if (j + 1 == K && p.best) greedy_logp<KB>(p, s_red, nbar, &s_fail);
+      if (j + 1 == K && p.best) greedy_logp<KB>(p, s_red);
     }
   }
   // ---- teardown: the asynchronous copies have landed (the fill: bounded), the MMAs are done
@@ -1593,7 +1610,7 @@ __global__ void __launch_bounds__(kRollThreadsAll, 1) rollout_kernel(const Rollo
     }
     if (!finish_step<KB>(p, j, st, s_red, s_tok, nbar, &s_fail, s_base, r_lo, r_n, rows_cta, false)) return;
   }
-  if (p.best) greedy_logp<KB>(p, s_red, nbar, &s_fail);
+  if (p.best) greedy_logp<KB>(p, s_red);
 }
 
 // ================================================================ launch
