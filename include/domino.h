@@ -258,7 +258,8 @@ DOMINO_API int domino_verify_tree_sample(const float* target_logits, const int32
 
 /* The greedy sequential draft loop, the paper's inference loop (section 4.1.2 and Fig. 3: each
  * draft token is chosen from the final logits and becomes the causal encoder's next input), as
- * a variant of domino_draft_step for callers that do not have the prefix:
+ * a variant of domino_draft_step for callers that do not have the prefix (V < 2^22, else
+ * DOMINO_ERR_UNSUPPORTED):
  *   t_0 = anchors[b]; for j = 0..K-1: S_j = the GRU state after emb[t_0..t_j];
  *   u_j = SiLU(W1 [hidden_j ; S_j] + b1); L_j = W_lm hidden_j + W2 u_j + b2;
  *   t_{j+1} = argmax L_j (equal values: the lowest id); logp_j = log-softmax(L_j)[t_{j+1}].
@@ -269,7 +270,8 @@ DOMINO_API int domino_verify_tree_sample(const float* target_logits, const int32
  *   per SM; a CTA's shared memory (at most 225 KB) holds u of every sequence (4 B r) and its
  *   share of the base logits (4 B ceil(V / SMs) rows), plus, for r <= 256, as many of its W2
  *   rows as fit (its first 512 W2 rows live in the tensor memory, all of it, of the SM for the
- *   whole call), or,
+ *   whole call; with the input table, B <= 2 and r a multiple of 64, 128-row W2 blocks in tensor
+ *   and shared memory instead, for the tensor cores), or,
  *   for r > 256, a 96 KB ring W2 streams through every step (those shares rounded up to whole
  *   ring chunks).  Sizes whose u and base-logit share alone exceed 225 KB return
  *   DOMINO_ERR_INVALID_ARG.

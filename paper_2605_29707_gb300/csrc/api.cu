@@ -936,6 +936,7 @@ int make_roll_plan(int B, int K, int H, int V, int Ds, int R, bool head, RollPla
   // head on: a W2 row must fit one 16 KB stage of the rollout's ring
   if (head && (Ds < 8 || (Ds & 7) || R < 8 || (R & 7) || R > 8192)) return DOMINO_ERR_INVALID_ARG;
   if (static_cast<long long>(B) * K * V > (1LL << 33)) return DOMINO_ERR_UNSUPPORTED;
+  if (V > static_cast<int>(dm::kGreedyIdMask)) return DOMINO_ERR_UNSUPPORTED;  // token ids below 2^22
   int sms = 0, major = 0, minor = 0;
   int rc = device_sms(&sms, &major, &minor);
   if (rc != DOMINO_OK) return rc;
@@ -1053,9 +1054,8 @@ int rollout_entry(const void* hidden, const int32_t* anchors, const float* unifo
   rp.barrier = reinterpret_cast<unsigned*>(ws + 64);
   rp.ucount = reinterpret_cast<unsigned*>(ws + 128);  // cleared with the status and the barrier
   rp.uhcount = reinterpret_cast<unsigned*>(ws + 192);
-  // greedy: the argmax keys of the sequences (cleared with them), ids below 2^22
-  rp.best = (!uniforms && V <= static_cast<int>(dm::kGreedyIdMask)) ? reinterpret_cast<unsigned long long*>(ws + 256)
-                                                                   : nullptr;
+  // greedy: the argmax keys of the sequences (cleared with them)
+  rp.best = uniforms ? nullptr : reinterpret_cast<unsigned long long*>(ws + 256);
   rp.tokens = tokens;
   rp.logp = logp;
   rp.status = status;

@@ -198,12 +198,11 @@ struct RolloutParams {
   const float* base;            // [B*K, V] W_lm hidden (fp32, from the store-mode GEMM)
   float* h;                     // [2][B][Ds] GRU states (cleared: h_{-1} = 0)
   float* u;                     // [B][R]
-  float* partials;              // float4 (max, sum exp, argmax bits, 0) per sequence: greedy with keys
-                                // [K][grid][kRollComputeWarps][kRollMaxB] (per warp); otherwise
+  float* partials;              // float4 (max, sum exp, argmax bits, 0) per sequence: greedy
+                                // [K][grid][kRollComputeWarps][kRollMaxB] (per warp); sampled
                                 // [2][grid][kRollMaxB] (per CTA), by step parity
   unsigned long long* best;     // greedy: [2][kRollMaxB] keys of each sequence's argmax by step parity
-                                // (cleared), or nullptr
-                                // (sampled mode, or V >= 2^22: every CTA combines the partials instead)
+                                // (cleared); nullptr in sampled mode (every CTA combines the partials)
   unsigned* barrier;            // grid barrier counter (cleared)
   int32_t* tokens;              // [B, K] t_1 .. t_K
   float* logp;                  // [B, K]

@@ -910,17 +910,17 @@ __device__ bool finish_greedy(const RolloutParams& p, int j, Lse (&st)[KB], int*
   return s_go != 0;
 }
 
-// End of step j: greedy with keys (p.best set), finish_greedy.  Otherwise this CTA's (max,
-// sum exp, argmax) per sequence go to the partials, and after a grid barrier every CTA combines
-// all of them and picks t_{j+1} (argmax, or sampled).  The partials and (sampled mode) the
-// final-logit copies alternate between two buffers by step parity: a CTA writes step j + 2's
-// only after every CTA has passed step j + 1's barrier, so after every read of step j's (with
-// the correction branch off no other barrier separates consecutive steps).
+// End of step j: greedy (p.best set), finish_greedy.  Sampled: this CTA's (max, sum exp, argmax)
+// per sequence go to the partials, and after a grid barrier every CTA combines all of them and
+// draws t_{j+1}.  The partials and the final-logit copies alternate between two buffers by step
+// parity: a CTA writes step j + 2's only after every CTA has passed step j + 1's barrier, so
+// after every read of step j's (with the correction branch off no other barrier separates
+// consecutive steps).
 template <int KB>
 __device__ __forceinline__ bool finish_step(const RolloutParams& p, int j, Lse (&st)[KB], Lse (*s_red)[kRollMaxB],
                                             int* s_tok, unsigned& nbar, volatile int* s_fail, float* s_logit,
                                             int r_lo, int r_n, int rows_cta, bool resident) {
-  const int B = p.B, K = p.K, V = p.V, tid = threadIdx.x;
+  const int B = p.B, V = p.V, tid = threadIdx.x;
   const int grid = static_cast<int>(gridDim.x);
   if (p.best != nullptr)
     return finish_greedy<KB>(p, j, st, s_tok, nbar, s_fail, (resident && p.fast_gates) ? s_logit : nullptr, r_lo,
@@ -959,29 +959,15 @@ __device__ __forceinline__ bool finish_step(const RolloutParams& p, int j, Lse (
     }
   }
   block_reduce(st, s_red, B);
-  if (p.uniforms) {
-    __shared__ float s_gmax[kRollMaxB], s_glz[kRollMaxB];
-    if (tid < B) {
-      Lse a = s_red[0][tid];
-      for (int w = 1; w < kRollWarps; ++w) lse_merge(a, s_red[w][tid]);
-      s_gmax[tid] = a.m;
-      s_glz[tid] = logf(a.s);
-    }
-    compute_sync();
-    sample_step<KB>(p, j, mine, lg, s_logit, rows_cta, s_tok, s_gmax, s_glz, resident);
-    return true;
-  }
+  __shared__ float s_gmax[kRollMaxB], s_glz[kRollMaxB];
   if (tid < B) {
     Lse a = s_red[0][tid];
     for (int w = 1; w < kRollWarps; ++w) lse_merge(a, s_red[w][tid]);
-    const int tok = a.i == 0x7fffffff ? 0 : a.i;
-    s_tok[tid] = tok;
-    if (blockIdx.x == 0) {
-      p.tokens[static_cast<size_t>(tid) * K + j] = tok;
-      p.logp[static_cast<size_t>(tid) * K + j] = -logf(a.s);  // the argmax's logit is the max
-    }
+    s_gmax[tid] = a.m;
+    s_glz[tid] = logf(a.s);
   }
   compute_sync();
+  sample_step<KB>(p, j, mine, lg, s_logit, rows_cta, s_tok, s_gmax, s_glz, resident);
   return true;
 }
 

@@ -172,6 +172,8 @@ def test_rollout_rejects_bad_anchor_and_sizes():
     assert binding.domino_rollout_greedy(hidden, bad, w["w_lm"], head, 1, 3, c.H, c.V, tokens, logp, ws,
                                          nbytes - 256, s) == binding.DOMINO_ERR_INVALID_ARG
     assert binding.domino_rollout_workspace_bytes(9, 3, c.H, c.V, c.Ds, c.R) == 0
+    # token ids must fit the greedy argmax key's 22 bits
+    assert binding.domino_rollout_workspace_bytes(1, 3, c.H, 1 << 22, c.Ds, c.R) == 0
 
 
 @pytest.mark.parametrize("name", ["qwen3-8b", "qwen3-1.7b"])
