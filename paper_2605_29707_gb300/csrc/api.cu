@@ -582,6 +582,9 @@ int run_step_launches(const Plan& P, const void* hidden, const int32_t* ids, con
     tp.bias = hw ? static_cast<const __nv_bfloat16*>(hw->b2) : nullptr;
     tp.out = reinterpret_cast<float*>(ws + P.off_part);
     tp.status = status;
+    // large M on CTA pairs: a programmatic dependent of u_finalize, waiting for it only before
+    // the W2 segment (the first tile's W_lm segment streams meanwhile)
+    if (P.head && !P.u_in_gru && !P.swap && P.mcast == 2) tp.pdl_wait = 3;
     ts = timing_open(DOMINO_KERNEL_VOCAB, st);
     if (P.overlap)
       rc = cuda_rc(dm::launch_tc_softmax_deferred(P.bn, P.kmax, maps, tp, P.grid, st));

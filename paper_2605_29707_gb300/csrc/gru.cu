@@ -784,6 +784,9 @@ cudaError_t launch_gru(const GruParams& p, const GruPlan& plan, cudaStream_t str
 
 // ---------------------------------------------------------------------------- u finalize
 __global__ void __launch_bounds__(256) u_finalize_kernel(const UFinalParams p) {
+  // the vocabulary GEMM launched after this kernel may start now: it streams its W_lm segment
+  // first and waits for this grid before it loads u
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const size_t n = static_cast<size_t>(p.M) * p.R;
   for (size_t e = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < n;
        e += static_cast<size_t>(gridDim.x) * blockDim.x) {

@@ -39,7 +39,8 @@ struct TcParams {
   int defer;      // softmax + swap only: number of leading tiles whose second segment waits for
                   // the preceding grid (0 = off); see the producer in tc_gemm.cuh
   int pdl_wait;   // launched as a programmatic dependent: 1 = wait for the preceding grid before
-                  // the first load, 2 = after the last load (0 = no wait)
+                  // the first load, 2 = after the last load, 3 = before the first load of the
+                  // second K segment (the pair kernel; 0 = no wait)
   int mcast;      // tokens-on-M orientation: CTAs per cluster sharing each weight box by TMA
                   // multicast (1 = off; 2 or 4, dividing tok_tiles); the weight maps' box is
                   // BN / mcast rows high

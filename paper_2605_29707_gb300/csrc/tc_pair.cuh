@@ -131,12 +131,19 @@ __global__ void __launch_bounds__(192, 1)
       uint32_t phase = 0;
       int issued = 0;
       bool ok = true;
+      bool waited = p.pdl_wait != 3;
       TcItem it;
       for (int i = 0; ok && tc_get_item<kModeSoftmax>(p, i, it); ++i) {
         for (int kb = 0; kb < it.kb1; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, p.status)) { ok = false; break; }
-          if (lead) mbar_arrive_expect_tx(&full[stage], 2 * C::kStageBytes);
           const bool seg2 = kb >= p.nkb1;
+          if (seg2 && !waited) {
+            // launched as a programmatic dependent of the kernel that writes u: the W_lm segment
+            // streamed meanwhile; this thread alone reads u (through TMA)
+            asm volatile("griddepcontrol.wait;" ::: "memory");
+            waited = true;
+          }
+          if (lead) mbar_arrive_expect_tx(&full[stage], 2 * C::kStageBytes);
           const int kx = (seg2 ? kb - p.nkb1 : kb) * 64;
           const uint32_t bar = lead_full + static_cast<uint32_t>(stage * sizeof(uint64_t));
           tma_load_2d_pair(sA + stage * C::kABytes, seg2 ? &tmA2 : &tmA1, bar, kx, it.tok * 128, pol_t);
@@ -283,13 +290,15 @@ cudaError_t launch_tc_vocab_pair_instance(const CUtensorMap* maps, const TcParam
   cfg.blockDim = dim3(192);
   cfg.dynamicSmemBytes = C::kSmemBytes;
   cfg.stream = stream;
-  cudaLaunchAttribute attrs[1];
+  cudaLaunchAttribute attrs[2];
   attrs[0].id = cudaLaunchAttributeClusterDimension;
   attrs[0].val.clusterDim.x = 2;
   attrs[0].val.clusterDim.y = 1;
   attrs[0].val.clusterDim.z = 1;
+  attrs[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attrs[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attrs;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = p.pdl_wait == 3 ? 2 : 1;
   cudaError_t e = cudaLaunchKernelEx(&cfg, kern, maps[0], maps[1], maps[2], maps[3], p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
