@@ -465,9 +465,13 @@ int run_step_launches(const Plan& P, const void* hidden, const int32_t* ids, con
       tp.tmem_cols = pow2_at_least(2 * g.bn, 32);
       tp.out = xpart; tp.ld_out = 3 * Ds;
       tp.status = status;
-      tp.pdl_wait = P.chain ? 1 : 0;  // E comes from the gather
+      // E comes from the gather: small M chained, and for many tokens a programmatic dependent
+      // of the gather
+      const bool dep = !P.chain && !g.swap && g.bn == 256;
+      tp.pdl_wait = (P.chain || dep) ? 1 : 0;
       ts = timing_open(DOMINO_KERNEL_GRU_INPUT, st);
       rc = cuda_rc(P.chain ? dm::launch_tc_store_chained(g.bn, maps, tp, g.grid, st)
+                   : dep   ? dm::launch_tc_store_dependent(maps, tp, g.grid, st)
                            : dm::launch_tc_gemm(dm::kModeStore, g.bn, g.swap, 16, maps, tp, g.grid, st));
       timing_close(ts, st);
       if (rc) return rc;
@@ -497,10 +501,13 @@ int run_step_launches(const Plan& P, const void* hidden, const int32_t* ids, con
       tp.out = upart; tp.ld_out = R;
       tp.status = status;
       const bool chained = P.chain && !both;
-      tp.pdl_wait = chained ? 2 : 0;  // reads nothing the kernel before it (X GEMM or gather)
-                                      // writes; completes after it
+      // many tokens: both halves after the GRU, a programmatic dependent of it (S is its output)
+      const bool dep = both && !g.swap && g.bn == 256;
+      tp.pdl_wait = chained ? 2 : (dep ? 1 : 0);  // chained: reads nothing the kernel before it
+                                                  // (X GEMM or gather) writes; completes after it
       const int slot = timing_open(DOMINO_KERNEL_W1_HIDDEN, st);
       const int r = cuda_rc(chained ? dm::launch_tc_store_chained(g.bn, maps, tp, g.grid, st)
+                            : dep   ? dm::launch_tc_store_dependent(maps, tp, g.grid, st)
                                     : dm::launch_tc_gemm(dm::kModeStore, g.bn, g.swap, 16, maps, tp, g.grid, st));
       timing_close(slot, st);
       return r;
@@ -543,8 +550,9 @@ int run_step_launches(const Plan& P, const void* hidden, const int32_t* ids, con
       gr.V = V;
     }
     ts = timing_open(DOMINO_KERNEL_GRU, st);
-    // no vocabulary CTA shares the GRU's SMs unless the two overlap
-    rc = cuda_rc(dm::launch_gru(gr, P.gru, st, P.chain && !P.fused, !P.overlap));
+    // no vocabulary CTA shares the GRU's SMs unless the two overlap; for many tokens the GRU is
+    // a programmatic dependent of the kernel before it (it waits for it before reading)
+    rc = cuda_rc(dm::launch_gru(gr, P.gru, st, (P.chain && !P.fused) || !P.u_in_gru, !P.overlap));
     timing_close(ts, st);
     if (rc) return rc;
     if (!P.u_in_gru) {
@@ -552,7 +560,7 @@ int run_step_launches(const Plan& P, const void* hidden, const int32_t* ids, con
       if (rc) return rc;
       dm::UFinalParams uf{upart, P.ug.splits, M, R, static_cast<const __nv_bfloat16*>(hw->b1), u};
       ts = timing_open(DOMINO_KERNEL_W1_HIDDEN, st);
-      rc = cuda_rc(dm::launch_u_finalize(uf, st));
+      rc = cuda_rc(dm::launch_u_finalize(uf, st, true));
       timing_close(ts, st);
       if (rc) return rc;
     }

@@ -787,6 +787,9 @@ __global__ void __launch_bounds__(256) u_finalize_kernel(const UFinalParams p) {
   // the vocabulary GEMM launched after this kernel may start now: it streams its W_lm segment
   // first and waits for this grid before it loads u
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  // launched as a programmatic dependent of the W1 GEMM: its partial sums are read below (a
+  // no-op otherwise)
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const size_t n = static_cast<size_t>(p.M) * p.R;
   for (size_t e = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < n;
        e += static_cast<size_t>(gridDim.x) * blockDim.x) {
@@ -797,11 +800,21 @@ __global__ void __launch_bounds__(256) u_finalize_kernel(const UFinalParams p) {
   }
 }
 
-cudaError_t launch_u_finalize(const UFinalParams& p, cudaStream_t stream) {
+cudaError_t launch_u_finalize(const UFinalParams& p, cudaStream_t stream, bool pdl) {
   const size_t n = static_cast<size_t>(p.M) * p.R;
   const size_t want = (n + 255) / 256;
   const int blocks = static_cast<int>(want < 1024 ? want : 1024);
-  u_finalize_kernel<<<blocks, 256, 0, stream>>>(p);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(blocks);
+  cfg.blockDim = dim3(256);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, u_finalize_kernel, p);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

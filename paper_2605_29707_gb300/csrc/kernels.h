@@ -56,6 +56,9 @@ constexpr int kSoftmaxRecWords(int kmax) { return 2 + 2 * kmax; }
 // Tensor maps in the order A1, B1, A2, B2 (A = 128-row operand, B = N-row operand).
 cudaError_t launch_tc_gemm(int mode, int bn, bool swap, int kmax, const CUtensorMap* maps,
                            const TcParams& p, int grid, cudaStream_t stream);
+// The store-mode GEMM for many tokens (bn 256, tokens on M) launched as a programmatic dependent
+// of the kernel before it (p.pdl_wait says where it waits for that kernel).
+cudaError_t launch_tc_store_dependent(const CUtensorMap* maps, const TcParams& p, int grid, cudaStream_t stream);
 // Deferred-segment vocabulary GEMM launched as a programmatic dependent of the GRU kernel
 // (bn 16 or 32; fewer pipeline stages so that its CTAs fit beside the GRU's on one SM).
 cudaError_t launch_tc_softmax_deferred(int bn, int kmax, const CUtensorMap* maps, const TcParams& p, int grid,
@@ -165,7 +168,8 @@ struct UFinalParams {
   const __nv_bfloat16* b1;
   __nv_bfloat16* u;
 };
-cudaError_t launch_u_finalize(const UFinalParams& p, cudaStream_t stream);
+// pdl: launched as a programmatic dependent of the W1 GEMM (it waits for it before reading)
+cudaError_t launch_u_finalize(const UFinalParams& p, cudaStream_t stream, bool pdl = false);
 
 // ---------------------------------------------------------------- merge + tree
 struct TreeParams {

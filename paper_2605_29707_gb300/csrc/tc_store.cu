@@ -34,6 +34,10 @@ int tc_store_chained_smem(int bn) {
   }
 }
 
+cudaError_t launch_tc_store_dependent(const CUtensorMap* maps, const TcParams& p, int grid, cudaStream_t s) {
+  return launch_tc_instance<256, false, kModeStore, 16>(maps, p, grid, s, true);
+}
+
 cudaError_t launch_tc_gemm(int mode, int bn, bool swap, int kmax, const CUtensorMap* maps, const TcParams& p,
                            int grid, cudaStream_t stream) {
   if (mode == kModeSoftmax) return launch_tc_softmax(bn, swap, kmax, maps, p, grid, stream);
