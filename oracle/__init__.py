@@ -60,6 +60,11 @@ def _load():
         _lib.oracle_verify_sample.argtypes = [P, I, I, ctypes.c_double, P, P, P, P, P, P, P]
         _lib.oracle_rollout_greedy.argtypes = [P] * 12 + [I] * 6 + [P, I, P, P, I]
         _lib.oracle_rollout_sample.argtypes = [P] * 13 + [I] * 6 + [P, I, P, P, I]
+        U64 = ctypes.c_uint64
+        _lib.oracle_philox4x32_10.restype = None
+        _lib.oracle_philox4x32_10.argtypes = [P, P, P]
+        _lib.oracle_gumbel_row.argtypes = [U64, I, I, I, P]
+        _lib.oracle_rollout_sample_gumbel.argtypes = [P, P, U64] + [P] * 10 + [I] * 6 + [P, I, P, P, I]
         _lib.oracle_max_threads.restype = I
         for name in ("oracle_embed", "oracle_gru", "oracle_lowrank", "oracle_logits",
                      "oracle_log_softmax", "oracle_topk", "oracle_tree", "oracle_draft_step"):
@@ -277,6 +282,46 @@ def rollout_sample(w, hidden, anchors, uniforms, seqs=None, nthreads=0):
                                          _p(w_hh), _p(g("b_ih")), _p(g("b_hh")), _p(g("w1")), _p(g("b1")), _p(w2),
                                          _p(g("b2")), B, K, H, V, Ds, R, _p(sq), nseq, _p(tokens), _p(logp),
                                          nthreads), "oracle_rollout_sample")
+    return tokens, logp
+
+
+def philox4x32_10(ctr, key):
+    """Philox-4x32-10 of a 4-word counter and a 2-word key (uint32 each); returns 4 words."""
+    c = np.ascontiguousarray(ctr, dtype=np.uint32).reshape(4)
+    k = np.ascontiguousarray(key, dtype=np.uint32).reshape(2)
+    out = np.empty(4, np.uint32)
+    _load().oracle_philox4x32_10(_p(c), _p(k), _p(out))
+    return out
+
+
+def gumbel_row(seed, b, j, V):
+    """The exponential-race perturbations g[0 .. V-1] of sequence b at step j (float64 [V])."""
+    g = np.empty(V, np.float64)
+    _check(_load().oracle_gumbel_row(int(seed), int(b), int(j), int(V), _p(g)), "oracle_gumbel_row")
+    return g
+
+
+def rollout_sample_gumbel(w, hidden, anchors, seed, seqs=None, nthreads=0):
+    """Sampled sequential draft loop by the exponential race (Gumbel-max) under a 64-bit seed:
+    t_{j+1} = argmax_v L_j[v] + gumbel_row(seed, b, j, V)[v].  Otherwise as rollout_greedy."""
+    hidden = _u16(hidden)
+    B, K, H = hidden.shape
+    anchors = _i32(anchors)
+    g = lambda n: _u16(w[n]) if w.get(n) is not None else None  # noqa: E731
+    w_lm = g("w_lm")
+    V = w_lm.shape[0]
+    w2 = g("w2")
+    R = w2.shape[1] if w2 is not None else 0
+    w_hh = g("w_hh")
+    Ds = w_hh.shape[1] if w_hh is not None else 0
+    sq = None if seqs is None else _i32(seqs)
+    nseq = B if sq is None else sq.shape[0]
+    tokens = np.empty((nseq, K), np.int32)
+    logp = np.empty((nseq, K), np.float64)
+    _check(_load().oracle_rollout_sample_gumbel(_p(hidden), _p(anchors), int(seed), _p(w_lm), _p(g("emb")),
+                                                _p(g("w_ih")), _p(w_hh), _p(g("b_ih")), _p(g("b_hh")), _p(g("w1")),
+                                                _p(g("b1")), _p(w2), _p(g("b2")), B, K, H, V, Ds, R, _p(sq), nseq,
+                                                _p(tokens), _p(logp), nthreads), "oracle_rollout_sample_gumbel")
     return tokens, logp
 
 

@@ -17,7 +17,8 @@
  *   section 3.1, verification of the draft (the step after it)     -> oracle_verify_greedy,
  *                                                                       oracle_verify_sample
  *   section 4.1.2 / Fig. 3, tokens chosen and fed back one by one   -> oracle_rollout_greedy,
- *                                                                       oracle_rollout_sample
+ *                                                                       oracle_rollout_sample,
+ *                                                                       oracle_rollout_sample_gumbel
  * Readings of points the paper leaves open (GRU gate convention, which ids feed which
  * position, tree tie-breaks) are listed in the design notes; the comments below state the
  * reading each function implements.
@@ -413,12 +414,54 @@ int oracle_verify_sample(const float* target, int N, int V, double T, const floa
   return oracle_tree_walk(N, parent, token, row_sample, nodes, n_acc, bonus);
 }
 
+/* O13: Philox-4x32-10.  One round multiplies words 0 and 2 by the two round constants (full
+   64-bit products), and the new words are (high product of word 2) ^ word 1 ^ key 0, (low product
+   of word 2), (high product of word 0) ^ word 3 ^ key 1, (low product of word 0); the key grows
+   by the two Weyl constants between rounds. */
+void oracle_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4]) {
+  const uint64_t M0 = 0xD2511F53u, M1 = 0xCD9E8D57u;
+  const uint32_t W0 = 0x9E3779B9u, W1 = 0xBB67AE85u;
+  uint32_t c0 = ctr[0], c1 = ctr[1], c2 = ctr[2], c3 = ctr[3];
+  uint32_t k0 = key[0], k1 = key[1];
+  for (int r = 0; r < 10; ++r) {
+    if (r > 0) {
+      k0 += W0;
+      k1 += W1;
+    }
+    const uint64_t p0 = M0 * (uint64_t)c0, p1 = M1 * (uint64_t)c2;
+    const uint32_t hi0 = (uint32_t)(p0 >> 32), lo0 = (uint32_t)p0;
+    const uint32_t hi1 = (uint32_t)(p1 >> 32), lo1 = (uint32_t)p1;
+    c0 = hi1 ^ c1 ^ k0;
+    c1 = lo1;
+    c2 = hi0 ^ c3 ^ k1;
+    c3 = lo0;
+  }
+  out[0] = c0; out[1] = c1; out[2] = c2; out[3] = c3;
+}
+
+/* O14: u from the top 23 bits of the word, centred in its interval (never 0 or 1), then the
+   Gumbel transform of the uniform. */
+int oracle_gumbel_row(uint64_t seed, int b, int j, int V, double* g) {
+  if (!g || b < 0 || j < 0 || V <= 0) return ORACLE_ERR_ARG;
+  const uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+  for (int v = 0; v < V; ++v) {
+    const uint32_t ctr[4] = {(uint32_t)v, (uint32_t)j, (uint32_t)(b / 4), 0u};
+    uint32_t x[4];
+    oracle_philox4x32_10(ctr, key, x);
+    const double u = ((double)(x[b % 4] >> 9) + 0.5) / 8388608.0;
+    g[v] = -log(-log(u));
+  }
+  return 0;
+}
+
 /* O9: the greedy sequential draft loop.  Each position is computed from scratch out of the
  * primitives above (the GRU re-run over the whole prefix chosen so far), so the only new step is
  * the feedback: the argmax of position j becomes the input of position j + 1. */
-/* The draft loop of section 4.1.2 / Fig. 3 for both selection rules: with `uniforms` NULL the
- * greedy choice (O9), otherwise the sampled one (O10). */
-static int rollout(const uint16_t* hidden, const int32_t* anchors, const float* uniforms, const uint16_t* w_lm,
+/* The draft loop of section 4.1.2 / Fig. 3 for every selection rule: with `uniforms` NULL and
+ * `gumbel` 0 the greedy choice (O9), with `uniforms` the inverse-CDF draw (O10), with `gumbel`
+ * the exponential race under `seed` (O15). */
+static int rollout(const uint16_t* hidden, const int32_t* anchors, const float* uniforms, int gumbel, uint64_t seed,
+                   const uint16_t* w_lm,
                    const uint16_t* emb, const uint16_t* w_ih, const uint16_t* w_hh, const uint16_t* b_ih,
                    const uint16_t* b_hh, const uint16_t* w1, const uint16_t* b1, const uint16_t* w2,
                    const uint16_t* b2, int B, int K, int H, int V, int Ds, int R, const int32_t* seqs, int nseq,
@@ -437,9 +480,10 @@ static int rollout(const uint16_t* hidden, const int32_t* anchors, const float* 
   double* u = use_head ? (double*)malloc((size_t)R * sizeof(double)) : NULL;
   double* z = (double*)malloc((size_t)V * sizeof(double));
   double* lp = (double*)malloc((size_t)V * sizeof(double));
+  double* gv = gumbel ? (double*)malloc((size_t)V * sizeof(double)) : NULL;
   double ls;
   int rc = 0;
-  if (!ids || !hid || !E || !z || !lp || (use_head && (!S || !u))) rc = ORACLE_ERR_ARG;
+  if (!ids || !hid || !E || !z || !lp || (use_head && (!S || !u)) || (gumbel && !gv)) rc = ORACLE_ERR_ARG;
 
   for (int si = 0; si < nseq && rc == 0; ++si) {
     const int b = seqs ? seqs[si] : si;
@@ -459,7 +503,13 @@ static int rollout(const uint16_t* hidden, const int32_t* anchors, const float* 
       if (!rc) rc = oracle_log_softmax(z, 1, V, lp, &ls);
       if (rc) break;
       int best = 0;
-      if (!uniforms) {
+      if (gumbel) {
+        /* O15: the largest perturbed logit; strict, so an equal value keeps the lower id */
+        rc = oracle_gumbel_row(seed, b, j, V, gv);
+        if (rc) break;
+        for (int v = 1; v < V; ++v)
+          if (z[v] + gv[v] > z[best] + gv[best]) best = v;
+      } else if (!uniforms) {
         for (int v = 1; v < V; ++v)
           if (z[v] > z[best]) best = v; /* strict: an equal value keeps the lower id */
       } else {
@@ -482,7 +532,7 @@ static int rollout(const uint16_t* hidden, const int32_t* anchors, const float* 
       logp[(long)si * K + j] = lp[best];
     }
   }
-  free(ids); free(hid); free(E); free(S); free(u); free(z); free(lp);
+  free(ids); free(hid); free(E); free(S); free(u); free(z); free(lp); free(gv);
   return rc;
 }
 
@@ -492,7 +542,7 @@ int oracle_rollout_greedy(const uint16_t* hidden, const int32_t* anchors, const 
                           const uint16_t* b1, const uint16_t* w2, const uint16_t* b2, int B, int K,
                           int H, int V, int Ds, int R, const int32_t* seqs, int nseq, int32_t* tokens,
                           double* logp, int nthreads) {
-  return rollout(hidden, anchors, NULL, w_lm, emb, w_ih, w_hh, b_ih, b_hh, w1, b1, w2, b2, B, K, H, V, Ds, R, seqs,
+  return rollout(hidden, anchors, NULL, 0, 0, w_lm, emb, w_ih, w_hh, b_ih, b_hh, w1, b1, w2, b2, B, K, H, V, Ds, R, seqs,
                  nseq, tokens, logp, nthreads);
 }
 
@@ -505,6 +555,16 @@ int oracle_rollout_sample(const uint16_t* hidden, const int32_t* anchors, const 
   if (!uniforms) return ORACLE_ERR_ARG;
   for (long i = 0; i < (long)B * K; ++i)
     if (!(uniforms[i] >= 0.0f && uniforms[i] < 1.0f)) return ORACLE_ERR_ARG;
-  return rollout(hidden, anchors, uniforms, w_lm, emb, w_ih, w_hh, b_ih, b_hh, w1, b1, w2, b2, B, K, H, V, Ds, R,
-                 seqs, nseq, tokens, logp, nthreads);
+  return rollout(hidden, anchors, uniforms, 0, 0, w_lm, emb, w_ih, w_hh, b_ih, b_hh, w1, b1, w2, b2, B, K, H, V, Ds,
+                 R, seqs, nseq, tokens, logp, nthreads);
+}
+
+int oracle_rollout_sample_gumbel(const uint16_t* hidden, const int32_t* anchors, uint64_t seed,
+                                 const uint16_t* w_lm, const uint16_t* emb, const uint16_t* w_ih,
+                                 const uint16_t* w_hh, const uint16_t* b_ih, const uint16_t* b_hh,
+                                 const uint16_t* w1, const uint16_t* b1, const uint16_t* w2, const uint16_t* b2,
+                                 int B, int K, int H, int V, int Ds, int R, const int32_t* seqs, int nseq,
+                                 int32_t* tokens, double* logp, int nthreads) {
+  return rollout(hidden, anchors, NULL, 1, seed, w_lm, emb, w_ih, w_hh, b_ih, b_hh, w1, b1, w2, b2, B, K, H, V, Ds,
+                 R, seqs, nseq, tokens, logp, nthreads);
 }

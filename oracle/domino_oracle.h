@@ -162,6 +162,28 @@ int oracle_rollout_sample(const uint16_t* hidden, const int32_t* anchors, const 
                           int B, int K, int H, int V, int Ds, int R, const int32_t* seqs, int nseq,
                           int32_t* tokens, double* logp, int nthreads);
 
+/* O13, the counter-based generator of the exponential-race sampler: Philox-4x32 with ten
+ * rounds, as published by Salmon, Moraes, Dror and Shaw ("Parallel random numbers: as easy as
+ * 1, 2, 3", SC 2011): ctr (4 words) and key (2 words) in, 4 words out. */
+void oracle_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4]);
+
+/* O14, the perturbation of vocabulary entry v at step j of sequence b under a 64-bit seed:
+ * x = word (b mod 4) of Philox-4x32-10 with counter (v, j, floor(b / 4), 0) and key (seed mod
+ * 2^32, floor(seed / 2^32)); u = (floor(x / 512) + 1/2) / 2^23, which lies in [2^-24, 1 - 2^-24];
+ * g = -log(-log(u)), a standard Gumbel draw.  Fills g[0 .. V-1] for v = 0 .. V-1. */
+int oracle_gumbel_row(uint64_t seed, int b, int j, int V, double* g);
+
+/* O15, the same loop as O10 with each token sampled by the exponential race (Gumbel-max): with
+ * g_j[v] the perturbation O14 of (seed, b, j, v), t_{j+1} = argmax_v (L_j[v] + g_j[v]) (equal
+ * values: the lowest id), a draw from softmax(L_j); logp_j = log-softmax(L_j)[t_{j+1}].
+ * Otherwise as oracle_rollout_greedy. */
+int oracle_rollout_sample_gumbel(const uint16_t* hidden, const int32_t* anchors, uint64_t seed,
+                                 const uint16_t* w_lm, const uint16_t* emb, const uint16_t* w_ih,
+                                 const uint16_t* w_hh, const uint16_t* b_ih, const uint16_t* b_hh,
+                                 const uint16_t* w1, const uint16_t* b1, const uint16_t* w2, const uint16_t* b2,
+                                 int B, int K, int H, int V, int Ds, int R, const int32_t* seqs, int nseq,
+                                 int32_t* tokens, double* logp, int nthreads);
+
 /* Number of OpenMP threads the oracle would use for nthreads <= 0 (all available). */
 int oracle_max_threads(void);
 

@@ -692,3 +692,77 @@ def test_rollout_head_off_is_the_base_argmax_and_rejects_bad_anchors():
     assert tokens.tolist() == np.argmax(z, axis=2).tolist()
     with pytest.raises(oracle.OracleError):
         oracle.rollout_greedy(w, hidden, np.array([3, V], np.int32))
+
+
+# ---------------------------------------------------------------------------- O13-O15 exponential race
+def test_philox_known_answer_vectors():
+    """O13 against the generator's published known-answer vectors."""
+    g = load("philox4x32_10_kat.json")
+    for v in g["vectors"]:
+        ctr = [int(x, 16) for x in v["ctr"]]
+        key = [int(x, 16) for x in v["key"]]
+        assert [int(x) for x in oracle.philox4x32_10(ctr, key)] == [int(x, 16) for x in v["out"]]
+
+
+def test_gumbel_rows_have_the_standard_gumbel_law():
+    """O14: 2^20 perturbations of one row follow the standard Gumbel law (mean = the
+    Euler-Mascheroni constant, variance pi^2 / 6, P(g <= 0) = 1/e, every value inside the range the
+    23-bit uniform allows), and rows of other sequences and steps are uncorrelated with it."""
+    n = 1 << 20
+    g = oracle.gumbel_row(0x0123456789ABCDEF, 5, 3, n)
+    assert np.isfinite(g).all()
+    lo, hi = -math.log(-math.log(2.0 ** -24)), -math.log(-math.log(1.0 - 2.0 ** -24))
+    assert lo - 1e-12 <= g.min() and g.max() <= hi + 1e-12
+    assert abs(g.mean() - 0.5772156649015329) < 5 * math.sqrt(math.pi ** 2 / 6 / n)
+    assert abs(g.var() - math.pi ** 2 / 6) < 0.02
+    assert abs(np.mean(g <= 0.0) - math.exp(-1.0)) < 5 * math.sqrt(math.exp(-1) * (1 - math.exp(-1)) / n)
+    for b, j in ((4, 3), (6, 3), (5, 2), (5, 4)):  # same word of another group; another word; other steps
+        other = oracle.gumbel_row(0x0123456789ABCDEF, b, j, n)
+        assert abs(np.corrcoef(g, other)[0, 1]) < 5 / math.sqrt(n)
+    assert abs(np.corrcoef(g, oracle.gumbel_row(0x0123456789ABCDF0, 5, 3, n))[0, 1]) < 5 / math.sqrt(n)
+
+
+def test_rollout_sample_gumbel_draws_follow_the_softmax():
+    """O15 with the correction branch off (the logits of a position do not depend on the tokens
+    drawn before it): over 6000 sequences with the same hidden rows, the tokens drawn at each
+    position have the softmax's frequencies (chi-square, 5 categories), and logp is the
+    log-softmax of the drawn token."""
+    rng = np.random.default_rng(11)
+    V, H, K, B = 5, 8, 2, 6000
+    w = {"w_lm": rand_bf16(rng, (V, H), 0.6)}
+    one = rand_bf16(rng, (1, K, H), 1.0)
+    hidden = np.repeat(one, B, axis=0)
+    anchors = np.zeros(B, np.int32)
+    tokens, logp = oracle.rollout_sample_gumbel(w, hidden, anchors, 77)
+    z = np.einsum("kh,vh->kv", to_f64(one[0]), to_f64(w["w_lm"]))
+    lp = z - np.log(np.exp(z - z.max(axis=1, keepdims=True)).sum(axis=1, keepdims=True)) - z.max(axis=1, keepdims=True)
+    for j in range(K):
+        p = np.exp(lp[j])
+        counts = np.bincount(tokens[:, j], minlength=V)
+        chi2 = float(np.sum((counts - B * p) ** 2 / (B * p)))
+        assert chi2 < 35.0, (j, counts.tolist(), (B * p).round(1).tolist())  # df 4: p < 1e-6 by chance
+        assert np.allclose(logp[:, j], lp[j][tokens[:, j]], atol=1e-12)
+
+
+@pytest.mark.parametrize("B,K,V,H,Ds,R,biases", [(2, 5, 40, 16, 6, 4, False), (5, 7, 13, 8, 3, 2, True)])
+def test_rollout_sample_gumbel_follows_the_teacher_forced_step(B, K, V, H, Ds, R, biases):
+    """Fed the drawn tokens as its prefix, the (pinned) draft step gives, at every position, a
+    distribution whose log-probabilities plus the (pinned) perturbations of that sequence and step
+    are largest at the drawn token, and the drawn token's log-probability; another seed draws
+    other tokens."""
+    rng = np.random.default_rng(B * 10000 + K)
+    w = _small_weights(rng, V, H, Ds, R, biases)
+    hidden = rand_bf16(rng, (B, K, H), 1.0)
+    anchors = rng.integers(0, V, B).astype(np.int32)
+    seed = 0xFEEDFACE12345678
+    tokens, logp = oracle.rollout_sample_gumbel(w, hidden, anchors, seed)
+    prefix = np.concatenate([anchors[:, None], tokens[:, :-1]], axis=1).astype(np.int32)
+    ref = oracle.draft_step(w, hidden, prefix, 1, 1, want_logp_full=True)
+    for b in range(B):
+        for j in range(K):
+            key = ref["logp_full"][b, j] + oracle.gumbel_row(seed, b, j, V)
+            t = int(tokens[b, j])
+            assert t == int(np.argmax(key)), (b, j)
+            assert logp[b, j] == pytest.approx(ref["logp_full"][b, j, t], abs=1e-12)
+    other, _ = oracle.rollout_sample_gumbel(w, hidden, anchors, seed + 1)
+    assert (other != tokens).any()
