@@ -385,7 +385,7 @@ def verify_timing(st, c, device, stream, reps=200):
 
 
 def rollout_timing(st, wl, c, hidden, device, stream, reps=50):
-    """The sequential draft loop (domino_rollout_greedy / _sample) on this workload's weights and
+    """The sequential draft loop (domino_rollout_greedy / _sample / _sample_gumbel) on this workload's weights and
     hidden states: device time per block of K tokens, split into the kernels by the library's
     per-kernel CUDA events.  Timed with the input-projection table emb . W_ih^T (built once,
     outside the timed region) and, for comparison, without it."""
@@ -412,7 +412,10 @@ def rollout_timing(st, wl, c, hidden, device, stream, reps=50):
 
     def timed(head, sampled, split=False):
         def run():
-            if sampled:
+            if sampled == "race":
+                rc = binding.domino_rollout_sample_gumbel(hidden, anchors, 0x5EED, w["w_lm"], head, c.B, c.K, c.H,
+                                                          c.V, tok, lp, ws, nb, stream)
+            elif sampled:
                 rc = binding.domino_rollout_sample(hidden, anchors, uni, w["w_lm"], head, c.B, c.K, c.H, c.V, tok,
                                                    lp, ws, nb, stream)
             else:
@@ -443,6 +446,7 @@ def rollout_timing(st, wl, c, hidden, device, stream, reps=50):
 
     us, split, status = timed(head_t, False, split=True)
     us_s, _, status_s = timed(head_t, True)
+    us_g, split_g, status_g = timed(head_t, "race", split=True)
     us_nt, split_nt, status_nt = timed(st.head, False, split=True)
     # every byte the loop needs once: W_lm (base GEMM), W1[:, :H] (its GEMM), W2, W_hh and
     # W1[:, H:] (step kernel: W2 on chip, the rest in L2 across steps), one table row per token
@@ -454,7 +458,11 @@ def rollout_timing(st, wl, c, hidden, device, stream, reps=50):
     return {"us_per_block": round(us, 2), "draft_tokens_per_s": round(c.B * c.K / (us * 1e-6), 1),
             "us_per_kernel": split, "status": status, "unique_bytes_per_block": unique,
             "sampled": {"us_per_block": round(us_s, 2), "draft_tokens_per_s": round(c.B * c.K / (us_s * 1e-6), 1),
-                        "status": status_s},
+                        "status": status_s, "rule": "inverse CDF of the caller's uniforms (domino_rollout_sample)"},
+            "sampled_race": {"us_per_block": round(us_g, 2), "draft_tokens_per_s": round(c.B * c.K / (us_g * 1e-6), 1),
+                             "us_per_kernel": split_g, "status": status_g,
+                             "frac_of_hbm_roofline": round(roof_us / us_g, 4),
+                             "rule": "exponential race / Gumbel-max under a 64-bit seed (domino_rollout_sample_gumbel)"},
             "input_table": {"bytes": table.numel() * 4, "build_s": round(build_s, 4),
                             "note": "emb . W_ih^T [V, 3 d_s] fp32, built once per set of weights (tensor cores)"},
             "without_table": {"us_per_block": round(us_nt, 2), "us_per_kernel": split_nt, "status": status_nt},

@@ -304,6 +304,22 @@ DOMINO_API int domino_rollout_greedy(const void* hidden, const int32_t* anchors,
                                      int32_t* tokens, float* logp, void* workspace, size_t workspace_bytes,
                                      void* stream);
 
+/* The same loop with every draft token SAMPLED from the final distribution (section 4.1.2: each
+ * draft token is sampled from the final logits; temperature 1) by the exponential race (Gumbel-
+ * max, the rule serving systems sample with): t_{j+1} = argmax_v L_j[v] + g_{b,j}[v], ties to the
+ * lowest id, where g_{b,j}[v] = -log(-log(u)) and u comes from Philox-4x32-10 (Salmon, Moraes,
+ * Dror and Shaw, SC 2011), key = seed (low word first), counter (v, j, floor(b / 4), 0), word
+ * b mod 4, u = (that word's top 23 bits + 1/2) / 2^23.  This draws t_{j+1} from softmax(L_j);
+ * logp_j = log-softmax(L_j)[t_{j+1}].  The perturbations are computed in fp32 on the device, so
+ * where two perturbed logits lie within rounding of each other either may win.  Unlike
+ * domino_rollout_sample it needs no per-step scan after the argmax: it costs what the greedy
+ * loop costs (one grid barrier per step on the fast path) plus the generator.  Arguments,
+ * outputs, workspace (domino_rollout_workspace_bytes) and errors as domino_rollout_greedy. */
+DOMINO_API int domino_rollout_sample_gumbel(const void* hidden, const int32_t* anchors, uint64_t seed,
+                                            const void* w_lm, const domino_head_weights* head, int B, int K,
+                                            int H, int V, int32_t* tokens, float* logp, void* workspace,
+                                            size_t workspace_bytes, void* stream);
+
 /* Draft step for callers that cannot allocate device memory.  Some callers cannot call
  * cudaMalloc or any allocator at all: code running inside a host framework that owns every
  * allocation, a plugin loaded into a process whose memory pool is fixed up front, or a

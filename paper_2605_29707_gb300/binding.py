@@ -27,7 +27,7 @@ SYMBOLS = ("domino_workspace_bytes", "domino_draft_step", "domino_workspace_byte
            "domino_draft_step_static_scratch", "domino_verify_tree_greedy", "domino_rollout_workspace_bytes",
            "domino_rollout_greedy", "domino_rollout_sample", "domino_input_table_bytes",
            "domino_build_input_table", "domino_launches_per_step_table", "domino_debug_hold",
-           "domino_verify_tree_sample")
+           "domino_verify_tree_sample", "domino_rollout_sample_gumbel")
 
 DOMINO_STATIC_SCRATCH_BYTES = 16 << 20
 
@@ -103,6 +103,9 @@ def load():
     lib.domino_rollout_sample.argtypes = [P, P, P, P, ctypes.POINTER(domino_head_weights)] + [I] * 4 + [
         P, P, P, ctypes.c_size_t, P]
     lib.domino_rollout_sample.restype = I
+    lib.domino_rollout_sample_gumbel.argtypes = [P, P, ctypes.c_uint64, P, ctypes.POINTER(domino_head_weights)] + [
+        I] * 4 + [P, P, P, ctypes.c_size_t, P]
+    lib.domino_rollout_sample_gumbel.restype = I
     lib.domino_input_table_bytes.argtypes = [I, I]
     lib.domino_input_table_bytes.restype = S
     lib.domino_build_input_table.argtypes = [P, P, I, I, I, P, P]
@@ -260,6 +263,15 @@ def domino_rollout_sample(hidden, anchors, uniforms, w_lm, head, B, K, H, V, tok
     return int(load().domino_rollout_sample(_addr(hidden), _addr(anchors), _addr(uniforms), _addr(w_lm), h, B, K, H,
                                             V, _addr(tokens), _addr(logp), _addr(workspace), int(workspace_bytes),
                                             _stream(stream)))
+
+
+def domino_rollout_sample_gumbel(hidden, anchors, seed, w_lm, head, B, K, H, V, tokens, logp, workspace,
+                                 workspace_bytes, stream=None) -> int:
+    """Sampled sequential draft loop by the exponential race under a 64-bit ``seed``."""
+    h = ctypes.byref(head) if head is not None else None
+    return int(load().domino_rollout_sample_gumbel(_addr(hidden), _addr(anchors), int(seed) & ((1 << 64) - 1),
+                                                   _addr(w_lm), h, B, K, H, V, _addr(tokens), _addr(logp),
+                                                   _addr(workspace), int(workspace_bytes), _stream(stream)))
 
 
 def domino_debug_hold(what, gru_cta=-1, step=-1) -> int:

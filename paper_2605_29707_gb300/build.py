@@ -17,7 +17,8 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libdomino.so")
-SOURCES = ["api.cu", "tc_softmax.cu", "tc_softmax_k8.cu", "tc_store.cu", "gru.cu", "tree.cu", "verify.cu", "rollout.cu"]
+SOURCES = ["api.cu", "tc_softmax.cu", "tc_softmax_k8.cu", "tc_store.cu", "gru.cu", "tree.cu", "verify.cu", "rollout.cu",
+           "rollout_race.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

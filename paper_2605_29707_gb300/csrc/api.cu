@@ -997,10 +997,11 @@ size_t domino_rollout_workspace_bytes(int B, int K, int H, int V, int Ds, int R)
 }
 
 namespace {
-// The greedy (uniforms NULL) and the sampled rollout.
-int rollout_entry(const void* hidden, const int32_t* anchors, const float* uniforms, const void* w_lm,
-                  const domino_head_weights* head, int B, int K, int H, int V, int32_t* tokens, float* logp,
-                  void* workspace, size_t workspace_bytes, void* stream) {
+// The greedy (uniforms NULL, race false), the inverse-CDF sampled (uniforms) and the seeded
+// exponential-race sampled (race) rollout.
+int rollout_entry(const void* hidden, const int32_t* anchors, const float* uniforms, bool race, uint64_t seed,
+                  const void* w_lm, const domino_head_weights* head, int B, int K, int H, int V, int32_t* tokens,
+                  float* logp, void* workspace, size_t workspace_bytes, void* stream) {
   const bool hd = head_active(head);
   if (!hidden || !anchors || !w_lm || !tokens || !logp || !workspace) return DOMINO_ERR_INVALID_ARG;
   if (hd && (!head->emb || !head->w_ih || !head->w_hh || !head->w1)) return DOMINO_ERR_INVALID_ARG;
@@ -1065,8 +1066,10 @@ int rollout_entry(const void* hidden, const int32_t* anchors, const float* unifo
   rp.barrier = reinterpret_cast<unsigned*>(ws + 64);
   rp.ucount = reinterpret_cast<unsigned*>(ws + 128);  // cleared with the status and the barrier
   rp.uhcount = reinterpret_cast<unsigned*>(ws + 192);
-  // greedy: the argmax keys of the sequences (cleared with them)
+  // greedy and race: the (perturbed) argmax keys of the sequences (cleared with them)
   rp.best = uniforms ? nullptr : reinterpret_cast<unsigned long long*>(ws + 256);
+  rp.race = race ? 1 : 0;
+  rp.seed = seed;
   rp.tokens = tokens;
   rp.logp = logp;
   rp.status = status;
@@ -1085,16 +1088,23 @@ int rollout_entry(const void* hidden, const int32_t* anchors, const float* unifo
 int domino_rollout_greedy(const void* hidden, const int32_t* anchors, const void* w_lm,
                           const domino_head_weights* head, int B, int K, int H, int V, int32_t* tokens,
                           float* logp, void* workspace, size_t workspace_bytes, void* stream) {
-  return rollout_entry(hidden, anchors, nullptr, w_lm, head, B, K, H, V, tokens, logp, workspace, workspace_bytes,
-                       stream);
+  return rollout_entry(hidden, anchors, nullptr, false, 0, w_lm, head, B, K, H, V, tokens, logp, workspace,
+                       workspace_bytes, stream);
 }
 
 int domino_rollout_sample(const void* hidden, const int32_t* anchors, const float* uniforms, const void* w_lm,
                           const domino_head_weights* head, int B, int K, int H, int V, int32_t* tokens,
                           float* logp, void* workspace, size_t workspace_bytes, void* stream) {
   if (!uniforms || (reinterpret_cast<uintptr_t>(uniforms) & 3u) != 0) return DOMINO_ERR_INVALID_ARG;
-  return rollout_entry(hidden, anchors, uniforms, w_lm, head, B, K, H, V, tokens, logp, workspace, workspace_bytes,
-                       stream);
+  return rollout_entry(hidden, anchors, uniforms, false, 0, w_lm, head, B, K, H, V, tokens, logp, workspace,
+                       workspace_bytes, stream);
+}
+
+int domino_rollout_sample_gumbel(const void* hidden, const int32_t* anchors, uint64_t seed, const void* w_lm,
+                                 const domino_head_weights* head, int B, int K, int H, int V, int32_t* tokens,
+                                 float* logp, void* workspace, size_t workspace_bytes, void* stream) {
+  return rollout_entry(hidden, anchors, nullptr, true, seed, w_lm, head, B, K, H, V, tokens, logp, workspace,
+                       workspace_bytes, stream);
 }
 
 int domino_launches_per_step(int B, int K, int H, int V, int Ds, int R, int k, int N) {

@@ -206,13 +206,17 @@ struct RolloutParams {
   float* partials;              // float4 (max, sum exp, argmax bits, 0) per sequence: greedy
                                 // [K][grid][kRollComputeWarps][kRollMaxB] (per warp); sampled
                                 // [2][grid][kRollMaxB] (per CTA), by step parity
-  unsigned long long* best;     // greedy: [2][kRollMaxB] keys of each sequence's argmax by step parity
-                                // (cleared); nullptr in sampled mode (every CTA combines the partials)
+  unsigned long long* best;     // greedy and race: [2][kRollMaxB] keys of each sequence's (perturbed)
+                                // argmax by step parity (cleared); nullptr in inverse-CDF mode (every CTA
+                                // combines the partials)
   unsigned* barrier;            // grid barrier counter (cleared)
   int32_t* tokens;              // [B, K] t_1 .. t_K
   float* logp;                  // [B, K]
   int* status;
-  const float* uniforms;        // [B, K] in [0, 1): sampled mode; nullptr: greedy
+  const float* uniforms;        // [B, K] in [0, 1): sampled mode (inverse CDF); nullptr: greedy or race
+  int race;                     // seeded sampled mode: t_{j+1} = argmax_v L_j[v] + Gumbel(seed, b, j, v)
+                                // (the exponential race); keys, partials and logp as greedy (best set)
+  unsigned long long seed;      // race: the generator's key
   float* lg;                    // [2][B][V] sampled mode: every CTA's final logits, by step parity
   const float* x_table;         // [V, 3 Ds] emb . W_ih^T, or nullptr (phase A projects emb[t] itself)
   float* uh;                    // [B*K][R] scratch for hidden . W1[:, :H]^T (resident kernel), or nullptr

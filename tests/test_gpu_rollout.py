@@ -341,3 +341,102 @@ def test_rollout_sample_uniform_ends_and_bad_pointer():
     h = ctypes.byref(head)
     assert f(hidden.data_ptr(), anchors.data_ptr(), bad, w["w_lm"].data_ptr(), h, c.B, c.K, c.H, c.V,
              out_t.data_ptr(), out_l.data_ptr(), ws.data_ptr(), nbytes, None) == binding.DOMINO_ERR_INVALID_ARG
+
+
+# ---------------------------------------------------------------------------- exponential race
+def _run_gpu_gumbel(wl, seed, head_on=True, table=False):
+    c = wl.cfg
+    dev = torch.device("cuda:0")
+    w, head = _device_weights(wl, dev, head_on, table)
+    hidden = torch.from_numpy(wl.hidden.view(np.int16)).view(torch.bfloat16).to(dev)
+    anchors = torch.from_numpy(np.ascontiguousarray(wl.prefix_ids[:, 0])).to(dev)
+    nbytes = binding.domino_rollout_workspace_bytes(c.B, c.K, c.H, c.V, c.Ds if head_on else 0, c.R if head_on else 0)
+    ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    tokens = torch.full((c.B, c.K), -7, dtype=torch.int32, device=dev)
+    logp = torch.full((c.B, c.K), 7.0, dtype=torch.float32, device=dev)
+    s = torch.cuda.current_stream(dev)
+    rc = binding.domino_rollout_sample_gumbel(hidden, anchors, seed, w["w_lm"], head, c.B, c.K, c.H, c.V, tokens,
+                                              logp, ws, nbytes, s)
+    assert rc == 0, binding.domino_status_string(rc)
+    assert binding.domino_check_status(ws, s) == 0
+    return tokens.cpu().numpy(), logp.cpu().numpy()
+
+
+def _check_gumbel(wl, seed, head_on=True, table=False):
+    """Teacher-forced, as _check with the perturbed log-probabilities: at every position, under
+    the oracle's step fed the GPU's own tokens, the GPU token's log-probability plus the oracle's
+    perturbation of that sequence, step and token is within GAP of the largest such sum, the
+    GPU's logp within LOGP_TOL of the token's log-probability; up to the first position whose two
+    largest sums are within GAP the tokens equal the oracle rollout's.  (The perturbations are a
+    function of (seed, sequence, step, token) alone, so a rollout that took another, equally
+    valid token keeps the same perturbations for the steps after it.)"""
+    c = wl.cfg
+    w = wl.weights if head_on else {"w_lm": wl.weights["w_lm"], "b2": wl.weights.get("b2")}
+    tokens, logp = _run_gpu_gumbel(wl, seed, head_on, table)
+    anchors = np.ascontiguousarray(wl.prefix_ids[:, 0]).astype(np.int32)
+    o_tok, _ = oracle.rollout_sample_gumbel(w, wl.hidden, anchors, seed)
+    excused = 0
+    for b in range(c.B):
+        prefix = np.concatenate([[anchors[b]], tokens[b, :-1]]).astype(np.int32)[None, :]
+        ref = oracle.draft_step(w, wl.hidden[b:b + 1], prefix, 1, 1, want_logp_full=True)
+        lp = ref["logp_full"][0]
+        same = True
+        for j in range(c.K):
+            t = int(tokens[b, j])
+            assert 0 <= t < c.V
+            key = lp[j] + oracle.gumbel_row(seed, b, j, c.V)
+            best = float(key.max())
+            assert key[t] >= best - GAP, (b, j, t, key[t], best)
+            assert abs(float(logp[b, j]) - lp[j, t]) <= LOGP_TOL, (b, j, logp[b, j], lp[j, t])
+            if same:
+                top2 = np.partition(key, -2)[-2:]
+                if abs(top2[1] - top2[0]) > GAP:
+                    assert t == int(o_tok[b, j]), (b, j, t, o_tok[b, j])
+                elif t != int(o_tok[b, j]):
+                    excused += 1
+                    same = False
+    return excused
+
+
+@pytest.mark.parametrize("cfg", [
+    inputs.CONFIGS["tiny"],
+    inputs.custom_config("race-b3", B=3, K=8, H=512, V=3000, Ds=64, R=64, seed=61, biases=True),
+    inputs.custom_config("race-b8", B=8, K=5, H=256, V=1000, Ds=32, R=16, seed=62),
+    inputs.custom_config("race-b5", B=5, K=4, H=256, V=2000, Ds=32, R=32, seed=63),
+    # r > 256: the streamed kernel
+    inputs.custom_config("race-wide", B=6, K=4, H=256, V=2500, Ds=32, R=512, seed=64, biases=True),
+    # tensor-memory, shared-memory and L2 rows of W2 in every CTA, a ragged last slice
+    inputs.custom_config("race-tiers", B=8, K=3, H=256, V=167001, Ds=32, R=256, seed=65),
+])
+def test_rollout_sample_gumbel_matches_oracle(cfg):
+    _check_gumbel(_full_emb(inputs.make_workload(cfg)), seed=0x9E3779B97F4A7C15)
+
+
+@pytest.mark.parametrize("cfg", [MMA_CASES[0], MMA_CASES[1], MMA_CASES[2], MMA_CASES[3]])
+def test_rollout_sample_gumbel_tensor_core_phase_c_matches_oracle(cfg):
+    _check_gumbel(_full_emb(inputs.make_workload(cfg)), seed=12345, table=True)
+
+
+def test_rollout_sample_gumbel_head_off():
+    _check_gumbel(inputs.make_workload(inputs.custom_config("race-off", B=6, K=6, H=256, V=2000, seed=66)), seed=3,
+                  head_on=False)
+
+
+def test_rollout_sample_gumbel_full_size():
+    _check_gumbel(_full_size("qwen3-8b"), seed=2026)
+
+
+def test_rollout_sample_gumbel_full_size_with_input_table():
+    _check_gumbel(_full_size("qwen3-8b"), seed=2027, table=True)
+
+
+def test_rollout_sample_gumbel_seed_is_the_draw():
+    """The same seed draws the same tokens and log-probabilities; a seed that differs in its high
+    word only draws other tokens."""
+    wl = _full_emb(inputs.make_workload(inputs.custom_config("race-seed", B=2, K=6, H=128, V=700, Ds=16, R=8,
+                                                             seed=67)))
+    a, la = _run_gpu_gumbel(wl, 1 << 40)
+    b, lb = _run_gpu_gumbel(wl, 1 << 40)
+    assert (a == b).all() and np.array_equal(la, lb)
+    c, _ = _run_gpu_gumbel(wl, (1 << 40) + (1 << 33))
+    assert (a != c).any()
