@@ -189,7 +189,7 @@ struct TreeParams {
 };
 cudaError_t launch_merge_tree(const TreeParams& p, cudaStream_t stream);
 
-// ---------------------------------------------------------------- greedy rollout (rollout.cu)
+// ---------------------------------------------------------------- sequential draft loop (rollout*.cu)
 constexpr int kRollMaxB = 8;  // sequences per rollout launch
 constexpr unsigned kGreedyIdMask = 0x3FFFFFu;  // greedy rollout keys: token ids below 2^22
 constexpr int kRollComputeWarps = 8;             // compute warps of a rollout CTA

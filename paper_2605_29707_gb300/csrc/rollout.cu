@@ -101,7 +101,8 @@ cudaError_t launch_rollout(const RolloutParams& p, int grid, cudaStream_t stream
   CUtensorMap tm;
   if (tm_w2 != nullptr) tm = *tm_w2;
   else memset(&tm, 0, sizeof(tm));  // never read: phase C stays on the CUDA cores
-  return pp.race ? launch_rollout_race(pp, grid, smem, stream, tm) : launch_rollout_b<false>(pp, grid, smem, stream, tm);
+  if (pp.race) return launch_rollout_race(pp, grid, smem, stream, tm);
+  return launch_rollout_b<false>(pp, grid, smem, stream, tm);
 }
 
 }  // namespace dm
