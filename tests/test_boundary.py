@@ -144,6 +144,10 @@ def test_rollout_rejects_bad_sizes_before_any_device_work():
     assert f(1, 4, 256, 100, 60, 64) == 0       # d_s not a multiple of 8
     assert binding.domino_rollout_greedy(None, None, None, None, 1, 4, 256, 100, None, None, None, 0) == \
         binding.DOMINO_ERR_INVALID_ARG
+    assert binding.domino_rollout_sample_gumbel(None, None, 1, None, None, 1, 4, 256, 100, None, None, None, 0) == \
+        binding.DOMINO_ERR_INVALID_ARG
+    assert binding.domino_rollout_sample_gumbel(None, None, (1 << 64) - 1, None, None, 1, 4, 256, 100, None, None,
+                                                None, 0) == binding.DOMINO_ERR_INVALID_ARG
 
 
 def test_debug_hold_argument_checks_and_header_constants():
