@@ -764,8 +764,10 @@ __device__ __forceinline__ void pass_push(const float (&dot)[kRowsPerPass * KB],
     const float logit = *x + d;
     *x = logit;  // the final logit, for the sampled mode's scan of this CTA's rows
     lse_push(mine, logit, vid0 + role.r);
-    if constexpr (kRace)
-      pick_push(pick, logit, race_gumbel(race_words(seed, role.b >> 2, j, vid0 + role.r), role.b & 3), vid0 + role.r);
+    if constexpr (kRace) {
+      const float g = race_gumbel(race_words(seed, role.b >> 2, j, vid0 + role.r), role.b & 3);
+      pick_push(pick, logit, g, vid0 + role.r);
+    }
   }
 }
 
