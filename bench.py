@@ -601,7 +601,8 @@ def measure_config(name, device, stream, steps, warmup, num_sms, peaks):
     input_table = {"us_per_step": round(us_tab, 2), "value": round(c.B * 1e6 / us_tab, 3),
                    "launches_per_step": st_tab.launches_per_step(),
                    "step_roofline_frac": step_roofline(c, peaks, us_tab)["frac"],
-                   "note": "the same step reading the GRU's input-gate sums from the table; us_per_step is without it"}
+                   "note": "us_per_step here: the same step reading the GRU's input-gate sums from the table; "
+                           "the config's own us_per_step is the step without it"}
     del st_tab
     out = {"config": config_dict(c), "us_per_step": round(us, 2), "value": round(c.B * 1e6 / us, 3), "unit": UNIT,
            "steps": steps, "warmup": max(3, warmup), "gpu_launches": steps * st.launches_per_step(),
@@ -748,7 +749,8 @@ def run_ours(args):
         us_tab = time_steps(st_tab, hidden, ids, stream, min(args.steps, 1000), args.warmup)
         input_table = {"us_per_step": round(us_tab, 2), "launches_per_step": st_tab.launches_per_step(),
                        "table_bytes": st_tab.x_table.numel() * 4,
-                       "note": "the same step reading the GRU's input-gate sums from the table; value is the step without it"}
+                       "note": "us_per_step here: the same step reading the GRU's input-gate sums from the table; "
+                               "the line's value and us_per_step are the step without it"}
         del st_tab
 
     # ---- the step after the draft: verification of this step's trees against synthetic target
