@@ -368,8 +368,8 @@ enum domino_kernel_kind {
                                      M <= 128) */
   DOMINO_KERNEL_VOCAB = 4,        /* [hidden | u] . [W_lm | W2]^T with online softmax / top-k */
   DOMINO_KERNEL_TREE = 5,         /* merge to log-probs and top-k; best-first tree */
-  DOMINO_KERNEL_ROLLOUT_BASE = 6, /* domino_rollout_greedy: W_lm hidden_j of every position */
-  DOMINO_KERNEL_ROLLOUT = 7,      /* domino_rollout_greedy: the K sequential steps */
+  DOMINO_KERNEL_ROLLOUT_BASE = 6, /* domino_rollout_*: W_lm hidden_j of every position */
+  DOMINO_KERNEL_ROLLOUT = 7,      /* domino_rollout_*: the K sequential steps */
   DOMINO_KERNEL_VERIFY = 8,       /* domino_verify_tree_greedy / _sample: row argmax or draw, and
                                      tree walk */
   DOMINO_KERNEL_KINDS = 9
