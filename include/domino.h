@@ -311,7 +311,9 @@ DOMINO_API int domino_rollout_greedy(const void* hidden, const int32_t* anchors,
  * Dror and Shaw, SC 2011), key = seed (low word first), counter (v, j, floor(b / 4), 0), word
  * b mod 4, u = (that word's top 23 bits + 1/2) / 2^23.  This draws t_{j+1} from softmax(L_j);
  * logp_j = log-softmax(L_j)[t_{j+1}].  The perturbations are computed in fp32 on the device, so
- * where two perturbed logits lie within rounding of each other either may win.  Unlike
+ * where two perturbed logits lie within rounding of each other either may win.  The draws depend
+ * on (seed, b, j, v) alone, so a call with the same seed repeats them: pass a new seed for every
+ * block (a running counter will do).  Unlike
  * domino_rollout_sample it needs no per-step scan after the argmax: it costs what the greedy
  * loop costs (one grid barrier per step on the fast path) plus the generator.  Arguments,
  * outputs, workspace (domino_rollout_workspace_bytes) and errors as domino_rollout_greedy. */
