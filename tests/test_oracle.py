@@ -766,3 +766,42 @@ def test_rollout_sample_gumbel_follows_the_teacher_forced_step(B, K, V, H, Ds, R
             assert logp[b, j] == pytest.approx(ref["logp_full"][b, j, t], abs=1e-12)
     other, _ = oracle.rollout_sample_gumbel(w, hidden, anchors, seed + 1)
     assert (other != tokens).any()
+
+
+def test_rollout_sample_gumbel_exact_tie_takes_the_lower_id():
+    """O15's tie rule: two ids whose perturbations coincide exactly (the 23-bit uniform repeats
+    about once per 2^23 pairs, so a row of 2^16 perturbations holds a few such pairs) and whose
+    logits are equal and far above the rest tie exactly; the lower id is drawn."""
+    seed = 99
+    g = oracle.gumbel_row(seed, 0, 0, 1 << 16)
+    order = np.argsort(g, kind="stable")
+    same = np.nonzero(g[order[1:]] == g[order[:-1]])[0]
+    assert same.size > 0
+    v1, v2 = sorted((int(order[same[0]]), int(order[same[0] + 1])))
+    V, H = v2 + 1, 8
+    w_lm = np.zeros((V, H), np.float32)
+    w_lm[v1, 0] = w_lm[v2, 0] = 30.0  # 30 + g > 27 beats 0 + g < 17 for every other id
+    hidden = np.zeros((1, 1, H), np.float32)
+    hidden[0, 0, 0] = 1.0
+    tokens, logp = oracle.rollout_sample_gumbel({"w_lm": bf16(w_lm)}, bf16(hidden), np.array([0], np.int32), seed)
+    assert int(tokens[0, 0]) == v1
+    z = np.zeros(V)
+    z[[v1, v2]] = 30.0
+    assert logp[0, 0] == pytest.approx(30.0 - (z.max() + np.log(np.exp(z - z.max()).sum())), abs=1e-9)
+
+
+def test_gumbel_row_reaches_both_ends_of_the_uniform_finitely():
+    """O14's uniform never reaches 0 or 1: the words whose top 23 bits are all zero or all one
+    (one in 2^23 each) give the smallest and largest perturbations, -log(-log(2^-24)) and
+    -log(-log(1 - 2^-24)), both finite; scanning rows of 2^22 perturbations finds both."""
+    lo, hi = -math.log(-math.log(2.0 ** -24)), -math.log(-math.log(1.0 - 2.0 ** -24))
+    found_lo = found_hi = False
+    for j in range(24):
+        g = oracle.gumbel_row(7, 1, j, 1 << 22)
+        assert np.isfinite(g).all(), j
+        assert g.min() >= lo - 1e-12 and g.max() <= hi + 1e-12
+        found_lo |= abs(float(g.min()) - lo) < 1e-12
+        found_hi |= abs(float(g.max()) - hi) < 1e-12
+        if found_lo and found_hi:
+            break
+    assert found_lo and found_hi
