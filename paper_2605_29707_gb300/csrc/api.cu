@@ -11,8 +11,10 @@
 // Other batches: memset (the control words: status, merge counters), gather (id check, state
 // words cleared; E = emb[ids] unless a table is given), tc store Xp = E . W_ih^T (not with a
 // table), tc store Up = hidden . W1[:, :H]^T, gru, tc soft, tree; large M moves the W1 GEMM
-// (both halves) and a SiLU kernel after the GRU.  With the correction branch off only memset, gather (id check), tc soft and
-// tree run.
+// (both halves) and a SiLU kernel (u_finalize) after the GRU, and launches X, GRU, W1,
+// u_finalize and the vocabulary GEMM on CTA pairs each as a programmatic dependent of the kernel
+// before it (the pair kernel waits for u only before its W2 segment).  With the correction
+// branch off only memset, gather (id check), tc soft and tree run.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
@@ -978,10 +980,10 @@ int make_roll_plan(int B, int K, int H, int V, int Ds, int R, bool head, RollPla
   p.off_h = take(static_cast<size_t>(2) * B * (p.Ds > 0 ? p.Ds : 1) * 4);
   p.clear_bytes = off;
   p.off_u = take(static_cast<size_t>(B) * (p.R > 0 ? p.R : 1) * 4);
-  // greedy: every step's, per warp (the log-probabilities are merged at the end); sampled: two,
-  // by step parity, per CTA
+  // greedy and race: every step's, per warp (the log-probabilities are merged at the end);
+  // inverse-CDF sampled: two, by step parity, per CTA
   p.off_part = take(static_cast<size_t>(K > 2 ? K : 2) * p.grid * dm::kRollComputeWarps * dm::kRollMaxB * 16);
-  p.off_lg = take(static_cast<size_t>(2) * B * V * 4);  // sampled mode: final logits, by step parity
+  p.off_lg = take(static_cast<size_t>(2) * B * V * 4);  // inverse-CDF sampling: final logits, by step parity
   p.off_base = take(static_cast<size_t>(p.M) * V * 4);
   p.off_uh = take(static_cast<size_t>(p.M) * (p.R > 0 ? p.R : 1) * 4);  // hidden . W1[:, :H]^T
   p.off_gh = take(static_cast<size_t>(2) * B * 3 * (p.Ds > 0 ? p.Ds : 1) * 4);  // W_hh h_j, by step parity
